@@ -1,0 +1,124 @@
+/*
+ * lpvit.h -- C ABI of liblpvit.so: block-sparse linear layers for LPViT-pruned vision
+ * transformers (Xu et al., "LPViT: Low-Power Semi-structured Pruning for Vision
+ * Transformers", arXiv 2407.02068), hand-written for NVIDIA GB300 (sm_103a).
+ *
+ * The operation (Sec. 3.1, block-structured pruning; Sec. 3.3, block-sparse matmul):
+ *
+ *     Y[m][o] = act( sum_i X[m][i] * W~[o][i] + bias[o] ),
+ *     W~[o][i] = W[o][i] if mask[o/b][i/b] != 0, else 0,
+ *
+ * with W stored [n = out features][k = in features] (PyTorch Linear layout), b x b blocks
+ * (b in {16, 32, 64}), act = identity (lpvit_bsr_linear) or the exact GELU
+ * 0.5*y*(1+erf(y/sqrt 2)) (lpvit_bsr_linear_gelu, the DeiT fc1 activation). Only the kept
+ * blocks are stored and multiplied: the work is proportional to the number of kept blocks,
+ * as in the power model of Sec. 3.3 (Eq. for P).
+ *
+ * Conventions for every call:
+ *  - All pointers except nnzb_host are DEVICE pointers owned by the caller; the library never
+ *    allocates, frees or keeps them. All calls are asynchronous on `stream` (a cudaStream_t
+ *    passed as void*, NULL = legacy default stream) unless stated otherwise.
+ *  - bf16 means IEEE-754 bfloat16 (raw 16-bit storage); all matrices are row-major.
+ *  - A status is returned synchronously for argument errors; CUDA launch errors map to
+ *    LPVIT_ERR_CUDA. Errors raised inside a running kernel (a bounded wait that ran out)
+ *    are recorded in the workspace and reported by lpvit_check().
+ *  - The GPU must be compute capability 10.3 (sm_103a); other devices get
+ *    LPVIT_ERR_UNSUPPORTED.
+ */
+#ifndef LPVIT_H
+#define LPVIT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  LPVIT_OK = 0,
+  LPVIT_ERR_INVALID_ARG = 1, /* bad shape, null pointer, misaligned pointer or stride      */
+  LPVIT_ERR_UNSUPPORTED = 2, /* b not in {16,32,64}, or not an sm_103 device               */
+  LPVIT_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed                          */
+  LPVIT_ERR_TIMEOUT = 4,     /* a device-side bounded wait ran out (see lpvit_check)       */
+  LPVIT_ERR_WORKSPACE = 5    /* workspace or schedule buffer smaller than required          */
+} lpvit_status;
+
+typedef enum { LPVIT_BF16 = 0, LPVIT_F32 = 1 } lpvit_dtype;
+
+/* Block-sparse (BSR) weight, filled by lpvit_pack_bsr. Every pointer is caller-owned device
+ * memory of the size stated; the struct itself is a plain host value.
+ *   row panel r = output rows [r*b, (r+1)*b);  n/b panels.
+ *   row_ptr [n/b + 1]          int32   exclusive prefix sum of kept blocks per panel
+ *   col_idx [nnzb_capacity]    int32   kept block columns of each panel, ascending
+ *   blocks  [nnzb_capacity][b][b] bf16 kept tiles of W, row-major inside the tile, bits unchanged
+ *   sched   [sched_bytes]      bytes   work list for lpvit_bsr_linear (layout private to the
+ *                                      library; see lpvit_sched_bytes)
+ * nnzb_capacity must be >= the number of kept blocks; (n/b)*(k/b) always suffices. */
+typedef struct {
+  int32_t n, k, b;
+  int32_t nnzb_capacity;
+  int32_t *row_ptr;
+  int32_t *col_idx;
+  void *blocks;
+  void *sched;
+  size_t sched_bytes;
+} lpvit_bsr;
+
+/* Bytes of the `sched` buffer needed for an n x k weight with b x b blocks (0 if the shape is
+ * invalid). The work list groups the row panels into 128-feature groups and lists, per group,
+ * the block columns where any panel of the group keeps a block (Sec. 3.3: one block matmul per
+ * kept block and token tile). */
+size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t b);
+
+/* Pack W (bf16 [n][k], row-major, 16-byte aligned) under the block mask (uint8 [n/b][k/b],
+ * nonzero = kept; Sec. 3.1 M_alpha) into bsr->row_ptr / col_idx / blocks and build the work
+ * list in bsr->sched. bsr->n, k, b, nnzb_capacity and all its pointers must be set by the
+ * caller. The contents of W inside removed blocks are never read.
+ * If nnzb_host is not NULL the call synchronises `stream` and stores the number of kept
+ * blocks there. If the mask keeps more blocks than nnzb_capacity, nothing beyond the capacity
+ * is written, the work list is marked invalid (linear calls on it then compute nothing and
+ * lpvit_check() reports LPVIT_ERR_WORKSPACE), and, when nnzb_host is given, this call returns
+ * LPVIT_ERR_WORKSPACE. A capacity of (n/b)*(k/b) never overflows.
+ * Errors: LPVIT_ERR_INVALID_ARG (shape, null or misaligned pointer), LPVIT_ERR_UNSUPPORTED
+ * (b), LPVIT_ERR_WORKSPACE (sched_bytes too small), LPVIT_ERR_CUDA. */
+lpvit_status lpvit_pack_bsr(const void *W, const uint8_t *mask, lpvit_bsr *bsr, int32_t *nnzb_host,
+                            void *stream);
+
+/* Bytes of device workspace lpvit_bsr_linear[_gelu] needs for m tokens. The workspace holds
+ * scheduler counters, the device error word and, for small m, fp32 partial sums of split
+ * work units. It must be zero-filled once before its first use (cudaMemset); every call
+ * leaves its counters at zero again. Calls that may run concurrently must not share a
+ * workspace. */
+size_t lpvit_workspace_bytes(const lpvit_bsr *bsr, int64_t m);
+
+/* Y = X W~^T + bias for m tokens.
+ *   X     bf16 [m][ldx], ldx >= k, ldx % 8 == 0, 16-byte aligned (the first k columns are used)
+ *   bias  float32 [n] or NULL (zero bias)
+ *   Y     [m][ldy] of y_dtype (bf16, round to nearest even, or float32), ldy >= n;
+ *         only columns [0, n) of rows [0, m) are written. X and Y must not overlap.
+ *   workspace / ws_bytes: see lpvit_workspace_bytes.
+ * Output columns of a panel with no kept block equal bias (or GELU(bias)).
+ * Errors: LPVIT_ERR_INVALID_ARG, LPVIT_ERR_UNSUPPORTED, LPVIT_ERR_WORKSPACE, LPVIT_ERR_CUDA. */
+lpvit_status lpvit_bsr_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias,
+                              void *Y, int64_t ldy, lpvit_dtype y_dtype, void *workspace, size_t ws_bytes,
+                              void *stream);
+
+/* As lpvit_bsr_linear, followed by the exact GELU 0.5*y*(1+erf(y/sqrt 2)) (the DeiT MLP fc1). */
+lpvit_status lpvit_bsr_linear_gelu(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx,
+                                   const float *bias, void *Y, int64_t ldy, lpvit_dtype y_dtype, void *workspace,
+                                   size_t ws_bytes, void *stream);
+
+/* Synchronises `stream`, then reads and clears the error word in `workspace`.
+ * Returns LPVIT_OK, LPVIT_ERR_TIMEOUT (a device-side bounded wait ran out; the kernel
+ * stopped early and its output is incomplete) or LPVIT_ERR_CUDA. */
+lpvit_status lpvit_check(void *workspace, void *stream);
+
+/* Static English description of a status code. */
+const char *lpvit_status_string(lpvit_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LPVIT_H */

@@ -1,0 +1,110 @@
+"""Block-sparse linear layers for LPViT-pruned vision transformers on GB300 (sm_103a).
+
+LPViT (arXiv 2407.02068) prunes each linear weight of a ViT in b x b blocks (Sec. 3.1) so that
+the layer becomes a block-sparse matmul whose work is proportional to the kept blocks
+(Sec. 3.3). This package wraps the C library ``liblpvit.so`` (include/lpvit.h):
+
+* ``pack_bsr(W, mask, b)``  -- mask -> BSR pack + work list, on the GPU
+* ``bsr_linear(w, X, bias, gelu=...)`` -- Y = act(X (W (.) M)^T + bias)
+
+PyTorch provides device memory and streams only; every step runs in the library's kernels.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import torch
+
+from . import _lib
+
+__all__ = ["BsrWeight", "pack_bsr", "workspace_for", "bsr_linear", "check", "LpvitError"]
+
+LpvitError = _lib.LpvitError
+
+
+def _stream_handle(stream) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return int(s.cuda_stream)
+
+
+@dataclass
+class BsrWeight:
+    """A packed block-sparse weight: device tensors owned by this object."""
+    n: int
+    k: int
+    b: int
+    capacity: int
+    row_ptr: torch.Tensor   # int32 [n/b + 1]
+    col_idx: torch.Tensor   # int32 [capacity]
+    blocks: torch.Tensor    # bf16 [capacity, b, b]
+    sched: torch.Tensor     # uint8 [sched_bytes]
+    nnzb: int | None = None
+
+    def struct(self) -> _lib.lpvit_bsr:
+        return _lib.lpvit_bsr(self.n, self.k, self.b, self.capacity, self.row_ptr.data_ptr(),
+                              self.col_idx.data_ptr(), self.blocks.data_ptr(), self.sched.data_ptr(),
+                              self.sched.numel())
+
+
+def pack_bsr(W: torch.Tensor, mask: torch.Tensor, b: int, capacity: int | None = None, count: bool = False,
+             stream=None) -> BsrWeight:
+    """Pack W (bf16 [n, k], CUDA) under the block mask (uint8 [n/b, k/b], CUDA, nonzero = kept)."""
+    if W.dtype != torch.bfloat16 or not W.is_cuda or W.dim() != 2:
+        raise ValueError("W must be a 2-D bf16 CUDA tensor")
+    W = W.contiguous()
+    mask = mask.to(device=W.device, dtype=torch.uint8).contiguous()
+    n, k = W.shape
+    if capacity is None:
+        capacity = (n // b) * (k // b) if b > 0 and n % b == 0 and k % b == 0 else 0
+    sb = _lib.lpvit_sched_bytes(n, k, b)
+    dev = W.device
+    w = BsrWeight(n, k, b, capacity,
+                  torch.empty(max(n // max(b, 1), 0) + 1, dtype=torch.int32, device=dev),
+                  torch.empty(max(capacity, 1), dtype=torch.int32, device=dev),
+                  torch.empty((max(capacity, 1), max(b, 1), max(b, 1)), dtype=torch.bfloat16, device=dev),
+                  torch.empty(max(sb, 16), dtype=torch.uint8, device=dev))
+    s = w.struct()
+    st, nnzb = _lib.lpvit_pack_bsr(W.data_ptr(), mask.data_ptr(), s, count, _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_pack_bsr")
+    w.nnzb = nnzb
+    return w
+
+
+def workspace_for(w: BsrWeight, m: int, device=None) -> torch.Tensor:
+    """A zero-filled workspace of lpvit_workspace_bytes(w, m) bytes (256-byte aligned)."""
+    nbytes = _lib.lpvit_workspace_bytes(w.struct(), m)
+    return torch.zeros(max(nbytes, 256), dtype=torch.uint8, device=device or w.blocks.device)
+
+
+def bsr_linear(w: BsrWeight, X: torch.Tensor, bias: torch.Tensor | None = None, gelu: bool = False,
+               out: torch.Tensor | None = None, out_dtype=torch.bfloat16, workspace: torch.Tensor | None = None,
+               stream=None) -> torch.Tensor:
+    """Y = act(X W~^T + bias). X: bf16 [m, k] CUDA (a row-strided view with unit column stride is
+    fine); bias: fp32 [n] or None. Returns Y [m, n] (or writes ``out``)."""
+    if X.dtype != torch.bfloat16 or X.dim() != 2 or X.stride(1) != 1:
+        raise ValueError("X must be a 2-D bf16 tensor with unit column stride")
+    m = X.shape[0]
+    if out is None:
+        out = torch.empty((m, w.n), dtype=out_dtype, device=X.device)
+    if out.dtype not in (torch.bfloat16, torch.float32) or out.stride(1) != 1:
+        raise ValueError("out must be bf16 or fp32 with unit column stride")
+    if bias is not None:
+        if bias.dtype != torch.float32 or not bias.is_contiguous():
+            raise ValueError("bias must be a contiguous fp32 tensor")
+    if workspace is None:
+        workspace = workspace_for(w, m, X.device)
+    fn = _lib.lpvit_bsr_linear_gelu if gelu else _lib.lpvit_bsr_linear
+    st = fn(w.struct(), X.data_ptr(), m, X.stride(0), bias.data_ptr() if bias is not None else None,
+            out.data_ptr(), out.stride(0), _lib.LPVIT_F32 if out.dtype == torch.float32 else _lib.LPVIT_BF16,
+            workspace.data_ptr(), workspace.numel(), _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_bsr_linear_gelu" if gelu else "lpvit_bsr_linear")
+    return out
+
+
+def check(workspace: torch.Tensor, stream=None) -> None:
+    """Synchronise and raise if a kernel that used ``workspace`` reported a device-side error."""
+    st = _lib.lpvit_check(workspace.data_ptr(), _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_check")

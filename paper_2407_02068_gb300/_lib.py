@@ -1,0 +1,113 @@
+"""ctypes binding of liblpvit.so: one Python function per C entry point, same names, argument
+marshalling only (every step of the layer runs in the library's CUDA kernels).
+
+The library must have been built (``paper_2407_02068_gb300.build.build()``); if it is missing,
+loading raises instead of falling back to anything else.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+from .build import LIB
+
+LPVIT_OK = 0
+LPVIT_ERR_INVALID_ARG = 1
+LPVIT_ERR_UNSUPPORTED = 2
+LPVIT_ERR_CUDA = 3
+LPVIT_ERR_TIMEOUT = 4
+LPVIT_ERR_WORKSPACE = 5
+LPVIT_BF16 = 0
+LPVIT_F32 = 1
+
+EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_workspace_bytes", "lpvit_bsr_linear",
+           "lpvit_bsr_linear_gelu", "lpvit_check", "lpvit_status_string")
+
+
+class lpvit_bsr(ctypes.Structure):
+    _fields_ = [
+        ("n", ctypes.c_int32), ("k", ctypes.c_int32), ("b", ctypes.c_int32),
+        ("nnzb_capacity", ctypes.c_int32),
+        ("row_ptr", ctypes.c_void_p), ("col_idx", ctypes.c_void_p), ("blocks", ctypes.c_void_p),
+        ("sched", ctypes.c_void_p), ("sched_bytes", ctypes.c_size_t),
+    ]
+
+
+class LpvitError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: status {status} ({status_string(status)})")
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def load(path: str | None = None):
+    """Load liblpvit.so (once). Raises if the library has not been built."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        p = path or LIB
+        if not os.path.exists(p):
+            raise RuntimeError(f"{p} is missing: build the CUDA library first "
+                               "(python -c 'import __graft_entry__ as g; g.build()')")
+        lib = ctypes.CDLL(p)
+        V, I32, I64, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+        BP = ctypes.POINTER(lpvit_bsr)
+        lib.lpvit_sched_bytes.restype = SZ
+        lib.lpvit_sched_bytes.argtypes = [I32, I32, I32]
+        lib.lpvit_pack_bsr.restype = ctypes.c_int
+        lib.lpvit_pack_bsr.argtypes = [V, V, BP, ctypes.POINTER(I32), V]
+        lib.lpvit_workspace_bytes.restype = SZ
+        lib.lpvit_workspace_bytes.argtypes = [BP, I64]
+        for name in ("lpvit_bsr_linear", "lpvit_bsr_linear_gelu"):
+            f = getattr(lib, name)
+            f.restype = ctypes.c_int
+            f.argtypes = [BP, V, I64, I64, V, V, I64, ctypes.c_int, V, SZ, V]
+        lib.lpvit_check.restype = ctypes.c_int
+        lib.lpvit_check.argtypes = [V, V]
+        lib.lpvit_status_string.restype = ctypes.c_char_p
+        lib.lpvit_status_string.argtypes = [ctypes.c_int]
+        _lib = lib
+        return lib
+
+
+def status_string(status: int) -> str:
+    return load().lpvit_status_string(int(status)).decode()
+
+
+def lpvit_sched_bytes(n: int, k: int, b: int) -> int:
+    return int(load().lpvit_sched_bytes(n, k, b))
+
+
+def lpvit_pack_bsr(W_ptr: int, mask_ptr: int, bsr: lpvit_bsr, want_count: bool, stream: int):
+    """Returns (status, nnzb or None)."""
+    cnt = ctypes.c_int32(0)
+    st = load().lpvit_pack_bsr(W_ptr, mask_ptr, ctypes.byref(bsr), ctypes.byref(cnt) if want_count else None,
+                               stream)
+    return st, (cnt.value if want_count else None)
+
+
+def lpvit_workspace_bytes(bsr: lpvit_bsr, m: int) -> int:
+    return int(load().lpvit_workspace_bytes(ctypes.byref(bsr), m))
+
+
+def lpvit_bsr_linear(bsr, X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, ws_ptr, ws_bytes, stream) -> int:
+    return load().lpvit_bsr_linear(ctypes.byref(bsr), X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, ws_ptr,
+                                   ws_bytes, stream)
+
+
+def lpvit_bsr_linear_gelu(bsr, X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, ws_ptr, ws_bytes, stream) -> int:
+    return load().lpvit_bsr_linear_gelu(ctypes.byref(bsr), X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, ws_ptr,
+                                        ws_bytes, stream)
+
+
+def lpvit_check(ws_ptr: int, stream: int) -> int:
+    return load().lpvit_check(ws_ptr, stream)
+
+
+def lpvit_status_string(status: int) -> str:
+    return status_string(status)

@@ -1,0 +1,282 @@
+// C ABI of liblpvit.so (declared in include/lpvit.h): argument checks, TMA tensor-map encoding,
+// work sizing, and launches on the caller's stream. No allocation happens here.
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "lpvit.h"
+#include "lpvit_device.cuh"
+
+namespace lpvit {
+
+namespace {
+
+constexpr int MAX_DIM = 65536;
+constexpr uint64_t TIMEOUT_NS = 2000000000ull;  // 2 s per wait: far above any legitimate stall
+
+struct DeviceInfo {
+  bool queried = false;
+  bool supported = false;
+  int sms = 0;
+};
+DeviceInfo g_dev[64];
+std::mutex g_mu;
+
+bool device_info(int *sms, lpvit_status *st) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    *st = LPVIT_ERR_CUDA;
+    return false;
+  }
+  std::lock_guard<std::mutex> lk(g_mu);
+  DeviceInfo &d = g_dev[dev];
+  if (!d.queried) {
+    int major = 0, minor = 0, n = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+      *st = LPVIT_ERR_CUDA;
+      return false;
+    }
+    d.supported = (major == 10 && minor == 3);
+    d.sms = n;
+    d.queried = true;
+  }
+  if (!d.supported) {
+    *st = LPVIT_ERR_UNSUPPORTED;
+    return false;
+  }
+  *sms = d.sms;
+  return true;
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+bool valid_b(int b) { return b == 16 || b == 32 || b == 64; }
+
+bool shape_ok(int n, int k, int b) {
+  return valid_b(b) && n > 0 && k > 0 && n <= MAX_DIM && k <= MAX_DIM && n % b == 0 && k % b == 0;
+}
+
+int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// Entries per slice. With enough (token tile, group) units to fill every SM twice, a unit covers
+// the whole group; otherwise the group's block columns are cut into slices so that about two
+// units per SM exist, and the slices are summed by the fix-up.
+int choose_slice(int64_t n_tt, int n_groups, int kb, int sms) {
+  const int64_t units = n_tt * n_groups;
+  if (units >= 2LL * sms) return kb;
+  const int64_t s = ceil_div((int64_t)kb * units, 2LL * sms);
+  return (int)(s < 1 ? 1 : (s > kb ? kb : s));
+}
+
+struct WsLayout {
+  size_t tickets_off, partials_off, total;
+};
+
+WsLayout ws_layout(int64_t m, int n, int k, int b, int sms) {
+  WsLayout L;
+  const int64_t n_tt = ceil_div(m, TOKENS_PER_TILE);
+  const int ng = (int)ceil_div(n, GROUP_FEATURES);
+  const int kb = k / b;
+  const int S = choose_slice(n_tt, ng, kb, sms);
+  L.tickets_off = sizeof(Control);
+  size_t off = L.tickets_off + (size_t)ceil_div(n_tt * ng * 4, 256) * 256;
+  L.partials_off = off;
+  if (S < kb) off += (size_t)n_tt * ng * ceil_div(kb, S) * TOKENS_PER_TILE * GROUP_FEATURES * sizeof(float);
+  L.total = off;
+  return L;
+}
+
+lpvit_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LPVIT_OK : LPVIT_ERR_CUDA; }
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias, void *Y,
+                        int64_t ldy, lpvit_dtype y_dtype, void *workspace, size_t ws_bytes, void *stream, int gelu) {
+  if (!bsr) return LPVIT_ERR_INVALID_ARG;
+  const int n = bsr->n, k = bsr->k, b = bsr->b;
+  if (!valid_b(b)) return LPVIT_ERR_UNSUPPORTED;
+  if (!shape_ok(n, k, b)) return LPVIT_ERR_INVALID_ARG;
+  if (m < 0) return LPVIT_ERR_INVALID_ARG;
+  if (y_dtype != LPVIT_BF16 && y_dtype != LPVIT_F32) return LPVIT_ERR_INVALID_ARG;
+  if (m == 0) return LPVIT_OK;
+  if (!X || !Y || !bsr->blocks || !bsr->sched || !workspace) return LPVIT_ERR_INVALID_ARG;
+  if (bsr->nnzb_capacity < 0) return LPVIT_ERR_INVALID_ARG;
+  if (ldx < k || ldx % 8 != 0 || !aligned(X, 16)) return LPVIT_ERR_INVALID_ARG;
+  const size_t ysz = y_dtype == LPVIT_F32 ? 4 : 2;
+  if (ldy < n || !aligned(Y, ysz) || !aligned(bsr->blocks, 16) || !aligned(bsr->sched, 16) ||
+      !aligned(workspace, 256))
+    return LPVIT_ERR_INVALID_ARG;
+  if (bias && !aligned(bias, 4)) return LPVIT_ERR_INVALID_ARG;
+  if (m > (int64_t)0x7fffff00) return LPVIT_ERR_INVALID_ARG;
+  // X and Y must not overlap
+  {
+    const uintptr_t x0 = reinterpret_cast<uintptr_t>(X), x1 = x0 + (size_t)((m - 1) * ldx + k) * 2;
+    const uintptr_t y0 = reinterpret_cast<uintptr_t>(Y), y1 = y0 + (size_t)((m - 1) * ldy + n) * ysz;
+    if (x0 < y1 && y0 < x1) return LPVIT_ERR_INVALID_ARG;
+  }
+  if (bsr->sched_bytes < lpvit_sched_bytes(n, k, b)) return LPVIT_ERR_WORKSPACE;
+  int sms = 0;
+  lpvit_status st = LPVIT_OK;
+  if (!device_info(&sms, &st)) return st;
+  const WsLayout W = ws_layout(m, n, k, b, sms);
+  if (ws_bytes < W.total) return LPVIT_ERR_WORKSPACE;
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return LPVIT_ERR_CUDA;
+
+  const CUtensorMapSwizzle swz =
+      b == 16 ? CU_TENSOR_MAP_SWIZZLE_32B : (b == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
+  CUtensorMap tmX, tmW;
+  {
+    cuuint64_t dims[2] = {(cuuint64_t)k, (cuuint64_t)m};
+    cuuint64_t strides[1] = {(cuuint64_t)ldx * 2};
+    cuuint32_t box[2] = {(cuuint32_t)b, (cuuint32_t)TOKENS_PER_TILE};
+    cuuint32_t es[2] = {1, 1};
+    if (enc(&tmX, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(X), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return LPVIT_ERR_INVALID_ARG;
+  }
+  {
+    const int64_t cap = bsr->nnzb_capacity > 0 ? bsr->nnzb_capacity : 1;
+    cuuint64_t dims[2] = {(cuuint64_t)b, (cuuint64_t)(cap * b)};
+    cuuint64_t strides[1] = {(cuuint64_t)b * 2};
+    cuuint32_t box[2] = {(cuuint32_t)b, (cuuint32_t)b};
+    cuuint32_t es[2] = {1, 1};
+    if (enc(&tmW, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, bsr->blocks, dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return LPVIT_ERR_INVALID_ARG;
+  }
+  LinearParams P;
+  P.sched = static_cast<const int32_t *>(bsr->sched);
+  P.bias = bias;
+  P.Y = Y;
+  P.ldy = ldy;
+  P.m = m;
+  P.n = n;
+  P.k = k;
+  P.n_tt = (int)ceil_div(m, TOKENS_PER_TILE);
+  P.n_groups = (int)ceil_div(n, GROUP_FEATURES);
+  P.S = choose_slice(P.n_tt, P.n_groups, k / b, sms);
+  P.y_f32 = y_dtype == LPVIT_F32;
+  P.gelu = gelu;
+  uint8_t *ws = static_cast<uint8_t *>(workspace);
+  P.ctl = reinterpret_cast<Control *>(ws);
+  P.tickets = reinterpret_cast<int32_t *>(ws + W.tickets_off);
+  P.partials = reinterpret_cast<float *>(ws + W.partials_off);
+  P.timeout_ns = TIMEOUT_NS;
+  const int64_t units_max = (int64_t)P.n_tt * P.n_groups * ceil_div(k / b, P.S);
+  const int grid = (int)(units_max < sms ? units_max : sms);
+  return cuda_status(launch_linear(b, tmX, tmW, P, grid,
+                                   static_cast<cudaStream_t>(stream)));
+}
+
+}  // namespace
+}  // namespace lpvit
+
+using namespace lpvit;
+
+extern "C" {
+
+size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t b) {
+  if (!shape_ok(n, k, b)) return 0;
+  const int ng = (int)ceil_div(n, GROUP_FEATURES);
+  return 4 * (size_t)sched_entries_offset_ints(ng) + 4 * (size_t)ENTRY_INTS * ng * (k / b);
+}
+
+lpvit_status lpvit_pack_bsr(const void *W, const uint8_t *mask, lpvit_bsr *bsr, int32_t *nnzb_host, void *stream) {
+  if (!bsr) return LPVIT_ERR_INVALID_ARG;
+  const int n = bsr->n, k = bsr->k, b = bsr->b;
+  if (!valid_b(b)) return LPVIT_ERR_UNSUPPORTED;
+  if (!shape_ok(n, k, b)) return LPVIT_ERR_INVALID_ARG;
+  if (!W || !mask || !bsr->row_ptr || !bsr->sched || bsr->nnzb_capacity < 0) return LPVIT_ERR_INVALID_ARG;
+  if (bsr->nnzb_capacity > 0 && (!bsr->col_idx || !bsr->blocks)) return LPVIT_ERR_INVALID_ARG;
+  if (!aligned(W, 16) || (bsr->blocks && !aligned(bsr->blocks, 16)) || !aligned(bsr->sched, 16) ||
+      !aligned(bsr->row_ptr, 4) || (bsr->col_idx && !aligned(bsr->col_idx, 4)))
+    return LPVIT_ERR_INVALID_ARG;
+  if (bsr->sched_bytes < lpvit_sched_bytes(n, k, b)) return LPVIT_ERR_WORKSPACE;
+  int sms = 0;
+  lpvit_status st = LPVIT_OK;
+  if (!device_info(&sms, &st)) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = launch_pack(W, mask, n, k, b, bsr->row_ptr, bsr->col_idx, bsr->nnzb_capacity, bsr->blocks,
+                              static_cast<int32_t *>(bsr->sched), sms, s);
+  if (e != cudaSuccess) return LPVIT_ERR_CUDA;
+  if (nnzb_host) {
+    int32_t v = 0;
+    e = cudaMemcpyAsync(&v, bsr->row_ptr + n / b, sizeof(v), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return LPVIT_ERR_CUDA;
+    *nnzb_host = v;
+    if (v > bsr->nnzb_capacity) return LPVIT_ERR_WORKSPACE;
+  }
+  return LPVIT_OK;
+}
+
+size_t lpvit_workspace_bytes(const lpvit_bsr *bsr, int64_t m) {
+  if (!bsr || !shape_ok(bsr->n, bsr->k, bsr->b) || m < 0) return 0;
+  int sms = 0;
+  lpvit_status st = LPVIT_OK;
+  if (!device_info(&sms, &st)) sms = 152;  // sizing only; the call itself reports the device error
+  return ws_layout(m > 0 ? m : 1, bsr->n, bsr->k, bsr->b, sms).total;
+}
+
+lpvit_status lpvit_bsr_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias,
+                              void *Y, int64_t ldy, lpvit_dtype y_dtype, void *workspace, size_t ws_bytes,
+                              void *stream) {
+  return run_linear(bsr, X, m, ldx, bias, Y, ldy, y_dtype, workspace, ws_bytes, stream, 0);
+}
+
+lpvit_status lpvit_bsr_linear_gelu(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx,
+                                   const float *bias, void *Y, int64_t ldy, lpvit_dtype y_dtype, void *workspace,
+                                   size_t ws_bytes, void *stream) {
+  return run_linear(bsr, X, m, ldx, bias, Y, ldy, y_dtype, workspace, ws_bytes, stream, 1);
+}
+
+lpvit_status lpvit_check(void *workspace, void *stream) {
+  if (!workspace) return LPVIT_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return LPVIT_ERR_CUDA;
+  Control *ctl = static_cast<Control *>(workspace);
+  unsigned int err = 0;
+  if (cudaMemcpy(&err, &ctl->err, sizeof(err), cudaMemcpyDeviceToHost) != cudaSuccess) return LPVIT_ERR_CUDA;
+  if (err) {
+    if (cudaMemset(&ctl->err, 0, sizeof(err)) != cudaSuccess) return LPVIT_ERR_CUDA;
+    if (err & (ERR_SCHED_OVERFLOW | ERR_BAD_SCHED)) return LPVIT_ERR_WORKSPACE;
+    return LPVIT_ERR_TIMEOUT;
+  }
+  return LPVIT_OK;
+}
+
+const char *lpvit_status_string(lpvit_status status) {
+  switch (status) {
+    case LPVIT_OK: return "ok";
+    case LPVIT_ERR_INVALID_ARG: return "invalid argument (shape, null or misaligned pointer or stride)";
+    case LPVIT_ERR_UNSUPPORTED: return "unsupported (block size not 16/32/64, or device is not sm_103)";
+    case LPVIT_ERR_CUDA: return "CUDA runtime or driver error";
+    case LPVIT_ERR_TIMEOUT: return "a device-side bounded wait ran out; the output is incomplete";
+    case LPVIT_ERR_WORKSPACE: return "workspace, schedule buffer or block capacity too small";
+  }
+  return "unknown status";
+}
+
+}  // extern "C"

@@ -1,0 +1,211 @@
+// Device-side building blocks for sm_103a: mbarriers with bounded waits, TMA (tensor and bulk),
+// tcgen05 (TMEM allocation, weight-stationary MMA with B-collector reuse, TMEM loads) and the
+// shared-memory matrix / instruction descriptors they take. All inline PTX, no libraries.
+#pragma once
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace lpvit {
+
+// Layout of the work list ("sched") shared by the pack and the GEMM.
+// header (16 int32): [0] nnzb, [1] n_groups, [2] total entries, [3] overflow flag, [4] n, [5] k, [6] b
+// then gent_ptr[n_groups + 1] (int32, entries of group g are [gent_ptr[g], gent_ptr[g+1]))
+// then entries, ENTRY_INTS int32 each: [0] = j | (panel mask << 16), [1 + p] = block index of the
+// group's p-th row panel at block column j, or -1.
+constexpr int SCHED_HDR_INTS = 16;
+constexpr int ENTRY_INTS = 12;
+constexpr int GROUP_FEATURES = 128;  // output features covered by one work unit
+constexpr int TOKENS_PER_TILE = 256; // tokens covered by one work unit (the .ws MMA N)
+
+__host__ __device__ inline int sched_gent_offset_ints() { return SCHED_HDR_INTS; }
+__host__ __device__ inline int64_t sched_entries_offset_ints(int n_groups) {
+  return ((int64_t)SCHED_HDR_INTS + n_groups + 1 + 3) / 4 * 4;  // 16-byte aligned entries
+}
+
+// Workspace control block (first 256 bytes of the caller's workspace).
+struct Control {
+  unsigned int next_unit;   // dynamic scheduler: next unit to hand out
+  unsigned int done_ctas;   // CTAs that found the queue empty; the last one resets both
+  unsigned int err;         // device error word (bit set per failing wait site), read by lpvit_check
+  unsigned int err_detail;
+  unsigned int pad[60];
+};
+static_assert(sizeof(Control) == 256, "control block is 256 bytes");
+
+// Parameter block of the linear kernel (host fills it, the kernel reads it by value).
+struct LinearParams {
+  const int32_t *sched;    // work list (header, gent_ptr, entries)
+  const float *bias;       // [n] or nullptr
+  void *Y;
+  int64_t ldy;
+  int64_t m;
+  int n, k;
+  int n_tt, n_groups, S;   // token tiles, 128-feature groups, max entries per slice
+  int y_f32, gelu;
+  Control *ctl;
+  int32_t *tickets;        // [n_tt * n_groups] arrival tickets of split units
+  float *partials;         // [slots][128 features][256 tokens] fp32 partial sums of split units
+  uint64_t timeout_ns;     // limit of every device-side wait
+};
+
+enum ErrBits : unsigned int {
+  ERR_PRODUCER_EMPTY = 1u << 0,
+  ERR_PRODUCER_UNIT = 1u << 1,
+  ERR_MMA_FULL = 1u << 2,
+  ERR_MMA_ACC = 1u << 3,
+  ERR_MMA_UNIT = 1u << 4,
+  ERR_EPI_ACC = 1u << 5,
+  ERR_EPI_UNIT = 1u << 6,
+  ERR_DRAIN = 1u << 7,
+  ERR_SCHED_OVERFLOW = 1u << 8,
+  ERR_BAD_SCHED = 1u << 9,
+};
+
+// Launchers (host side, defined next to their kernels).
+cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int b, int32_t *row_ptr, int32_t *col_idx,
+                        int cap, void *blocks, int32_t *sched, int num_sms, cudaStream_t s);
+cudaError_t launch_linear(int b, const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
+                          cudaStream_t s);
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ uint32_t elect_one() {
+  uint32_t pred = 0;
+  asm volatile("{.reg .b32 rx; .reg .pred px; elect.sync rx|px, 0xffffffff; selp.u32 %0, 1, 0, px;}" : "=r"(pred));
+  return pred;
+}
+
+// ------------------------------------------------------------------ mbarrier
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(bar), "r"(count));
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" :: "r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile("{.reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p;}"
+               : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+  return ok != 0;
+}
+
+// Bounded wait: returns false after `limit_ns` without completion, or as soon as another role of
+// this CTA has raised the abort flag. Never spins forever.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const volatile int *abort_flag,
+                                          uint64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (;;) {
+#pragma unroll 1
+    for (int i = 0; i < 32; ++i)
+      if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer_ns() - t0 > limit_ns) return false;
+  }
+}
+
+// ------------------------------------------------------------------ TMA
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int32_t x, int32_t y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+      :: "r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar) : "memory");
+}
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map) {
+  asm volatile("prefetch.tensormap [%0];" :: "l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// ------------------------------------------------------------------ tcgen05
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" :: "r"(dst_smem), "r"(ncols));
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" :: "r"(taddr), "r"(ncols));
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" :: "r"(bar) : "memory");
+}
+
+// Shared-memory matrix descriptor for a K-major operand tile whose rows are `row_bytes`
+// (32, 64 or 128) long and stored with the matching TMA swizzle; 8-row atoms are contiguous.
+template <int ROW_BYTES>
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
+  static_assert(ROW_BYTES == 32 || ROW_BYTES == 64 || ROW_BYTES == 128, "row bytes");
+  constexpr uint64_t layout = ROW_BYTES == 128 ? 2 : (ROW_BYTES == 64 ? 4 : 6);  // SW128 / SW64 / SW32
+  constexpr uint64_t sbo = 8 * ROW_BYTES;                                     // bytes between 8-row atoms
+  return (uint64_t)((saddr & 0x3FFFF) >> 4) | ((uint64_t)1 << 16) | ((sbo >> 4) << 32) | ((uint64_t)1 << 46) |
+         (layout << 61);
+}
+
+// Instruction descriptor, kind::f16: bf16 x bf16 -> fp32, both operands K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// Weight-stationary MMA D[M x N] (+)= A[M x 16] * B[N x 16]^T with the B operand held in
+// collector buffer BUF: fill (load and keep), use (reuse), lastuse (reuse and release), or none.
+enum Coll { COLL_NONE = 0, COLL_FILL = 1, COLL_USE = 2, COLL_LAST = 3 };
+
+#define LPVIT_WS_MMA(QUAL)                                                                            \
+  asm volatile("{.reg .pred p; setp.ne.b32 p, %4, 0;\n"                                              \
+               "tcgen05.mma.ws.cta_group::1.kind::f16" QUAL " [%0], %1, %2, %3, p;}\n"               \
+               :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate))
+
+template <int BUF>
+__device__ __forceinline__ void ws_mma(int coll, uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                       uint32_t accumulate) {
+  static_assert(BUF >= 0 && BUF < 4, "collector buffer");
+  if (coll == COLL_NONE) {
+    LPVIT_WS_MMA("");
+  } else if (BUF == 0) {
+    if (coll == COLL_FILL) LPVIT_WS_MMA(".collector::b0::fill");
+    else if (coll == COLL_USE) LPVIT_WS_MMA(".collector::b0::use");
+    else LPVIT_WS_MMA(".collector::b0::lastuse");
+  } else if (BUF == 1) {
+    if (coll == COLL_FILL) LPVIT_WS_MMA(".collector::b1::fill");
+    else if (coll == COLL_USE) LPVIT_WS_MMA(".collector::b1::use");
+    else LPVIT_WS_MMA(".collector::b1::lastuse");
+  } else if (BUF == 2) {
+    if (coll == COLL_FILL) LPVIT_WS_MMA(".collector::b2::fill");
+    else if (coll == COLL_USE) LPVIT_WS_MMA(".collector::b2::use");
+    else LPVIT_WS_MMA(".collector::b2::lastuse");
+  } else {
+    if (coll == COLL_FILL) LPVIT_WS_MMA(".collector::b3::fill");
+    else if (coll == COLL_USE) LPVIT_WS_MMA(".collector::b3::use");
+    else LPVIT_WS_MMA(".collector::b3::lastuse");
+  }
+}
+#undef LPVIT_WS_MMA
+
+// TMEM -> registers: 32 lanes x 32 consecutive 32-bit columns (one lane per thread).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+}  // namespace lpvit

@@ -1,0 +1,545 @@
+// Block-sparse linear Y = act(X W~^T + bias) on sm_103a (Sec. 3.1 block mask, Sec. 3.3
+// block-sparse matmul: one block matmul per kept block and token tile, nothing for removed
+// blocks).
+//
+// Work unit = 256 tokens x one 128-feature group of row panels (x one slice of the group's block
+// columns when the problem is too small to fill the GPU). Per CTA (one per SM, persistent):
+//   warp 0      producer: takes units from a global atomic queue, walks the unit's work-list
+//               entries and, per entry (one block column j), TMA-loads the X tile
+//               [256 tokens x b] and every kept W block of the group at column j.
+//   warp 1      MMA issuer: per entry and per 16-wide k step, one weight-stationary tcgen05 MMA
+//               per present panel, D[panel rows x 256 tokens] += W_blk * X_tile^T, fp32 in TMEM.
+//               The X chunk is loaded once into a B collector buffer (fill) and reused by the
+//               other panels of the entry (use / lastuse).
+//   warps 2..9  epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
+//               type, stores of 64-byte row segments; split slices are summed in slice order
+//               by the last slice to finish (ticket), which makes the result deterministic.
+// Accumulators are double-buffered in TMEM (2 x 256 columns) so the epilogue of one unit overlaps
+// the MMAs of the next. Every wait is bounded: on timeout the CTA records an error bit, drains its
+// own copies and MMAs, frees TMEM and returns.
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "lpvit_device.cuh"
+
+namespace lpvit {
+
+template <int B>
+struct Cfg {
+  static constexpr int MP = (B == 64) ? 64 : 32;            // MMA M: features per MMA panel
+  static constexpr int PPM = MP / B;                        // BSR row panels per MMA panel
+  static constexpr int G = GROUP_FEATURES / MP;             // MMA panels per group
+  static constexpr int GB = GROUP_FEATURES / B;             // BSR row panels per group
+  static constexpr int KSTEPS = B / 16;                     // 16-wide k steps per block
+  static constexpr int ROW_BYTES = B * 2;                   // bytes of one tile row (bf16)
+  static constexpr int TT = TOKENS_PER_TILE;                // MMA N: tokens per unit
+  static constexpr int ACC_COLS = TT * MP / 128;            // TMEM columns per MMA-panel accumulator
+  static constexpr int BUF_COLS = G * ACC_COLS;             // TMEM columns per accumulator buffer
+  static constexpr int X_BYTES = TT * ROW_BYTES;            // X tile [256 x b]
+  static constexpr int BLK_BYTES = B * ROW_BYTES;           // one W block [b x b]
+  static constexpr int A_BYTES = MP * ROW_BYTES;            // one MMA-panel A tile [MP x b]
+  static constexpr int STAGE_BYTES = X_BYTES + G * A_BYTES;
+  static constexpr int NSTAGES = 196608 / STAGE_BYTES;      // 192 KB of stages
+  static constexpr int UR = 4;                              // unit-info ring depth
+  static constexpr int VPT = TT * MP / 128 / 2;             // accumulator values per epilogue thread and panel
+  static constexpr uint32_t IDESC = idesc_bf16(MP, TT);
+  static_assert(BUF_COLS == 256, "two accumulator buffers fill the 512 TMEM columns");
+  static_assert(NSTAGES >= 4, "pipeline depth");
+};
+
+constexpr int NUM_THREADS = 320;   // 10 warps
+constexpr int EPI_WARPS = 8;
+constexpr int MAX_GROUPS = 512;    // n <= 65536
+
+struct UnitInfo {
+  int tt, g, s, nsl, e0, e1, touched, pad;
+};
+
+
+template <int B>
+struct Smem {
+  // stages first (1024-byte aligned), then the control area
+  static constexpr int CTRL_OFF = Cfg<B>::NSTAGES * Cfg<B>::STAGE_BYTES;
+  static constexpr int NS = Cfg<B>::NSTAGES, UR = Cfg<B>::UR;
+  static constexpr int BAR_OFF = CTRL_OFF;
+  // barriers: full[NS], empty[NS], accf[2], acce[2], unitf[UR], unite[UR], drain, episync
+  static constexpr int NBARS = 2 * NS + 4 + 2 * UR + 2;
+  static constexpr int META_OFF = BAR_OFF + 8 * NBARS;
+  static constexpr int RING_OFF = (META_OFF + 4 * NS + 31) / 32 * 32;
+  static constexpr int SLICE_OFF = RING_OFF + (int)sizeof(UnitInfo) * UR;
+  static constexpr int MISC_OFF = SLICE_OFF + 4 * (MAX_GROUPS + 1);
+  static constexpr int END = MISC_OFF + 64;
+  static constexpr int BYTES = END + 1024;  // + alignment slack for the dynamic smem base
+};
+
+__device__ __forceinline__ void store_out(void *Y, int64_t idx, float y, int y_f32) {
+  if (y_f32) static_cast<float *>(Y)[idx] = y;
+  else static_cast<__nv_bfloat16 *>(Y)[idx] = __float2bfloat16_rn(y);
+}
+
+template <int B>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
+                  const LinearParams P) {
+  using C = Cfg<B>;
+  using L = Smem<B>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t smem_base = smem_u32(smem);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  const uint32_t bar0 = smem_base + L::BAR_OFF;
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (L::NS + s); };
+  auto accf_bar = [&](int b) { return bar0 + 8u * (2 * L::NS + b); };
+  auto acce_bar = [&](int b) { return bar0 + 8u * (2 * L::NS + 2 + b); };
+  auto unitf_bar = [&](int u) { return bar0 + 8u * (2 * L::NS + 4 + u); };
+  auto unite_bar = [&](int u) { return bar0 + 8u * (2 * L::NS + 4 + L::UR + u); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * L::NS + 4 + 2 * L::UR);
+  const uint32_t episync_bar = drain_bar + 8u;
+  volatile int *meta = reinterpret_cast<volatile int *>(smem + L::META_OFF);
+  UnitInfo *ring = reinterpret_cast<UnitInfo *>(smem + L::RING_OFF);
+  int *slice_ptr = reinterpret_cast<int *>(smem + L::SLICE_OFF);
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + L::MISC_OFF);
+  volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 4);
+  volatile int *last_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 8);
+  volatile int *never_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 12);  // stays 0
+
+  const int32_t *gent = P.sched + SCHED_HDR_INTS;
+  const int32_t *entries = P.sched + sched_entries_offset_ints(P.n_groups);
+  const uint64_t tmo = P.timeout_ns;
+
+  // ---------------------------------------------------------------- prologue
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), 512);
+    tmem_relinquish();
+  }
+  if (tid == 0) {
+    for (int s = 0; s < L::NS; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(accf_bar(b), 1);
+      mbar_init(acce_bar(b), EPI_WARPS);
+    }
+    for (int u = 0; u < L::UR; ++u) {
+      mbar_init(unitf_bar(u), 1);
+      mbar_init(unite_bar(u), EPI_WARPS);
+    }
+    mbar_init(drain_bar, 1);
+    mbar_init(episync_bar, EPI_WARPS);
+    *abort_flag = 0;
+    *last_flag = 0;
+    *never_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmX);
+    prefetch_tensormap(&tmW);
+  }
+  const bool sched_ok = P.sched[3] == 0 && P.sched[1] == P.n_groups;
+  if (warp == 2) {
+    // slices per group = max(1, ceil(entries / S)); exclusive prefix into slice_ptr
+    int run = 0;
+    for (int base = 0; base < P.n_groups; base += 32) {
+      const int g = base + lane;
+      int c = 0;
+      if (g < P.n_groups) {
+        const int cnt = gent[g + 1] - gent[g];
+        c = cnt <= 0 ? 1 : (cnt + P.S - 1) / P.S;
+      }
+      int incl = c;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+      }
+      if (g < P.n_groups) slice_ptr[g] = run + incl - c;
+      run += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) slice_ptr[P.n_groups] = run;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int total_slices = slice_ptr[P.n_groups];
+  const uint32_t total_units = sched_ok ? (uint32_t)P.n_tt * (uint32_t)total_slices : 0u;
+  if (!sched_ok && tid == 0) atomicOr(&P.ctl->err, P.sched[3] ? ERR_SCHED_OVERFLOW : ERR_BAD_SCHED);
+
+  if (warp == 0) {
+    // ============================================================== producer
+    uint32_t it = 0, ui = 0;
+    bool ok = true;
+    while (true) {
+      uint32_t u = 0;
+      if (lane == 0) u = atomicAdd(&P.ctl->next_unit, 1u);
+      u = __shfl_sync(0xffffffffu, u, 0);
+      const uint32_t slot = ui % L::UR, uph = (ui / L::UR) & 1u;
+      if (!mbar_wait(unite_bar(slot), uph ^ 1u, abort_flag, tmo)) {
+        ok = false;
+        if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_UNIT);
+        break;
+      }
+      if (u >= total_units) {
+        if (lane == 0) {
+          ring[slot].tt = -1;
+          mbar_arrive(unitf_bar(slot));
+        }
+        break;
+      }
+      const int tt = (int)(u / (uint32_t)total_slices);
+      const int rr = (int)(u % (uint32_t)total_slices);
+      int lo = 0, hi = P.n_groups - 1;  // group g with slice_ptr[g] <= rr < slice_ptr[g+1]
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (slice_ptr[mid] <= rr) lo = mid;
+        else hi = mid - 1;
+      }
+      const int g = lo, s = rr - slice_ptr[g], nsl = slice_ptr[g + 1] - slice_ptr[g];
+      const int ge0 = gent[g], ge1 = gent[g + 1];
+      const int e0 = min(ge0 + s * P.S, ge1), e1 = min(e0 + P.S, ge1);
+      // MMA panels touched by this unit
+      unsigned touched = 0;
+      for (int e = e0 + lane; e < e1; e += 32) touched |= (unsigned)entries[(int64_t)e * ENTRY_INTS] >> 16;
+      touched = __reduce_or_sync(0xffffffffu, touched);
+      unsigned tmask = 0;
+#pragma unroll
+      for (int p = 0; p < C::G; ++p)
+        tmask |= ((touched >> (p * C::PPM)) & ((1u << C::PPM) - 1u)) ? (1u << p) : 0u;
+      if (lane == 0) {
+        UnitInfo inf;
+        inf.tt = tt; inf.g = g; inf.s = s; inf.nsl = nsl; inf.e0 = e0; inf.e1 = e1; inf.touched = (int)tmask;
+        inf.pad = 0;
+        ring[slot] = inf;
+        mbar_arrive(unitf_bar(slot));
+      }
+      for (int base = e0; base < e1 && ok; base += 32) {
+        const int e = base + lane;
+        int w0 = 0;
+        int blk[C::GB];
+#pragma unroll
+        for (int p = 0; p < C::GB; ++p) blk[p] = -1;
+        if (e < e1) {
+          const int32_t *ep = entries + (int64_t)e * ENTRY_INTS;
+          w0 = ep[0];
+#pragma unroll
+          for (int p = 0; p < C::GB; ++p) blk[p] = ep[1 + p];
+        }
+        const int cnt = min(32, e1 - base);
+        for (int i = 0; i < cnt; ++i) {
+          const uint32_t stage = it % L::NS, ph = (it / L::NS) & 1u;
+          if (!mbar_wait(empty_bar(stage), ph ^ 1u, abort_flag, tmo)) {
+            ok = false;
+            if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_EMPTY);
+            break;
+          }
+          const int wi = __shfl_sync(0xffffffffu, w0, i);
+          int bi[C::GB];
+#pragma unroll
+          for (int p = 0; p < C::GB; ++p) bi[p] = __shfl_sync(0xffffffffu, blk[p], i);
+          const int j = wi & 0xffff;
+          const uint32_t pm = (uint32_t)wi >> 16;
+          uint8_t *st = smem + stage * C::STAGE_BYTES;
+          if (C::PPM == 2) {
+            // an MMA panel with exactly one of its two row panels present: zero the other half
+            bool wrote = false;
+#pragma unroll
+            for (int p = 0; p < C::G; ++p) {
+              const uint32_t two = (pm >> (2 * p)) & 3u;
+              if (two == 1u || two == 2u) {
+                const int half = two == 1u ? 1 : 0;
+                reinterpret_cast<int4 *>(st + C::X_BYTES + p * C::A_BYTES + half * C::BLK_BYTES)[lane] =
+                    make_int4(0, 0, 0, 0);
+                wrote = true;
+              }
+            }
+            if (wrote) fence_proxy_async_smem();
+            __syncwarp();
+          }
+          if (lane == 0) {
+            meta[stage] = (int)pm;
+            const uint32_t bytes = C::X_BYTES + __popc(pm) * C::BLK_BYTES;
+            const uint32_t fb = full_bar(stage);
+            mbar_arrive_expect_tx(fb, bytes);
+            const uint32_t st_u32 = smem_u32(st);
+            tma_load_2d(st_u32, &tmX, j * B, tt * C::TT, fb);
+#pragma unroll
+            for (int bp = 0; bp < C::GB; ++bp) {
+              if ((pm >> bp) & 1u) {
+                const int p = bp / C::PPM, half = bp % C::PPM;
+                tma_load_2d(st_u32 + C::X_BYTES + p * C::A_BYTES + half * C::BLK_BYTES, &tmW, 0, bi[bp] * B, fb);
+              }
+            }
+          }
+          __syncwarp();
+          ++it;
+        }
+      }
+      if (!ok) break;
+      ++ui;
+    }
+    if (!ok && lane == 0) *abort_flag = 1;
+    // queue bookkeeping: the last CTA to leave resets the counters for the next launch
+    if (lane == 0) {
+      __threadfence();
+      if (atomicAdd(&P.ctl->done_ctas, 1u) == gridDim.x - 1) {
+        P.ctl->next_unit = 0;
+        P.ctl->done_ctas = 0;
+        __threadfence();
+      }
+    }
+    // make sure no TMA write into this CTA's smem is still in flight
+    const uint32_t first = it > (uint32_t)L::NS ? it - L::NS : 0u;
+    for (uint32_t i = first; i < it; ++i)
+      if (!mbar_wait(full_bar(i % L::NS), (i / L::NS) & 1u, never_flag, tmo)) break;
+  } else if (warp == 1) {
+    // ============================================================== MMA issuer
+    uint32_t it = 0, ui = 0;
+    bool ok = true;
+    while (ok) {
+      const uint32_t slot = ui % L::UR, uph = (ui / L::UR) & 1u;
+      if (!mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)) {
+        ok = false;
+        if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_UNIT);
+        break;
+      }
+      const UnitInfo inf = ring[slot];
+      if (inf.tt < 0) break;
+      const uint32_t buf = ui & 1u, aph = (ui >> 1) & 1u;
+      if (!mbar_wait(acce_bar(buf), aph ^ 1u, abort_flag, tmo)) {
+        ok = false;
+        if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_ACC);
+        break;
+      }
+      tc_fence_after();
+      const uint32_t dbase = tmem_base + buf * C::BUF_COLS;
+      uint32_t touched = 0;
+      for (int e = inf.e0; e < inf.e1; ++e) {
+        const uint32_t stage = it % L::NS, ph = (it / L::NS) & 1u;
+        if (!mbar_wait(full_bar(stage), ph, abort_flag, tmo)) {
+          ok = false;
+          if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_FULL);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t pm = (uint32_t)meta[stage];
+        uint32_t mm = 0;
+#pragma unroll
+        for (int p = 0; p < C::G; ++p) mm |= ((pm >> (p * C::PPM)) & ((1u << C::PPM) - 1u)) ? (1u << p) : 0u;
+        const uint32_t st_u32 = smem_base + stage * C::STAGE_BYTES;
+        if (elect_one()) {
+          const int np = __popc(mm);
+#pragma unroll
+          for (int kk = 0; kk < C::KSTEPS; ++kk) {
+            const uint64_t bdesc = smem_desc<C::ROW_BYTES>(st_u32 + kk * 32);
+            uint32_t rem = mm;
+            int i = 0;
+            while (rem) {
+              const int p = __ffs(rem) - 1;
+              rem &= rem - 1u;
+              const uint64_t adesc = smem_desc<C::ROW_BYTES>(st_u32 + C::X_BYTES + p * C::A_BYTES + kk * 32);
+              const uint32_t d = dbase + (uint32_t)(p * C::ACC_COLS);
+              const uint32_t acc = (kk > 0 || ((touched >> p) & 1u)) ? 1u : 0u;
+              const int coll = np == 1 ? COLL_NONE : (i == 0 ? COLL_FILL : (rem == 0 ? COLL_LAST : COLL_USE));
+              if (kk == 0) ws_mma<0>(coll, d, adesc, bdesc, C::IDESC, acc);
+              else if (kk == 1) ws_mma<1>(coll, d, adesc, bdesc, C::IDESC, acc);
+              else if (kk == 2) ws_mma<2>(coll, d, adesc, bdesc, C::IDESC, acc);
+              else ws_mma<3>(coll, d, adesc, bdesc, C::IDESC, acc);
+              ++i;
+            }
+          }
+          tc_commit(empty_bar(stage));
+        }
+        __syncwarp();
+        touched |= mm;
+        ++it;
+      }
+      if (!ok) break;
+      if (elect_one()) {
+        if (inf.e1 > inf.e0) tc_commit(accf_bar(buf));
+        else mbar_arrive(accf_bar(buf));
+      }
+      __syncwarp();
+      ++ui;
+    }
+    if (!ok && lane == 0) *abort_flag = 1;
+    // wait for every MMA this thread issued before TMEM can be freed
+    if (elect_one()) tc_commit(drain_bar);
+    __syncwarp();
+    if (!mbar_wait(drain_bar, 0, never_flag, tmo) && lane == 0) atomicOr(&P.ctl->err, ERR_DRAIN);
+  } else {
+    // ============================================================== epilogue
+    const int ew = warp - 2;       // 0..7
+    const int q = warp & 3;        // TMEM lane quarter this warp may access
+    const int h = ew >> 2;         // column half
+    const int r = (C::MP == 32) ? lane : 32 * (q & 1) + lane;          // feature row in the MMA panel
+    const int tok0 = (C::MP == 32) ? 64 * q + 32 * h : 128 * (q >> 1) + 64 * h;  // first token of this thread
+    const int col0 = (C::MP == 32) ? 32 * h : 64 * h;                  // first column in the accumulator
+    uint32_t ui = 0, sync_phase = 0;
+    const float kInvSqrt2 = 0.70710678118654752440f;
+    while (true) {
+      const uint32_t slot = ui % L::UR, uph = (ui / L::UR) & 1u;
+      if (!mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)) {
+        if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_UNIT); *abort_flag = 1; }
+        break;
+      }
+      const UnitInfo inf = ring[slot];
+      if (inf.tt < 0) break;
+      const uint32_t buf = ui & 1u, aph = (ui >> 1) & 1u;
+      if (!mbar_wait(accf_bar(buf), aph, abort_flag, tmo)) {
+        if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_ACC); *abort_flag = 1; }
+        break;
+      }
+      tc_fence_after();
+      const bool split = inf.nsl > 1;
+      const int64_t tok_base = (int64_t)inf.tt * C::TT + tok0;
+      float *part = nullptr;
+      if (split)
+        part = P.partials + ((int64_t)inf.tt * total_slices + slice_ptr[inf.g] + inf.s) * (int64_t)(C::TT * 128);
+#pragma unroll 1
+      for (int p = 0; p < C::G; ++p) {
+        const int f = inf.g * GROUP_FEATURES + p * C::MP + r;
+        const uint32_t taddr = tmem_base + ((uint32_t)(32 * q) << 16) + buf * C::BUF_COLS + p * C::ACC_COLS + col0;
+        const bool has = (inf.touched >> p) & 1;
+#pragma unroll
+        for (int c = 0; c < C::VPT; c += 32) {
+          float v[32];
+          if (has) {
+            tmem_ld32(taddr + c, v);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+          }
+          if (split) {
+            float4 *dst = reinterpret_cast<float4 *>(part + (int64_t)(p * C::MP + r) * C::TT + tok0 + c);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+          } else if (f < P.n) {
+            const float bb = P.bias ? __ldg(P.bias + f) : 0.f;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int64_t tok = tok_base + c + i;
+              if (tok < P.m) {
+                float y = v[i] + bb;
+                if (P.gelu) y = 0.5f * y * (1.f + erff(y * kInvSqrt2));
+                store_out(P.Y, tok * P.ldy + f, y, P.y_f32);
+              }
+            }
+          }
+        }
+      }
+      // accumulator buffer and unit slot are free again
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(acce_bar(buf));
+        mbar_arrive(unite_bar(slot));
+      }
+      if (split) {
+        // make the partial visible, take a ticket; the last slice sums all partials in order
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(episync_bar);
+        if (!mbar_wait(episync_bar, sync_phase, abort_flag, tmo)) {
+          if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_UNIT); *abort_flag = 1; }
+          break;
+        }
+        sync_phase ^= 1u;
+        if (ew == 0 && lane == 0) {
+          int32_t *tk = P.tickets + (int64_t)inf.tt * P.n_groups + inf.g;
+          const int old = atomicAdd(tk, 1);
+          const int last = old == inf.nsl - 1;
+          if (last) atomicExch(tk, 0);
+          *last_flag = last;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(episync_bar);
+        if (!mbar_wait(episync_bar, sync_phase, abort_flag, tmo)) {
+          if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_UNIT); *abort_flag = 1; }
+          break;
+        }
+        sync_phase ^= 1u;
+        const int last = *last_flag;
+        if (last) {
+          __threadfence();
+          const float *base0 =
+              P.partials + ((int64_t)inf.tt * total_slices + slice_ptr[inf.g]) * (int64_t)(C::TT * 128);
+#pragma unroll 1
+          for (int p = 0; p < C::G; ++p) {
+            const int f = inf.g * GROUP_FEATURES + p * C::MP + r;
+            if (f >= P.n) continue;
+            const float bb = P.bias ? __ldg(P.bias + f) : 0.f;
+#pragma unroll 1
+            for (int c = 0; c < C::VPT; c += 32) {
+              float v[32];
+#pragma unroll
+              for (int i = 0; i < 32; ++i) v[i] = 0.f;
+              for (int s2 = 0; s2 < inf.nsl; ++s2) {
+                const float4 *src = reinterpret_cast<const float4 *>(
+                    base0 + (int64_t)s2 * (C::TT * 128) + (int64_t)(p * C::MP + r) * C::TT + tok0 + c);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                  const float4 t = __ldcg(src + i);
+                  v[4 * i] += t.x; v[4 * i + 1] += t.y; v[4 * i + 2] += t.z; v[4 * i + 3] += t.w;
+                }
+              }
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                const int64_t tok = tok_base + c + i;
+                if (tok < P.m) {
+                  float y = v[i] + bb;
+                  if (P.gelu) y = 0.5f * y * (1.f + erff(y * kInvSqrt2));
+                  store_out(P.Y, tok * P.ldy + f, y, P.y_f32);
+                }
+              }
+            }
+          }
+        }
+      }
+      ++ui;
+    }
+  }
+
+  // ---------------------------------------------------------------- teardown
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, 512);
+}
+
+// ------------------------------------------------------------------------------------ host side
+
+template <int B>
+int smem_bytes() { return Smem<B>::BYTES; }
+
+template <int B>
+cudaError_t launch_linear_t(const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
+                            cudaStream_t s) {
+  static bool attr_done[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(bsr_linear_kernel<B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         Smem<B>::BYTES);
+    if (e != cudaSuccess) return e;
+    attr_done[dev] = true;
+  }
+  bsr_linear_kernel<B><<<grid, NUM_THREADS, Smem<B>::BYTES, s>>>(tmX, tmW, P);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_linear(int b, const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
+                          cudaStream_t s) {
+  switch (b) {
+    case 16: return launch_linear_t<16>(tmX, tmW, P, grid, s);
+    case 32: return launch_linear_t<32>(tmX, tmW, P, grid, s);
+    case 64: return launch_linear_t<64>(tmX, tmW, P, grid, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace lpvit

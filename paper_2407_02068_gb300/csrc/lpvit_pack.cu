@@ -1,0 +1,217 @@
+// Mask -> BSR pack and work-list build (Sec. 3.1 block mask; Sec. 1 / Sec. 3.3: only the kept
+// blocks are stored, moved and multiplied).
+//
+// plan kernel (one CTA): per row panel r, cnt[r] = number of kept blocks (warp reductions);
+//   row_ptr = exclusive prefix sum of cnt (warp-shuffle scan + a scan of warp totals);
+//   col_idx = kept block columns of each panel in ascending order (ballot compaction);
+//   work list: panels are grouped 128 output features at a time; for every group, one entry per
+//   block column where any panel of the group keeps a block, with that column's block index in
+//   each panel (or -1). The GEMM walks these entries.
+// copy kernel (grid-stride over kept blocks): blocks[t] = W[r*b:(r+1)*b, j*b:(j+1)*b], 16-byte
+//   vector copies; the bits are moved unchanged.
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "lpvit_device.cuh"
+
+namespace lpvit {
+
+constexpr int PLAN_THREADS = 1024;
+constexpr int PLAN_WARPS = PLAN_THREADS / 32;
+
+// Exclusive block-wide scan of v[0..count) in shared memory (in place); returns the total.
+// All threads of the CTA must call it.
+__device__ int block_exclusive_scan(int *v, int count, int *warp_tot) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int per = (count + PLAN_THREADS - 1) / PLAN_THREADS;
+  const int beg = min(count, tid * per), end = min(count, beg + per);
+  int local = 0;
+  for (int i = beg; i < end; ++i) local += v[i];
+  int incl = local;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  if (lane == 31) warp_tot[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    int w = warp_tot[lane];
+    int wi = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, wi, o);
+      if (lane >= o) wi += t;
+    }
+    warp_tot[lane] = wi - w;  // exclusive prefix of warp totals
+    if (lane == 31) warp_tot[32] = wi;
+  }
+  __syncthreads();
+  int run = warp_tot[warp] + incl - local;
+  for (int i = beg; i < end; ++i) {
+    const int c = v[i];
+    v[i] = run;
+    run += c;
+  }
+  const int total = warp_tot[32];
+  __syncthreads();
+  return total;
+}
+
+__global__ void __launch_bounds__(PLAN_THREADS, 1)
+plan_kernel(const uint8_t *__restrict__ mask, int n, int k, int b, int32_t *__restrict__ row_ptr,
+            int32_t *__restrict__ col_idx, int cap, int32_t *__restrict__ sched) {
+  extern __shared__ int plan_smem[];
+  const int np = n / b, kb = k / b;
+  const int gb = GROUP_FEATURES / b;  // row panels per group
+  const int ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
+  int *cnt = plan_smem;            // [np + 1]
+  int *gcnt = cnt + np + 1;        // [ng + 1]
+  int *warp_tot = gcnt + ng + 1;   // [33]
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const unsigned lt = (1u << lane) - 1u;
+
+  // 1. kept blocks per panel
+  for (int r = warp; r < np; r += PLAN_WARPS) {
+    int c = 0;
+    for (int j = lane; j < kb; j += 32) c += mask[(int64_t)r * kb + j] != 0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+    if (lane == 0) cnt[r] = c;
+  }
+  __syncthreads();
+  // 2. row_ptr = exclusive scan
+  const int nnzb = block_exclusive_scan(cnt, np, warp_tot);
+  for (int r = tid; r < np; r += PLAN_THREADS) row_ptr[r] = cnt[r];
+  if (tid == 0) {
+    row_ptr[np] = nnzb;
+    cnt[np] = nnzb;
+  }
+  __syncthreads();
+  // 3. col_idx, ascending within each panel
+  for (int r = warp; r < np; r += PLAN_WARPS) {
+    int run = cnt[r];
+    for (int base = 0; base < kb; base += 32) {
+      const int j = base + lane;
+      const bool keep = j < kb && mask[(int64_t)r * kb + j] != 0;
+      const unsigned bal = __ballot_sync(0xffffffffu, keep);
+      if (keep) {
+        const int pos = run + __popc(bal & lt);
+        if (pos < cap) col_idx[pos] = j;
+      }
+      run += __popc(bal);
+    }
+  }
+  // 4a. entries per group: block columns where any panel of the group keeps a block
+  for (int g = warp; g < ng; g += PLAN_WARPS) {
+    int c = 0;
+    for (int base = 0; base < kb; base += 32) {
+      const int j = base + lane;
+      unsigned any = 0;
+      for (int p = 0; p < gb; ++p) {
+        const int r = g * gb + p;
+        const bool keep = r < np && j < kb && mask[(int64_t)r * kb + j] != 0;
+        any |= __ballot_sync(0xffffffffu, keep);
+      }
+      c += __popc(any);
+    }
+    if (lane == 0) gcnt[g] = c;
+  }
+  __syncthreads();
+  const int total_entries = block_exclusive_scan(gcnt, ng, warp_tot);
+  int32_t *gent = sched + SCHED_HDR_INTS;
+  int32_t *entries = sched + sched_entries_offset_ints(ng);
+  for (int g = tid; g < ng; g += PLAN_THREADS) gent[g] = gcnt[g];
+  if (tid == 0) {
+    gent[ng] = total_entries;
+    sched[0] = nnzb;
+    sched[1] = ng;
+    sched[2] = total_entries;
+    sched[3] = nnzb > cap ? 1 : 0;
+    sched[4] = n;
+    sched[5] = k;
+    sched[6] = b;
+    for (int i = 7; i < SCHED_HDR_INTS; ++i) sched[i] = 0;
+  }
+  // 4b. entries: j | (panel mask << 16), then the block index of each panel of the group (or -1)
+  for (int g = warp; g < ng; g += PLAN_WARPS) {
+    int e_run = gcnt[g];
+    int p_run[8];
+#pragma unroll
+    for (int p = 0; p < 8; ++p) p_run[p] = (p < gb && g * gb + p < np) ? cnt[g * gb + p] : 0;
+    for (int base = 0; base < kb; base += 32) {
+      const int j = base + lane;
+      unsigned bal[8];
+      unsigned any = 0;
+#pragma unroll
+      for (int p = 0; p < 8; ++p) {
+        const int r = g * gb + p;
+        const bool keep = p < gb && r < np && j < kb && mask[(int64_t)r * kb + j] != 0;
+        bal[p] = __ballot_sync(0xffffffffu, keep);
+        any |= bal[p];
+      }
+      if ((any >> lane) & 1u) {
+        int32_t *e = entries + (int64_t)(e_run + __popc(any & lt)) * ENTRY_INTS;
+        unsigned pm = 0;
+#pragma unroll
+        for (int p = 0; p < 8; ++p) {
+          const bool keep = (bal[p] >> lane) & 1u;
+          pm |= (keep ? 1u : 0u) << p;
+          e[1 + p] = keep ? p_run[p] + __popc(bal[p] & lt) : -1;
+        }
+        e[0] = (int32_t)((unsigned)j | (pm << 16));
+        e[9] = 0;
+        e[10] = 0;
+        e[11] = 0;
+      }
+      e_run += __popc(any);
+#pragma unroll
+      for (int p = 0; p < 8; ++p) p_run[p] += __popc(bal[p]);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(128)
+copy_blocks_kernel(const uint16_t *__restrict__ W, int n, int k, int b, const int32_t *__restrict__ row_ptr,
+                   const int32_t *__restrict__ col_idx, int cap, uint16_t *__restrict__ blocks) {
+  const int np = n / b;
+  const int nnzb = min(row_ptr[np], cap);
+  const int vec_per_row = b / 8;  // 16-byte vectors per block row
+  const int vecs = b * vec_per_row;
+  for (int t = blockIdx.x; t < nnzb; t += gridDim.x) {
+    int lo = 0, hi = np - 1;  // largest r with row_ptr[r] <= t (that panel holds block t)
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (row_ptr[mid] <= t) lo = mid;
+      else hi = mid - 1;
+    }
+    const int r = lo, j = col_idx[t];
+    for (int v = threadIdx.x; v < vecs; v += blockDim.x) {
+      const int c = v / vec_per_row, cv = v - c * vec_per_row;
+      const int4 *src = reinterpret_cast<const int4 *>(W + ((int64_t)r * b + c) * k + (int64_t)j * b + cv * 8);
+      int4 *dst = reinterpret_cast<int4 *>(blocks + ((int64_t)t * b + c) * b + cv * 8);
+      *dst = __ldg(src);
+    }
+  }
+}
+
+size_t plan_smem_bytes(int n, int b) {
+  const int np = n / b, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
+  return sizeof(int) * (size_t)(np + 1 + ng + 1 + 33);
+}
+
+cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int b, int32_t *row_ptr, int32_t *col_idx,
+                        int cap, void *blocks, int32_t *sched, int num_sms, cudaStream_t s) {
+  const size_t smem = plan_smem_bytes(n, b);
+  plan_kernel<<<1, PLAN_THREADS, smem, s>>>(mask, n, k, b, row_ptr, col_idx, cap, sched);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int max_blocks = (n / b) * (k / b);
+  int grid = max_blocks < num_sms * 16 ? max_blocks : num_sms * 16;
+  if (grid < 1) grid = 1;
+  copy_blocks_kernel<<<grid, 128, 0, s>>>(static_cast<const uint16_t *>(W), n, k, b, row_ptr, col_idx, cap,
+                                         static_cast<uint16_t *>(blocks));
+  return cudaGetLastError();
+}
+
+}  // namespace lpvit

@@ -1,0 +1,60 @@
+"""CPU checks of the C ABI: the library builds, loads, exports every function include/lpvit.h
+declares, and rejects bad arguments before touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2407_02068_gb300 import _lib, build
+    build.build()
+    return _lib
+
+
+def _declared_functions():
+    src = open(os.path.join(ROOT, "include", "lpvit.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(lpvit_[a-z_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared_functions()
+    assert {"lpvit_pack_bsr", "lpvit_bsr_linear", "lpvit_bsr_linear_gelu"} <= set(names)
+    raw = ctypes.CDLL(lib.LIB)
+    for name in names:
+        assert hasattr(raw, name), name
+    assert set(names) == set(lib.EXPORTS)
+
+
+def test_sched_bytes_and_status_strings(lib):
+    assert lib.lpvit_sched_bytes(1152, 384, 32) > 0
+    assert lib.lpvit_sched_bytes(1152, 384, 24) == 0      # unsupported block size
+    assert lib.lpvit_sched_bytes(1000, 384, 32) == 0      # n not a multiple of b
+    for st in range(6):
+        assert lib.status_string(st)
+
+
+def test_bad_arguments_are_rejected_without_a_gpu(lib):
+    bsr = lib.lpvit_bsr(1152, 384, 32, 432, None, None, None, None, 0)
+    st, _ = lib.lpvit_pack_bsr(None, None, bsr, False, None)
+    assert st == lib.LPVIT_ERR_INVALID_ARG
+    bad_b = lib.lpvit_bsr(1152, 384, 24, 432, None, None, None, None, 0)
+    st, _ = lib.lpvit_pack_bsr(None, None, bad_b, False, None)
+    assert st == lib.LPVIT_ERR_UNSUPPORTED
+    assert lib.lpvit_bsr_linear(bsr, None, 197, 384, None, None, 1152, 0, None, 0, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert lib.lpvit_bsr_linear(bsr, None, -1, 384, None, None, 1152, 0, None, 0, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert lib.lpvit_bsr_linear(bsr, None, 0, 384, None, None, 1152, 0, None, 0, None) == lib.LPVIT_OK  # empty
+    assert lib.lpvit_bsr_linear_gelu(bad_b, None, 4, 384, None, None, 1152, 0, None, 0, None) == \
+        lib.LPVIT_ERR_UNSUPPORTED
+    # misaligned X (not 16-byte aligned) / ldx not a multiple of 8
+    fake = ctypes.c_void_p(0x1000)
+    assert lib.lpvit_bsr_linear(bsr, 0x1002, 4, 384, None, 0x200000, 1152, 0, 0x100000, 1 << 20, None) == \
+        lib.LPVIT_ERR_INVALID_ARG
+    assert lib.lpvit_bsr_linear(bsr, fake.value, 4, 388, None, 0x200000, 1152, 0, 0x100000, 1 << 20, None) == \
+        lib.LPVIT_ERR_INVALID_ARG
+    assert lib.lpvit_check(None, None) == lib.LPVIT_ERR_INVALID_ARG

@@ -1,0 +1,283 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 CPU oracle.
+
+Gates (from the method's stated bar): BSR pack bit-exact; GEMM with fp32 output within
+max|y - y_ref| / rms(y_ref) <= 1e-2 (and, as a tighter diagnostic, <= 1e-4, since fp32
+accumulation of bf16 products is accurate to ~1e-6); bf16 output within one bf16 ulp of the
+exact value element-wise; integer-exact inputs bit-exact."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2407_02068_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+NORM_TOL = 1e-2      # max|y - y_ref| / rms(y_ref), fp32 output
+TIGHT_TOL = 1e-4
+
+
+@pytest.fixture(scope="module")
+def lp():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2407_02068_gb300 as lp
+    from paper_2407_02068_gb300 import build
+    build.build()
+    return lp
+
+
+def _bits(t):
+    return inputs.bf16_bits(t)
+
+
+def _oracle(X, W, mask, b, bias, gelu=False, rows=None):
+    Xb = _bits(X if rows is None else X[rows])
+    return oracle.linear(Xb, _bits(W), mask.cpu().numpy(), b, None if bias is None else bias.cpu().numpy(), gelu)
+
+
+def _norm_err(y, ref):
+    rms = np.sqrt(np.mean(ref ** 2))
+    return np.max(np.abs(y - ref)) / max(rms, 1e-30)
+
+
+def _ulp_bf16(x):
+    a = np.abs(x)
+    e = np.floor(np.log2(np.maximum(a, 2.0 ** -126)))
+    return 2.0 ** (e - 7)
+
+
+def _acc_bound(X, W, mask, b, bias):
+    """Bound on the fp32 accumulation error of any summation order: k * 2^-24 * sum_k |x w~|."""
+    keep = mask.repeat_interleave(b, 0).repeat_interleave(b, 1).bool()
+    Wa = torch.where(keep, W, torch.zeros_like(W)).double().abs().cpu()
+    S = X.double().abs().cpu() @ Wa.T + bias.double().abs().cpu()
+    return (W.shape[1] * 2.0 ** -24 * S).numpy()
+
+
+def _bf16_tol(ref, X, W, mask, b, bias, gelu=False):
+    """One bf16 ulp of the exact value, plus the fp32 accumulation bound (scaled by max|gelu'| = 1.13),
+    plus 4 fp32 ulps for erff."""
+    acc = _acc_bound(X, W, mask, b, bias)
+    return _ulp_bf16(ref) + (1.13 * acc + 4 * 2.0 ** -23 * np.abs(ref) if gelu else acc)
+
+
+def _case(m, n, k, b, sp, seed, device="cuda", int_valued=False, mask_kind="uniform"):
+    g = torch.Generator().manual_seed(seed)
+    if int_valued:
+        X = torch.randint(-4, 5, (m, k), generator=g).float().to(torch.bfloat16)
+        W = (torch.randint(-4, 5, (n, k), generator=g).float() / 16).to(torch.bfloat16)
+        bias = torch.randint(-8, 9, (n,), generator=g).float() / 8
+    else:
+        X = torch.randn(m, k, generator=g).to(torch.bfloat16)
+        W = (torch.randn(n, k, generator=g) * 0.02).to(torch.bfloat16)
+        bias = torch.randn(n, generator=g) * 0.02
+    if mask_kind == "uniform":
+        mask = inputs.uniform_mask(n, k, b, sp, seed + 1)
+    else:
+        mask = inputs.zipf_mask(n, k, b, sp, seed + 1)
+    return X.to(device), W.to(device), bias.to(device), mask.to(device)
+
+
+# ------------------------------------------------------------------------------------- pack
+
+@pytest.mark.parametrize("n,k,b,sp", [(1152, 384, 32, 0.5), (384, 1536, 16, 0.5), (768, 3072, 64, 0.3),
+                                      (3072, 768, 32, 0.0), (256, 256, 16, 1.0), (64, 48, 16, 0.4)])
+def test_pack_bit_exact(lp, n, k, b, sp):
+    X, W, bias, mask = _case(4, n, k, b, sp, 11)
+    mask[0] = 0  # an empty panel
+    w = lp.pack_bsr(W, mask, b, count=True)
+    rp, ci, bl = oracle.pack(_bits(W), mask.cpu().numpy(), b)
+    assert w.nnzb == len(ci)
+    assert np.array_equal(w.row_ptr.cpu().numpy(), rp)
+    assert np.array_equal(w.col_idx[:w.nnzb].cpu().numpy(), ci)
+    got = w.blocks[:w.nnzb].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+    assert np.array_equal(got, bl)
+
+
+def _decode_sched(w):
+    raw = w.sched.cpu().numpy().view(np.int32)
+    ng = int(raw[1])
+    gent = raw[16:16 + ng + 1]
+    off = (16 + ng + 1 + 3) // 4 * 4
+    ent = raw[off:off + int(gent[-1]) * 12].reshape(-1, 12)
+    return raw[:16], gent, ent
+
+
+@pytest.mark.parametrize("n,k,b", [(1152, 384, 32), (384, 1536, 16), (768, 3072, 64), (200 * 16, 64, 16)])
+def test_work_list_covers_every_kept_block_once(lp, n, k, b):
+    X, W, bias, mask = _case(4, n, k, b, 0.55, 12)
+    w = lp.pack_bsr(W, mask, b, count=True)
+    hdr, gent, ent = _decode_sched(w)
+    gb = 128 // b
+    M = mask.cpu().numpy()
+    rp, ci, _ = oracle.pack(_bits(W), M, b)
+    seen = set()
+    for g in range(int(hdr[1])):
+        js = []
+        for e in ent[gent[g]:gent[g + 1]]:
+            j, pm = int(e[0]) & 0xFFFF, (int(e[0]) >> 16) & 0xFFFF
+            js.append(j)
+            for p in range(gb):
+                r = g * gb + p
+                if (pm >> p) & 1:
+                    t = int(e[1 + p])
+                    assert r < n // b and M[r, j] and ci[t] == j and rp[r] <= t < rp[r + 1]
+                    seen.add(t)
+                else:
+                    assert e[1 + p] == -1 and (r >= n // b or not M[r, j])
+        assert js == sorted(set(js))
+        want = sorted(set(np.nonzero(M[g * gb:(g + 1) * gb].any(axis=0))[0].tolist()))
+        assert js == want
+    assert seen == set(range(len(ci)))
+
+
+# ------------------------------------------------------------------------------------- GEMM
+
+@pytest.mark.parametrize("b", [16, 32, 64])
+@pytest.mark.parametrize("m", [1, 197, 300, 777])
+def test_linear_fp32_out(lp, b, m):
+    n, k = 384, 256
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 100 + b + m)
+    w = lp.pack_bsr(W, mask, b)
+    Y = lp.bsr_linear(w, X, bias, out_dtype=torch.float32)
+    ws = lp.workspace_for(w, m)
+    lp.check(ws)
+    ref = _oracle(X, W, mask, b, bias)
+    err = _norm_err(Y.cpu().double().numpy(), ref)
+    assert err <= NORM_TOL
+    assert err <= TIGHT_TOL
+
+
+@pytest.mark.parametrize("b", [16, 32, 64])
+def test_linear_integer_inputs_bit_exact(lp, b):
+    m, n, k = 520, 256, 512
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 200 + b, int_valued=True)
+    w = lp.pack_bsr(W, mask, b)
+    Y = lp.bsr_linear(w, X, bias, out_dtype=torch.float32)
+    ref = _oracle(X, W, mask, b, bias)
+    assert np.array_equal(Y.cpu().double().numpy(), ref)
+
+
+@pytest.mark.parametrize("b", [16, 32, 64])
+def test_linear_bf16_out_within_one_ulp(lp, b):
+    m, n, k = 600, 512, 384
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 300 + b)
+    w = lp.pack_bsr(W, mask, b)
+    Y = lp.bsr_linear(w, X, bias)
+    ref = _oracle(X, W, mask, b, bias)
+    y = Y.float().cpu().double().numpy()
+    assert np.all(np.abs(y - ref) <= _bf16_tol(ref, X, W, mask, b, bias))
+
+
+@pytest.mark.parametrize("b", [16, 32, 64])
+def test_linear_gelu(lp, b):
+    m, n, k = 333, 256, 256
+    X, W, bias, mask = _case(m, n, k, b, 0.4, 400 + b)
+    w = lp.pack_bsr(W, mask, b)
+    Y = lp.bsr_linear(w, X, bias, gelu=True, out_dtype=torch.float32)
+    ref = _oracle(X, W, mask, b, bias, gelu=True)
+    assert _norm_err(Y.cpu().double().numpy(), ref) <= TIGHT_TOL
+    Yb = lp.bsr_linear(w, X, bias, gelu=True)
+    assert np.all(np.abs(Yb.float().cpu().double().numpy() - ref) <= _bf16_tol(ref, X, W, mask, b, bias, gelu=True))
+
+
+@pytest.mark.parametrize("b", [16, 32, 64])
+def test_all_zero_mask_is_bias(lp, b):
+    m, n, k = 260, 256, 128
+    X, W, bias, _ = _case(m, n, k, b, 0.5, 500 + b)
+    mask = torch.zeros(n // b, k // b, dtype=torch.uint8, device="cuda")
+    w = lp.pack_bsr(W, mask, b)
+    Y = lp.bsr_linear(w, X, bias, out_dtype=torch.float32)
+    assert torch.equal(Y, bias.expand(m, n))
+    Yg = lp.bsr_linear(w, X, bias, gelu=True, out_dtype=torch.float32)
+    ref = oracle.gelu(bias.cpu().double().numpy())
+    assert np.allclose(Yg[0].cpu().double().numpy(), ref, rtol=1e-6, atol=1e-9)
+    Yn = lp.bsr_linear(w, X, None, out_dtype=torch.float32)
+    assert torch.count_nonzero(Yn) == 0
+
+
+@pytest.mark.parametrize("b", [16, 32, 64])
+def test_pruned_blocks_never_read(lp, b):
+    m, n, k = 300, 256, 256
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 600 + b)
+    keep = mask.repeat_interleave(b, 0).repeat_interleave(b, 1).bool()
+    Wp = W.clone()
+    Wp[~keep] = float("nan")
+    Wz = W.clone()
+    Wz[~keep] = 0
+    Yp = lp.bsr_linear(lp.pack_bsr(Wp, mask, b), X, bias, out_dtype=torch.float32)
+    Yz = lp.bsr_linear(lp.pack_bsr(Wz, mask, b), X, bias, out_dtype=torch.float32)
+    assert torch.equal(Yp, Yz) and torch.isfinite(Yp).all()
+
+
+def test_single_block_closed_form(lp):
+    m, n, k, b = 290, 256, 256, 32
+    X, W, bias, _ = _case(m, n, k, b, 0.5, 700, int_valued=True)
+    mask = torch.zeros(n // b, k // b, dtype=torch.uint8, device="cuda")
+    mask[3, 5] = 1
+    Y = lp.bsr_linear(lp.pack_bsr(W, mask, b), X, bias, out_dtype=torch.float32)
+    Xd, Wd = X.double().cpu(), W.double().cpu()
+    expect = bias.double().cpu().expand(m, n).clone()
+    expect[:, 96:128] += Xd[:, 160:192] @ Wd[96:128, 160:192].T
+    assert torch.equal(Y.double().cpu(), expect)
+
+
+def test_strided_input_output_and_guard_band(lp):
+    m, n, k, b = 400, 256, 128, 32
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 800)
+    Xw = torch.zeros(m, k + 64, dtype=torch.bfloat16, device="cuda")
+    Xw[:, 64:] = X
+    canary = -12345.0
+    Yw = torch.full((m + 7, n + 32), canary, dtype=torch.float32, device="cuda")
+    w = lp.pack_bsr(W, mask, b)
+    lp.bsr_linear(w, Xw[:, 64:], bias, out=Yw[:m, 16:16 + n])
+    ref = _oracle(X, W, mask, b, bias)
+    assert _norm_err(Yw[:m, 16:16 + n].cpu().double().numpy(), ref) <= TIGHT_TOL
+    assert torch.all(Yw[m:] == canary) and torch.all(Yw[:, :16] == canary) and torch.all(Yw[:, 16 + n:] == canary)
+
+
+def test_deterministic_repeats(lp):
+    m, n, k, b = 197, 768, 3072, 32   # small m: split slices + fix-up path
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 900)
+    w = lp.pack_bsr(W, mask, b)
+    ws = lp.workspace_for(w, m)
+    Y1 = lp.bsr_linear(w, X, bias, out_dtype=torch.float32, workspace=ws)
+    Y2 = lp.bsr_linear(w, X, bias, out_dtype=torch.float32, workspace=ws)
+    lp.check(ws)
+    assert torch.equal(Y1, Y2)
+    ref = _oracle(X, W, mask, b, bias)
+    assert _norm_err(Y1.cpu().double().numpy(), ref) <= TIGHT_TOL
+
+
+@pytest.mark.parametrize("b", [16, 64])
+def test_zipf_imbalanced_masks(lp, b):
+    m, n, k = 513, 768, 3072
+    X, W, bias, mask = _case(m, n, k, b, 0.6, 1000 + b, mask_kind="zipf")
+    w = lp.pack_bsr(W, mask, b)
+    Y = lp.bsr_linear(w, X, bias, gelu=True, out_dtype=torch.float32)
+    ref = _oracle(X, W, mask, b, bias, gelu=True)
+    assert _norm_err(Y.cpu().double().numpy(), ref) <= TIGHT_TOL
+
+
+def test_empty_input_rows(lp):
+    X, W, bias, mask = _case(4, 128, 128, 32, 0.5, 1100)
+    w = lp.pack_bsr(W, mask, 32)
+    Y = lp.bsr_linear(w, X[:0], bias)
+    assert Y.shape == (0, 128)
+
+
+def test_full_size_deit_b_fc1_sampled_rows(lp):
+    """DeiT-B fc1 at batch 256 (M = 50432), 32x32 blocks, 50% sparsity, launched as in the bench;
+    the oracle checks a seeded sample of rows plus the first and last token tile."""
+    m, k, n, b = 50432, 768, 3072, 32
+    X = inputs.activations(m, k, inputs.seed(3, 0, "X"), "cuda")
+    W = inputs.weight(n, k, inputs.seed(3, 0, "W"), "cuda")
+    bias = inputs.bias(n, inputs.seed(3, 0, "bias"), "cuda")
+    mask = inputs.uniform_mask(n, k, b, 0.5, inputs.seed(3, 0, "mask"))
+    w = lp.pack_bsr(W, mask.cuda(), b)
+    Y = lp.bsr_linear(w, X, bias, gelu=True, out_dtype=torch.float32)
+    rows = np.unique(np.concatenate([np.random.default_rng(0).choice(m, 96, replace=False),
+                                     np.arange(0, 8), np.arange(m - 8, m)]))
+    ref = _oracle(X, W, mask, b, bias, gelu=True, rows=torch.from_numpy(rows).cuda())
+    assert _norm_err(Y[torch.from_numpy(rows).cuda()].cpu().double().numpy(), ref) <= TIGHT_TOL
