@@ -1,0 +1,406 @@
+#!/usr/bin/env python
+"""Benchmark: effective TFLOP/s and % of roofline for block-sparse DeiT linears on GB300.
+
+Workload (one "step" = one pass of the whole block-sparse path over one batch): the 12-layer
+DeiT-B linear stack (48 GEMMs: qkv 768->2304, proj 768->768, fc1 768->3072 + GELU,
+fc2 3072->768) at batch 256 (M = 50432 tokens), 32x32 blocks, per-GEMM block sparsity drawn
+U[30%, 70%] as antithetic layer pairs (mean exactly 50%); every weight is packed (mask -> BSR +
+work list) and every linear runs, chained layer to layer. Inputs are seeded synthetic bf16 tensors
+resident in HBM; each step streams ~15 GB, far more than the 129 MB L2, so no flush is needed.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl lpvit|reference]
+
+Prints one JSON line (rank 0). ``--impl reference`` times the CPU oracle (fp64 C loops on the
+host cores) on a bounded row sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "effective TFLOP/s and % of roofline for block-sparse DeiT linears"
+UNIT = "TFLOP/s"
+M_TOKENS = 50432          # DeiT-B, batch 256 x 197 tokens
+BLOCK = 32
+CONFIG_ID = 4             # seeds of the 12-layer stack workload
+WORKLOAD = "deit_b_12layer_linear_stack_batch256"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "bsr_linear_deit_b_stack_traffic.txt")
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=400)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", choices=["lpvit", "reference"], default="lpvit")
+    p.add_argument("--e2e-steps", type=int, default=None)
+    p.add_argument("--cpu-budget-s", type=float, default=15.0, help="CPU seconds for the oracle baseline sample")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-dense", action="store_true")
+    return p.parse_args()
+
+
+# ----------------------------------------------------------------------------------------- helpers
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for name in ("lpvit_linear.cu", "lpvit_device.cuh"):
+        with open(os.path.join(ROOT, "paper_2407_02068_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic():
+    """DRAM bytes per launch of the linear kernel from the committed ncu summary, if it was
+    taken on the current kernel source (else None)."""
+    try:
+        kv = {}
+        with open(PROFILE_TRAFFIC) as f:
+            for line in f:
+                if ":" in line and not line.startswith("#"):
+                    k, v = line.split(":", 1)
+                    kv[k.strip()] = v.strip()
+        if kv.get("kernel_source_sha") != kernel_source_hash():
+            return None
+        return float(kv["dram_bytes_per_stack_linear_launch"])
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling every 200 ms while the timed region runs."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.t.join(timeout=2)
+        sm, smax, pw, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+                pw.append(float(parts[3]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "power_w_median": statistics.median(pw) if pw else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ------------------------------------------------------------------------------------ CPU oracle
+
+def oracle_layers_from(stack_layers):
+    """Host copies (bf16 bits, masks, biases) of the stack for the oracle."""
+    from paper_2407_02068_gb300 import inputs
+    out = []
+    for L in stack_layers:
+        out.append({name: (inputs.bf16_bits(L[name]["W"]), L[name]["mask"].cpu().numpy().astype("uint8"),
+                           L[name]["bias"].cpu().numpy(), L[name]["b"]) for name in ("qkv", "proj", "fc1", "fc2")})
+    return out
+
+
+def oracle_step(olayers, h_rows, nthreads):
+    """One oracle pass over a row sample: pack every weight, then the chained stack on the rows."""
+    import oracle
+    for L in olayers:
+        for name in ("qkv", "proj", "fc1", "fc2"):
+            W, Mk, _, b = L[name]
+            oracle.pack(W, Mk, b)
+    return oracle.deit_stack_rows(h_rows, olayers, nthreads)
+
+
+def eff_flops_rows(olayers, rows):
+    return sum(2 * rows * int((L[n][1] != 0).sum()) * L[n][3] ** 2 for L in olayers for n in L)
+
+
+def calibrate_rows(olayers, h_bits, nthreads, budget_s, steps):
+    """Rows per oracle step so that `steps` steps (pack + chain) take about `budget_s` seconds."""
+    import oracle
+    t0 = time.perf_counter()
+    for L in olayers:
+        for name in ("qkv", "proj", "fc1", "fc2"):
+            W, Mk, _, b = L[name]
+            oracle.pack(W, Mk, b)
+    t_pack = time.perf_counter() - t0
+    r0 = min(len(h_bits), max(1, nthreads))
+    t0 = time.perf_counter()
+    oracle.deit_stack_rows(h_bits[:r0], olayers, nthreads)
+    rate = r0 / max(time.perf_counter() - t0, 1e-6)          # rows per second on all threads
+    per_step = budget_s / max(steps, 1) - t_pack
+    rows = int(max(per_step, 0.0) * rate)
+    if rows >= nthreads:
+        rows -= rows % nthreads
+    return max(1, min(len(h_bits), rows))
+
+
+def run_reference(args, world, rank):
+    """The reference arm: the CPU oracle as it stands, on this host's cores, bounded sample per step."""
+    if rank != 0:
+        return
+    import numpy as np
+    import oracle
+    from paper_2407_02068_gb300 import inputs
+    oracle.build()
+    layers = inputs.deit_b_stack(CONFIG_ID, BLOCK, "cpu")
+    olayers = oracle_layers_from(layers)
+    cores = os.cpu_count() or 1
+    total = args.warmup + args.steps
+    budget = min(150.0, 6.0 * total)  # whole run within a few minutes
+    h_all = inputs.bf16_bits(inputs.activations(4096, 768, inputs.seed(CONFIG_ID, 0, "X")))
+    rows = calibrate_rows(olayers, h_all, cores, budget, total)
+    rng = np.random.default_rng(0)
+    for _ in range(args.warmup):
+        oracle_step(olayers, h_all[rng.choice(len(h_all), rows, replace=False)], cores)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_step(olayers, h_all[rng.choice(len(h_all), rows, replace=False)], cores)
+    dt = time.perf_counter() - t0
+    flops = eff_flops_rows(olayers, rows) * args.steps
+    value = flops / dt / 1e12
+    sample = (f"{rows} token rows per step through all 48 GEMMs (+ packing all 48 weights) of the batch-256 "
+              f"DeiT-B stack, fp64 C oracle, {cores} threads")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": WORKLOAD, "M": M_TOKENS, "block": BLOCK, "gemms": 48,
+                                            "sample_rows_per_step": rows},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------------ GPU arm
+
+def run_gpu(args, world, rank, local):
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2407_02068_gb300 import inputs
+    from paper_2407_02068_gb300.stack import DeitLinearStack
+
+    layers = inputs.deit_b_stack(CONFIG_ID, BLOCK, dev)
+    stack = DeitLinearStack(M_TOKENS, layers, dev)
+    # each rank works on its own batch (weak scaling: per-GPU work fixed); weights are replicated
+    h0 = inputs.activations(M_TOKENS, 768, inputs.seed(CONFIG_ID, 0, "X") + 7 * rank, dev)
+    stack.h_in.copy_(h0)
+    s = torch.cuda.current_stream()
+    ngemm = len(stack.gemms)
+
+    for _ in range(max(args.warmup, 3)):
+        stack.step()
+    stack.check()
+    torch.cuda.synchronize()
+
+    # ---------------- timed region: K steps, per-linear events on the launching stream
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(ngemm)]
+          for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    start.record(s)
+    for k in range(args.steps):
+        stack.step(events=ev[k])
+    end.record(s)
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop()
+    stack.check()
+    elapsed_ms = start.elapsed_time(end)
+    lin_ms = sum(a.elapsed_time(b) for row in ev for (a, b) in row)
+    elapsed_max = max_over_ranks(elapsed_ms, world, dev)
+    flops_step = stack.effective_flops()
+    value = flops_step * args.steps * world / (elapsed_max / 1e3) / 1e12
+    lin_flops = flops_step * args.steps
+    achieved = lin_flops / (lin_ms / 1e3) / 1e12
+    peaks, peak_src = load_peaks()
+    peak = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    traffic = profiled_traffic()
+    linear_launches = ngemm * args.steps
+
+    # ---------------- e2e through the public API: pinned host in, pinned host out, every step
+    e2e_steps = args.e2e_steps or max(10, min(args.steps, 100))
+    h0_host = h0.cpu().pin_memory()
+    out_host = torch.empty_like(h0_host).pin_memory()
+    for _ in range(2):
+        stack.h_in.copy_(h0_host, non_blocking=True)
+        out = stack.step()
+        out_host.copy_(out, non_blocking=True)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    e0.record(s)
+    for _ in range(e2e_steps):
+        stack.h_in.copy_(h0_host, non_blocking=True)
+        out = stack.step()
+        out_host.copy_(out, non_blocking=True)
+    e1.record(s)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_value = flops_step * e2e_steps * world / (e2e_ms / 1e3) / 1e12
+    io_bytes = h0_host.numel() * h0_host.element_size()
+
+    # ---------------- dense comparator (torch bf16 F.linear on W (.) M, same chain)
+    dense = None
+    if not args.no_dense:
+        for _ in range(3):
+            stack.dense_forward(h0)
+        torch.cuda.synchronize()
+        d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        nd = max(5, min(args.steps, 50))
+        d0.record(s)
+        for _ in range(nd):
+            stack.dense_forward(h0)
+        d1.record(s)
+        torch.cuda.synchronize()
+        dense_ms = d0.elapsed_time(d1) / nd
+        stack_lin_ms = lin_ms / args.steps
+        dense = {"dense_torch_ms_per_step": dense_ms, "speedup_linears_vs_dense": dense_ms / stack_lin_ms,
+                 "speedup_step_vs_dense": dense_ms / (elapsed_ms / args.steps)}
+
+    # ---------------- CPU oracle baseline (rank 0, N = 1)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        olayers = oracle_layers_from(layers)
+        cores = os.cpu_count() or 1
+        h_bits = inputs.bf16_bits(h0[:8192])
+        rows = calibrate_rows(olayers, h_bits, cores, args.cpu_budget_s, 1)
+        t0 = time.perf_counter()
+        oracle_step(olayers, h_bits[:rows], cores)
+        dt = time.perf_counter() - t0
+        cpu = {"value": eff_flops_rows(olayers, rows) / dt / 1e12, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"first {rows} token rows through all 48 GEMMs (+ packing all 48 weights), one pass, "
+                         f"fp64 C oracle on {cores} threads, {dt:.1f} s"}
+
+    if rank != 0:
+        return
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": max(args.warmup, 3), "ms_per_step": elapsed_max / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "M": M_TOKENS, "block": BLOCK, "gemms": ngemm,
+                   "sparsity": "per-GEMM U[0.30,0.70], antithetic layer pairs, mean 0.50",
+                   "step": "pack all 48 weights + 48 chained block-sparse linears (fc1 with GELU)",
+                   "l2": "no flush: each step streams ~15 GB (> 129 MB L2)",
+                   "parallelism": f"replicas x{world} (token batches per rank, no collective)"},
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)",
+                     "kernel": "lpvit::bsr_linear_kernel<32>", "launches_timed": linear_launches,
+                     "frac_of_burst_peak": achieved / float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))},
+        "linear_ms_per_step": lin_ms / args.steps,
+        "pack_and_gaps_ms_per_step": (elapsed_ms - lin_ms) / args.steps,
+        "hbm_gbs_linears": stack.algorithmic_bytes() * args.steps / (lin_ms / 1e3) / 1e9,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": io_bytes, "d2h_bytes_per_step": io_bytes,
+                "steps": e2e_steps},
+        "gpu_launches": args.steps * ngemm * 3,
+        "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
+                   "power_w_median": clk.get("power_w_median"), "samples": clk["samples"]},
+        "cpu_baseline": cpu,
+    }
+    if dense:
+        line.update(dense)
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    world, rank, local = dist_setup(args)
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+        return
+    run_gpu(args, world, rank, local)
+
+
+if __name__ == "__main__":
+    main()

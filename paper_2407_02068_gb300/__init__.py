@@ -17,7 +17,8 @@ import torch
 
 from . import _lib
 
-__all__ = ["BsrWeight", "pack_bsr", "workspace_for", "bsr_linear", "check", "LpvitError"]
+__all__ = ["BsrWeight", "alloc_bsr", "pack_bsr", "pack_bsr_into", "workspace_for", "bsr_linear", "check",
+           "LpvitError"]
 
 LpvitError = _lib.LpvitError
 
@@ -46,29 +47,42 @@ class BsrWeight:
                               self.sched.numel())
 
 
+def alloc_bsr(n: int, k: int, b: int, capacity: int | None = None, device="cuda") -> BsrWeight:
+    """Device buffers for a packed n x k weight with b x b blocks (capacity defaults to every block)."""
+    if capacity is None:
+        capacity = (n // b) * (k // b) if b > 0 and n % b == 0 and k % b == 0 else 0
+    sb = _lib.lpvit_sched_bytes(n, k, b)
+    return BsrWeight(n, k, b, capacity,
+                     torch.empty(max(n // max(b, 1), 0) + 1, dtype=torch.int32, device=device),
+                     torch.empty(max(capacity, 1), dtype=torch.int32, device=device),
+                     torch.empty((max(capacity, 1), max(b, 1), max(b, 1)), dtype=torch.bfloat16, device=device),
+                     torch.empty(max(sb, 16), dtype=torch.uint8, device=device))
+
+
+def pack_bsr_into(w: BsrWeight, W: torch.Tensor, mask: torch.Tensor, count: bool = False, stream=None) -> BsrWeight:
+    """Pack W (bf16 [n, k], contiguous CUDA) under the block mask (uint8 [n/b, k/b], contiguous CUDA,
+    nonzero = kept) into the buffers of ``w``; asynchronous unless ``count``."""
+    if W.dtype != torch.bfloat16 or not W.is_cuda or W.dim() != 2 or not W.is_contiguous():
+        raise ValueError("W must be a contiguous 2-D bf16 CUDA tensor")
+    if mask.dtype != torch.uint8 or not mask.is_contiguous() or mask.device != W.device:
+        raise ValueError("mask must be a contiguous uint8 tensor on W's device")
+    st, nnzb = _lib.lpvit_pack_bsr(W.data_ptr(), mask.data_ptr(), w.struct(), count, _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_pack_bsr")
+    w.nnzb = nnzb
+    return w
+
+
 def pack_bsr(W: torch.Tensor, mask: torch.Tensor, b: int, capacity: int | None = None, count: bool = False,
              stream=None) -> BsrWeight:
-    """Pack W (bf16 [n, k], CUDA) under the block mask (uint8 [n/b, k/b], CUDA, nonzero = kept)."""
+    """Pack W (bf16 [n, k], CUDA) under the block mask (uint8 [n/b, k/b], nonzero = kept)."""
     if W.dtype != torch.bfloat16 or not W.is_cuda or W.dim() != 2:
         raise ValueError("W must be a 2-D bf16 CUDA tensor")
     W = W.contiguous()
     mask = mask.to(device=W.device, dtype=torch.uint8).contiguous()
     n, k = W.shape
-    if capacity is None:
-        capacity = (n // b) * (k // b) if b > 0 and n % b == 0 and k % b == 0 else 0
-    sb = _lib.lpvit_sched_bytes(n, k, b)
-    dev = W.device
-    w = BsrWeight(n, k, b, capacity,
-                  torch.empty(max(n // max(b, 1), 0) + 1, dtype=torch.int32, device=dev),
-                  torch.empty(max(capacity, 1), dtype=torch.int32, device=dev),
-                  torch.empty((max(capacity, 1), max(b, 1), max(b, 1)), dtype=torch.bfloat16, device=dev),
-                  torch.empty(max(sb, 16), dtype=torch.uint8, device=dev))
-    s = w.struct()
-    st, nnzb = _lib.lpvit_pack_bsr(W.data_ptr(), mask.data_ptr(), s, count, _stream_handle(stream))
-    if st != _lib.LPVIT_OK:
-        raise LpvitError(st, "lpvit_pack_bsr")
-    w.nnzb = nnzb
-    return w
+    w = alloc_bsr(n, k, b, capacity, W.device)
+    return pack_bsr_into(w, W, mask, count, stream)
 
 
 def workspace_for(w: BsrWeight, m: int, device=None) -> torch.Tensor:
