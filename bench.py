@@ -36,6 +36,13 @@ CONFIG_ID = 4             # seeds of the 12-layer stack workload
 WORKLOAD = "deit_b_12layer_linear_stack_batch256"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "bsr_linear_deit_b_stack_traffic.txt")
+# single GEMMs of the stack's shapes (profiling cases): (k, n, b, sparsity, gelu, m)
+CASES = {
+    "fc1": (768, 3072, 32, 0.5, True, M_TOKENS),
+    "fc2": (3072, 768, 32, 0.5, False, M_TOKENS),
+    "qkv": (768, 2304, 32, 0.5, False, M_TOKENS),
+    "proj": (768, 768, 32, 0.5, False, M_TOKENS),
+}
 
 
 def parse_args():
@@ -48,6 +55,8 @@ def parse_args():
     p.add_argument("--cpu-budget-s", type=float, default=15.0, help="CPU seconds for the oracle baseline sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-dense", action="store_true")
+    p.add_argument("--case", default="stack", choices=["stack"] + sorted(CASES),
+                   help="stack (the benchmarked workload) or one GEMM of it, for profiling")
     return p.parse_args()
 
 
@@ -393,11 +402,54 @@ def run_gpu(args, world, rank, local):
         dist.destroy_process_group()
 
 
+def run_case(args, local):
+    """One GEMM of the stack's shapes, pack + linear per step (for ncu and per-shape numbers)."""
+    import torch
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2407_02068_gb300 as lp
+    from paper_2407_02068_gb300 import inputs
+    k, n, b, sp, gelu, m = CASES[args.case]
+    g = inputs.make_gemm(CONFIG_ID, 0, m, k, n, b, sp, device=dev)
+    mask = g["mask"].to(dev).contiguous()
+    w = lp.alloc_bsr(n, k, b, device=dev)
+    Y = torch.empty(m, n, dtype=torch.bfloat16, device=dev)
+    lp.pack_bsr_into(w, g["W"], mask)
+    ws = lp.workspace_for(w, m)
+    for _ in range(max(args.warmup, 1)):
+        lp.pack_bsr_into(w, g["W"], mask)
+        lp.bsr_linear(w, g["X"], g["bias"], gelu=gelu, out=Y, workspace=ws)
+    lp.check(ws)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for e0, e1 in ev:
+        lp.pack_bsr_into(w, g["W"], mask)
+        e0.record()
+        lp.bsr_linear(w, g["X"], g["bias"], gelu=gelu, out=Y, workspace=ws)
+        e1.record()
+    torch.cuda.synchronize()
+    lp.check(ws)
+    ms = sum(a.elapsed_time(b_) for a, b_ in ev) / len(ev)
+    nnzb = int((g["mask"] != 0).sum())
+    flops = 2 * m * nnzb * b * b
+    byts = 2 * m * k + 2 * m * n + 2 * nnzb * b * b + 4 * nnzb + 4 * (n // b + 1) + 4 * n
+    peaks, src = load_peaks()
+    print(json.dumps({"case": args.case, "m": m, "k": k, "n": n, "b": b, "sparsity": sp, "gelu": gelu,
+                      "linear_ms": ms, "eff_tflops": flops / ms / 1e9, "gbs": byts / ms / 1e6,
+                      "frac_tensor_burst": flops / ms / 1e9 / float(peaks.get("bf16_tflops", 1900.0)),
+                      "frac_hbm": byts / ms / 1e6 / float(peaks.get("hbm_gbs", 6800.0)), "peaks": src}),
+          flush=True)
+
+
 def main():
     args = parse_args()
     world, rank, local = dist_setup(args)
     if args.impl == "reference":
         run_reference(args, world, rank)
+        return
+    if args.case != "stack":
+        run_case(args, local)
         return
     run_gpu(args, world, rank, local)
 

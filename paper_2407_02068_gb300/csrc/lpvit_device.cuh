@@ -159,6 +159,8 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
 
 // Weight-stationary MMA D[M x N] (+)= A[M x 16] * B[N x 16]^T with the B operand held in
 // collector buffer BUF: fill (load and keep), use (reuse), lastuse (reuse and release), or none.
+// COLL and BUF are compile-time so that every call site is one straight-line instruction; the
+// caller computes the (warp-uniform) operands with the whole warp and lets one elected lane issue.
 enum Coll { COLL_NONE = 0, COLL_FILL = 1, COLL_USE = 2, COLL_LAST = 3 };
 
 #define LPVIT_WS_MMA(QUAL)                                                                            \
@@ -166,27 +168,27 @@ enum Coll { COLL_NONE = 0, COLL_FILL = 1, COLL_USE = 2, COLL_LAST = 3 };
                "tcgen05.mma.ws.cta_group::1.kind::f16" QUAL " [%0], %1, %2, %3, p;}\n"               \
                :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate))
 
-template <int BUF>
-__device__ __forceinline__ void ws_mma(int coll, uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+template <int BUF, int COLL>
+__device__ __forceinline__ void ws_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                        uint32_t accumulate) {
   static_assert(BUF >= 0 && BUF < 4, "collector buffer");
-  if (coll == COLL_NONE) {
+  if constexpr (COLL == COLL_NONE) {
     LPVIT_WS_MMA("");
-  } else if (BUF == 0) {
-    if (coll == COLL_FILL) LPVIT_WS_MMA(".collector::b0::fill");
-    else if (coll == COLL_USE) LPVIT_WS_MMA(".collector::b0::use");
+  } else if constexpr (BUF == 0) {
+    if constexpr (COLL == COLL_FILL) LPVIT_WS_MMA(".collector::b0::fill");
+    else if constexpr (COLL == COLL_USE) LPVIT_WS_MMA(".collector::b0::use");
     else LPVIT_WS_MMA(".collector::b0::lastuse");
-  } else if (BUF == 1) {
-    if (coll == COLL_FILL) LPVIT_WS_MMA(".collector::b1::fill");
-    else if (coll == COLL_USE) LPVIT_WS_MMA(".collector::b1::use");
+  } else if constexpr (BUF == 1) {
+    if constexpr (COLL == COLL_FILL) LPVIT_WS_MMA(".collector::b1::fill");
+    else if constexpr (COLL == COLL_USE) LPVIT_WS_MMA(".collector::b1::use");
     else LPVIT_WS_MMA(".collector::b1::lastuse");
-  } else if (BUF == 2) {
-    if (coll == COLL_FILL) LPVIT_WS_MMA(".collector::b2::fill");
-    else if (coll == COLL_USE) LPVIT_WS_MMA(".collector::b2::use");
+  } else if constexpr (BUF == 2) {
+    if constexpr (COLL == COLL_FILL) LPVIT_WS_MMA(".collector::b2::fill");
+    else if constexpr (COLL == COLL_USE) LPVIT_WS_MMA(".collector::b2::use");
     else LPVIT_WS_MMA(".collector::b2::lastuse");
   } else {
-    if (coll == COLL_FILL) LPVIT_WS_MMA(".collector::b3::fill");
-    else if (coll == COLL_USE) LPVIT_WS_MMA(".collector::b3::use");
+    if constexpr (COLL == COLL_FILL) LPVIT_WS_MMA(".collector::b3::fill");
+    else if constexpr (COLL == COLL_USE) LPVIT_WS_MMA(".collector::b3::use");
     else LPVIT_WS_MMA(".collector::b3::lastuse");
   }
 }

@@ -79,6 +79,56 @@ __device__ __forceinline__ void store_out(void *Y, int64_t idx, float y, int y_f
   else static_cast<__nv_bfloat16 *>(Y)[idx] = __float2bfloat16_rn(y);
 }
 
+
+// All MMAs of one work-list entry: for every 16-wide k step, one weight-stationary MMA per present
+// MMA panel, the X chunk filled into collector buffer kk by the first panel and reused by the rest.
+// Every operand is computed by the whole warp (uniform values); one elected lane issues.
+template <int B, int KK>
+__device__ __forceinline__ void issue_kstep(uint32_t mm, uint32_t touched, uint32_t st_u32, uint32_t dbase) {
+  using C = Cfg<B>;
+  const uint64_t bdesc = smem_desc<C::ROW_BYTES>(st_u32 + KK * 32);
+  const uint32_t a0 = st_u32 + C::X_BYTES + KK * 32;
+  const int p_first = __ffs(mm) - 1;
+  const int p_last = 31 - __clz(mm);
+  auto acc_of = [&](int p) -> uint32_t { return (KK > 0 || ((touched >> p) & 1u)) ? 1u : 0u; };
+  if (p_first == p_last) {
+    const uint64_t ad = smem_desc<C::ROW_BYTES>(a0 + p_first * C::A_BYTES);
+    const uint32_t d = dbase + (uint32_t)(p_first * C::ACC_COLS), acc = acc_of(p_first);
+    if (elect_one()) ws_mma<KK, COLL_NONE>(d, ad, bdesc, C::IDESC, acc);
+    __syncwarp();
+    return;
+  }
+  {
+    const uint64_t ad = smem_desc<C::ROW_BYTES>(a0 + p_first * C::A_BYTES);
+    const uint32_t d = dbase + (uint32_t)(p_first * C::ACC_COLS), acc = acc_of(p_first);
+    if (elect_one()) ws_mma<KK, COLL_FILL>(d, ad, bdesc, C::IDESC, acc);
+    __syncwarp();
+  }
+  uint32_t mid = mm & ~(1u << p_first) & ~(1u << p_last);
+  while (mid) {
+    const int p = __ffs(mid) - 1;
+    mid &= mid - 1u;
+    const uint64_t ad = smem_desc<C::ROW_BYTES>(a0 + p * C::A_BYTES);
+    const uint32_t d = dbase + (uint32_t)(p * C::ACC_COLS), acc = acc_of(p);
+    if (elect_one()) ws_mma<KK, COLL_USE>(d, ad, bdesc, C::IDESC, acc);
+    __syncwarp();
+  }
+  {
+    const uint64_t ad = smem_desc<C::ROW_BYTES>(a0 + p_last * C::A_BYTES);
+    const uint32_t d = dbase + (uint32_t)(p_last * C::ACC_COLS), acc = acc_of(p_last);
+    if (elect_one()) ws_mma<KK, COLL_LAST>(d, ad, bdesc, C::IDESC, acc);
+    __syncwarp();
+  }
+}
+
+template <int B>
+__device__ __forceinline__ void issue_entry(uint32_t mm, uint32_t touched, uint32_t st_u32, uint32_t dbase) {
+  issue_kstep<B, 0>(mm, touched, st_u32, dbase);
+  if constexpr (Cfg<B>::KSTEPS > 1) issue_kstep<B, 1>(mm, touched, st_u32, dbase);
+  if constexpr (Cfg<B>::KSTEPS > 2) issue_kstep<B, 2>(mm, touched, st_u32, dbase);
+  if constexpr (Cfg<B>::KSTEPS > 3) issue_kstep<B, 3>(mm, touched, st_u32, dbase);
+}
+
 template <int B>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
 bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
@@ -331,29 +381,8 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
 #pragma unroll
         for (int p = 0; p < C::G; ++p) mm |= ((pm >> (p * C::PPM)) & ((1u << C::PPM) - 1u)) ? (1u << p) : 0u;
         const uint32_t st_u32 = smem_base + stage * C::STAGE_BYTES;
-        if (elect_one()) {
-          const int np = __popc(mm);
-#pragma unroll
-          for (int kk = 0; kk < C::KSTEPS; ++kk) {
-            const uint64_t bdesc = smem_desc<C::ROW_BYTES>(st_u32 + kk * 32);
-            uint32_t rem = mm;
-            int i = 0;
-            while (rem) {
-              const int p = __ffs(rem) - 1;
-              rem &= rem - 1u;
-              const uint64_t adesc = smem_desc<C::ROW_BYTES>(st_u32 + C::X_BYTES + p * C::A_BYTES + kk * 32);
-              const uint32_t d = dbase + (uint32_t)(p * C::ACC_COLS);
-              const uint32_t acc = (kk > 0 || ((touched >> p) & 1u)) ? 1u : 0u;
-              const int coll = np == 1 ? COLL_NONE : (i == 0 ? COLL_FILL : (rem == 0 ? COLL_LAST : COLL_USE));
-              if (kk == 0) ws_mma<0>(coll, d, adesc, bdesc, C::IDESC, acc);
-              else if (kk == 1) ws_mma<1>(coll, d, adesc, bdesc, C::IDESC, acc);
-              else if (kk == 2) ws_mma<2>(coll, d, adesc, bdesc, C::IDESC, acc);
-              else ws_mma<3>(coll, d, adesc, bdesc, C::IDESC, acc);
-              ++i;
-            }
-          }
-          tc_commit(empty_bar(stage));
-        }
+        issue_entry<B>(mm, touched, st_u32, dbase);
+        if (elect_one()) tc_commit(empty_bar(stage));
         __syncwarp();
         touched |= mm;
         ++it;
