@@ -109,6 +109,29 @@ lpvit_status lpvit_bsr_linear_gelu(const lpvit_bsr *bsr, const void *X, int64_t 
                                    const float *bias, void *Y, int64_t ldy, lpvit_dtype y_dtype, void *workspace,
                                    size_t ws_bytes, void *stream);
 
+/* Size of the library-held scratch array used by lpvit_bsr_linear_noalloc (8 MiB). */
+#define LPVIT_NOALLOC_SCRATCH_BYTES (8 * 1024 * 1024)
+
+/* As lpvit_bsr_linear (gelu == 0) or lpvit_bsr_linear_gelu (gelu != 0), for callers that cannot
+ * allocate device memory where they run this layer: code that has no allocator of its own because
+ * another runtime owns all device memory, code recorded while a stream is being captured, or
+ * latency-critical paths that must not take the allocator's implicit synchronisation. This entry
+ * point has no counterpart in the paper; it only changes who holds the workspace.
+ * The workspace is a library-owned device array of LPVIT_NOALLOC_SCRATCH_BYTES that every GPU
+ * loading the library keeps until the process exits; the call allocates nothing (no cudaMalloc,
+ * cudaFree or allocating library routine). The first call on a device looks up the array's device
+ * address (cudaGetSymbolAddress, with that device current) and caches it; make that first call
+ * before any stream capture. Each call clears the array's counters on `stream` before launching.
+ * All calls share the one array: calls whose kernels may overlap on the GPU (other streams,
+ * other host threads) race and give wrong results; serialise them.
+ * Errors: as lpvit_bsr_linear, plus LPVIT_ERR_WORKSPACE when lpvit_workspace_bytes(bsr, m)
+ * exceeds LPVIT_NOALLOC_SCRATCH_BYTES (large-m calls need well under 1 MiB; small-m calls whose
+ * work is split need up to n_tiles * groups * slices * 128 KiB). A device-side timeout is not
+ * reported by this entry point (its error word lives in the shared array). */
+lpvit_status lpvit_bsr_linear_noalloc(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx,
+                                      const float *bias, void *Y, int64_t ldy, lpvit_dtype y_dtype, int gelu,
+                                      void *stream);
+
 /* Synchronises `stream`, then reads and clears the error word in `workspace`.
  * Returns LPVIT_OK, LPVIT_ERR_TIMEOUT (a device-side bounded wait ran out; the kernel
  * stopped early and its output is incomplete) or LPVIT_ERR_CUDA. */

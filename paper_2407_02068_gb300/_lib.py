@@ -22,7 +22,8 @@ LPVIT_BF16 = 0
 LPVIT_F32 = 1
 
 EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_workspace_bytes", "lpvit_bsr_linear",
-           "lpvit_bsr_linear_gelu", "lpvit_check", "lpvit_status_string")
+           "lpvit_bsr_linear_gelu", "lpvit_bsr_linear_noalloc", "lpvit_check", "lpvit_status_string")
+LPVIT_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 
 class lpvit_bsr(ctypes.Structure):
@@ -67,6 +68,8 @@ def load(path: str | None = None):
             f = getattr(lib, name)
             f.restype = ctypes.c_int
             f.argtypes = [BP, V, I64, I64, V, V, I64, ctypes.c_int, V, SZ, V]
+        lib.lpvit_bsr_linear_noalloc.restype = ctypes.c_int
+        lib.lpvit_bsr_linear_noalloc.argtypes = [BP, V, I64, I64, V, V, I64, ctypes.c_int, ctypes.c_int, V]
         lib.lpvit_check.restype = ctypes.c_int
         lib.lpvit_check.argtypes = [V, V]
         lib.lpvit_status_string.restype = ctypes.c_char_p
@@ -103,6 +106,12 @@ def lpvit_bsr_linear(bsr, X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, ws_ptr, 
 def lpvit_bsr_linear_gelu(bsr, X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, ws_ptr, ws_bytes, stream) -> int:
     return load().lpvit_bsr_linear_gelu(ctypes.byref(bsr), X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, ws_ptr,
                                         ws_bytes, stream)
+
+
+def lpvit_bsr_linear_noalloc(bsr, X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, gelu, stream) -> int:
+    """The linear with the library's own scratch array as workspace (no allocation by anyone)."""
+    return load().lpvit_bsr_linear_noalloc(ctypes.byref(bsr), X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype,
+                                           1 if gelu else 0, stream)
 
 
 def lpvit_check(ws_ptr: int, stream: int) -> int:
