@@ -179,6 +179,7 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.S = choose_slice(P.n_tt, P.n_groups, k / b, sms);
   P.y_f32 = y_dtype == LPVIT_F32;
   P.gelu = gelu;
+  P.y_vec16 = (aligned(Y, 16) && ldy % 8 == 0) ? 1 : 0;
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   P.ctl = reinterpret_cast<Control *>(ws);
   P.tickets = reinterpret_cast<int32_t *>(ws + W.tickets_off);

@@ -11,17 +11,21 @@ namespace lpvit {
 // Layout of the work list ("sched") shared by the pack and the GEMM.
 // header (16 int32): [0] nnzb, [1] n_groups, [2] total entries, [3] overflow flag, [4] n, [5] k, [6] b
 // then gent_ptr[n_groups + 1] (int32, entries of group g are [gent_ptr[g], gent_ptr[g+1]))
-// then entries, ENTRY_INTS int32 each: [0] = j | (panel mask << 16), [1 + p] = block index of the
-// group's p-th row panel at block column j, or -1.
+// then entries, ENTRY_INTS int32 each: [0] = j | (row-panel mask << 16), [1 + p] = block index of
+// the group's p-th row panel at block column j, or -1 (p < GROUP_FEATURES / b <= 8).
 constexpr int SCHED_HDR_INTS = 16;
 constexpr int ENTRY_INTS = 12;
-constexpr int GROUP_FEATURES = 128;  // output features covered by one work unit
-constexpr int TOKENS_PER_TILE = 256; // tokens covered by one work unit (the .ws MMA N)
+constexpr int GROUP_FEATURES = 128;   // output features covered by one work unit
+constexpr int MAX_GROUP_PANELS = GROUP_FEATURES / 16;
+constexpr int TOKENS_PER_TILE = 256;  // tokens covered by one work unit (the .ws MMA N)
 
 __host__ __device__ inline int sched_gent_offset_ints() { return SCHED_HDR_INTS; }
 __host__ __device__ inline int64_t sched_entries_offset_ints(int n_groups) {
   return ((int64_t)SCHED_HDR_INTS + n_groups + 1 + 3) / 4 * 4;  // 16-byte aligned entries
 }
+
+static_assert(GROUP_FEATURES / 16 <= MAX_GROUP_PANELS, "entry holds every row panel of a group");
+static_assert(1 + MAX_GROUP_PANELS <= ENTRY_INTS, "entry size");
 
 // Workspace control block (first 256 bytes of the caller's workspace).
 struct Control {
@@ -43,6 +47,7 @@ struct LinearParams {
   int n, k;
   int n_tt, n_groups, S;   // token tiles, 128-feature groups, max entries per slice
   int y_f32, gelu;
+  int y_vec16;             // bf16 output rows may take 16-byte stores (Y 16-byte aligned, ldy % 8 == 0)
   Control *ctl;
   int32_t *tickets;        // [n_tt * n_groups] arrival tickets of split units
   float *partials;         // [slots][128 features][256 tokens] fp32 partial sums of split units

@@ -43,6 +43,9 @@ struct Cfg {
   static constexpr int STAGE_BYTES = X_BYTES + G * A_BYTES;
   static constexpr int NSTAGES = 196608 / STAGE_BYTES;      // 192 KB of stages
   static constexpr int UR = 4;                              // unit-info ring depth
+  static constexpr int BATCH = NSTAGES >= 16 ? 8 : NSTAGES / 2;  // most entries per lane-parallel TMA batch
+  static constexpr int OPS = 1 + GB;                        // lane slots per entry: X tile + one per row panel
+  static constexpr int NBMAX = BATCH < 32 / OPS ? BATCH : 32 / OPS;  // entries per batch
   static constexpr int VPT = TT * MP / 128 / 2;             // accumulator values per epilogue thread and panel
   static constexpr uint32_t IDESC = idesc_bf16(MP, TT);
   static_assert(BUF_COLS == 256, "two accumulator buffers fill the 512 TMEM columns");
@@ -70,55 +73,95 @@ struct Smem {
   static constexpr int RING_OFF = (META_OFF + 4 * NS + 31) / 32 * 32;
   static constexpr int SLICE_OFF = RING_OFF + (int)sizeof(UnitInfo) * UR;
   static constexpr int MISC_OFF = SLICE_OFF + 4 * (MAX_GROUPS + 1);
-  static constexpr int END = MISC_OFF + 64;
+  static constexpr int EPI_OFF = (MISC_OFF + 64 + 127) / 128 * 128;
+  static constexpr int EPI_TILE = 32 * 80;  // per epilogue warp: 32 token rows x 32 bf16, rows padded to 80 B
+  static constexpr int END = EPI_OFF + 8 * EPI_TILE;
   static constexpr int BYTES = END + 1024;  // + alignment slack for the dynamic smem base
 };
 
-__device__ __forceinline__ void store_out(void *Y, int64_t idx, float y, int y_f32) {
-  if (y_f32) static_cast<float *>(Y)[idx] = y;
-  else static_cast<__nv_bfloat16 *>(Y)[idx] = __float2bfloat16_rn(y);
+// Epilogue of one 32 x 32 block held by a warp: v[i] = accumulator of token tok_base + i for feature
+// f0 + lane. Adds the bias, applies GELU, rounds, and stores rows [tok_base, min(tok_base + 32, m)).
+// bf16 output is staged through this warp's shared tile (rows padded to 80 bytes, conflict-free) so
+// that every token row leaves as 16-byte vector stores; fp32 output is stored directly (a warp
+// writes 128 contiguous bytes per token).
+__device__ __forceinline__ void emit32(const float (&v)[32], int f0, int64_t tok_base, const LinearParams &P,
+                                       uint8_t *tile) {
+  const int lane = threadIdx.x & 31;
+  const int f = f0 + lane;
+  const bool fvalid = f < P.n;
+  const float bb = (P.bias != nullptr && fvalid) ? __ldg(P.bias + f) : 0.f;
+  const int64_t left = P.m - tok_base;
+  const int rows = left >= 32 ? 32 : (left > 0 ? (int)left : 0);
+  float y[32];
+  if (P.gelu) {
+    const float kInvSqrt2 = 0.70710678118654752440f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const float t = v[i] + bb;
+      y[i] = 0.5f * t * (1.f + erff(t * kInvSqrt2));
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) y[i] = v[i] + bb;
+  }
+  if (P.y_f32) {
+    float *dst = static_cast<float *>(P.Y) + tok_base * P.ldy + f;
+    if (fvalid) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i)
+        if (i < rows) dst[(int64_t)i * P.ldy] = y[i];
+    }
+    return;
+  }
+  __nv_bfloat16 *t = reinterpret_cast<__nv_bfloat16 *>(tile);
+#pragma unroll
+  for (int i = 0; i < 32; ++i) t[i * 40 + lane] = __float2bfloat16_rn(y[i]);
+  __syncwarp();
+  const int ch = lane & 3;
+  const bool cvalid = f0 + ch * 8 < P.n;
+#pragma unroll
+  for (int it = 0; it < 4; ++it) {
+    const int row = 8 * it + (lane >> 2);
+    const int4 val = *reinterpret_cast<const int4 *>(tile + row * 80 + ch * 16);
+    if (row < rows && cvalid) {
+      __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(P.Y) + (tok_base + row) * P.ldy + f0 + ch * 8;
+      if (P.y_vec16) {
+        *reinterpret_cast<int4 *>(dst) = val;
+      } else {
+        const __nv_bfloat16 *src = reinterpret_cast<const __nv_bfloat16 *>(&val);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) dst[e] = src[e];
+      }
+    }
+  }
+  __syncwarp();
 }
 
 
-// All MMAs of one work-list entry: for every 16-wide k step, one weight-stationary MMA per present
-// MMA panel, the X chunk filled into collector buffer kk by the first panel and reused by the rest.
-// Every operand is computed by the whole warp (uniform values); one elected lane issues.
+// All MMAs of one work-list entry, issued by one elected thread: for every 16-wide k step, one
+// weight-stationary MMA per present MMA panel; the X chunk is filled into collector buffer KK by the
+// first panel and reused by the others. Collector variants are compile-time, panel order ascending.
 template <int B, int KK>
 __device__ __forceinline__ void issue_kstep(uint32_t mm, uint32_t touched, uint32_t st_u32, uint32_t dbase) {
   using C = Cfg<B>;
   const uint64_t bdesc = smem_desc<C::ROW_BYTES>(st_u32 + KK * 32);
-  const uint32_t a0 = st_u32 + C::X_BYTES + KK * 32;
+  const uint64_t a0 = smem_desc<C::ROW_BYTES>(st_u32 + C::X_BYTES + KK * 32);
   const int p_first = __ffs(mm) - 1;
   const int p_last = 31 - __clz(mm);
   auto acc_of = [&](int p) -> uint32_t { return (KK > 0 || ((touched >> p) & 1u)) ? 1u : 0u; };
+  auto adesc = [&](int p) -> uint64_t { return a0 + (uint64_t)((p * C::A_BYTES) >> 4); };
   if (p_first == p_last) {
-    const uint64_t ad = smem_desc<C::ROW_BYTES>(a0 + p_first * C::A_BYTES);
-    const uint32_t d = dbase + (uint32_t)(p_first * C::ACC_COLS), acc = acc_of(p_first);
-    if (elect_one()) ws_mma<KK, COLL_NONE>(d, ad, bdesc, C::IDESC, acc);
-    __syncwarp();
+    ws_mma<KK, COLL_NONE>(dbase + (uint32_t)(p_first * C::ACC_COLS), adesc(p_first), bdesc, C::IDESC, acc_of(p_first));
     return;
   }
-  {
-    const uint64_t ad = smem_desc<C::ROW_BYTES>(a0 + p_first * C::A_BYTES);
-    const uint32_t d = dbase + (uint32_t)(p_first * C::ACC_COLS), acc = acc_of(p_first);
-    if (elect_one()) ws_mma<KK, COLL_FILL>(d, ad, bdesc, C::IDESC, acc);
-    __syncwarp();
-  }
+  ws_mma<KK, COLL_FILL>(dbase + (uint32_t)(p_first * C::ACC_COLS), adesc(p_first), bdesc, C::IDESC, acc_of(p_first));
   uint32_t mid = mm & ~(1u << p_first) & ~(1u << p_last);
   while (mid) {
     const int p = __ffs(mid) - 1;
     mid &= mid - 1u;
-    const uint64_t ad = smem_desc<C::ROW_BYTES>(a0 + p * C::A_BYTES);
-    const uint32_t d = dbase + (uint32_t)(p * C::ACC_COLS), acc = acc_of(p);
-    if (elect_one()) ws_mma<KK, COLL_USE>(d, ad, bdesc, C::IDESC, acc);
-    __syncwarp();
+    ws_mma<KK, COLL_USE>(dbase + (uint32_t)(p * C::ACC_COLS), adesc(p), bdesc, C::IDESC, acc_of(p));
   }
-  {
-    const uint64_t ad = smem_desc<C::ROW_BYTES>(a0 + p_last * C::A_BYTES);
-    const uint32_t d = dbase + (uint32_t)(p_last * C::ACC_COLS), acc = acc_of(p_last);
-    if (elect_one()) ws_mma<KK, COLL_LAST>(d, ad, bdesc, C::IDESC, acc);
-    __syncwarp();
-  }
+  ws_mma<KK, COLL_LAST>(dbase + (uint32_t)(p_last * C::ACC_COLS), adesc(p_last), bdesc, C::IDESC, acc_of(p_last));
 }
 
 template <int B>
@@ -280,53 +323,76 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
           for (int p = 0; p < C::GB; ++p) blk[p] = ep[1 + p];
         }
         const int cnt = min(32, e1 - base);
-        for (int i = 0; i < cnt; ++i) {
-          const uint32_t stage = it % L::NS, ph = (it / L::NS) & 1u;
-          if (!mbar_wait(empty_bar(stage), ph ^ 1u, abort_flag, tmo)) {
+        for (int i = 0; i < cnt && ok;) {
+          // One batch = NBMAX consecutive entries. Lane k*OPS + o issues op o of entry k (op 0: the X
+          // tile, op o >= 1: the block of row panel o-1 if kept), all in one instruction: a thread's
+          // bulk copies are processed one after another, copies from different threads overlap.
+          const int nb = min(C::NBMAX, cnt - i);
+          bool wok = true;
+          if (lane < nb) {
+            const uint32_t itk = it + lane;
+            wok = mbar_wait(empty_bar(itk % L::NS), ((itk / L::NS) & 1u) ^ 1u, abort_flag, tmo);
+          }
+          if (!__all_sync(0xffffffffu, wok)) {
             ok = false;
             if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_EMPTY);
             break;
           }
-          const int wi = __shfl_sync(0xffffffffu, w0, i);
-          int bi[C::GB];
-#pragma unroll
-          for (int p = 0; p < C::GB; ++p) bi[p] = __shfl_sync(0xffffffffu, blk[p], i);
-          const int j = wi & 0xffff;
-          const uint32_t pm = (uint32_t)wi >> 16;
-          uint8_t *st = smem + stage * C::STAGE_BYTES;
           if (C::PPM == 2) {
             // an MMA panel with exactly one of its two row panels present: zero the other half
             bool wrote = false;
+            for (int k = 0; k < nb; ++k) {
+              const uint32_t pmk = (uint32_t)__shfl_sync(0xffffffffu, w0, min(i + k, 31)) >> 16;
+              uint8_t *stk = smem + ((it + k) % L::NS) * C::STAGE_BYTES;
 #pragma unroll
-            for (int p = 0; p < C::G; ++p) {
-              const uint32_t two = (pm >> (2 * p)) & 3u;
-              if (two == 1u || two == 2u) {
-                const int half = two == 1u ? 1 : 0;
-                reinterpret_cast<int4 *>(st + C::X_BYTES + p * C::A_BYTES + half * C::BLK_BYTES)[lane] =
-                    make_int4(0, 0, 0, 0);
-                wrote = true;
+              for (int p = 0; p < C::G; ++p) {
+                const uint32_t two = (pmk >> (2 * p)) & 3u;
+                if (two == 1u || two == 2u) {
+                  const int half = two == 1u ? 1 : 0;
+                  reinterpret_cast<int4 *>(stk + C::X_BYTES + p * C::A_BYTES + half * C::BLK_BYTES)[lane] =
+                      make_int4(0, 0, 0, 0);
+                  wrote = true;
+                }
               }
             }
             if (wrote) fence_proxy_async_smem();
             __syncwarp();
           }
-          if (lane == 0) {
-            meta[stage] = (int)pm;
-            const uint32_t bytes = C::X_BYTES + __popc(pm) * C::BLK_BYTES;
-            const uint32_t fb = full_bar(stage);
-            mbar_arrive_expect_tx(fb, bytes);
-            const uint32_t st_u32 = smem_u32(st);
-            tma_load_2d(st_u32, &tmX, j * B, tt * C::TT, fb);
-#pragma unroll
-            for (int bp = 0; bp < C::GB; ++bp) {
-              if ((pm >> bp) & 1u) {
-                const int p = bp / C::PPM, half = bp % C::PPM;
-                tma_load_2d(st_u32 + C::X_BYTES + p * C::A_BYTES + half * C::BLK_BYTES, &tmW, 0, bi[bp] * B, fb);
-              }
+          {
+            const int wk = __shfl_sync(0xffffffffu, w0, min(i + lane, 31));
+            if (lane < nb) {
+              const uint32_t stk = (it + lane) % L::NS;
+              const uint32_t pmk = (uint32_t)wk >> 16;
+              meta[stk] = (int)pmk;
+              mbar_arrive_expect_tx(full_bar(stk), C::X_BYTES + __popc(pmk) * C::BLK_BYTES);
             }
           }
           __syncwarp();
-          ++it;
+          {
+            const int k = lane / C::OPS, o = lane - k * C::OPS;
+            const int srck = min(i + k, 31);
+            const int wsrc = __shfl_sync(0xffffffffu, w0, srck);
+            const uint32_t pm_k = (uint32_t)wsrc >> 16;
+            int bidx = 0;
+#pragma unroll
+            for (int q = 0; q < C::GB; ++q) {
+              const int v = __shfl_sync(0xffffffffu, blk[q], srck);
+              if (q == o - 1) bidx = v;
+            }
+            const bool is_x = o == 0;
+            if (k < nb && (is_x || ((pm_k >> (o - 1)) & 1u))) {
+              const uint32_t stk = (it + k) % L::NS;
+              const uint32_t st_u32 = smem_base + stk * C::STAGE_BYTES;
+              const int bp = o - 1;
+              const uint32_t dst =
+                  is_x ? st_u32 : st_u32 + C::X_BYTES + (bp / C::PPM) * C::A_BYTES + (bp % C::PPM) * C::BLK_BYTES;
+              tma_load_2d(dst, is_x ? &tmX : &tmW, is_x ? (wsrc & 0xffff) * B : 0, is_x ? tt * C::TT : bidx * B,
+                          full_bar(stk));
+            }
+          }
+          __syncwarp();
+          it += nb;
+          i += nb;
         }
       }
       if (!ok) break;
@@ -381,8 +447,10 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
 #pragma unroll
         for (int p = 0; p < C::G; ++p) mm |= ((pm >> (p * C::PPM)) & ((1u << C::PPM) - 1u)) ? (1u << p) : 0u;
         const uint32_t st_u32 = smem_base + stage * C::STAGE_BYTES;
-        issue_entry<B>(mm, touched, st_u32, dbase);
-        if (elect_one()) tc_commit(empty_bar(stage));
+        if (elect_one()) {
+          issue_entry<B>(mm, touched, st_u32, dbase);
+          tc_commit(empty_bar(stage));
+        }
         __syncwarp();
         touched |= mm;
         ++it;
@@ -409,7 +477,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     const int tok0 = (C::MP == 32) ? 64 * q + 32 * h : 128 * (q >> 1) + 64 * h;  // first token of this thread
     const int col0 = (C::MP == 32) ? 32 * h : 64 * h;                  // first column in the accumulator
     uint32_t ui = 0, sync_phase = 0;
-    const float kInvSqrt2 = 0.70710678118654752440f;
+    uint8_t *epi_tile = smem + L::EPI_OFF + ew * L::EPI_TILE;
     while (true) {
       const uint32_t slot = ui % L::UR, uph = (ui / L::UR) & 1u;
       if (!mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)) {
@@ -447,17 +515,8 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
             float4 *dst = reinterpret_cast<float4 *>(part + (int64_t)(p * C::MP + r) * C::TT + tok0 + c);
 #pragma unroll
             for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-          } else if (f < P.n) {
-            const float bb = P.bias ? __ldg(P.bias + f) : 0.f;
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int64_t tok = tok_base + c + i;
-              if (tok < P.m) {
-                float y = v[i] + bb;
-                if (P.gelu) y = 0.5f * y * (1.f + erff(y * kInvSqrt2));
-                store_out(P.Y, tok * P.ldy + f, y, P.y_f32);
-              }
-            }
+          } else {
+            emit32(v, f - lane, tok_base + c, P, epi_tile);
           }
         }
       }
@@ -500,8 +559,6 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
 #pragma unroll 1
           for (int p = 0; p < C::G; ++p) {
             const int f = inf.g * GROUP_FEATURES + p * C::MP + r;
-            if (f >= P.n) continue;
-            const float bb = P.bias ? __ldg(P.bias + f) : 0.f;
 #pragma unroll 1
             for (int c = 0; c < C::VPT; c += 32) {
               float v[32];
@@ -516,15 +573,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
                   v[4 * i] += t.x; v[4 * i + 1] += t.y; v[4 * i + 2] += t.z; v[4 * i + 3] += t.w;
                 }
               }
-#pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                const int64_t tok = tok_base + c + i;
-                if (tok < P.m) {
-                  float y = v[i] + bb;
-                  if (P.gelu) y = 0.5f * y * (1.f + erff(y * kInvSqrt2));
-                  store_out(P.Y, tok * P.ldy + f, y, P.y_f32);
-                }
-              }
+              emit32(v, f - lane, tok_base + c, P, epi_tile);
             }
           }
         }

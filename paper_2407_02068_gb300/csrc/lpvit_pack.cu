@@ -136,15 +136,15 @@ plan_kernel(const uint8_t *__restrict__ mask, int n, int k, int b, int32_t *__re
   // 4b. entries: j | (panel mask << 16), then the block index of each panel of the group (or -1)
   for (int g = warp; g < ng; g += PLAN_WARPS) {
     int e_run = gcnt[g];
-    int p_run[8];
+    int p_run[MAX_GROUP_PANELS];
 #pragma unroll
-    for (int p = 0; p < 8; ++p) p_run[p] = (p < gb && g * gb + p < np) ? cnt[g * gb + p] : 0;
+    for (int p = 0; p < MAX_GROUP_PANELS; ++p) p_run[p] = (p < gb && g * gb + p < np) ? cnt[g * gb + p] : 0;
     for (int base = 0; base < kb; base += 32) {
       const int j = base + lane;
-      unsigned bal[8];
+      unsigned bal[MAX_GROUP_PANELS];
       unsigned any = 0;
 #pragma unroll
-      for (int p = 0; p < 8; ++p) {
+      for (int p = 0; p < MAX_GROUP_PANELS; ++p) {
         const int r = g * gb + p;
         const bool keep = p < gb && r < np && j < kb && mask[(int64_t)r * kb + j] != 0;
         bal[p] = __ballot_sync(0xffffffffu, keep);
@@ -154,19 +154,18 @@ plan_kernel(const uint8_t *__restrict__ mask, int n, int k, int b, int32_t *__re
         int32_t *e = entries + (int64_t)(e_run + __popc(any & lt)) * ENTRY_INTS;
         unsigned pm = 0;
 #pragma unroll
-        for (int p = 0; p < 8; ++p) {
+        for (int p = 0; p < MAX_GROUP_PANELS; ++p) {
           const bool keep = (bal[p] >> lane) & 1u;
           pm |= (keep ? 1u : 0u) << p;
           e[1 + p] = keep ? p_run[p] + __popc(bal[p] & lt) : -1;
         }
         e[0] = (int32_t)((unsigned)j | (pm << 16));
-        e[9] = 0;
-        e[10] = 0;
-        e[11] = 0;
+#pragma unroll
+        for (int q = 1 + MAX_GROUP_PANELS; q < ENTRY_INTS; ++q) e[q] = 0;
       }
       e_run += __popc(any);
 #pragma unroll
-      for (int p = 0; p < 8; ++p) p_run[p] += __popc(bal[p]);
+      for (int p = 0; p < MAX_GROUP_PANELS; ++p) p_run[p] += __popc(bal[p]);
     }
   }
 }
