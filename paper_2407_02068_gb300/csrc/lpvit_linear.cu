@@ -7,11 +7,12 @@
 //   warp 0      producer: takes units from a global atomic queue, walks the unit's work-list
 //               entries and, per entry (one block column j), TMA-loads the X tile
 //               [256 tokens x b] and every kept W block of the group at column j.
-//   warp 1      MMA issuer: per entry and per 16-wide k step, one weight-stationary tcgen05 MMA
-//               per present panel, D[panel rows x 256 tokens] += W_blk * X_tile^T, fp32 in TMEM.
-//               The X chunk is loaded once into a B collector buffer (fill) and reused by the
-//               other panels of the entry (use / lastuse).
-//   warps 2..9  epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
+//   warps 1,2   MMA issuers, each owning half of the group's MMA panels: per entry and per 16-wide
+//               k step, one weight-stationary tcgen05 MMA per present panel, D[panel rows x 256
+//               tokens] += W_blk * X_tile^T, fp32 in TMEM. Within an issuer the X chunk is loaded
+//               once into a B collector buffer (fill) and reused by its other panels (use /
+//               lastuse); the two issuers use disjoint collector buffers.
+//   warps 3..10 epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
 //               type, stores of 64-byte row segments; split slices are summed in slice order
 //               by the last slice to finish (ticket), which makes the result deterministic.
 // Accumulators are double-buffered in TMEM (2 x 256 columns) so the epilogue of one unit overlaps
@@ -52,8 +53,10 @@ struct Cfg {
   static_assert(NSTAGES >= 4, "pipeline depth");
 };
 
-constexpr int NUM_THREADS = 320;   // 10 warps
+constexpr int MMA_WARPS = 2;       // MMA issuers, each owning half of the group's MMA panels
+constexpr int FIRST_EPI = 1 + MMA_WARPS;
 constexpr int EPI_WARPS = 8;
+constexpr int NUM_THREADS = 32 * (FIRST_EPI + EPI_WARPS);   // 352
 constexpr int MAX_GROUPS = 512;    // n <= 65536
 
 struct UnitInfo {
@@ -141,9 +144,10 @@ __device__ __forceinline__ void emit32(const float (&v)[32], int f0, int64_t tok
 // All MMAs of one work-list entry, issued by one elected thread: for every 16-wide k step, one
 // weight-stationary MMA per present MMA panel; the X chunk is filled into collector buffer KK by the
 // first panel and reused by the others. Collector variants are compile-time, panel order ascending.
-template <int B, int KK>
+template <int B, int KK, int BUFBASE>
 __device__ __forceinline__ void issue_kstep(uint32_t mm, uint32_t touched, uint32_t st_u32, uint32_t dbase) {
   using C = Cfg<B>;
+  constexpr int BUF = (KK + BUFBASE) % 4;  // collector buffer of this issuer and k step
   const uint64_t bdesc = smem_desc<C::ROW_BYTES>(st_u32 + KK * 32);
   const uint64_t a0 = smem_desc<C::ROW_BYTES>(st_u32 + C::X_BYTES + KK * 32);
   const int p_first = __ffs(mm) - 1;
@@ -151,25 +155,28 @@ __device__ __forceinline__ void issue_kstep(uint32_t mm, uint32_t touched, uint3
   auto acc_of = [&](int p) -> uint32_t { return (KK > 0 || ((touched >> p) & 1u)) ? 1u : 0u; };
   auto adesc = [&](int p) -> uint64_t { return a0 + (uint64_t)((p * C::A_BYTES) >> 4); };
   if (p_first == p_last) {
-    ws_mma<KK, COLL_NONE>(dbase + (uint32_t)(p_first * C::ACC_COLS), adesc(p_first), bdesc, C::IDESC, acc_of(p_first));
+    ws_mma<BUF, COLL_NONE>(dbase + (uint32_t)(p_first * C::ACC_COLS), adesc(p_first), bdesc, C::IDESC, acc_of(p_first));
     return;
   }
-  ws_mma<KK, COLL_FILL>(dbase + (uint32_t)(p_first * C::ACC_COLS), adesc(p_first), bdesc, C::IDESC, acc_of(p_first));
+  ws_mma<BUF, COLL_FILL>(dbase + (uint32_t)(p_first * C::ACC_COLS), adesc(p_first), bdesc, C::IDESC, acc_of(p_first));
   uint32_t mid = mm & ~(1u << p_first) & ~(1u << p_last);
   while (mid) {
     const int p = __ffs(mid) - 1;
     mid &= mid - 1u;
-    ws_mma<KK, COLL_USE>(dbase + (uint32_t)(p * C::ACC_COLS), adesc(p), bdesc, C::IDESC, acc_of(p));
+    ws_mma<BUF, COLL_USE>(dbase + (uint32_t)(p * C::ACC_COLS), adesc(p), bdesc, C::IDESC, acc_of(p));
   }
-  ws_mma<KK, COLL_LAST>(dbase + (uint32_t)(p_last * C::ACC_COLS), adesc(p_last), bdesc, C::IDESC, acc_of(p_last));
+  ws_mma<BUF, COLL_LAST>(dbase + (uint32_t)(p_last * C::ACC_COLS), adesc(p_last), bdesc, C::IDESC, acc_of(p_last));
 }
 
-template <int B>
+// BUFBASE separates the collector buffers of the two issuers (b0/b1 and b2/b3). With 64-wide
+// blocks each issuer owns one panel, so its MMAs never use a collector buffer.
+template <int B, int BUFBASE>
 __device__ __forceinline__ void issue_entry(uint32_t mm, uint32_t touched, uint32_t st_u32, uint32_t dbase) {
-  issue_kstep<B, 0>(mm, touched, st_u32, dbase);
-  if constexpr (Cfg<B>::KSTEPS > 1) issue_kstep<B, 1>(mm, touched, st_u32, dbase);
-  if constexpr (Cfg<B>::KSTEPS > 2) issue_kstep<B, 2>(mm, touched, st_u32, dbase);
-  if constexpr (Cfg<B>::KSTEPS > 3) issue_kstep<B, 3>(mm, touched, st_u32, dbase);
+  static_assert(Cfg<B>::KSTEPS <= 2 || Cfg<B>::G <= MMA_WARPS, "collector buffers per issuer");
+  issue_kstep<B, 0, BUFBASE>(mm, touched, st_u32, dbase);
+  if constexpr (Cfg<B>::KSTEPS > 1) issue_kstep<B, 1, BUFBASE>(mm, touched, st_u32, dbase);
+  if constexpr (Cfg<B>::KSTEPS > 2) issue_kstep<B, 2, BUFBASE>(mm, touched, st_u32, dbase);
+  if constexpr (Cfg<B>::KSTEPS > 3) issue_kstep<B, 3, BUFBASE>(mm, touched, st_u32, dbase);
 }
 
 template <int B>
@@ -212,17 +219,17 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
   if (tid == 0) {
     for (int s = 0; s < L::NS; ++s) {
       mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), 1);
+      mbar_init(empty_bar(s), MMA_WARPS);
     }
     for (int b = 0; b < 2; ++b) {
-      mbar_init(accf_bar(b), 1);
+      mbar_init(accf_bar(b), MMA_WARPS);
       mbar_init(acce_bar(b), EPI_WARPS);
     }
     for (int u = 0; u < L::UR; ++u) {
       mbar_init(unitf_bar(u), 1);
       mbar_init(unite_bar(u), EPI_WARPS);
     }
-    mbar_init(drain_bar, 1);
+    mbar_init(drain_bar, MMA_WARPS);
     mbar_init(episync_bar, EPI_WARPS);
     *abort_flag = 0;
     *last_flag = 0;
@@ -412,8 +419,13 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     const uint32_t first = it > (uint32_t)L::NS ? it - L::NS : 0u;
     for (uint32_t i = first; i < it; ++i)
       if (!mbar_wait(full_bar(i % L::NS), (i / L::NS) & 1u, never_flag, tmo)) break;
-  } else if (warp == 1) {
-    // ============================================================== MMA issuer
+  } else if (warp < FIRST_EPI) {
+    // ============================================================== MMA issuers
+    // Warp 1 + w owns MMA panels [w G/2, (w + 1) G/2) of the group: two independent issuers keep
+    // the tensor pipe fed while each one waits, branches and commits. Each arrives on a stage's
+    // empty barrier once per entry (a commit when it issued MMAs there).
+    const int mw = warp - 1;
+    const uint32_t own = ((1u << (C::G / MMA_WARPS)) - 1u) << (mw * (C::G / MMA_WARPS));
     uint32_t it = 0, ui = 0;
     bool ok = true;
     while (ok) {
@@ -447,17 +459,23 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
 #pragma unroll
         for (int p = 0; p < C::G; ++p) mm |= ((pm >> (p * C::PPM)) & ((1u << C::PPM) - 1u)) ? (1u << p) : 0u;
         const uint32_t st_u32 = smem_base + stage * C::STAGE_BYTES;
-        if (elect_one()) {
-          issue_entry<B>(mm, touched, st_u32, dbase);
-          tc_commit(empty_bar(stage));
+        const uint32_t mine = mm & own;
+        if (mine) {
+          if (elect_one()) {
+            if (mw == 0) issue_entry<B, 0>(mine, touched, st_u32, dbase);
+            else issue_entry<B, 2>(mine, touched, st_u32, dbase);
+            tc_commit(empty_bar(stage));
+          }
+        } else {
+          if (elect_one()) mbar_arrive(empty_bar(stage));
         }
         __syncwarp();
-        touched |= mm;
+        touched |= mine;
         ++it;
       }
       if (!ok) break;
       if (elect_one()) {
-        if (inf.e1 > inf.e0) tc_commit(accf_bar(buf));
+        if (touched) tc_commit(accf_bar(buf));
         else mbar_arrive(accf_bar(buf));
       }
       __syncwarp();
@@ -470,7 +488,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     if (!mbar_wait(drain_bar, 0, never_flag, tmo) && lane == 0) atomicOr(&P.ctl->err, ERR_DRAIN);
   } else {
     // ============================================================== epilogue
-    const int ew = warp - 2;       // 0..7
+    const int ew = warp - FIRST_EPI;  // 0..7
     const int q = warp & 3;        // TMEM lane quarter this warp may access
     const int h = ew >> 2;         // column half
     const int r = (C::MP == 32) ? lane : 32 * (q & 1) + lane;          // feature row in the MMA panel
