@@ -137,6 +137,18 @@ lpvit_status lpvit_bsr_linear_noalloc(const lpvit_bsr *bsr, const void *X, int64
  * stopped early and its output is incomplete) or LPVIT_ERR_CUDA. */
 lpvit_status lpvit_check(void *workspace, void *stream);
 
+/* Diagnostic of the failure path; it has no counterpart in the paper. Launches, on `stream`, a
+ * kernel whose one thread waits on an mbarrier that nothing arrives on, with the bounded wait every
+ * role of the GEMM uses: the wait gives up after limit_ns, or after abort_after_ns when that is
+ * nonzero (a second thread then raises the CTA's abort flag, as a failing role of the GEMM does).
+ * The timeout is recorded in `workspace` (a zero-filled workspace as for lpvit_bsr_linear, 256-byte
+ * aligned): the error word, which lpvit_check() then reports as LPVIT_ERR_TIMEOUT and clears, and the
+ * microseconds waited, in the 32-bit word at byte offset 12. Nothing else is in flight, so the kernel
+ * ends cleanly and the context stays usable.
+ * Errors: LPVIT_ERR_INVALID_ARG (null or misaligned workspace, limit_ns 0 or above 10 s,
+ * abort_after_ns >= limit_ns), LPVIT_ERR_CUDA (launch failure). */
+lpvit_status lpvit_selftest_wait(void *workspace, uint64_t limit_ns, uint64_t abort_after_ns, void *stream);
+
 /* Static English description of a status code. */
 const char *lpvit_status_string(lpvit_status status);
 

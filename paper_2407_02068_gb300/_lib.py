@@ -22,7 +22,8 @@ LPVIT_BF16 = 0
 LPVIT_F32 = 1
 
 EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_workspace_bytes", "lpvit_bsr_linear",
-           "lpvit_bsr_linear_gelu", "lpvit_bsr_linear_noalloc", "lpvit_check", "lpvit_status_string")
+           "lpvit_bsr_linear_gelu", "lpvit_bsr_linear_noalloc", "lpvit_check", "lpvit_status_string",
+           "lpvit_selftest_wait")
 LPVIT_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 
@@ -72,6 +73,8 @@ def load(path: str | None = None):
         lib.lpvit_bsr_linear_noalloc.argtypes = [BP, V, I64, I64, V, V, I64, ctypes.c_int, ctypes.c_int, V]
         lib.lpvit_check.restype = ctypes.c_int
         lib.lpvit_check.argtypes = [V, V]
+        lib.lpvit_selftest_wait.restype = ctypes.c_int
+        lib.lpvit_selftest_wait.argtypes = [V, ctypes.c_uint64, ctypes.c_uint64, V]
         lib.lpvit_status_string.restype = ctypes.c_char_p
         lib.lpvit_status_string.argtypes = [ctypes.c_int]
         _lib = lib
@@ -116,6 +119,11 @@ def lpvit_bsr_linear_noalloc(bsr, X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, 
 
 def lpvit_check(ws_ptr: int, stream: int) -> int:
     return load().lpvit_check(ws_ptr, stream)
+
+
+def lpvit_selftest_wait(ws_ptr: int, limit_ns: int, abort_after_ns: int, stream: int) -> int:
+    """Force the bounded device wait to run out (diagnostic of the failure path)."""
+    return load().lpvit_selftest_wait(ws_ptr, limit_ns, abort_after_ns, stream)
 
 
 def lpvit_status_string(status: int) -> str:

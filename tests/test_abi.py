@@ -58,3 +58,9 @@ def test_bad_arguments_are_rejected_without_a_gpu(lib):
     assert lib.lpvit_bsr_linear(bsr, fake.value, 4, 388, None, 0x200000, 1152, 0, 0x100000, 1 << 20, None) == \
         lib.LPVIT_ERR_INVALID_ARG
     assert lib.lpvit_check(None, None) == lib.LPVIT_ERR_INVALID_ARG
+    # the wait self-test validates before launching anything
+    assert lib.lpvit_selftest_wait(0, 10 ** 6, 0, None) == lib.LPVIT_ERR_INVALID_ARG          # no workspace
+    assert lib.lpvit_selftest_wait(0x100010, 10 ** 6, 0, None) == lib.LPVIT_ERR_INVALID_ARG   # misaligned
+    assert lib.lpvit_selftest_wait(0x100000, 0, 0, None) == lib.LPVIT_ERR_INVALID_ARG         # no limit
+    assert lib.lpvit_selftest_wait(0x100000, 11 * 10 ** 9, 0, None) == lib.LPVIT_ERR_INVALID_ARG  # > 10 s
+    assert lib.lpvit_selftest_wait(0x100000, 10 ** 6, 10 ** 6, None) == lib.LPVIT_ERR_INVALID_ARG  # abort >= limit
