@@ -65,7 +65,6 @@ enum ErrBits : unsigned int {
   ERR_DRAIN = 1u << 7,
   ERR_SCHED_OVERFLOW = 1u << 8,
   ERR_BAD_SCHED = 1u << 9,
-  ERR_SELFTEST_WAIT = 1u << 10,  // lpvit_selftest_wait: its wait ran out as intended
 };
 
 // Launchers (host side, defined next to their kernels).
