@@ -12,7 +12,7 @@
 //               tokens] += W_blk * X_tile^T, fp32 in TMEM. Within an issuer the X chunk is loaded
 //               once into a B collector buffer (fill) and reused by its other panels (use /
 //               lastuse); the two issuers use disjoint collector buffers.
-//   warps 3..10 epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
+//   warps 3..14 epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
 //               type, stores of 64-byte row segments; split slices are summed in slice order
 //               by the last slice to finish (ticket), which makes the result deterministic.
 // Accumulators are double-buffered in TMEM (2 x 256 columns) so the epilogue of one unit overlaps
@@ -55,7 +55,8 @@ struct Cfg {
 
 constexpr int MMA_WARPS = 2;       // MMA issuers, each owning half of the group's MMA panels
 constexpr int FIRST_EPI = 1 + MMA_WARPS;
-constexpr int EPI_WARPS = 8;
+constexpr int EPI_WARPS = 12;      // three per TMEM lane quarter
+static_assert(EPI_WARPS % 4 == 0, "epilogue warps come in whole sets of four lane quarters");
 constexpr int NUM_THREADS = 32 * (FIRST_EPI + EPI_WARPS);   // 352
 constexpr int MAX_GROUPS = 512;    // n <= 65536
 
@@ -78,16 +79,17 @@ struct Smem {
   static constexpr int MISC_OFF = SLICE_OFF + 4 * (MAX_GROUPS + 1);
   static constexpr int EPI_OFF = (MISC_OFF + 64 + 127) / 128 * 128;
   static constexpr int EPI_TILE = 32 * 80;  // per epilogue warp: 32 token rows x 32 bf16, rows padded to 80 B
-  static constexpr int END = EPI_OFF + 8 * EPI_TILE;
+  static constexpr int END = EPI_OFF + EPI_WARPS * EPI_TILE;
   static constexpr int BYTES = END + 1024;  // + alignment slack for the dynamic smem base
+  static_assert(BYTES <= 227 * 1024, "shared memory per CTA");
 };
 
-// Epilogue of one 32 x 32 block held by a warp: v[i] = accumulator of token tok_base + i for feature
-// f0 + lane. Adds the bias, applies GELU, rounds, and stores rows [tok_base, min(tok_base + 32, m)).
+// Epilogue of one 32 x 32 block held by a warp: y[i] = accumulator of token tok_base + i for feature
+// f0 + lane (turned into the output in place). Adds the bias, applies GELU, rounds, and stores rows [tok_base, min(tok_base + 32, m)).
 // bf16 output is staged through this warp's shared tile (rows padded to 80 bytes, conflict-free) so
 // that every token row leaves as 16-byte vector stores; fp32 output is stored directly (a warp
 // writes 128 contiguous bytes per token).
-__device__ __forceinline__ void emit32(const float (&v)[32], int f0, int64_t tok_base, const LinearParams &P,
+__device__ __forceinline__ void emit32(float (&y)[32], int f0, int64_t tok_base, const LinearParams &P,
                                        uint8_t *tile) {
   const int lane = threadIdx.x & 31;
   const int f = f0 + lane;
@@ -95,17 +97,16 @@ __device__ __forceinline__ void emit32(const float (&v)[32], int f0, int64_t tok
   const float bb = (P.bias != nullptr && fvalid) ? __ldg(P.bias + f) : 0.f;
   const int64_t left = P.m - tok_base;
   const int rows = left >= 32 ? 32 : (left > 0 ? (int)left : 0);
-  float y[32];
   if (P.gelu) {
     const float kInvSqrt2 = 0.70710678118654752440f;
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
-      const float t = v[i] + bb;
+      const float t = y[i] + bb;
       y[i] = 0.5f * t * (1.f + erff(t * kInvSqrt2));
     }
   } else {
 #pragma unroll
-    for (int i = 0; i < 32; ++i) y[i] = v[i] + bb;
+    for (int i = 0; i < 32; ++i) y[i] += bb;
   }
   if (P.y_f32) {
     float *dst = static_cast<float *>(P.Y) + tok_base * P.ldy + f;
@@ -488,12 +489,14 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     if (!mbar_wait(drain_bar, 0, never_flag, tmo) && lane == 0) atomicOr(&P.ctl->err, ERR_DRAIN);
   } else {
     // ============================================================== epilogue
-    const int ew = warp - FIRST_EPI;  // 0..7
-    const int q = warp & 3;        // TMEM lane quarter this warp may access
-    const int h = ew >> 2;         // column half
-    const int r = (C::MP == 32) ? lane : 32 * (q & 1) + lane;          // feature row in the MMA panel
-    const int tok0 = (C::MP == 32) ? 64 * q + 32 * h : 128 * (q >> 1) + 64 * h;  // first token of this thread
-    const int col0 = (C::MP == 32) ? 32 * h : 64 * h;                  // first column in the accumulator
+    // A unit's accumulators form, per TMEM lane quarter, 2 column halves x G panels x CPP chunks =
+    // 8 blocks of 32 tokens x 32 features; the quarter's EPI_WARPS / 4 warps take them in turn.
+    const int ew = warp - FIRST_EPI;             // 0 .. EPI_WARPS - 1
+    const int q = warp & 3;                      // TMEM lane quarter this warp may access
+    const int wq = ew >> 2;                      // this warp's turn within its quarter
+    constexpr int CPP = C::VPT / 32;             // 32-column chunks per panel and column half
+    constexpr int QBLK = 2 * C::G * CPP;         // blocks per lane quarter
+    const int r = (C::MP == 32) ? lane : 32 * (q & 1) + lane;  // feature row in the MMA panel
     uint32_t ui = 0, sync_phase = 0;
     uint8_t *epi_tile = smem + L::EPI_OFF + ew * L::EPI_TILE;
     while (true) {
@@ -511,31 +514,29 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       }
       tc_fence_after();
       const bool split = inf.nsl > 1;
-      const int64_t tok_base = (int64_t)inf.tt * C::TT + tok0;
       float *part = nullptr;
       if (split)
         part = P.partials + ((int64_t)inf.tt * total_slices + slice_ptr[inf.g] + inf.s) * (int64_t)(C::TT * 128);
 #pragma unroll 1
-      for (int p = 0; p < C::G; ++p) {
+      for (int j = wq; j < QBLK; j += EPI_WARPS / 4) {
+        const int h = j / (C::G * CPP), p = (j / CPP) % C::G, c = 32 * (j % CPP);
+        const int tok0 = (C::MP == 32) ? 64 * q + 32 * h : 128 * (q >> 1) + 64 * h;  // first token of the block
+        const int col0 = (C::MP == 32) ? 32 * h : 64 * h;                              // its accumulator column
         const int f = inf.g * GROUP_FEATURES + p * C::MP + r;
         const uint32_t taddr = tmem_base + ((uint32_t)(32 * q) << 16) + buf * C::BUF_COLS + p * C::ACC_COLS + col0;
-        const bool has = (inf.touched >> p) & 1;
+        float v[32];
+        if ((inf.touched >> p) & 1) {
+          tmem_ld32(taddr + c, v);
+        } else {
 #pragma unroll
-        for (int c = 0; c < C::VPT; c += 32) {
-          float v[32];
-          if (has) {
-            tmem_ld32(taddr + c, v);
-          } else {
+          for (int i = 0; i < 32; ++i) v[i] = 0.f;
+        }
+        if (split) {
+          float4 *dst = reinterpret_cast<float4 *>(part + (int64_t)(p * C::MP + r) * C::TT + tok0 + c);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0.f;
-          }
-          if (split) {
-            float4 *dst = reinterpret_cast<float4 *>(part + (int64_t)(p * C::MP + r) * C::TT + tok0 + c);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-          } else {
-            emit32(v, f - lane, tok_base + c, P, epi_tile);
-          }
+          for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        } else {
+          emit32(v, f - lane, (int64_t)inf.tt * C::TT + tok0 + c, P, epi_tile);
         }
       }
       // accumulator buffer and unit slot are free again
@@ -575,24 +576,23 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
           const float *base0 =
               P.partials + ((int64_t)inf.tt * total_slices + slice_ptr[inf.g]) * (int64_t)(C::TT * 128);
 #pragma unroll 1
-          for (int p = 0; p < C::G; ++p) {
+          for (int j = wq; j < QBLK; j += EPI_WARPS / 4) {
+            const int h = j / (C::G * CPP), p = (j / CPP) % C::G, c = 32 * (j % CPP);
+            const int tok0 = (C::MP == 32) ? 64 * q + 32 * h : 128 * (q >> 1) + 64 * h;
             const int f = inf.g * GROUP_FEATURES + p * C::MP + r;
-#pragma unroll 1
-            for (int c = 0; c < C::VPT; c += 32) {
-              float v[32];
+            float v[32];
 #pragma unroll
-              for (int i = 0; i < 32; ++i) v[i] = 0.f;
-              for (int s2 = 0; s2 < inf.nsl; ++s2) {
-                const float4 *src = reinterpret_cast<const float4 *>(
-                    base0 + (int64_t)s2 * (C::TT * 128) + (int64_t)(p * C::MP + r) * C::TT + tok0 + c);
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+            for (int s2 = 0; s2 < inf.nsl; ++s2) {
+              const float4 *src = reinterpret_cast<const float4 *>(
+                  base0 + (int64_t)s2 * (C::TT * 128) + (int64_t)(p * C::MP + r) * C::TT + tok0 + c);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                  const float4 t = __ldcg(src + i);
-                  v[4 * i] += t.x; v[4 * i + 1] += t.y; v[4 * i + 2] += t.z; v[4 * i + 3] += t.w;
-                }
+              for (int i = 0; i < 8; ++i) {
+                const float4 t = __ldcg(src + i);
+                v[4 * i] += t.x; v[4 * i + 1] += t.y; v[4 * i + 2] += t.z; v[4 * i + 3] += t.w;
               }
-              emit32(v, f - lane, tok_base + c, P, epi_tile);
             }
+            emit32(v, f - lane, (int64_t)inf.tt * C::TT + tok0 + c, P, epi_tile);
           }
         }
       }

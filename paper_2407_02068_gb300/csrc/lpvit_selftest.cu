@@ -12,7 +12,7 @@
 namespace lpvit {
 
 constexpr uint64_t SELFTEST_MAX_NS = 10000000000ull;  // 10 s
-constexpr unsigned int ERR_SELFTEST_WAIT = 1u << 10;   // next to the GEMM's ErrBits, none of them
+constexpr unsigned int ERR_SELFTEST_WAIT = 1u << 10;   // a bit the GEMM error bits leave free
 
 __global__ void wait_selftest_kernel(Control *ctl, uint64_t limit_ns, uint64_t abort_after_ns) {
   __shared__ __align__(8) uint64_t bar;
