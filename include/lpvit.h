@@ -85,6 +85,18 @@ size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t b);
 lpvit_status lpvit_pack_bsr(const void *W, const uint8_t *mask, lpvit_bsr *bsr, int32_t *nnzb_host,
                             void *stream);
 
+/* lpvit_pack_bsr for `count` weights at once, asynchronously on `stream`: W[i] and mask[i] (host
+ * arrays of device pointers) are packed into bsr[i] (a host array of count descriptors, set up as
+ * for lpvit_pack_bsr). Every job is checked as lpvit_pack_bsr checks its arguments before anything
+ * is launched; the first failing check is returned and nothing runs. The jobs travel in the launch
+ * parameters (96 per launch), so the call allocates nothing: all plans run in one launch, one CTA
+ * per weight, then all block copies in one more. Results are bit-identical to count calls of
+ * lpvit_pack_bsr. There is no kept-block count output; a capacity overflow is reported as for
+ * lpvit_pack_bsr (the work list is marked invalid and lpvit_check reports it after a linear).
+ * Errors: as lpvit_pack_bsr, and LPVIT_ERR_INVALID_ARG for count < 0 or null arrays. */
+lpvit_status lpvit_pack_bsr_many(int32_t count, const void *const *W, const uint8_t *const *mask, lpvit_bsr *bsr,
+                                 void *stream);
+
 /* Bytes of device workspace lpvit_bsr_linear[_gelu] needs for m tokens. The workspace holds
  * scheduler counters, the device error word and, for small m, fp32 partial sums of split
  * work units. It must be zero-filled once before its first use (cudaMemset); every call

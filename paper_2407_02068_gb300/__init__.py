@@ -5,6 +5,7 @@ the layer becomes a block-sparse matmul whose work is proportional to the kept b
 (Sec. 3.3). This package wraps the C library ``liblpvit.so`` (include/lpvit.h):
 
 * ``pack_bsr(W, mask, b)``  -- mask -> BSR pack + work list, on the GPU
+* ``pack_bsr_many_into(ws, Ws, masks)`` -- the same for a list of weights in two launches
 * ``bsr_linear(w, X, bias, gelu=...)`` -- Y = act(X (W (.) M)^T + bias)
 
 PyTorch provides device memory and streams only; every step runs in the library's kernels.
@@ -17,8 +18,8 @@ import torch
 
 from . import _lib
 
-__all__ = ["BsrWeight", "alloc_bsr", "pack_bsr", "pack_bsr_into", "workspace_for", "bsr_linear", "check",
-           "LpvitError"]
+__all__ = ["BsrWeight", "alloc_bsr", "pack_bsr", "pack_bsr_into", "pack_bsr_many_into", "workspace_for",
+           "bsr_linear", "check", "LpvitError"]
 
 LpvitError = _lib.LpvitError
 
@@ -71,6 +72,23 @@ def pack_bsr_into(w: BsrWeight, W: torch.Tensor, mask: torch.Tensor, count: bool
         raise LpvitError(st, "lpvit_pack_bsr")
     w.nnzb = nnzb
     return w
+
+
+def pack_bsr_many_into(ws: list, Ws: list, masks: list, stream=None) -> list:
+    """Pack Ws[i] under masks[i] into ws[i] for all i in two launches (lpvit_pack_bsr_many);
+    asynchronous. Tensors as for pack_bsr_into."""
+    if not (len(ws) == len(Ws) == len(masks)):
+        raise ValueError("ws, Ws and masks must have the same length")
+    for W, mask in zip(Ws, masks):
+        if W.dtype != torch.bfloat16 or not W.is_cuda or W.dim() != 2 or not W.is_contiguous():
+            raise ValueError("every W must be a contiguous 2-D bf16 CUDA tensor")
+        if mask.dtype != torch.uint8 or not mask.is_contiguous() or mask.device != W.device:
+            raise ValueError("every mask must be a contiguous uint8 tensor on its W's device")
+    st = _lib.lpvit_pack_bsr_many([W.data_ptr() for W in Ws], [m.data_ptr() for m in masks],
+                                  [w.struct() for w in ws], _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_pack_bsr_many")
+    return ws
 
 
 def pack_bsr(W: torch.Tensor, mask: torch.Tensor, b: int, capacity: int | None = None, count: bool = False,

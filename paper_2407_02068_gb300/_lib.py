@@ -23,7 +23,7 @@ LPVIT_F32 = 1
 
 EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_workspace_bytes", "lpvit_bsr_linear",
            "lpvit_bsr_linear_gelu", "lpvit_bsr_linear_noalloc", "lpvit_check", "lpvit_status_string",
-           "lpvit_selftest_wait")
+           "lpvit_selftest_wait", "lpvit_pack_bsr_many")
 LPVIT_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 
@@ -63,6 +63,8 @@ def load(path: str | None = None):
         lib.lpvit_sched_bytes.argtypes = [I32, I32, I32]
         lib.lpvit_pack_bsr.restype = ctypes.c_int
         lib.lpvit_pack_bsr.argtypes = [V, V, BP, ctypes.POINTER(I32), V]
+        lib.lpvit_pack_bsr_many.restype = ctypes.c_int
+        lib.lpvit_pack_bsr_many.argtypes = [I32, ctypes.POINTER(V), ctypes.POINTER(V), BP, V]
         lib.lpvit_workspace_bytes.restype = SZ
         lib.lpvit_workspace_bytes.argtypes = [BP, I64]
         for name in ("lpvit_bsr_linear", "lpvit_bsr_linear_gelu"):
@@ -95,6 +97,19 @@ def lpvit_pack_bsr(W_ptr: int, mask_ptr: int, bsr: lpvit_bsr, want_count: bool, 
     st = load().lpvit_pack_bsr(W_ptr, mask_ptr, ctypes.byref(bsr), ctypes.byref(cnt) if want_count else None,
                                stream)
     return st, (cnt.value if want_count else None)
+
+
+def lpvit_pack_bsr_many(W_ptrs, mask_ptrs, bsrs, stream: int) -> int:
+    """Pack len(bsrs) weights in two launches. ``bsrs``: a ctypes array of lpvit_bsr (or a list)."""
+    n = len(bsrs)
+    if not isinstance(bsrs, ctypes.Array):
+        arr = (lpvit_bsr * n)()
+        for i, b in enumerate(bsrs):
+            arr[i] = b
+        bsrs = arr
+    Wa = (ctypes.c_void_p * n)(*W_ptrs)
+    Ma = (ctypes.c_void_p * n)(*mask_ptrs)
+    return load().lpvit_pack_bsr_many(n, Wa, Ma, bsrs, stream)
 
 
 def lpvit_workspace_bytes(bsr: lpvit_bsr, m: int) -> int:

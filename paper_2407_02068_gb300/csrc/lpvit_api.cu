@@ -3,6 +3,7 @@
 #include <cstdint>
 #include <cstring>
 #include <mutex>
+#include <vector>
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -191,6 +192,21 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
                                    static_cast<cudaStream_t>(stream)));
 }
 
+// The checks lpvit_pack_bsr applies to one weight.
+lpvit_status check_pack_args(const void *W, const uint8_t *mask, const lpvit_bsr *bsr) {
+  if (!bsr) return LPVIT_ERR_INVALID_ARG;
+  const int n = bsr->n, k = bsr->k, b = bsr->b;
+  if (!valid_b(b)) return LPVIT_ERR_UNSUPPORTED;
+  if (!shape_ok(n, k, b)) return LPVIT_ERR_INVALID_ARG;
+  if (!W || !mask || !bsr->row_ptr || !bsr->sched || bsr->nnzb_capacity < 0) return LPVIT_ERR_INVALID_ARG;
+  if (bsr->nnzb_capacity > 0 && (!bsr->col_idx || !bsr->blocks)) return LPVIT_ERR_INVALID_ARG;
+  if (!aligned(W, 16) || (bsr->blocks && !aligned(bsr->blocks, 16)) || !aligned(bsr->sched, 16) ||
+      !aligned(bsr->row_ptr, 4) || (bsr->col_idx && !aligned(bsr->col_idx, 4)))
+    return LPVIT_ERR_INVALID_ARG;
+  if (bsr->sched_bytes < lpvit_sched_bytes(n, k, b)) return LPVIT_ERR_WORKSPACE;
+  return LPVIT_OK;
+}
+
 }  // namespace
 }  // namespace lpvit
 
@@ -204,17 +220,11 @@ size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t b) {
   return 4 * (size_t)sched_entries_offset_ints(ng) + 4 * (size_t)ENTRY_INTS * ng * (k / b);
 }
 
+
 lpvit_status lpvit_pack_bsr(const void *W, const uint8_t *mask, lpvit_bsr *bsr, int32_t *nnzb_host, void *stream) {
-  if (!bsr) return LPVIT_ERR_INVALID_ARG;
+  const lpvit_status chk = check_pack_args(W, mask, bsr);
+  if (chk != LPVIT_OK) return chk;
   const int n = bsr->n, k = bsr->k, b = bsr->b;
-  if (!valid_b(b)) return LPVIT_ERR_UNSUPPORTED;
-  if (!shape_ok(n, k, b)) return LPVIT_ERR_INVALID_ARG;
-  if (!W || !mask || !bsr->row_ptr || !bsr->sched || bsr->nnzb_capacity < 0) return LPVIT_ERR_INVALID_ARG;
-  if (bsr->nnzb_capacity > 0 && (!bsr->col_idx || !bsr->blocks)) return LPVIT_ERR_INVALID_ARG;
-  if (!aligned(W, 16) || (bsr->blocks && !aligned(bsr->blocks, 16)) || !aligned(bsr->sched, 16) ||
-      !aligned(bsr->row_ptr, 4) || (bsr->col_idx && !aligned(bsr->col_idx, 4)))
-    return LPVIT_ERR_INVALID_ARG;
-  if (bsr->sched_bytes < lpvit_sched_bytes(n, k, b)) return LPVIT_ERR_WORKSPACE;
   int sms = 0;
   lpvit_status st = LPVIT_OK;
   if (!device_info(&sms, &st)) return st;
@@ -231,6 +241,35 @@ lpvit_status lpvit_pack_bsr(const void *W, const uint8_t *mask, lpvit_bsr *bsr, 
     if (v > bsr->nnzb_capacity) return LPVIT_ERR_WORKSPACE;
   }
   return LPVIT_OK;
+}
+
+lpvit_status lpvit_pack_bsr_many(int32_t count, const void *const *W, const uint8_t *const *mask, lpvit_bsr *bsr,
+                                 void *stream) {
+  if (count < 0) return LPVIT_ERR_INVALID_ARG;
+  if (count == 0) return LPVIT_OK;
+  if (!W || !mask || !bsr) return LPVIT_ERR_INVALID_ARG;
+  for (int32_t i = 0; i < count; ++i) {
+    const lpvit_status chk = check_pack_args(W[i], mask[i], &bsr[i]);
+    if (chk != LPVIT_OK) return chk;
+  }
+  int sms = 0;
+  lpvit_status st = LPVIT_OK;
+  if (!device_info(&sms, &st)) return st;
+  std::vector<PackJob> jobs((size_t)count);
+  for (int32_t i = 0; i < count; ++i) {
+    PackJob &j = jobs[(size_t)i];
+    j.W = static_cast<const uint16_t *>(W[i]);
+    j.mask = mask[i];
+    j.row_ptr = bsr[i].row_ptr;
+    j.col_idx = bsr[i].col_idx;
+    j.blocks = static_cast<uint16_t *>(bsr[i].blocks);
+    j.sched = static_cast<int32_t *>(bsr[i].sched);
+    j.n = bsr[i].n;
+    j.k = bsr[i].k;
+    j.b = bsr[i].b;
+    j.cap = bsr[i].nnzb_capacity;
+  }
+  return cuda_status(launch_pack_many(jobs.data(), count, sms, static_cast<cudaStream_t>(stream)));
 }
 
 size_t lpvit_workspace_bytes(const lpvit_bsr *bsr, int64_t m) {

@@ -70,6 +70,23 @@ enum ErrBits : unsigned int {
 // Launchers (host side, defined next to their kernels).
 cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int b, int32_t *row_ptr, int32_t *col_idx,
                         int cap, void *blocks, int32_t *sched, int num_sms, cudaStream_t s);
+
+// One weight of a batched pack; the whole table travels in the kernel parameters.
+struct PackJob {
+  const uint16_t *W;
+  const uint8_t *mask;
+  int32_t *row_ptr;
+  int32_t *col_idx;
+  uint16_t *blocks;
+  int32_t *sched;
+  int n, k, b, cap;
+};
+constexpr int PACK_MAX_JOBS = 96;  // jobs per launch (6 KB of parameters)
+struct PackJobs {
+  int count;
+  PackJob job[PACK_MAX_JOBS];
+};
+cudaError_t launch_pack_many(const PackJob *jobs, int count, int num_sms, cudaStream_t s);
 cudaError_t launch_linear(int b, const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
                           cudaStream_t s);
 

@@ -58,10 +58,10 @@ __device__ int block_exclusive_scan(int *v, int count, int *warp_tot) {
   return total;
 }
 
-__global__ void __launch_bounds__(PLAN_THREADS, 1)
-plan_kernel(const uint8_t *__restrict__ mask, int n, int k, int b, int32_t *__restrict__ row_ptr,
-            int32_t *__restrict__ col_idx, int cap, int32_t *__restrict__ sched) {
-  extern __shared__ int plan_smem[];
+// The plan of one weight, computed by one CTA of PLAN_THREADS threads (plan_smem: plan_smem_bytes).
+__device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int n, int k, int b,
+                                          int32_t *__restrict__ row_ptr, int32_t *__restrict__ col_idx, int cap,
+                                          int32_t *__restrict__ sched, int *plan_smem) {
   const int np = n / b, kb = k / b;
   const int gb = GROUP_FEATURES / b;  // row panels per group
   const int ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
@@ -170,14 +170,29 @@ plan_kernel(const uint8_t *__restrict__ mask, int n, int k, int b, int32_t *__re
   }
 }
 
-__global__ void __launch_bounds__(128)
-copy_blocks_kernel(const uint16_t *__restrict__ W, int n, int k, int b, const int32_t *__restrict__ row_ptr,
-                   const int32_t *__restrict__ col_idx, int cap, uint16_t *__restrict__ blocks) {
+__global__ void __launch_bounds__(PLAN_THREADS, 1)
+plan_kernel(const uint8_t *__restrict__ mask, int n, int k, int b, int32_t *__restrict__ row_ptr,
+            int32_t *__restrict__ col_idx, int cap, int32_t *__restrict__ sched) {
+  extern __shared__ int plan_smem[];
+  plan_body(mask, n, k, b, row_ptr, col_idx, cap, sched, plan_smem);
+}
+
+// Several weights at once: CTA j plans job j.
+__global__ void __launch_bounds__(PLAN_THREADS, 1) plan_many_kernel(const __grid_constant__ PackJobs J) {
+  extern __shared__ int plan_smem[];
+  const PackJob &w = J.job[blockIdx.x];
+  plan_body(w.mask, w.n, w.k, w.b, w.row_ptr, w.col_idx, w.cap, w.sched, plan_smem);
+}
+
+// Kept blocks t = cta, cta + ncta, ... of one weight.
+__device__ __forceinline__ void copy_body(const uint16_t *__restrict__ W, int n, int k, int b,
+                                          const int32_t *__restrict__ row_ptr, const int32_t *__restrict__ col_idx,
+                                          int cap, uint16_t *__restrict__ blocks, int cta, int ncta) {
   const int np = n / b;
   const int nnzb = min(row_ptr[np], cap);
   const int vec_per_row = b / 8;  // 16-byte vectors per block row
   const int vecs = b * vec_per_row;
-  for (int t = blockIdx.x; t < nnzb; t += gridDim.x) {
+  for (int t = cta; t < nnzb; t += ncta) {
     int lo = 0, hi = np - 1;  // largest r with row_ptr[r] <= t (that panel holds block t)
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
@@ -191,6 +206,20 @@ copy_blocks_kernel(const uint16_t *__restrict__ W, int n, int k, int b, const in
       int4 *dst = reinterpret_cast<int4 *>(blocks + ((int64_t)t * b + c) * b + cv * 8);
       *dst = __ldg(src);
     }
+  }
+}
+
+__global__ void __launch_bounds__(128)
+copy_blocks_kernel(const uint16_t *__restrict__ W, int n, int k, int b, const int32_t *__restrict__ row_ptr,
+                   const int32_t *__restrict__ col_idx, int cap, uint16_t *__restrict__ blocks) {
+  copy_body(W, n, k, b, row_ptr, col_idx, cap, blocks, blockIdx.x, gridDim.x);
+}
+
+// Several weights at once: every CTA takes its share of every job's kept blocks.
+__global__ void __launch_bounds__(128) copy_many_kernel(const __grid_constant__ PackJobs J) {
+  for (int j = 0; j < J.count; ++j) {
+    const PackJob &w = J.job[j];
+    if (w.cap > 0) copy_body(w.W, w.n, w.k, w.b, w.row_ptr, w.col_idx, w.cap, w.blocks, blockIdx.x, gridDim.x);
   }
 }
 
@@ -211,6 +240,41 @@ cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int b,
   copy_blocks_kernel<<<grid, 128, 0, s>>>(static_cast<const uint16_t *>(W), n, k, b, row_ptr, col_idx, cap,
                                          static_cast<uint16_t *>(blocks));
   return cudaGetLastError();
+}
+
+cudaError_t launch_pack_many(const PackJob *jobs, int count, int num_sms, cudaStream_t s) {
+  static bool attr_done[64] = {false};
+  for (int first = 0; first < count; first += PACK_MAX_JOBS) {
+    PackJobs J;
+    J.count = count - first < PACK_MAX_JOBS ? count - first : PACK_MAX_JOBS;
+    size_t smem = 0;
+    int64_t blocks_max = 0;
+    for (int j = 0; j < J.count; ++j) {
+      J.job[j] = jobs[first + j];
+      const size_t sj = plan_smem_bytes(J.job[j].n, J.job[j].b);
+      smem = sj > smem ? sj : smem;
+      blocks_max += (int64_t)(J.job[j].n / J.job[j].b) * (J.job[j].k / J.job[j].b);
+    }
+    if (smem > 48 * 1024) {
+      int dev = 0;
+      cudaGetDevice(&dev);
+      if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(plan_many_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             200 * 1024);
+        if (e != cudaSuccess) return e;
+        attr_done[dev] = true;
+      }
+    }
+    plan_many_kernel<<<J.count, PLAN_THREADS, smem, s>>>(J);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    int64_t grid = blocks_max < (int64_t)num_sms * 16 ? blocks_max : (int64_t)num_sms * 16;
+    if (grid < 1) grid = 1;
+    copy_many_kernel<<<(int)grid, 128, 0, s>>>(J);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace lpvit

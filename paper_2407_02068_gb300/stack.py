@@ -2,7 +2,8 @@
 each a pruned linear (Sec. 3.1) run as a block-sparse matmul (Sec. 3.3).
 
 One ``step`` is one pass of the whole block-sparse path over one batch: every weight is packed
-(mask -> BSR + work list) and every linear runs, chained layer to layer on one stream:
+(mask -> BSR + work list, all weights in one batched call) and every linear runs, chained layer to
+layer on one stream:
 
     qkv  = X~qkv(h)                     [M, 3D]
     proj = X~proj(qkv[:, 2D:3D])        the V third stands in for the attention output
@@ -31,6 +32,7 @@ class DeitLinearStack:
         self.layers = layers
         lib = _lib.load()
         self._pack_fn = lib.lpvit_pack_bsr
+        self._pack_many_fn = lib.lpvit_pack_bsr_many
         self._lin = {False: lib.lpvit_bsr_linear, True: lib.lpvit_bsr_linear_gelu}
         d = layers[0]["qkv"]["W"].shape[1]
         h = layers[0]["fc1"]["W"].shape[0]
@@ -74,6 +76,10 @@ class DeitLinearStack:
     def _build_calls(self, stream: int):
         V = ctypes.c_void_p
         calls = []
+        n = len(self.gemms)
+        self._pack_many_args = (ctypes.c_int32(n), (V * n)(*[G["W"].data_ptr() for G in self.gemms]),
+                                (V * n)(*[G["mask"].data_ptr() for G in self.gemms]),
+                                (_lib.lpvit_bsr * n)(*[G["struct"] for G in self.gemms]), V(stream))
         ws = V(self.ws.data_ptr())
         wsn = ctypes.c_size_t(self.ws.numel())
         st = V(stream)
@@ -103,6 +109,15 @@ class DeitLinearStack:
         return self._calls[1]
 
     def pack_all(self, stream=None):
+        """Pack every weight: one lpvit_pack_bsr_many call (two launches for the whole stack)."""
+        s = int((stream or torch.cuda.current_stream()).cuda_stream)
+        self._calls_for(s)
+        rc = self._pack_many_fn(*self._pack_many_args)
+        if rc != 0:
+            raise _lib.LpvitError(rc, "lpvit_pack_bsr_many")
+
+    def pack_each(self, stream=None):
+        """Pack every weight with its own lpvit_pack_bsr call (the per-weight path)."""
         s = int((stream or torch.cuda.current_stream()).cuda_stream)
         for pack_args, _, _ in self._calls_for(s):
             rc = self._pack_fn(*pack_args)

@@ -58,6 +58,12 @@ def test_bad_arguments_are_rejected_without_a_gpu(lib):
     assert lib.lpvit_bsr_linear(bsr, fake.value, 4, 388, None, 0x200000, 1152, 0, 0x100000, 1 << 20, None) == \
         lib.LPVIT_ERR_INVALID_ARG
     assert lib.lpvit_check(None, None) == lib.LPVIT_ERR_INVALID_ARG
+    # the batched pack checks every job before launching anything
+    assert lib.load().lpvit_pack_bsr_many(0, None, None, None, None) == lib.LPVIT_OK
+    assert lib.load().lpvit_pack_bsr_many(-1, None, None, None, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert lib.load().lpvit_pack_bsr_many(1, None, None, None, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert lib.lpvit_pack_bsr_many([0x1000], [0x2000], [bad_b], None) == lib.LPVIT_ERR_UNSUPPORTED
+    assert lib.lpvit_pack_bsr_many([0x1000, 0], [0x2000, 0x2000], [bsr, bsr], None) == lib.LPVIT_ERR_INVALID_ARG
     # the wait self-test validates before launching anything
     assert lib.lpvit_selftest_wait(0, 10 ** 6, 0, None) == lib.LPVIT_ERR_INVALID_ARG          # no workspace
     assert lib.lpvit_selftest_wait(0x100010, 10 ** 6, 0, None) == lib.LPVIT_ERR_INVALID_ARG   # misaligned

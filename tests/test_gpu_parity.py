@@ -132,6 +132,35 @@ def test_work_list_covers_every_kept_block_once(lp, n, k, b):
     assert seen == set(range(len(ci)))
 
 
+@pytest.mark.parametrize("count", [1, 5, 100])
+def test_pack_many_matches_single_packs(lp, count):
+    """The batched pack (all plans in one launch, all copies in another; 100 jobs span two launches
+    of 96) gives, weight by weight, the bits of single packs and of the oracle."""
+    shapes = [(384, 256, 32), (208, 128, 16), (384, 768, 64), (768, 3072, 32), (96, 64, 32)]
+    Ws, masks, wm, ws = [], [], [], []
+    for i in range(count):
+        n, k, b = shapes[i % len(shapes)]
+        X, W, bias, mask = _case(4, n, k, b, 0.3 + 0.1 * (i % 5), 2000 + i)
+        Ws.append(W.contiguous())
+        masks.append(mask.contiguous())
+        wm.append(lp.alloc_bsr(n, k, b))
+        ws.append(lp.pack_bsr(W, mask, b, count=True))
+    lp.pack_bsr_many_into(wm, Ws, masks)
+    torch.cuda.synchronize()
+    for i in range(count):
+        a, s1 = wm[i], ws[i]
+        n, k, b = a.n, a.k, a.b
+        nnzb = s1.nnzb
+        assert torch.equal(a.row_ptr, s1.row_ptr)
+        assert torch.equal(a.col_idx[:nnzb], s1.col_idx[:nnzb])
+        assert torch.equal(a.blocks[:nnzb].view(torch.int16), s1.blocks[:nnzb].view(torch.int16))
+        # header, group pointers and entries (the words padding the entries to 16 bytes are not defined)
+        ha, hs, ea, es = _decode_sched(a)[0], _decode_sched(s1)[0], _decode_sched(a), _decode_sched(s1)
+        assert np.array_equal(ha, hs) and np.array_equal(ea[1], es[1]) and np.array_equal(ea[2], es[2])
+        rp, ci, bl = oracle.pack(_bits(Ws[i]), masks[i].cpu().numpy(), b)
+        assert np.array_equal(a.row_ptr.cpu().numpy(), rp) and np.array_equal(a.col_idx[:nnzb].cpu().numpy(), ci)
+
+
 # ------------------------------------------------------------------------------------- GEMM
 
 @pytest.mark.parametrize("b", [16, 32, 64])
