@@ -389,7 +389,7 @@ def run_gpu(args, world, rank, local):
         "hbm_gbs_linears": stack.algorithmic_bytes() * args.steps / (lin_ms / 1e3) / 1e9,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": io_bytes, "d2h_bytes_per_step": io_bytes,
                 "steps": e2e_steps},
-        "gpu_launches": args.steps * ngemm * 3,
+        "gpu_launches": args.steps * stack.launches_per_step(),
         "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
                    "power_w_median": clk.get("power_w_median"), "samples": clk["samples"]},
         "cpu_baseline": cpu,

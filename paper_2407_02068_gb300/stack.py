@@ -72,6 +72,11 @@ class DeitLinearStack:
             tot += 2 * self.m * k + 2 * self.m * n + 2 * G["nnzb"] * b * b + 4 * G["nnzb"] + 4 * (n // b + 1) + 4 * n
         return tot
 
+    def launches_per_step(self) -> int:
+        """Kernel launches of one step: one per linear, two per batched pack of up to 96 weights."""
+        n = len(self.gemms)
+        return n + 2 * ((n + 95) // 96)
+
     # ------------------------------------------------------------------ launches
     def _build_calls(self, stream: int):
         V = ctypes.c_void_p
