@@ -174,6 +174,17 @@ def barrier(world: int):
         dist.barrier()
 
 
+def rank_input_seed(rank: int) -> int:
+    """Seed of the activations of rank ``rank``: every rank runs its own batch (weak scaling)."""
+    from paper_2407_02068_gb300 import inputs
+    return inputs.seed(CONFIG_ID, 0, "X") + 7 * rank
+
+
+def weak_scaling_value(flops_per_rank_step: float, steps: int, world: int, elapsed_max_ms: float) -> float:
+    """Whole-job TFLOP/s: the effective FLOPs all ranks processed over the slowest rank's time."""
+    return flops_per_rank_step * steps * world / (elapsed_max_ms / 1e3) / 1e12
+
+
 # ------------------------------------------------------------------------------------ CPU oracle
 
 def oracle_layers_from(stack_layers):
@@ -273,7 +284,7 @@ def run_gpu(args, world, rank, local):
     layers = inputs.deit_b_stack(CONFIG_ID, BLOCK, dev)
     stack = DeitLinearStack(M_TOKENS, layers, dev)
     # each rank works on its own batch (weak scaling: per-GPU work fixed); weights are replicated
-    h0 = inputs.activations(M_TOKENS, 768, inputs.seed(CONFIG_ID, 0, "X") + 7 * rank, dev)
+    h0 = inputs.activations(M_TOKENS, 768, rank_input_seed(rank), dev)
     stack.h_in.copy_(h0)
     s = torch.cuda.current_stream()
     ngemm = len(stack.gemms)
@@ -304,7 +315,7 @@ def run_gpu(args, world, rank, local):
     lin_ms = sum(a.elapsed_time(b) for row in ev for (a, b) in row)
     elapsed_max = max_over_ranks(elapsed_ms, world, dev)
     flops_step = stack.effective_flops()
-    value = flops_step * args.steps * world / (elapsed_max / 1e3) / 1e12
+    value = weak_scaling_value(flops_step, args.steps, world, elapsed_max)
     lin_flops = flops_step * args.steps
     achieved = lin_flops / (lin_ms / 1e3) / 1e12
     peaks, peak_src = load_peaks()
@@ -331,7 +342,7 @@ def run_gpu(args, world, rank, local):
     e1.record(s)
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
-    e2e_value = flops_step * e2e_steps * world / (e2e_ms / 1e3) / 1e12
+    e2e_value = weak_scaling_value(flops_step, e2e_steps, world, e2e_ms)
     io_bytes = h0_host.numel() * h0_host.element_size()
 
     # ---------------- dense comparator (torch bf16 F.linear on W (.) M, same chain)
