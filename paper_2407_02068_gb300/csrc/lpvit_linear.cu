@@ -12,7 +12,7 @@
 //               tokens] += W_blk * X_tile^T, fp32 in TMEM. Within an issuer the X chunk is loaded
 //               once into a B collector buffer (fill) and reused by its other panels (use /
 //               lastuse); the two issuers use disjoint collector buffers.
-//   warps 3..14 epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
+//   warps 3..18 epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
 //               type, stores of 64-byte row segments; split slices are summed in slice order
 //               by the last slice to finish (ticket), which makes the result deterministic.
 // Accumulators are double-buffered in TMEM (2 x 256 columns) so the epilogue of one unit overlaps
@@ -55,7 +55,7 @@ struct Cfg {
 
 constexpr int MMA_WARPS = 2;       // MMA issuers, each owning half of the group's MMA panels
 constexpr int FIRST_EPI = 1 + MMA_WARPS;
-constexpr int EPI_WARPS = 12;      // three per TMEM lane quarter
+constexpr int EPI_WARPS = 16;      // four per TMEM lane quarter
 static_assert(EPI_WARPS % 4 == 0, "epilogue warps come in whole sets of four lane quarters");
 constexpr int NUM_THREADS = 32 * (FIRST_EPI + EPI_WARPS);   // 352
 constexpr int MAX_GROUPS = 512;    // n <= 65536
@@ -78,7 +78,7 @@ struct Smem {
   static constexpr int SLICE_OFF = RING_OFF + (int)sizeof(UnitInfo) * UR;
   static constexpr int MISC_OFF = SLICE_OFF + 4 * (MAX_GROUPS + 1);
   static constexpr int EPI_OFF = (MISC_OFF + 64 + 127) / 128 * 128;
-  static constexpr int EPI_TILE = 32 * 80;  // per epilogue warp: 32 token rows x 32 bf16, rows padded to 80 B
+  static constexpr int EPI_TILE = 16 * 80;  // per epilogue warp: 16 token rows x 32 bf16, rows padded to 80 B
   static constexpr int END = EPI_OFF + EPI_WARPS * EPI_TILE;
   static constexpr int BYTES = END + 1024;  // + alignment slack for the dynamic smem base
   static_assert(BYTES <= 227 * 1024, "shared memory per CTA");
@@ -118,27 +118,30 @@ __device__ __forceinline__ void emit32(float (&y)[32], int f0, int64_t tok_base,
     return;
   }
   __nv_bfloat16 *t = reinterpret_cast<__nv_bfloat16 *>(tile);
-#pragma unroll
-  for (int i = 0; i < 32; ++i) t[i * 40 + lane] = __float2bfloat16_rn(y[i]);
-  __syncwarp();
   const int ch = lane & 3;
   const bool cvalid = f0 + ch * 8 < P.n;
 #pragma unroll
-  for (int it = 0; it < 4; ++it) {
-    const int row = 8 * it + (lane >> 2);
-    const int4 val = *reinterpret_cast<const int4 *>(tile + row * 80 + ch * 16);
-    if (row < rows && cvalid) {
-      __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(P.Y) + (tok_base + row) * P.ldy + f0 + ch * 8;
-      if (P.y_vec16) {
-        *reinterpret_cast<int4 *>(dst) = val;
-      } else {
-        const __nv_bfloat16 *src = reinterpret_cast<const __nv_bfloat16 *>(&val);
+  for (int half = 0; half < 2; ++half) {  // 16 token rows at a time through the warp's tile
 #pragma unroll
-        for (int e = 0; e < 8; ++e) dst[e] = src[e];
+    for (int i = 0; i < 16; ++i) t[i * 40 + lane] = __float2bfloat16_rn(y[16 * half + i]);
+    __syncwarp();
+#pragma unroll
+    for (int it = 0; it < 2; ++it) {
+      const int rt = 8 * it + (lane >> 2), row = 16 * half + rt;
+      const int4 val = *reinterpret_cast<const int4 *>(tile + rt * 80 + ch * 16);
+      if (row < rows && cvalid) {
+        __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(P.Y) + (tok_base + row) * P.ldy + f0 + ch * 8;
+        if (P.y_vec16) {
+          *reinterpret_cast<int4 *>(dst) = val;
+        } else {
+          const __nv_bfloat16 *src = reinterpret_cast<const __nv_bfloat16 *>(&val);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) dst[e] = src[e];
+        }
       }
     }
+    __syncwarp();
   }
-  __syncwarp();
 }
 
 
