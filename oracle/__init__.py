@@ -11,6 +11,8 @@ contraction); this module compiles it with gcc on first use and wraps it with ct
 * ``linear``   -- y = [gelu](X (W (.) M)^T + bias) in float64 (Sec. 3.1 mask, Sec. 3.3 matmul)
 * ``pack``     -- BSR packing of the surviving blocks (Sec. 1, Sec. 3.3)
 * ``round_bf16`` / ``bf16_to_f64`` / ``gelu``
+* ``block_scores`` / ``prune_count`` / ``taylor_mask`` -- the block mask from first-order Taylor
+  scores (Sec. 3.1): |W . grad W| average-pooled per block, bottom alpha of the blocks eliminated
 * ``deit_stack_rows`` -- the 48-GEMM DeiT linear stack on a subset of token rows
 """
 from __future__ import annotations
@@ -61,6 +63,12 @@ def _load():
             lib.lpvit_oracle_linear.argtypes = [P, ctypes.c_int64, ctypes.c_int64, P, P, ctypes.c_int32,
                                                 ctypes.c_int32, ctypes.c_int32, P, ctypes.c_int, P,
                                                 ctypes.c_int64, ctypes.c_int]
+            lib.lpvit_oracle_block_scores.restype = ctypes.c_int
+            lib.lpvit_oracle_block_scores.argtypes = [P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, P]
+            lib.lpvit_oracle_prune_count.restype = ctypes.c_int64
+            lib.lpvit_oracle_prune_count.argtypes = [ctypes.c_double, ctypes.c_int64]
+            lib.lpvit_oracle_taylor_mask.restype = ctypes.c_int
+            lib.lpvit_oracle_taylor_mask.argtypes = [P, ctypes.c_int64, ctypes.c_int64, P]
             lib.lpvit_oracle_round_bf16_array.restype = None
             lib.lpvit_oracle_round_bf16_array.argtypes = [P, P, ctypes.c_int64]
             _lib = lib
@@ -114,6 +122,36 @@ def pack(W_bits: np.ndarray, mask: np.ndarray, b: int):
     if nnzb < 0:
         raise ValueError("oracle pack rejected the arguments")
     return row_ptr, col_idx[:nnzb].copy(), blocks[:nnzb].copy()
+
+
+def block_scores(W_bits: np.ndarray, G: np.ndarray, b: int) -> np.ndarray:
+    """Sec. 3.1 block scores: the average of |W . G| over each b x b block, float64 [n/b, k/b].
+    W_bits: uint16 bf16 bits [n, k]; G: float32 gradient [n, k]."""
+    W_bits = np.ascontiguousarray(W_bits, dtype=np.uint16)
+    G = np.ascontiguousarray(G, dtype=np.float32)
+    n, k = W_bits.shape
+    if G.shape != (n, k):
+        raise ValueError("shape mismatch")
+    out = np.empty((n // b, k // b), dtype=np.float64)
+    if _load().lpvit_oracle_block_scores(_ptr(W_bits), _ptr(G), n, k, b, _ptr(out)) != 0:
+        raise ValueError("oracle block_scores rejected the arguments")
+    return out
+
+
+def prune_count(alpha: float, count: int) -> int:
+    """Blocks eliminated at pruning ratio alpha: round(alpha * count), half away from zero."""
+    return int(_load().lpvit_oracle_prune_count(float(alpha), int(count)))
+
+
+def taylor_mask(scores: np.ndarray, alpha: float) -> np.ndarray:
+    """Sec. 3.1 block mask: rank the blocks by score (ties: lower linear index first) and eliminate
+    the bottom prune_count(alpha, blocks). Returns uint8 of the scores' shape, 1 = kept."""
+    scores = np.ascontiguousarray(scores, dtype=np.float64)
+    mask = np.empty(scores.shape, dtype=np.uint8)
+    if _load().lpvit_oracle_taylor_mask(_ptr(scores), scores.size, prune_count(alpha, scores.size),
+                                        _ptr(mask)) != 0:
+        raise ValueError("oracle taylor_mask rejected the arguments")
+    return mask
 
 
 def linear(X_bits: np.ndarray, W_bits: np.ndarray, mask: np.ndarray, b: int, bias: np.ndarray | None,

@@ -31,6 +31,16 @@
  *  - Round-to-nearest-even conversion of a double to bfloat16 (8 significant bits,
  *    the float32 exponent range, subnormals below 2^-126), written from that definition.
  *
+ *  - Block mask from first-order Taylor scores, Sec. 3.1 ("Block-structured Pruning within
+ *    layer"): the neuron score S = |W . grad_W f| element by element, a 2D average pooling
+ *    with the block as window and stride gives one score per block, the blocks are ranked by
+ *    that score and the bottom ones are eliminated at the layer's pruning ratio alpha.
+ *    Readings where the paper is silent: the number eliminated is round(alpha * blocks),
+ *    half away from zero; equal scores rank by linear block index r * (k/b) + j, the lower
+ *    index first (kept first); a block's sum runs over its elements in row-major order in
+ *    double (each product of a bf16 weight and a float32 gradient is exact in double), then
+ *    divides by b * b.
+ *
  * Inputs X and W arrive as bfloat16 bit patterns (the same bits the GPU reads); bias as
  * float32. Widening bf16 -> double is exact.
  */
@@ -167,4 +177,60 @@ int lpvit_oracle_linear(const uint16_t *X, int64_t m, int64_t ldx, const uint16_
 /* Element-wise double -> bf16 bits (round to nearest even). */
 void lpvit_oracle_round_bf16_array(const double *y, uint16_t *out, int64_t count) {
   for (int64_t i = 0; i < count; ++i) out[i] = lpvit_oracle_round_bf16(y[i]);
+}
+
+/* Sec. 3.1: block score S'[r][j] = average over the block of |W[i][l] * G[i][l]|, summed in
+ * row-major order within the block, in double. W: bf16 bits [n][k]; G: float32 [n][k];
+ * out: [n/b][k/b]. Returns 0, or -1 for a shape that is not a multiple of b. */
+int lpvit_oracle_block_scores(const uint16_t *W, const float *G, int32_t n, int32_t k, int32_t b, double *out) {
+  if (b <= 0 || n % b || k % b) return -1;
+  const int32_t np = n / b, kb = k / b;
+  for (int32_t r = 0; r < np; ++r) {
+    for (int32_t j = 0; j < kb; ++j) {
+      double sum = 0.0;
+      for (int32_t i = 0; i < b; ++i) {
+        for (int32_t l = 0; l < b; ++l) {
+          const int64_t e = (int64_t)(r * b + i) * k + (int64_t)j * b + l;
+          sum += fabs(lpvit_oracle_bf16_to_f64(W[e]) * (double)G[e]);
+        }
+      }
+      out[(int64_t)r * kb + j] = sum / ((double)b * (double)b);
+    }
+  }
+  return 0;
+}
+
+typedef struct {
+  double score;
+  int64_t index;
+} scored_block;
+
+/* higher score first; equal scores: lower linear index first */
+static int rank_order(const void *pa, const void *pb) {
+  const scored_block *a = (const scored_block *)pa, *b = (const scored_block *)pb;
+  if (a->score > b->score) return -1;
+  if (a->score < b->score) return 1;
+  return (a->index > b->index) - (a->index < b->index);
+}
+
+/* Number of blocks eliminated at pruning ratio alpha: round(alpha * count), half away from zero. */
+int64_t lpvit_oracle_prune_count(double alpha, int64_t count) {
+  const double x = alpha * (double)count;
+  return (int64_t)floor(x + 0.5);
+}
+
+/* Sec. 3.1: rank the blocks by score and eliminate the bottom `prune` of them. scores: [count];
+ * mask out: [count], 1 = kept. Returns 0, or -1 for bad arguments. */
+int lpvit_oracle_taylor_mask(const double *scores, int64_t count, int64_t prune, uint8_t *mask) {
+  if (count < 0 || prune < 0 || prune > count) return -1;
+  scored_block *order = (scored_block *)malloc(sizeof(scored_block) * (size_t)(count > 0 ? count : 1));
+  if (!order) return -1;
+  for (int64_t t = 0; t < count; ++t) {
+    order[t].score = scores[t];
+    order[t].index = t;
+  }
+  qsort(order, (size_t)count, sizeof(scored_block), rank_order);
+  for (int64_t t = 0; t < count; ++t) mask[order[t].index] = t < count - prune ? 1 : 0;
+  free(order);
+  return 0;
 }

@@ -288,3 +288,71 @@ def test_deit_stack_rows_is_row_independent_chain():
     qkv = X @ (oracle.bf16_to_f64(W) * _expand(M, b)).T + bias
     assert np.array_equal(oracle.round_bf16(oracle.linear(h0, W, M, b, bias)),
                           oracle.round_bf16(qkv)) or np.allclose(qkv, oracle.linear(h0, W, M, b, bias))
+
+
+# ------------------------------------------------------------- block mask from Taylor scores
+
+def _golden_taylor():
+    rows = [l.split() for l in open(os.path.join(GOLDEN, "taylor_mask_tiny.txt")) if l.strip() and not l.startswith("#")]
+    W = np.array([float(v) for v in rows[0][1:]], dtype=np.float32).reshape(4, 4)
+    G = np.array([float(v) for v in rows[1][1:]], dtype=np.float32).reshape(4, 4)
+    scores = np.array([float(v) for v in rows[2][1:]]).reshape(2, 2)
+    cases = [(float(r[1]), int(r[2]), np.array([int(v) for v in r[3:]], dtype=np.uint8).reshape(2, 2)) for r in rows[3:]]
+    return W, G, scores, cases
+
+
+def _bits(a):
+    """bf16 bits of a float32 array (round to nearest even, as the inputs module rounds)."""
+    return inputs.bf16_bits(torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16))
+
+
+def test_taylor_scores_and_masks_match_the_hand_worked_example():
+    W, G, scores, cases = _golden_taylor()
+    got = oracle.block_scores(_bits(W), G, 2)
+    assert np.array_equal(got, scores)
+    for alpha, pruned, mask in cases:
+        assert oracle.prune_count(alpha, 4) == pruned
+        assert np.array_equal(oracle.taylor_mask(got, alpha), mask), alpha
+
+
+def test_taylor_mask_equal_scores_keep_the_lowest_indices():
+    s = np.full((3, 5), 0.75)
+    for alpha in (0.2, 0.4, 0.6, 0.8):
+        keep = 15 - oracle.prune_count(alpha, 15)
+        assert np.array_equal(oracle.taylor_mask(s, alpha).ravel(), (np.arange(15) < keep).astype(np.uint8))
+
+
+def test_taylor_scores_are_local_and_scale_exactly():
+    rng = np.random.default_rng(5)
+    W = (rng.standard_normal((64, 96)) * 0.02).astype(np.float32)
+    G = (rng.standard_normal((64, 96)) * 1e-3).astype(np.float32)
+    Wb = _bits(W)
+    s = oracle.block_scores(Wb, G, 32)
+    # a power-of-two factor on the gradient scales every score exactly and keeps the mask
+    s4 = oracle.block_scores(Wb, G * np.float32(4.0), 32)
+    assert np.array_equal(s4, 4.0 * s)
+    assert np.array_equal(oracle.taylor_mask(s4, 0.5), oracle.taylor_mask(s, 0.5))
+    # changing one block changes only that block's score
+    G2 = G.copy()
+    G2[32:64, 0:32] *= 3
+    s2 = oracle.block_scores(Wb, G2, 32)
+    changed = s2 != s
+    assert changed[1, 0] and changed.sum() == 1
+
+
+def test_taylor_scores_brute_force_and_mask_order():
+    rng = np.random.default_rng(6)
+    for b in (16, 32):
+        W = (rng.standard_normal((4 * b, 3 * b)) * 0.02).astype(np.float32)
+        G = rng.standard_normal((4 * b, 3 * b)).astype(np.float32)
+        Wb = _bits(W)
+        Wd = oracle.bf16_to_f64(Wb)
+        want = np.abs(Wd * G.astype(np.float64)).reshape(4, b, 3, b).sum(axis=(1, 3)) / (b * b)
+        s = oracle.block_scores(Wb, G, b)
+        assert np.allclose(s, want, rtol=1e-13, atol=0)
+        for alpha in (0.0, 0.25, 0.5, 0.75, 1.0):
+            m = oracle.taylor_mask(s, alpha)
+            kept, pruned = s[m == 1], s[m == 0]
+            assert m.sum() == 12 - oracle.prune_count(alpha, 12)
+            if kept.size and pruned.size:
+                assert kept.min() >= pruned.max()
