@@ -97,6 +97,23 @@ lpvit_status lpvit_pack_bsr(const void *W, const uint8_t *mask, lpvit_bsr *bsr, 
 lpvit_status lpvit_pack_bsr_many(int32_t count, const void *const *W, const uint8_t *const *mask, lpvit_bsr *bsr,
                                  void *stream);
 
+/* The block mask of Sec. 3.1 ("Block-structured Pruning within layer") from first-order Taylor
+ * scores: the neuron score |W . grad W|, a 2D average pooling with the b x b block as window and
+ * stride, and the bottom-ranked blocks eliminated at pruning ratio `prune_ratio` (alpha).
+ *   W       bf16 [n][k] row-major, 16-byte aligned (the weight, as for lpvit_pack_bsr)
+ *   G       float32 [n][k] row-major, 16-byte aligned (the gradient of the loss with respect to W)
+ *   scores  out: double [n/b][k/b], 8-byte aligned: the block scores. Each is the sum of |w * g|
+ *           over the block in row-major order in double (every product is exact), divided by b*b,
+ *           so it is bit-identical to that sequential sum.
+ *   mask    out: uint8 [n/b][k/b], 1 = kept, 0 = eliminated; it can be passed to lpvit_pack_bsr.
+ * Exactly round(alpha * blocks), half away from zero, blocks are eliminated: those ranked lowest,
+ * where blocks rank by score and equal scores by linear block index r*(k/b)+j, the lower first
+ * (kept first). W and G must hold finite values. Asynchronous on `stream`; allocates nothing.
+ * Errors: LPVIT_ERR_UNSUPPORTED (b not in {16,32,64}, more than 2^20 blocks), LPVIT_ERR_INVALID_ARG
+ * (shape, alpha outside [0, 1], null or misaligned pointer), LPVIT_ERR_CUDA. */
+lpvit_status lpvit_taylor_block_mask(const void *W, const float *G, int32_t n, int32_t k, int32_t b,
+                                     double prune_ratio, double *scores, uint8_t *mask, void *stream);
+
 /* Bytes of device workspace lpvit_bsr_linear[_gelu] needs for m tokens. The workspace holds
  * scheduler counters, the device error word and, for small m, fp32 partial sums of split
  * work units. It must be zero-filled once before its first use (cudaMemset); every call

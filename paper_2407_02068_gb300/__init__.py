@@ -4,6 +4,7 @@ LPViT (arXiv 2407.02068) prunes each linear weight of a ViT in b x b blocks (Sec
 the layer becomes a block-sparse matmul whose work is proportional to the kept blocks
 (Sec. 3.3). This package wraps the C library ``liblpvit.so`` (include/lpvit.h):
 
+* ``taylor_block_mask(W, G, b, alpha)`` -- the block mask from first-order Taylor scores (Sec. 3.1)
 * ``pack_bsr(W, mask, b)``  -- mask -> BSR pack + work list, on the GPU
 * ``pack_bsr_many_into(ws, Ws, masks)`` -- the same for a list of weights in two launches
 * ``bsr_linear(w, X, bias, gelu=...)`` -- Y = act(X (W (.) M)^T + bias)
@@ -18,8 +19,8 @@ import torch
 
 from . import _lib
 
-__all__ = ["BsrWeight", "alloc_bsr", "pack_bsr", "pack_bsr_into", "pack_bsr_many_into", "workspace_for",
-           "bsr_linear", "check", "LpvitError"]
+__all__ = ["BsrWeight", "alloc_bsr", "pack_bsr", "pack_bsr_into", "pack_bsr_many_into", "taylor_block_mask",
+           "workspace_for", "bsr_linear", "check", "LpvitError"]
 
 LpvitError = _lib.LpvitError
 
@@ -72,6 +73,26 @@ def pack_bsr_into(w: BsrWeight, W: torch.Tensor, mask: torch.Tensor, count: bool
         raise LpvitError(st, "lpvit_pack_bsr")
     w.nnzb = nnzb
     return w
+
+
+def taylor_block_mask(W: torch.Tensor, G: torch.Tensor, b: int, prune_ratio: float, stream=None):
+    """Block mask of Sec. 3.1 from first-order Taylor scores: W bf16 [n, k], G (the gradient)
+    float32 [n, k], both contiguous CUDA. Returns (mask uint8 [n/b, k/b], 1 = kept; scores float64
+    [n/b, k/b]); round(prune_ratio * blocks) of the lowest-scored blocks are eliminated."""
+    if W.dtype != torch.bfloat16 or not W.is_cuda or W.dim() != 2 or not W.is_contiguous():
+        raise ValueError("W must be a contiguous 2-D bf16 CUDA tensor")
+    if G.dtype != torch.float32 or G.shape != W.shape or not G.is_contiguous() or G.device != W.device:
+        raise ValueError("G must be a contiguous float32 tensor shaped like W on W's device")
+    n, k = W.shape
+    if b <= 0 or n % b or k % b:
+        raise ValueError("n and k must be multiples of b")
+    scores = torch.empty((n // b, k // b), dtype=torch.float64, device=W.device)
+    mask = torch.empty((n // b, k // b), dtype=torch.uint8, device=W.device)
+    st = _lib.lpvit_taylor_block_mask(W.data_ptr(), G.data_ptr(), n, k, b, prune_ratio, scores.data_ptr(),
+                                      mask.data_ptr(), _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_taylor_block_mask")
+    return mask, scores
 
 
 def pack_bsr_many_into(ws: list, Ws: list, masks: list, stream=None) -> list:

@@ -23,7 +23,7 @@ LPVIT_F32 = 1
 
 EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_workspace_bytes", "lpvit_bsr_linear",
            "lpvit_bsr_linear_gelu", "lpvit_bsr_linear_noalloc", "lpvit_check", "lpvit_status_string",
-           "lpvit_selftest_wait", "lpvit_pack_bsr_many")
+           "lpvit_selftest_wait", "lpvit_pack_bsr_many", "lpvit_taylor_block_mask")
 LPVIT_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 
@@ -63,6 +63,8 @@ def load(path: str | None = None):
         lib.lpvit_sched_bytes.argtypes = [I32, I32, I32]
         lib.lpvit_pack_bsr.restype = ctypes.c_int
         lib.lpvit_pack_bsr.argtypes = [V, V, BP, ctypes.POINTER(I32), V]
+        lib.lpvit_taylor_block_mask.restype = ctypes.c_int
+        lib.lpvit_taylor_block_mask.argtypes = [V, V, I32, I32, I32, ctypes.c_double, V, V, V]
         lib.lpvit_pack_bsr_many.restype = ctypes.c_int
         lib.lpvit_pack_bsr_many.argtypes = [I32, ctypes.POINTER(V), ctypes.POINTER(V), BP, V]
         lib.lpvit_workspace_bytes.restype = SZ
@@ -110,6 +112,10 @@ def lpvit_pack_bsr_many(W_ptrs, mask_ptrs, bsrs, stream: int) -> int:
     Wa = (ctypes.c_void_p * n)(*W_ptrs)
     Ma = (ctypes.c_void_p * n)(*mask_ptrs)
     return load().lpvit_pack_bsr_many(n, Wa, Ma, bsrs, stream)
+
+
+def lpvit_taylor_block_mask(W_ptr, G_ptr, n, k, b, prune_ratio, scores_ptr, mask_ptr, stream) -> int:
+    return load().lpvit_taylor_block_mask(W_ptr, G_ptr, n, k, b, float(prune_ratio), scores_ptr, mask_ptr, stream)
 
 
 def lpvit_workspace_bytes(bsr: lpvit_bsr, m: int) -> int:

@@ -64,6 +64,15 @@ def test_bad_arguments_are_rejected_without_a_gpu(lib):
     assert lib.load().lpvit_pack_bsr_many(1, None, None, None, None) == lib.LPVIT_ERR_INVALID_ARG
     assert lib.lpvit_pack_bsr_many([0x1000], [0x2000], [bad_b], None) == lib.LPVIT_ERR_UNSUPPORTED
     assert lib.lpvit_pack_bsr_many([0x1000, 0], [0x2000, 0x2000], [bsr, bsr], None) == lib.LPVIT_ERR_INVALID_ARG
+    # the Taylor block mask validates before launching anything
+    tm = lib.lpvit_taylor_block_mask
+    assert tm(0x1000, 0x2000, 64, 64, 24, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_UNSUPPORTED
+    assert tm(0x1000, 0x2000, 64, 48, 32, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG   # k % b
+    for bad_alpha in (-0.1, 1.5, float("nan")):
+        assert tm(0x1000, 0x2000, 64, 64, 32, bad_alpha, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert tm(0, 0x2000, 64, 64, 32, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert tm(0x1008, 0x2000, 64, 64, 32, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG     # W alignment
+    assert tm(0x1000, 0x2000, 65536, 65536, 16, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_UNSUPPORTED  # > 2^20
     # the wait self-test validates before launching anything
     assert lib.lpvit_selftest_wait(0, 10 ** 6, 0, None) == lib.LPVIT_ERR_INVALID_ARG          # no workspace
     assert lib.lpvit_selftest_wait(0x100010, 10 ** 6, 0, None) == lib.LPVIT_ERR_INVALID_ARG   # misaligned
