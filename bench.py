@@ -57,6 +57,8 @@ def parse_args():
     p.add_argument("--no-dense", action="store_true")
     p.add_argument("--case", default="stack", choices=["stack"] + sorted(CASES),
                    help="stack (the benchmarked workload) or one GEMM of it, for profiling")
+    p.add_argument("--calibrate", action="store_true",
+                   help="fit measured GEMM time to the block-tile count of the paper's power model")
     return p.parse_args()
 
 
@@ -453,11 +455,77 @@ def run_case(args, local):
           flush=True)
 
 
+def run_calibrate(args, local):
+    """Cost-model calibration (Sec. 3.3, Eq. for P: p_m (M/B_m) ceil((1 - alpha) N K / (B_n B_k))):
+    time each DeiT GEMM shape over a block-density sweep and fit, per shape, the least-squares line
+    T = a + p * tiles * nnzb (tiles = ceil(M / 256), the kernel's token tile; nnzb = kept blocks).
+    Prints one JSON line per shape with a, p (ns per block-tile), R^2 and the largest relative
+    residual, and a final line with the fit over all shapes of each block size."""
+    import numpy as np
+    import torch
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2407_02068_gb300 as lp
+    from paper_2407_02068_gb300 import inputs
+    shapes = [("deit_b_fc1", 50432, 768, 3072, 32, True), ("deit_b_fc2", 50432, 3072, 768, 32, False),
+              ("deit_b_qkv", 50432, 768, 2304, 32, False), ("deit_b_proj", 50432, 768, 768, 32, False),
+              ("deit_s_fc1", 12608, 384, 1536, 16, True), ("deit_s_fc2", 12608, 1536, 384, 16, False)]
+    densities = [1.0, 0.7, 0.5, 0.3, 0.2]
+    reps = max(args.steps, 5)
+    pooled = {}
+    for si, (name, m, k, n, b, gelu) in enumerate(shapes):
+        X = inputs.activations(m, k, inputs.seed(6, si, "X"), dev)
+        W = inputs.weight(n, k, inputs.seed(6, si, "W"), dev)
+        bias = inputs.bias(n, inputs.seed(6, si, "bias"), dev)
+        Y = torch.empty(m, n, dtype=torch.bfloat16, device=dev)
+        xs, ts = [], []
+        for d in densities:
+            mask = inputs.uniform_mask(n, k, b, 1.0 - d, inputs.seed(6, si, "mask")).to(dev)
+            w = lp.pack_bsr(W, mask, b, count=True)
+            ws = lp.workspace_for(w, m)
+            for _ in range(3):
+                lp.bsr_linear(w, X, bias, gelu=gelu, out=Y, workspace=ws)
+            times = []
+            for _ in range(reps):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                lp.bsr_linear(w, X, bias, gelu=gelu, out=Y, workspace=ws)
+                e1.record()
+                e1.synchronize()
+                times.append(e0.elapsed_time(e1))
+            lp.check(ws)
+            xs.append(-(-m // 256) * w.nnzb)
+            ts.append(float(np.median(times)) * 1e6)  # ns
+        xs_a, ts_a = np.array(xs, dtype=np.float64), np.array(ts)
+        A = np.stack([np.ones_like(xs_a), xs_a], axis=1)
+        (a, p_), *_ = np.linalg.lstsq(A, ts_a, rcond=None)
+        pred = a + p_ * xs_a
+        r2 = 1 - np.sum((ts_a - pred) ** 2) / np.sum((ts_a - ts_a.mean()) ** 2)
+        print(json.dumps({"shape": name, "m": m, "k": k, "n": n, "b": b, "gelu": gelu, "densities": densities,
+                          "block_tiles": xs, "median_ns": ts, "a_ns": a, "p_ns_per_block_tile": p_, "r2": r2,
+                          "max_rel_residual": float(np.max(np.abs(ts_a - pred) / ts_a))}), flush=True)
+        pooled.setdefault(b, []).extend(zip(xs, ts))
+    for b, pts in pooled.items():
+        xs_a = np.array([x for x, _ in pts], dtype=np.float64)
+        ts_a = np.array([t for _, t in pts])
+        A = np.stack([np.ones_like(xs_a), xs_a], axis=1)
+        (a, p_), *_ = np.linalg.lstsq(A, ts_a, rcond=None)
+        pred = a + p_ * xs_a
+        r2 = 1 - np.sum((ts_a - pred) ** 2) / np.sum((ts_a - ts_a.mean()) ** 2)
+        print(json.dumps({"pooled_over_shapes_b": b, "a_ns": a, "p_ns_per_block_tile": p_, "r2": r2,
+                          "max_rel_residual": float(np.max(np.abs(ts_a - pred) / ts_a))}), flush=True)
+
+
 def main():
     args = parse_args()
     world, rank, local = dist_setup(args)
     if args.impl == "reference":
         run_reference(args, world, rank)
+        return
+    if args.calibrate:
+        run_calibrate(args, local)
         return
     if args.case != "stack":
         run_case(args, local)
