@@ -68,7 +68,9 @@ typedef struct {
 /* Bytes of the `sched` buffer needed for an n x k weight with b x b blocks (0 if the shape is
  * invalid). The work list groups the row panels into 128-feature groups and lists, per group,
  * the block columns where any panel of the group keeps a block (Sec. 3.3: one block matmul per
- * kept block and token tile). */
+ * kept block and token tile). It also holds a second copy of the kept weights, arranged entry
+ * by entry as the GEMM's tensor-core tiles, so that the GEMM reads `sched` and never `blocks`;
+ * that copy is sized for a dense weight: about 2*k*ceil(n/128)*128 bytes plus the list. */
 size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t b);
 
 /* Pack W (bf16 [n][k], row-major, 16-byte aligned) under the block mask (uint8 [n/b][k/b],

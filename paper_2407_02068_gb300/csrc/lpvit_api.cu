@@ -119,12 +119,11 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   if (m < 0) return LPVIT_ERR_INVALID_ARG;
   if (y_dtype != LPVIT_BF16 && y_dtype != LPVIT_F32) return LPVIT_ERR_INVALID_ARG;
   if (m == 0) return LPVIT_OK;
-  if (!X || !Y || !bsr->blocks || !bsr->sched || !workspace) return LPVIT_ERR_INVALID_ARG;
+  if (!X || !Y || !bsr->sched || !workspace) return LPVIT_ERR_INVALID_ARG;
   if (bsr->nnzb_capacity < 0) return LPVIT_ERR_INVALID_ARG;
   if (ldx < k || ldx % 8 != 0 || !aligned(X, 16)) return LPVIT_ERR_INVALID_ARG;
   const size_t ysz = y_dtype == LPVIT_F32 ? 4 : 2;
-  if (ldy < n || !aligned(Y, ysz) || !aligned(bsr->blocks, 16) || !aligned(bsr->sched, 16) ||
-      !aligned(workspace, 256))
+  if (ldy < n || !aligned(Y, ysz) || !aligned(bsr->sched, 16) || !aligned(workspace, 256))
     return LPVIT_ERR_INVALID_ARG;
   if (bias && !aligned(bias, 4)) return LPVIT_ERR_INVALID_ARG;
   if (m > (int64_t)0x7fffff00) return LPVIT_ERR_INVALID_ARG;
@@ -145,7 +144,7 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
 
   const CUtensorMapSwizzle swz =
       b == 16 ? CU_TENSOR_MAP_SWIZZLE_32B : (b == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
-  CUtensorMap tmX, tmW;
+  CUtensorMap tmX;
   {
     cuuint64_t dims[2] = {(cuuint64_t)k, (cuuint64_t)m};
     cuuint64_t strides[1] = {(cuuint64_t)ldx * 2};
@@ -156,19 +155,11 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return LPVIT_ERR_INVALID_ARG;
   }
-  {
-    const int64_t cap = bsr->nnzb_capacity > 0 ? bsr->nnzb_capacity : 1;
-    cuuint64_t dims[2] = {(cuuint64_t)b, (cuuint64_t)(cap * b)};
-    cuuint64_t strides[1] = {(cuuint64_t)b * 2};
-    cuuint32_t box[2] = {(cuuint32_t)b, (cuuint32_t)b};
-    cuuint32_t es[2] = {1, 1};
-    if (enc(&tmW, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, bsr->blocks, dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return LPVIT_ERR_INVALID_ARG;
-  }
   LinearParams P;
+  const int ng = (int)ceil_div(n, GROUP_FEATURES);
   P.sched = static_cast<const int32_t *>(bsr->sched);
+  P.wstream = static_cast<const uint8_t *>(bsr->sched) + sched_stream_offset_bytes(ng, k / b);
+  P.stream_tiles = sched_stream_tiles(ng, k / b, b);
   P.bias = bias;
   P.Y = Y;
   P.ldy = ldy;
@@ -176,7 +167,7 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.n = n;
   P.k = k;
   P.n_tt = (int)ceil_div(m, TOKENS_PER_TILE);
-  P.n_groups = (int)ceil_div(n, GROUP_FEATURES);
+  P.n_groups = ng;
   P.S = choose_slice(P.n_tt, P.n_groups, k / b, sms);
   P.y_f32 = y_dtype == LPVIT_F32;
   P.gelu = gelu;
@@ -188,8 +179,7 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.timeout_ns = TIMEOUT_NS;
   const int64_t units_max = (int64_t)P.n_tt * P.n_groups * ceil_div(k / b, P.S);
   const int grid = (int)(units_max < sms ? units_max : sms);
-  return cuda_status(launch_linear(b, tmX, tmW, P, grid,
-                                   static_cast<cudaStream_t>(stream)));
+  return cuda_status(launch_linear(b, tmX, P, grid, static_cast<cudaStream_t>(stream)));
 }
 
 // The checks lpvit_pack_bsr applies to one weight.
@@ -217,7 +207,7 @@ extern "C" {
 size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t b) {
   if (!shape_ok(n, k, b)) return 0;
   const int ng = (int)ceil_div(n, GROUP_FEATURES);
-  return 4 * (size_t)sched_entries_offset_ints(ng) + 4 * (size_t)ENTRY_INTS * ng * (k / b);
+  return (size_t)sched_stream_offset_bytes(ng, k / b) + (size_t)sched_stream_tiles(ng, k / b, b) * stream_tile_bytes(b);
 }
 
 

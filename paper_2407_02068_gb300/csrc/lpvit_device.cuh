@@ -1,6 +1,6 @@
 // Device-side building blocks for sm_103a: mbarriers with bounded waits, TMA (tensor and bulk),
-// tcgen05 (TMEM allocation, weight-stationary MMA with B-collector reuse, TMEM loads) and the
-// shared-memory matrix / instruction descriptors they take. All inline PTX, no libraries.
+// tcgen05 (TMEM allocation, MMA from shared memory, TMEM loads) and the shared-memory matrix /
+// instruction descriptors they take. All inline PTX, no libraries.
 #pragma once
 #include <cstdint>
 #include <cuda.h>
@@ -12,9 +12,17 @@ namespace lpvit {
 // header (16 int32): [0] nnzb, [1] n_groups, [2] total entries, [3] overflow flag, [4] n, [5] k, [6] b
 // then gent_ptr[n_groups + 1] (int32, entries of group g are [gent_ptr[g], gent_ptr[g+1]))
 // then entries, ENTRY_INTS int32 each: [0] = j | (row-panel mask << 16), [1 + p] = block index of
-// the group's p-th row panel at block column j, or -1 (p < GROUP_FEATURES / b <= 8).
+// the group's p-th row panel at block column j, or -1 (p < GROUP_FEATURES / b <= 8),
+// [ENTRY_TILE_WORD] = index of the entry's first tile in the weight stream;
+// then, at sched_stream_offset_bytes (1024-byte aligned), the weight stream: for every entry in
+// order, one tile per MMA panel of the group that keeps a block at column j (ascending panel
+// order; with MP = 128 that is exactly one tile per entry). A tile is W[g*128 + q*MP + r][j*b + c]
+// for r < MP, c < b (MP = mma_panel_rows(b)), with the rows of removed row panels zero, stored as
+// MP rows of 2b bytes whose 16-byte chunks are permuted by stream_chunk_swizzle: the arrangement
+// the MMA's shared-memory descriptor reads, so that one bulk copy moves all of an entry's weights.
 constexpr int SCHED_HDR_INTS = 16;
 constexpr int ENTRY_INTS = 12;
+constexpr int ENTRY_TILE_WORD = 9;
 constexpr int GROUP_FEATURES = 128;   // output features covered by one work unit
 constexpr int MAX_GROUP_PANELS = GROUP_FEATURES / 16;
 constexpr int TOKENS_PER_TILE = 256;  // tokens covered by one work unit (the .ws MMA N)
@@ -23,9 +31,38 @@ __host__ __device__ inline int sched_gent_offset_ints() { return SCHED_HDR_INTS;
 __host__ __device__ inline int64_t sched_entries_offset_ints(int n_groups) {
   return ((int64_t)SCHED_HDR_INTS + n_groups + 1 + 3) / 4 * 4;  // 16-byte aligned entries
 }
+__host__ __device__ inline int64_t sched_stream_offset_bytes(int n_groups, int kb) {
+  const int64_t end = 4 * (sched_entries_offset_ints(n_groups) + (int64_t)n_groups * kb * ENTRY_INTS);
+  return (end + 1023) / 1024 * 1024;
+}
+// Output features per MMA (its M): the whole 128-feature group, so that one MMA per 16-wide k step
+// covers every row panel of the group (those without a block at the column contribute zero rows)
+// and the X chunk it reads from shared memory serves all 128 features.
+__host__ __device__ constexpr int mma_panel_rows(int b) { return b > 0 ? GROUP_FEATURES : 0; }
+__host__ __device__ constexpr int stream_tile_bytes(int b) { return mma_panel_rows(b) * b * 2; }
+// Tiles the stream region holds: every MMA panel of every group at every block column.
+__host__ __device__ inline int64_t sched_stream_tiles(int n_groups, int kb, int b) {
+  return (int64_t)n_groups * kb * (GROUP_FEATURES / mma_panel_rows(b));
+}
+// Position of 16-byte chunk c in tile row r (rows of row_bytes = 32, 64 or 128 bytes): c XOR the
+// row's address bits 7.. above the chunk bits, i.e. the 32/64/128-byte TMA swizzle of a tile
+// placed at a 1024-byte aligned shared-memory address.
+__host__ __device__ constexpr int stream_chunk_swizzle(int r, int row_bytes) {
+  return ((r * row_bytes) >> 7) & (row_bytes / 16 - 1);
+}
+// MMA-panel mask of an entry from its row-panel mask (MMA panel q covers row panels
+// [q*PPM, (q+1)*PPM), PPM = mma_panel_rows(b) / b).
+__host__ __device__ inline uint32_t mma_panel_mask(uint32_t pm, int b) {
+  const int ppm = mma_panel_rows(b) / b;
+  if (ppm == 1) return pm;
+  const uint32_t pair = (1u << ppm) - 1u;
+  uint32_t mm = 0;
+  for (int q = 0; q * ppm < MAX_GROUP_PANELS; ++q) mm |= ((pm >> (ppm * q)) & pair) ? (1u << q) : 0u;
+  return mm;
+}
 
 static_assert(GROUP_FEATURES / 16 <= MAX_GROUP_PANELS, "entry holds every row panel of a group");
-static_assert(1 + MAX_GROUP_PANELS <= ENTRY_INTS, "entry size");
+static_assert(1 + MAX_GROUP_PANELS <= ENTRY_TILE_WORD && ENTRY_TILE_WORD < ENTRY_INTS, "entry size");
 
 // Workspace control block (first 256 bytes of the caller's workspace).
 struct Control {
@@ -40,6 +77,8 @@ static_assert(sizeof(Control) == 256, "control block is 256 bytes");
 // Parameter block of the linear kernel (host fills it, the kernel reads it by value).
 struct LinearParams {
   const int32_t *sched;    // work list (header, gent_ptr, entries)
+  const uint8_t *wstream;  // weight stream inside sched (16-byte aligned)
+  int64_t stream_tiles;    // tiles the stream region holds (bound on every entry's tile range)
   const float *bias;       // [n] or nullptr
   void *Y;
   int64_t ldy;
@@ -87,8 +126,7 @@ struct PackJobs {
   PackJob job[PACK_MAX_JOBS];
 };
 cudaError_t launch_pack_many(const PackJob *jobs, int count, int num_sms, cudaStream_t s);
-cudaError_t launch_linear(int b, const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
-                          cudaStream_t s);
+cudaError_t launch_linear(int b, const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s);
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
@@ -142,6 +180,11 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
       :: "r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar) : "memory");
 }
+// Untiled bulk copy global -> shared: both addresses 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               :: "r"(dst), "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar) : "memory");
+}
 __device__ __forceinline__ void prefetch_tensormap(const CUtensorMap *map) {
   asm volatile("prefetch.tensormap [%0];" :: "l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
@@ -179,42 +222,15 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
-// Weight-stationary MMA D[M x N] (+)= A[M x 16] * B[N x 16]^T with the B operand held in
-// collector buffer BUF: fill (load and keep), use (reuse), lastuse (reuse and release), or none.
-// COLL and BUF are compile-time so that every call site is one straight-line instruction; the
-// caller computes the (warp-uniform) operands with the whole warp and lets one elected lane issue.
-enum Coll { COLL_NONE = 0, COLL_FILL = 1, COLL_USE = 2, COLL_LAST = 3 };
-
-#define LPVIT_WS_MMA(QUAL)                                                                            \
-  asm volatile("{.reg .pred p; setp.ne.b32 p, %4, 0;\n"                                              \
-               "tcgen05.mma.ws.cta_group::1.kind::f16" QUAL " [%0], %1, %2, %3, p;}\n"               \
-               :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate))
-
-template <int BUF, int COLL>
-__device__ __forceinline__ void ws_mma(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
-                                       uint32_t accumulate) {
-  static_assert(BUF >= 0 && BUF < 4, "collector buffer");
-  if constexpr (COLL == COLL_NONE) {
-    LPVIT_WS_MMA("");
-  } else if constexpr (BUF == 0) {
-    if constexpr (COLL == COLL_FILL) LPVIT_WS_MMA(".collector::b0::fill");
-    else if constexpr (COLL == COLL_USE) LPVIT_WS_MMA(".collector::b0::use");
-    else LPVIT_WS_MMA(".collector::b0::lastuse");
-  } else if constexpr (BUF == 1) {
-    if constexpr (COLL == COLL_FILL) LPVIT_WS_MMA(".collector::b1::fill");
-    else if constexpr (COLL == COLL_USE) LPVIT_WS_MMA(".collector::b1::use");
-    else LPVIT_WS_MMA(".collector::b1::lastuse");
-  } else if constexpr (BUF == 2) {
-    if constexpr (COLL == COLL_FILL) LPVIT_WS_MMA(".collector::b2::fill");
-    else if constexpr (COLL == COLL_USE) LPVIT_WS_MMA(".collector::b2::use");
-    else LPVIT_WS_MMA(".collector::b2::lastuse");
-  } else {
-    if constexpr (COLL == COLL_FILL) LPVIT_WS_MMA(".collector::b3::fill");
-    else if constexpr (COLL == COLL_USE) LPVIT_WS_MMA(".collector::b3::use");
-    else LPVIT_WS_MMA(".collector::b3::lastuse");
-  }
+// MMA D[M x N] (+)= A[M x 16] * B[N x 16]^T, A and B K-major in shared memory (descriptors), D
+// fp32 in TMEM (row i in lane i, column j in column j); `accumulate` = 0 overwrites D. One thread
+// issues it; the caller computes the warp-uniform operands with the whole warp.
+__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile("{.reg .pred p; setp.ne.b32 p, %4, 0;\n"
+               "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;}\n"
+               :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
 }
-#undef LPVIT_WS_MMA
 
 // TMEM -> registers: 32 lanes x 32 consecutive 32-bit columns (one lane per thread).
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {

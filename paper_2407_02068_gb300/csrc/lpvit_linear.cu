@@ -5,14 +5,14 @@
 // Work unit = 256 tokens x one 128-feature group of row panels (x one slice of the group's block
 // columns when the problem is too small to fill the GPU). Per CTA (one per SM, persistent):
 //   warp 0      producer: takes units from a global atomic queue, walks the unit's work-list
-//               entries and, per entry (one block column j), TMA-loads the X tile
-//               [256 tokens x b] and every kept W block of the group at column j.
-//   warps 1,2   MMA issuers, each owning half of the group's MMA panels: per entry and per 16-wide
-//               k step, one weight-stationary tcgen05 MMA per present panel, D[panel rows x 256
-//               tokens] += W_blk * X_tile^T, fp32 in TMEM. Within an issuer the X chunk is loaded
-//               once into a B collector buffer (fill) and reused by its other panels (use /
-//               lastuse); the two issuers use disjoint collector buffers.
-//   warps 3..18 epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
+//               entries and, per entry (one block column j), loads the X tile [256 tokens x b]
+//               (TMA tensor copy) and the entry's weight tiles, one per MMA panel keeping a block
+//               at column j, stored back to back in the work list's weight stream (one bulk copy).
+//   warp 1      MMA issuer: per entry and per 16-wide k step, one tcgen05 MMA (M = 128, N = 256,
+//               K = 16, both operands from shared memory): D[128 features x 256 tokens] +=
+//               W_tile * X_tile^T, fp32 in TMEM. The W tile covers the whole group, with zero rows
+//               for the row panels that keep no block at this column.
+//   warps 2..17 epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
 //               type, stores of 64-byte row segments; split slices are summed in slice order
 //               by the last slice to finish (ticket), which makes the result deterministic.
 // Accumulators are double-buffered in TMEM (2 x 256 columns) so the epilogue of one unit overlaps
@@ -29,35 +29,32 @@ namespace lpvit {
 
 template <int B>
 struct Cfg {
-  static constexpr int MP = (B == 64) ? 64 : 32;            // MMA M: features per MMA panel
-  static constexpr int PPM = MP / B;                        // BSR row panels per MMA panel
-  static constexpr int G = GROUP_FEATURES / MP;             // MMA panels per group
-  static constexpr int GB = GROUP_FEATURES / B;             // BSR row panels per group
-  static constexpr int KSTEPS = B / 16;                     // 16-wide k steps per block
+  static constexpr int MP = mma_panel_rows(B);              // MMA M: the group's 128 features
+  static constexpr int PPM = MP / B;                        // BSR row panels per MMA tile
+  static constexpr int KSTEPS = B / 16;                     // 16-wide k steps per block column
   static constexpr int ROW_BYTES = B * 2;                   // bytes of one tile row (bf16)
   static constexpr int TT = TOKENS_PER_TILE;                // MMA N: tokens per unit
-  static constexpr int ACC_COLS = TT * MP / 128;            // TMEM columns per MMA-panel accumulator
-  static constexpr int BUF_COLS = G * ACC_COLS;             // TMEM columns per accumulator buffer
+  static constexpr int BUF_COLS = TT;                       // TMEM columns per accumulator buffer
   static constexpr int X_BYTES = TT * ROW_BYTES;            // X tile [256 x b]
-  static constexpr int BLK_BYTES = B * ROW_BYTES;           // one W block [b x b]
-  static constexpr int A_BYTES = MP * ROW_BYTES;            // one MMA-panel A tile [MP x b]
-  static constexpr int STAGE_BYTES = X_BYTES + G * A_BYTES;
+  static constexpr int A_BYTES = MP * ROW_BYTES;            // W tile [128 x b]
+  static constexpr int STAGE_BYTES = X_BYTES + A_BYTES;
   static constexpr int NSTAGES = 196608 / STAGE_BYTES;      // 192 KB of stages
   static constexpr int UR = 4;                              // unit-info ring depth
   static constexpr int BATCH = NSTAGES >= 16 ? 8 : NSTAGES / 2;  // most entries per lane-parallel TMA batch
-  static constexpr int OPS = 1 + GB;                        // lane slots per entry: X tile + one per row panel
+  static constexpr int OPS = 2;                             // lane slots per entry: X tile, W tile
   static constexpr int NBMAX = BATCH < 32 / OPS ? BATCH : 32 / OPS;  // entries per batch
-  static constexpr int VPT = TT * MP / 128 / 2;             // accumulator values per epilogue thread and panel
   static constexpr uint32_t IDESC = idesc_bf16(MP, TT);
-  static_assert(BUF_COLS == 256, "two accumulator buffers fill the 512 TMEM columns");
+  static_assert(MP == GROUP_FEATURES && A_BYTES == stream_tile_bytes(B), "weight-stream tile geometry");
+  static_assert(2 * BUF_COLS == 512, "two accumulator buffers fill the 512 TMEM columns");
   static_assert(NSTAGES >= 4, "pipeline depth");
+  static_assert(X_BYTES % 1024 == 0 && A_BYTES % 1024 == 0, "tiles stay on their swizzle alignment");
 };
 
-constexpr int MMA_WARPS = 2;       // MMA issuers, each owning half of the group's MMA panels
+constexpr int MMA_WARPS = 1;       // one MMA issuer
 constexpr int FIRST_EPI = 1 + MMA_WARPS;
 constexpr int EPI_WARPS = 16;      // four per TMEM lane quarter
 static_assert(EPI_WARPS % 4 == 0, "epilogue warps come in whole sets of four lane quarters");
-constexpr int NUM_THREADS = 32 * (FIRST_EPI + EPI_WARPS);   // 352
+constexpr int NUM_THREADS = 32 * (FIRST_EPI + EPI_WARPS);   // 576
 constexpr int MAX_GROUPS = 512;    // n <= 65536
 
 struct UnitInfo {
@@ -145,48 +142,22 @@ __device__ __forceinline__ void emit32(float (&y)[32], int f0, int64_t tok_base,
 }
 
 
-// All MMAs of one work-list entry, issued by one elected thread: for every 16-wide k step, one
-// weight-stationary MMA per present MMA panel; the X chunk is filled into collector buffer KK by the
-// first panel and reused by the others. Collector variants are compile-time, panel order ascending.
-template <int B, int KK, int BUFBASE>
-__device__ __forceinline__ void issue_kstep(uint32_t mm, uint32_t touched, uint32_t st_u32, uint32_t dbase) {
+// The MMAs of one work-list entry, issued by one elected thread: for every 16-wide k step,
+// D[128 x 256] (+)= W_tile[128 x 16] * X_tile[256 x 16]^T, both tiles in the stage (X first).
+template <int B>
+__device__ __forceinline__ void issue_entry(uint32_t st_u32, uint32_t dbase, uint32_t accumulate) {
   using C = Cfg<B>;
-  constexpr int BUF = (KK + BUFBASE) % 4;  // collector buffer of this issuer and k step
-  const uint64_t bdesc = smem_desc<C::ROW_BYTES>(st_u32 + KK * 32);
-  const uint64_t a0 = smem_desc<C::ROW_BYTES>(st_u32 + C::X_BYTES + KK * 32);
-  const int p_first = __ffs(mm) - 1;
-  const int p_last = 31 - __clz(mm);
-  auto acc_of = [&](int p) -> uint32_t { return (KK > 0 || ((touched >> p) & 1u)) ? 1u : 0u; };
-  auto adesc = [&](int p) -> uint64_t { return a0 + (uint64_t)((p * C::A_BYTES) >> 4); };
-  if (p_first == p_last) {
-    ws_mma<BUF, COLL_NONE>(dbase + (uint32_t)(p_first * C::ACC_COLS), adesc(p_first), bdesc, C::IDESC, acc_of(p_first));
-    return;
+#pragma unroll
+  for (int kk = 0; kk < C::KSTEPS; ++kk) {
+    const uint64_t bdesc = smem_desc<C::ROW_BYTES>(st_u32 + kk * 32);
+    const uint64_t adesc = smem_desc<C::ROW_BYTES>(st_u32 + C::X_BYTES + kk * 32);
+    umma_f16(dbase, adesc, bdesc, C::IDESC, (kk > 0 || accumulate) ? 1u : 0u);
   }
-  ws_mma<BUF, COLL_FILL>(dbase + (uint32_t)(p_first * C::ACC_COLS), adesc(p_first), bdesc, C::IDESC, acc_of(p_first));
-  uint32_t mid = mm & ~(1u << p_first) & ~(1u << p_last);
-  while (mid) {
-    const int p = __ffs(mid) - 1;
-    mid &= mid - 1u;
-    ws_mma<BUF, COLL_USE>(dbase + (uint32_t)(p * C::ACC_COLS), adesc(p), bdesc, C::IDESC, acc_of(p));
-  }
-  ws_mma<BUF, COLL_LAST>(dbase + (uint32_t)(p_last * C::ACC_COLS), adesc(p_last), bdesc, C::IDESC, acc_of(p_last));
-}
-
-// BUFBASE separates the collector buffers of the two issuers (b0/b1 and b2/b3). With 64-wide
-// blocks each issuer owns one panel, so its MMAs never use a collector buffer.
-template <int B, int BUFBASE>
-__device__ __forceinline__ void issue_entry(uint32_t mm, uint32_t touched, uint32_t st_u32, uint32_t dbase) {
-  static_assert(Cfg<B>::KSTEPS <= 2 || Cfg<B>::G <= MMA_WARPS, "collector buffers per issuer");
-  issue_kstep<B, 0, BUFBASE>(mm, touched, st_u32, dbase);
-  if constexpr (Cfg<B>::KSTEPS > 1) issue_kstep<B, 1, BUFBASE>(mm, touched, st_u32, dbase);
-  if constexpr (Cfg<B>::KSTEPS > 2) issue_kstep<B, 2, BUFBASE>(mm, touched, st_u32, dbase);
-  if constexpr (Cfg<B>::KSTEPS > 3) issue_kstep<B, 3, BUFBASE>(mm, touched, st_u32, dbase);
 }
 
 template <int B>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
-                  const LinearParams P) {
+bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P) {
   using C = Cfg<B>;
   using L = Smem<B>;
   extern __shared__ uint8_t smem_raw[];
@@ -240,10 +211,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     *never_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 0 && lane == 0) {
-    prefetch_tensormap(&tmX);
-    prefetch_tensormap(&tmW);
-  }
+  if (warp == 0 && lane == 0) prefetch_tensormap(&tmX);
   const bool sched_ok = P.sched[3] == 0 && P.sched[1] == P.n_groups;
   if (warp == 2) {
     // slices per group = max(1, ceil(entries / S)); exclusive prefix into slice_ptr
@@ -306,14 +274,11 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       const int g = lo, s = rr - slice_ptr[g], nsl = slice_ptr[g + 1] - slice_ptr[g];
       const int ge0 = gent[g], ge1 = gent[g + 1];
       const int e0 = min(ge0 + s * P.S, ge1), e1 = min(e0 + P.S, ge1);
-      // MMA panels touched by this unit
+      // whether any entry of this unit keeps a block (else the accumulator is never written)
       unsigned touched = 0;
       for (int e = e0 + lane; e < e1; e += 32) touched |= (unsigned)entries[(int64_t)e * ENTRY_INTS] >> 16;
       touched = __reduce_or_sync(0xffffffffu, touched);
-      unsigned tmask = 0;
-#pragma unroll
-      for (int p = 0; p < C::G; ++p)
-        tmask |= ((touched >> (p * C::PPM)) & ((1u << C::PPM) - 1u)) ? (1u << p) : 0u;
+      const unsigned tmask = touched ? 1u : 0u;
       if (lane == 0) {
         UnitInfo inf;
         inf.tt = tt; inf.g = g; inf.s = s; inf.nsl = nsl; inf.e0 = e0; inf.e1 = e1; inf.touched = (int)tmask;
@@ -323,21 +288,17 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       }
       for (int base = e0; base < e1 && ok; base += 32) {
         const int e = base + lane;
-        int w0 = 0;
-        int blk[C::GB];
-#pragma unroll
-        for (int p = 0; p < C::GB; ++p) blk[p] = -1;
+        int w0 = 0, toff = -1;
         if (e < e1) {
           const int32_t *ep = entries + (int64_t)e * ENTRY_INTS;
           w0 = ep[0];
-#pragma unroll
-          for (int p = 0; p < C::GB; ++p) blk[p] = ep[1 + p];
+          toff = ep[ENTRY_TILE_WORD];
         }
         const int cnt = min(32, e1 - base);
         for (int i = 0; i < cnt && ok;) {
-          // One batch = NBMAX consecutive entries. Lane k*OPS + o issues op o of entry k (op 0: the X
-          // tile, op o >= 1: the block of row panel o-1 if kept), all in one instruction: a thread's
-          // bulk copies are processed one after another, copies from different threads overlap.
+          // One batch = NBMAX consecutive entries. Lanes 2k and 2k+1 issue the two copies of entry k
+          // (its X tile, its weight tiles), all in one instruction: a thread's bulk copies are
+          // processed one after another, copies from different threads overlap.
           const int nb = min(C::NBMAX, cnt - i);
           bool wok = true;
           if (lane < nb) {
@@ -349,57 +310,28 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
             if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_EMPTY);
             break;
           }
-          if (C::PPM == 2) {
-            // an MMA panel with exactly one of its two row panels present: zero the other half
-            bool wrote = false;
-            for (int k = 0; k < nb; ++k) {
-              const uint32_t pmk = (uint32_t)__shfl_sync(0xffffffffu, w0, min(i + k, 31)) >> 16;
-              uint8_t *stk = smem + ((it + k) % L::NS) * C::STAGE_BYTES;
-#pragma unroll
-              for (int p = 0; p < C::G; ++p) {
-                const uint32_t two = (pmk >> (2 * p)) & 3u;
-                if (two == 1u || two == 2u) {
-                  const int half = two == 1u ? 1 : 0;
-                  reinterpret_cast<int4 *>(stk + C::X_BYTES + p * C::A_BYTES + half * C::BLK_BYTES)[lane] =
-                      make_int4(0, 0, 0, 0);
-                  wrote = true;
-                }
-              }
-            }
-            if (wrote) fence_proxy_async_smem();
-            __syncwarp();
-          }
-          {
-            const int wk = __shfl_sync(0xffffffffu, w0, min(i + lane, 31));
-            if (lane < nb) {
-              const uint32_t stk = (it + lane) % L::NS;
-              const uint32_t pmk = (uint32_t)wk >> 16;
-              meta[stk] = (int)pmk;
-              mbar_arrive_expect_tx(full_bar(stk), C::X_BYTES + __popc(pmk) * C::BLK_BYTES);
-            }
+          const int k2 = lane >> 1;
+          const int src = min(i + k2, 31);
+          const int wk = __shfl_sync(0xffffffffu, w0, src);
+          const int tk = __shfl_sync(0xffffffffu, toff, src);
+          uint32_t mm = mma_panel_mask((uint32_t)wk >> 16, B) & 1u;
+          // a tile range outside the stream region means a corrupt work list: flag it, load no weights
+          const bool tiles_ok = tk >= 0 && (int64_t)tk + __popc(mm) <= P.stream_tiles;
+          if (!tiles_ok) mm = 0;
+          const uint32_t stk = (it + k2) % L::NS;
+          const uint32_t st_u32 = smem_base + stk * C::STAGE_BYTES;
+          if (k2 < nb && (lane & 1) == 0) {
+            if (!tiles_ok) atomicOr(&P.ctl->err, ERR_BAD_SCHED);
+            meta[stk] = (int)mm;
+            mbar_arrive_expect_tx(full_bar(stk), C::X_BYTES + __popc(mm) * C::A_BYTES);
           }
           __syncwarp();
-          {
-            const int k = lane / C::OPS, o = lane - k * C::OPS;
-            const int srck = min(i + k, 31);
-            const int wsrc = __shfl_sync(0xffffffffu, w0, srck);
-            const uint32_t pm_k = (uint32_t)wsrc >> 16;
-            int bidx = 0;
-#pragma unroll
-            for (int q = 0; q < C::GB; ++q) {
-              const int v = __shfl_sync(0xffffffffu, blk[q], srck);
-              if (q == o - 1) bidx = v;
-            }
-            const bool is_x = o == 0;
-            if (k < nb && (is_x || ((pm_k >> (o - 1)) & 1u))) {
-              const uint32_t stk = (it + k) % L::NS;
-              const uint32_t st_u32 = smem_base + stk * C::STAGE_BYTES;
-              const int bp = o - 1;
-              const uint32_t dst =
-                  is_x ? st_u32 : st_u32 + C::X_BYTES + (bp / C::PPM) * C::A_BYTES + (bp % C::PPM) * C::BLK_BYTES;
-              tma_load_2d(dst, is_x ? &tmX : &tmW, is_x ? (wsrc & 0xffff) * B : 0, is_x ? tt * C::TT : bidx * B,
-                          full_bar(stk));
-            }
+          if (k2 < nb) {
+            if ((lane & 1) == 0)
+              tma_load_2d(st_u32, &tmX, (wk & 0xffff) * B, tt * C::TT, full_bar(stk));
+            else if (mm)
+              bulk_load(st_u32 + C::X_BYTES, P.wstream + (int64_t)tk * C::A_BYTES, __popc(mm) * C::A_BYTES,
+                        full_bar(stk));
           }
           __syncwarp();
           it += nb;
@@ -424,12 +356,8 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     for (uint32_t i = first; i < it; ++i)
       if (!mbar_wait(full_bar(i % L::NS), (i / L::NS) & 1u, never_flag, tmo)) break;
   } else if (warp < FIRST_EPI) {
-    // ============================================================== MMA issuers
-    // Warp 1 + w owns MMA panels [w G/2, (w + 1) G/2) of the group: two independent issuers keep
-    // the tensor pipe fed while each one waits, branches and commits. Each arrives on a stage's
-    // empty barrier once per entry (a commit when it issued MMAs there).
-    const int mw = warp - 1;
-    const uint32_t own = ((1u << (C::G / MMA_WARPS)) - 1u) << (mw * (C::G / MMA_WARPS));
+    // ============================================================== MMA issuer
+    // Arrives on a stage's empty barrier once per entry: a commit when it issued MMAs there.
     uint32_t it = 0, ui = 0;
     bool ok = true;
     while (ok) {
@@ -458,23 +386,18 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
           break;
         }
         tc_fence_after();
-        const uint32_t pm = (uint32_t)meta[stage];
-        uint32_t mm = 0;
-#pragma unroll
-        for (int p = 0; p < C::G; ++p) mm |= ((pm >> (p * C::PPM)) & ((1u << C::PPM) - 1u)) ? (1u << p) : 0u;
+        const uint32_t mm = (uint32_t)meta[stage];  // 1: the stage holds this entry's W tile
         const uint32_t st_u32 = smem_base + stage * C::STAGE_BYTES;
-        const uint32_t mine = mm & own;
-        if (mine) {
+        if (mm) {
           if (elect_one()) {
-            if (mw == 0) issue_entry<B, 0>(mine, touched, st_u32, dbase);
-            else issue_entry<B, 2>(mine, touched, st_u32, dbase);
+            issue_entry<B>(st_u32, dbase, touched);
             tc_commit(empty_bar(stage));
           }
         } else {
           if (elect_one()) mbar_arrive(empty_bar(stage));
         }
         __syncwarp();
-        touched |= mine;
+        touched |= mm;
         ++it;
       }
       if (!ok) break;
@@ -492,14 +415,13 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     if (!mbar_wait(drain_bar, 0, never_flag, tmo) && lane == 0) atomicOr(&P.ctl->err, ERR_DRAIN);
   } else {
     // ============================================================== epilogue
-    // A unit's accumulators form, per TMEM lane quarter, 2 column halves x G panels x CPP chunks =
-    // 8 blocks of 32 tokens x 32 features; the quarter's EPI_WARPS / 4 warps take them in turn.
+    // A unit's accumulator is 128 features (TMEM lanes) x 256 tokens (columns). Per TMEM lane
+    // quarter (32 features) it forms 8 blocks of 32 tokens; the quarter's EPI_WARPS / 4 warps take
+    // them in turn.
     const int ew = warp - FIRST_EPI;             // 0 .. EPI_WARPS - 1
     const int q = warp & 3;                      // TMEM lane quarter this warp may access
     const int wq = ew >> 2;                      // this warp's turn within its quarter
-    constexpr int CPP = C::VPT / 32;             // 32-column chunks per panel and column half
-    constexpr int QBLK = 2 * C::G * CPP;         // blocks per lane quarter
-    const int r = (C::MP == 32) ? lane : 32 * (q & 1) + lane;  // feature row in the MMA panel
+    constexpr int QBLK = C::TT / 32;             // blocks per lane quarter
     uint32_t ui = 0, sync_phase = 0;
     uint8_t *epi_tile = smem + L::EPI_OFF + ew * L::EPI_TILE;
     while (true) {
@@ -520,26 +442,24 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       float *part = nullptr;
       if (split)
         part = P.partials + ((int64_t)inf.tt * total_slices + slice_ptr[inf.g] + inf.s) * (int64_t)(C::TT * 128);
+      const int f0 = inf.g * GROUP_FEATURES + 32 * q;  // first feature of this warp's blocks
 #pragma unroll 1
       for (int j = wq; j < QBLK; j += EPI_WARPS / 4) {
-        const int h = j / (C::G * CPP), p = (j / CPP) % C::G, c = 32 * (j % CPP);
-        const int tok0 = (C::MP == 32) ? 64 * q + 32 * h : 128 * (q >> 1) + 64 * h;  // first token of the block
-        const int col0 = (C::MP == 32) ? 32 * h : 64 * h;                              // its accumulator column
-        const int f = inf.g * GROUP_FEATURES + p * C::MP + r;
-        const uint32_t taddr = tmem_base + ((uint32_t)(32 * q) << 16) + buf * C::BUF_COLS + p * C::ACC_COLS + col0;
+        const int tok0 = 32 * j;  // first token of the block (its accumulator column)
+        const uint32_t taddr = tmem_base + ((uint32_t)(32 * q) << 16) + buf * C::BUF_COLS + tok0;
         float v[32];
-        if ((inf.touched >> p) & 1) {
-          tmem_ld32(taddr + c, v);
+        if (inf.touched) {
+          tmem_ld32(taddr, v);
         } else {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = 0.f;
         }
         if (split) {
-          float4 *dst = reinterpret_cast<float4 *>(part + (int64_t)(p * C::MP + r) * C::TT + tok0 + c);
+          float4 *dst = reinterpret_cast<float4 *>(part + (int64_t)(32 * q + lane) * C::TT + tok0);
 #pragma unroll
           for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
         } else {
-          emit32(v, f - lane, (int64_t)inf.tt * C::TT + tok0 + c, P, epi_tile);
+          emit32(v, f0, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
         }
       }
       // accumulator buffer and unit slot are free again
@@ -580,22 +500,20 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
               P.partials + ((int64_t)inf.tt * total_slices + slice_ptr[inf.g]) * (int64_t)(C::TT * 128);
 #pragma unroll 1
           for (int j = wq; j < QBLK; j += EPI_WARPS / 4) {
-            const int h = j / (C::G * CPP), p = (j / CPP) % C::G, c = 32 * (j % CPP);
-            const int tok0 = (C::MP == 32) ? 64 * q + 32 * h : 128 * (q >> 1) + 64 * h;
-            const int f = inf.g * GROUP_FEATURES + p * C::MP + r;
+            const int tok0 = 32 * j;
             float v[32];
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = 0.f;
             for (int s2 = 0; s2 < inf.nsl; ++s2) {
               const float4 *src = reinterpret_cast<const float4 *>(
-                  base0 + (int64_t)s2 * (C::TT * 128) + (int64_t)(p * C::MP + r) * C::TT + tok0 + c);
+                  base0 + (int64_t)s2 * (C::TT * 128) + (int64_t)(32 * q + lane) * C::TT + tok0);
 #pragma unroll
               for (int i = 0; i < 8; ++i) {
                 const float4 t = __ldcg(src + i);
                 v[4 * i] += t.x; v[4 * i + 1] += t.y; v[4 * i + 2] += t.z; v[4 * i + 3] += t.w;
               }
             }
-            emit32(v, f - lane, (int64_t)inf.tt * C::TT + tok0 + c, P, epi_tile);
+            emit32(v, f0, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
           }
         }
       }
@@ -616,8 +534,7 @@ template <int B>
 int smem_bytes() { return Smem<B>::BYTES; }
 
 template <int B>
-cudaError_t launch_linear_t(const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
-                            cudaStream_t s) {
+cudaError_t launch_linear_t(const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s) {
   static bool attr_done[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
@@ -627,16 +544,15 @@ cudaError_t launch_linear_t(const CUtensorMap &tmX, const CUtensorMap &tmW, cons
     if (e != cudaSuccess) return e;
     attr_done[dev] = true;
   }
-  bsr_linear_kernel<B><<<grid, NUM_THREADS, Smem<B>::BYTES, s>>>(tmX, tmW, P);
+  bsr_linear_kernel<B><<<grid, NUM_THREADS, Smem<B>::BYTES, s>>>(tmX, P);
   return cudaGetLastError();
 }
 
-cudaError_t launch_linear(int b, const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
-                          cudaStream_t s) {
+cudaError_t launch_linear(int b, const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s) {
   switch (b) {
-    case 16: return launch_linear_t<16>(tmX, tmW, P, grid, s);
-    case 32: return launch_linear_t<32>(tmX, tmW, P, grid, s);
-    case 64: return launch_linear_t<64>(tmX, tmW, P, grid, s);
+    case 16: return launch_linear_t<16>(tmX, P, grid, s);
+    case 32: return launch_linear_t<32>(tmX, P, grid, s);
+    case 64: return launch_linear_t<64>(tmX, P, grid, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -6,9 +6,11 @@
 //   col_idx = kept block columns of each panel in ascending order (ballot compaction);
 //   work list: panels are grouped 128 output features at a time; for every group, one entry per
 //   block column where any panel of the group keeps a block, with that column's block index in
-//   each panel (or -1). The GEMM walks these entries.
-// copy kernel (grid-stride over kept blocks): blocks[t] = W[r*b:(r+1)*b, j*b:(j+1)*b], 16-byte
-//   vector copies; the bits are moved unchanged.
+//   each panel (or -1) and the index of its first tile in the weight stream (an exclusive scan of
+//   the entries' MMA-panel counts). The GEMM walks these entries.
+// copy kernel (grid-stride): blocks[t] = W[r*b:(r+1)*b, j*b:(j+1)*b], 16-byte vector copies, bits
+//   unchanged; then the weight stream, the same bits once more, entry by entry in the tiles the
+//   GEMM's MMAs read (rows of removed row panels zero, 16-byte chunks swizzled).
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -65,9 +67,11 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
   const int np = n / b, kb = k / b;
   const int gb = GROUP_FEATURES / b;  // row panels per group
   const int ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
+  const int ppm = mma_panel_rows(b) / b;  // row panels per MMA panel
   int *cnt = plan_smem;            // [np + 1]
   int *gcnt = cnt + np + 1;        // [ng + 1]
-  int *warp_tot = gcnt + ng + 1;   // [33]
+  int *gtile = gcnt + ng + 1;      // [ng + 1]
+  int *warp_tot = gtile + ng + 1;  // [33]
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const unsigned lt = (1u << lane) - 1u;
 
@@ -102,23 +106,34 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
       run += __popc(bal);
     }
   }
-  // 4a. entries per group: block columns where any panel of the group keeps a block
+  // 4a. entries per group (block columns where any panel of the group keeps a block) and stream
+  //     tiles per group (MMA panels keeping a block, summed over those columns)
   for (int g = warp; g < ng; g += PLAN_WARPS) {
-    int c = 0;
+    int c = 0, t = 0;
     for (int base = 0; base < kb; base += 32) {
       const int j = base + lane;
-      unsigned any = 0;
+      unsigned any = 0, qany = 0;
       for (int p = 0; p < gb; ++p) {
         const int r = g * gb + p;
         const bool keep = r < np && j < kb && mask[(int64_t)r * kb + j] != 0;
-        any |= __ballot_sync(0xffffffffu, keep);
+        const unsigned bal = __ballot_sync(0xffffffffu, keep);
+        any |= bal;
+        qany |= bal;
+        if (p % ppm == ppm - 1) {
+          t += __popc(qany);
+          qany = 0;
+        }
       }
       c += __popc(any);
     }
-    if (lane == 0) gcnt[g] = c;
+    if (lane == 0) {
+      gcnt[g] = c;
+      gtile[g] = t;
+    }
   }
   __syncthreads();
   const int total_entries = block_exclusive_scan(gcnt, ng, warp_tot);
+  block_exclusive_scan(gtile, ng, warp_tot);
   int32_t *gent = sched + SCHED_HDR_INTS;
   int32_t *entries = sched + sched_entries_offset_ints(ng);
   for (int g = tid; g < ng; g += PLAN_THREADS) gent[g] = gcnt[g];
@@ -133,9 +148,11 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
     sched[6] = b;
     for (int i = 7; i < SCHED_HDR_INTS; ++i) sched[i] = 0;
   }
-  // 4b. entries: j | (panel mask << 16), then the block index of each panel of the group (or -1)
+  // 4b. entries: j | (panel mask << 16), then the block index of each panel of the group (or -1),
+  //     then the first stream tile
   for (int g = warp; g < ng; g += PLAN_WARPS) {
     int e_run = gcnt[g];
+    int t_run = gtile[g];
     int p_run[MAX_GROUP_PANELS];
 #pragma unroll
     for (int p = 0; p < MAX_GROUP_PANELS; ++p) p_run[p] = (p < gb && g * gb + p < np) ? cnt[g * gb + p] : 0;
@@ -150,20 +167,31 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
         bal[p] = __ballot_sync(0xffffffffu, keep);
         any |= bal[p];
       }
+      unsigned pm = 0;
+#pragma unroll
+      for (int p = 0; p < MAX_GROUP_PANELS; ++p) pm |= ((bal[p] >> lane) & 1u) << p;
+      // this lane's stream tiles, and the exclusive prefix over the lanes before it
+      const int tc = __popc(mma_panel_mask(pm, b));
+      int tincl = tc;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(0xffffffffu, tincl, o);
+        if (lane >= o) tincl += v;
+      }
       if ((any >> lane) & 1u) {
         int32_t *e = entries + (int64_t)(e_run + __popc(any & lt)) * ENTRY_INTS;
-        unsigned pm = 0;
 #pragma unroll
         for (int p = 0; p < MAX_GROUP_PANELS; ++p) {
           const bool keep = (bal[p] >> lane) & 1u;
-          pm |= (keep ? 1u : 0u) << p;
           e[1 + p] = keep ? p_run[p] + __popc(bal[p] & lt) : -1;
         }
         e[0] = (int32_t)((unsigned)j | (pm << 16));
 #pragma unroll
         for (int q = 1 + MAX_GROUP_PANELS; q < ENTRY_INTS; ++q) e[q] = 0;
+        e[ENTRY_TILE_WORD] = t_run + tincl - tc;
       }
       e_run += __popc(any);
+      t_run += __shfl_sync(0xffffffffu, tincl, 31);
 #pragma unroll
       for (int p = 0; p < MAX_GROUP_PANELS; ++p) p_run[p] += __popc(bal[p]);
     }
@@ -209,23 +237,70 @@ __device__ __forceinline__ void copy_body(const uint16_t *__restrict__ W, int n,
   }
 }
 
-__global__ void __launch_bounds__(128)
-copy_blocks_kernel(const uint16_t *__restrict__ W, int n, int k, int b, const int32_t *__restrict__ row_ptr,
-                   const int32_t *__restrict__ col_idx, int cap, uint16_t *__restrict__ blocks) {
-  copy_body(W, n, k, b, row_ptr, col_idx, cap, blocks, blockIdx.x, gridDim.x);
+// Weight-stream tiles of entries e = cta, cta + ncta, ... of one weight (after its plan).
+__device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int n, int k, int b,
+                                            const int32_t *__restrict__ sched, int cta, int ncta) {
+  const int kb = k / b, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
+  if (sched[1] != ng || sched[3] != 0) return;  // not this shape's plan, or blocks overflowed
+  const int total = sched[2];
+  const int mp = mma_panel_rows(b), row_bytes = 2 * b, cpr = row_bytes / 16, chunks = mp * cpr;
+  const int tile_bytes = stream_tile_bytes(b);
+  const int64_t max_tiles = sched_stream_tiles(ng, kb, b);
+  const int32_t *gent = sched + SCHED_HDR_INTS;
+  const int32_t *ent = sched + sched_entries_offset_ints(ng);
+  uint8_t *stream = reinterpret_cast<uint8_t *>(const_cast<int32_t *>(sched)) + sched_stream_offset_bytes(ng, kb);
+  for (int e = cta; e < total; e += ncta) {
+    int lo = 0, hi = ng - 1;  // largest g with gent[g] <= e (the group holding entry e)
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (gent[mid] <= e) lo = mid;
+      else hi = mid - 1;
+    }
+    const int g = lo;
+    const int32_t *ep = ent + (int64_t)e * ENTRY_INTS;
+    const int j = ep[0] & 0xffff;
+    const uint32_t pm = (uint32_t)ep[0] >> 16;
+    const int toff = ep[ENTRY_TILE_WORD];
+    const uint32_t mm = mma_panel_mask(pm, b);
+    const int nt = __popc(mm);
+    if (j >= kb || toff < 0 || (int64_t)toff + nt > max_tiles) continue;
+    for (int v = threadIdx.x; v < nt * chunks; v += blockDim.x) {
+      const int i = v / chunks, ch = v - i * chunks;
+      uint32_t rest = mm;  // the i-th present MMA panel
+      for (int s2 = 0; s2 < i; ++s2) rest &= rest - 1u;
+      const int q = __ffs(rest) - 1;
+      const int r = ch / cpr, c = ch - r * cpr;
+      const int row = g * GROUP_FEATURES + q * mp + r;
+      int4 val = make_int4(0, 0, 0, 0);
+      if (((pm >> ((q * mp + r) / b)) & 1u) && row < n)
+        val = __ldg(reinterpret_cast<const int4 *>(W + (int64_t)row * k + (int64_t)j * b + c * 8));
+      int4 *dst = reinterpret_cast<int4 *>(stream + (int64_t)(toff + i) * tile_bytes + r * row_bytes) +
+                  (c ^ stream_chunk_swizzle(r, row_bytes));
+      *dst = val;
+    }
+  }
 }
 
-// Several weights at once: every CTA takes its share of every job's kept blocks.
+__global__ void __launch_bounds__(128)
+copy_blocks_kernel(const uint16_t *__restrict__ W, int n, int k, int b, const int32_t *__restrict__ row_ptr,
+                   const int32_t *__restrict__ col_idx, int cap, uint16_t *__restrict__ blocks,
+                   const int32_t *__restrict__ sched) {
+  copy_body(W, n, k, b, row_ptr, col_idx, cap, blocks, blockIdx.x, gridDim.x);
+  stream_body(W, n, k, b, sched, blockIdx.x, gridDim.x);
+}
+
+// Several weights at once: every CTA takes its share of every job's kept blocks and stream tiles.
 __global__ void __launch_bounds__(128) copy_many_kernel(const __grid_constant__ PackJobs J) {
   for (int j = 0; j < J.count; ++j) {
     const PackJob &w = J.job[j];
     if (w.cap > 0) copy_body(w.W, w.n, w.k, w.b, w.row_ptr, w.col_idx, w.cap, w.blocks, blockIdx.x, gridDim.x);
+    stream_body(w.W, w.n, w.k, w.b, w.sched, blockIdx.x, gridDim.x);
   }
 }
 
 size_t plan_smem_bytes(int n, int b) {
   const int np = n / b, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
-  return sizeof(int) * (size_t)(np + 1 + ng + 1 + 33);
+  return sizeof(int) * (size_t)(np + 1 + 2 * (ng + 1) + 33);
 }
 
 cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int b, int32_t *row_ptr, int32_t *col_idx,
@@ -238,7 +313,7 @@ cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int b,
   int grid = max_blocks < num_sms * 16 ? max_blocks : num_sms * 16;
   if (grid < 1) grid = 1;
   copy_blocks_kernel<<<grid, 128, 0, s>>>(static_cast<const uint16_t *>(W), n, k, b, row_ptr, col_idx, cap,
-                                         static_cast<uint16_t *>(blocks));
+                                         static_cast<uint16_t *>(blocks), sched);
   return cudaGetLastError();
 }
 

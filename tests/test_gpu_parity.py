@@ -132,6 +132,47 @@ def test_work_list_covers_every_kept_block_once(lp, n, k, b):
     assert seen == set(range(len(ci)))
 
 
+def _check_weight_stream(w, W, mask):
+    """The work list's weight stream: entry by entry, the 128-row tile of the entry's group at its
+    block column (W's rows there, removed row panels zero), tiles contiguous in entry order,
+    16-byte chunk c of tile row r stored at chunk c ^ ((r * rowbytes >> 7) & (rowbytes / 16 - 1))."""
+    n, k, b = w.n, w.k, w.b
+    hdr, gent, ent = _decode_sched(w)
+    ng, kb = int(hdr[1]), k // b
+    mp = 128
+    rb, cpr = 2 * b, 2 * b // 16
+    raw = w.sched.cpu().numpy().view(np.uint8)
+    ent_end = 4 * ((16 + ng + 1 + 3) // 4 * 4 + ng * kb * 12)
+    stream = raw[(ent_end + 1023) // 1024 * 1024:]
+    Wb = _bits(W).reshape(n, k)
+    M = mask.cpu().numpy()
+    t_next = 0
+    for g in range(ng):
+        for e in ent[gent[g]:gent[g + 1]]:
+            j, pm = int(e[0]) & 0xFFFF, (int(e[0]) >> 16) & 0xFFFF
+            assert int(e[9]) == t_next
+            panels = [q for q in range(128 // mp) if any((pm >> ((q * mp + r) // b)) & 1 for r in range(0, mp, b))]
+            for i, q in enumerate(panels):
+                tile = stream[(t_next + i) * mp * rb:(t_next + i + 1) * mp * rb].reshape(mp, cpr, 16)
+                for r in range(mp):
+                    row = g * 128 + q * mp + r
+                    kept = (pm >> ((q * mp + r) // b)) & 1
+                    want = Wb[row, j * b:(j + 1) * b] if kept else np.zeros(b, np.uint16)
+                    if kept:
+                        assert M[row // b, j]
+                    sw = ((r * rb) >> 7) & (cpr - 1)
+                    got = np.concatenate([tile[r, c ^ sw] for c in range(cpr)]).view(np.uint16)
+                    assert np.array_equal(got, want), (g, j, q, r)
+            t_next += len(panels)
+
+
+@pytest.mark.parametrize("n,k,b", [(384, 256, 32), (208, 128, 16), (384, 192, 64), (96, 64, 32)])
+def test_weight_stream_holds_every_entry_tile(lp, n, k, b):
+    X, W, bias, mask = _case(4, n, k, b, 0.5, 31)
+    w = lp.pack_bsr(W, mask, b, count=True)
+    _check_weight_stream(w, W, mask)
+
+
 @pytest.mark.parametrize("count", [1, 5, 100])
 def test_pack_many_matches_single_packs(lp, count):
     """The batched pack (all plans in one launch, all copies in another; 100 jobs span two launches
@@ -157,6 +198,8 @@ def test_pack_many_matches_single_packs(lp, count):
         # header, group pointers and entries (the words padding the entries to 16 bytes are not defined)
         ha, hs, ea, es = _decode_sched(a)[0], _decode_sched(s1)[0], _decode_sched(a), _decode_sched(s1)
         assert np.array_equal(ha, hs) and np.array_equal(ea[1], es[1]) and np.array_equal(ea[2], es[2])
+        if i < 5:
+            _check_weight_stream(a, Ws[i], masks[i])
         rp, ci, bl = oracle.pack(_bits(Ws[i]), masks[i].cpu().numpy(), b)
         assert np.array_equal(a.row_ptr.cpu().numpy(), rp) and np.array_equal(a.col_idx[:nnzb].cpu().numpy(), ci)
 
