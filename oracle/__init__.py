@@ -58,13 +58,15 @@ def _load():
             lib.lpvit_oracle_gelu.restype = ctypes.c_double
             lib.lpvit_oracle_gelu.argtypes = [ctypes.c_double]
             lib.lpvit_oracle_pack.restype = ctypes.c_int64
-            lib.lpvit_oracle_pack.argtypes = [P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, P, P, P]
+            lib.lpvit_oracle_pack.argtypes = [P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                              P, P, P]
             lib.lpvit_oracle_linear.restype = ctypes.c_int
             lib.lpvit_oracle_linear.argtypes = [P, ctypes.c_int64, ctypes.c_int64, P, P, ctypes.c_int32,
-                                                ctypes.c_int32, ctypes.c_int32, P, ctypes.c_int, P,
+                                                ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, P, ctypes.c_int, P,
                                                 ctypes.c_int64, ctypes.c_int]
             lib.lpvit_oracle_block_scores.restype = ctypes.c_int
-            lib.lpvit_oracle_block_scores.argtypes = [P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, P]
+            lib.lpvit_oracle_block_scores.argtypes = [P, P, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                                      ctypes.c_int32, P]
             lib.lpvit_oracle_prune_count.restype = ctypes.c_int64
             lib.lpvit_oracle_prune_count.argtypes = [ctypes.c_double, ctypes.c_int64]
             lib.lpvit_oracle_taylor_mask.restype = ctypes.c_int
@@ -77,6 +79,17 @@ def _load():
 
 def _ptr(a: np.ndarray | None):
     return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def block_shape(b) -> tuple[int, int]:
+    """A block given as b (square, b x b) or (bn, bk): bn output rows by bk input columns."""
+    if isinstance(b, (tuple, list)):
+        bn, bk = int(b[0]), int(b[1])
+    else:
+        bn = bk = int(b)
+    if bn <= 0 or bk <= 0:
+        raise ValueError("block sides must be positive")
+    return bn, bk
 
 
 def bf16_to_f64(bits) -> np.ndarray:
@@ -104,36 +117,39 @@ def gelu(y) -> np.ndarray:
     return np.vectorize(lib.lpvit_oracle_gelu, otypes=[np.float64])(y)
 
 
-def pack(W_bits: np.ndarray, mask: np.ndarray, b: int):
-    """BSR pack of W (uint16 bf16 bits [n, k]) under the block mask ([n/b, k/b], nonzero = kept).
+def pack(W_bits: np.ndarray, mask: np.ndarray, b):
+    """BSR pack of W (uint16 bf16 bits [n, k]) under the block mask ([n/bn, k/bk], nonzero = kept);
+    b is the block: an int (square) or (bn, bk).
 
-    Returns (row_ptr int32[n/b+1], col_idx int32[nnzb], blocks uint16[nnzb, b, b])."""
+    Returns (row_ptr int32[n/bn+1], col_idx int32[nnzb], blocks uint16[nnzb, bn, bk])."""
+    bn, bk = block_shape(b)
     W_bits = np.ascontiguousarray(W_bits, dtype=np.uint16)
     mask = np.ascontiguousarray(mask, dtype=np.uint8)
     n, k = W_bits.shape
-    if n % b or k % b or mask.shape != (n // b, k // b):
+    if n % bn or k % bk or mask.shape != (n // bn, k // bk):
         raise ValueError("shape mismatch")
-    cap = (n // b) * (k // b)
-    row_ptr = np.zeros(n // b + 1, dtype=np.int32)
+    cap = (n // bn) * (k // bk)
+    row_ptr = np.zeros(n // bn + 1, dtype=np.int32)
     col_idx = np.zeros(max(cap, 1), dtype=np.int32)
-    blocks = np.zeros((max(cap, 1), b, b), dtype=np.uint16)
-    nnzb = _load().lpvit_oracle_pack(_ptr(W_bits), _ptr(mask), n, k, b, _ptr(row_ptr), _ptr(col_idx),
+    blocks = np.zeros((max(cap, 1), bn, bk), dtype=np.uint16)
+    nnzb = _load().lpvit_oracle_pack(_ptr(W_bits), _ptr(mask), n, k, bn, bk, _ptr(row_ptr), _ptr(col_idx),
                                      _ptr(blocks))
     if nnzb < 0:
         raise ValueError("oracle pack rejected the arguments")
     return row_ptr, col_idx[:nnzb].copy(), blocks[:nnzb].copy()
 
 
-def block_scores(W_bits: np.ndarray, G: np.ndarray, b: int) -> np.ndarray:
-    """Sec. 3.1 block scores: the average of |W . G| over each b x b block, float64 [n/b, k/b].
-    W_bits: uint16 bf16 bits [n, k]; G: float32 gradient [n, k]."""
+def block_scores(W_bits: np.ndarray, G: np.ndarray, b) -> np.ndarray:
+    """Sec. 3.1 block scores: the average of |W . G| over each bn x bk block (b = int or (bn, bk)),
+    float64 [n/bn, k/bk]. W_bits: uint16 bf16 bits [n, k]; G: float32 gradient [n, k]."""
+    bn, bk = block_shape(b)
     W_bits = np.ascontiguousarray(W_bits, dtype=np.uint16)
     G = np.ascontiguousarray(G, dtype=np.float32)
     n, k = W_bits.shape
-    if G.shape != (n, k):
+    if G.shape != (n, k) or n % bn or k % bk:
         raise ValueError("shape mismatch")
-    out = np.empty((n // b, k // b), dtype=np.float64)
-    if _load().lpvit_oracle_block_scores(_ptr(W_bits), _ptr(G), n, k, b, _ptr(out)) != 0:
+    out = np.empty((n // bn, k // bk), dtype=np.float64)
+    if _load().lpvit_oracle_block_scores(_ptr(W_bits), _ptr(G), n, k, bn, bk, _ptr(out)) != 0:
         raise ValueError("oracle block_scores rejected the arguments")
     return out
 
@@ -154,12 +170,14 @@ def taylor_mask(scores: np.ndarray, alpha: float) -> np.ndarray:
     return mask
 
 
-def linear(X_bits: np.ndarray, W_bits: np.ndarray, mask: np.ndarray, b: int, bias: np.ndarray | None,
+def linear(X_bits: np.ndarray, W_bits: np.ndarray, mask: np.ndarray, b, bias: np.ndarray | None,
            gelu: bool = False, nthreads: int | None = None) -> np.ndarray:
     """y = [gelu](X (W (.) M)^T + bias) in float64.
 
-    X_bits: uint16 [m, k] (a row-strided view is fine); W_bits: uint16 [n, k]; mask: uint8
-    [n/b, k/b]; bias: float32 [n] or None. Returns float64 [m, n]."""
+    X_bits: uint16 [m, k] (a row-strided view is fine); W_bits: uint16 [n, k]; b: the block, int
+    (square) or (bn, bk); mask: uint8 [n/bn, k/bk]; bias: float32 [n] or None. Returns float64
+    [m, n]."""
+    bn, bk = block_shape(b)
     X_bits = np.asarray(X_bits, dtype=np.uint16)
     if X_bits.ndim != 2 or X_bits.strides[1] != 2:
         X_bits = np.ascontiguousarray(X_bits)
@@ -168,14 +186,14 @@ def linear(X_bits: np.ndarray, W_bits: np.ndarray, mask: np.ndarray, b: int, bia
     mask = np.ascontiguousarray(mask, dtype=np.uint8)
     m, k = X_bits.shape
     n = W_bits.shape[0]
-    if W_bits.shape[1] != k or mask.shape != (n // b, k // b):
+    if W_bits.shape[1] != k or n % bn or k % bk or mask.shape != (n // bn, k // bk):
         raise ValueError("shape mismatch")
     if bias is not None:
         bias = np.ascontiguousarray(bias, dtype=np.float32)
     Y = np.empty((m, n), dtype=np.float64)
     if nthreads is None:
         nthreads = os.cpu_count() or 1
-    rc = _load().lpvit_oracle_linear(_ptr(X_bits), m, ldx, _ptr(W_bits), _ptr(mask), n, k, b, _ptr(bias),
+    rc = _load().lpvit_oracle_linear(_ptr(X_bits), m, ldx, _ptr(W_bits), _ptr(mask), n, k, bn, bk, _ptr(bias),
                                      1 if gelu else 0, _ptr(Y), n, int(nthreads))
     if rc != 0:
         raise ValueError("oracle linear rejected the arguments")

@@ -10,7 +10,9 @@
  *  - Block-structured pruning mask, Sec. 3.1 ("Block-structured Pruning within layer"):
  *      W~[i][j] = W[i][j] (.) M[ceil(i/B_h)][ceil(j/B_w)]
  *    The paper indexes blocks 1-based with a ceiling; with 0-based indices the block of
- *    element (i, j) is (floor(i/b), floor(j/b)). A nonzero mask byte keeps the block; a
+ *    element (i, j) is (floor(i/bn), floor(j/bk)), a block being bn output rows by bk input
+ *    columns (B_n x B_k in Eq. for P; Table 2 uses 32x32, 64x32, 16x32 and 16x16, and a
+ *    square b x b block is bn = bk = b). A nonzero mask byte keeps the block; a
  *    zero byte removes it, and a removed weight is exactly zero whatever W holds there
  *    (the pruned value is never multiplied, so NaN or Inf in a pruned block has no effect).
  *
@@ -23,10 +25,10 @@
  *    erf form is used): gelu(y) = 0.5 * y * (1 + erf(y / sqrt(2))).
  *
  *  - Block-sparse packing of the surviving blocks (BSR), Sec. 1 and Sec. 3.3 (only the
- *    surviving blocks are stored and moved): for each row panel r (b consecutive output
+ *    surviving blocks are stored and moved): for each row panel r (bn consecutive output
  *    rows), cnt[r] = number of kept blocks, row_ptr = exclusive prefix sum of cnt,
  *    col_idx lists the kept block columns of panel r in ascending order, and blocks[t]
- *    is the b x b tile of W copied row-major with its bf16 bits unchanged.
+ *    is the bn x bk tile of W copied row-major with its bf16 bits unchanged.
  *
  *  - Round-to-nearest-even conversion of a double to bfloat16 (8 significant bits,
  *    the float32 exponent range, subnormals below 2^-126), written from that definition.
@@ -36,10 +38,10 @@
  *    with the block as window and stride gives one score per block, the blocks are ranked by
  *    that score and the bottom ones are eliminated at the layer's pruning ratio alpha.
  *    Readings where the paper is silent: the number eliminated is round(alpha * blocks),
- *    half away from zero; equal scores rank by linear block index r * (k/b) + j, the lower
+ *    half away from zero; equal scores rank by linear block index r * (k/bk) + j, the lower
  *    index first (kept first); a block's sum runs over its elements in row-major order in
  *    double (each product of a bf16 weight and a float32 gradient is exact in double), then
- *    divides by b * b.
+ *    divides by bn * bk.
  *
  * Inputs X and W arrive as bfloat16 bit patterns (the same bits the GPU reads); bias as
  * float32. Widening bf16 -> double is exact.
@@ -86,21 +88,21 @@ uint16_t lpvit_oracle_round_bf16(double y) {
 
 double lpvit_oracle_gelu(double y) { return 0.5 * y * (1.0 + erf(y / sqrt(2.0))); }
 
-/* BSR pack by the definition above. col_idx and blocks must hold (n/b)*(k/b) entries.
- * Returns nnzb, or -1 on bad arguments. */
-int64_t lpvit_oracle_pack(const uint16_t *W, const uint8_t *mask, int32_t n, int32_t k, int32_t b,
+/* BSR pack by the definition above, bn x bk blocks. col_idx and blocks must hold
+ * (n/bn)*(k/bk) entries. Returns nnzb, or -1 on bad arguments. */
+int64_t lpvit_oracle_pack(const uint16_t *W, const uint8_t *mask, int32_t n, int32_t k, int32_t bn, int32_t bk,
                           int32_t *row_ptr, int32_t *col_idx, uint16_t *blocks) {
-  if (b <= 0 || n % b != 0 || k % b != 0) return -1;
-  const int32_t np = n / b, kb = k / b;
+  if (bn <= 0 || bk <= 0 || n % bn != 0 || k % bk != 0) return -1;
+  const int32_t np = n / bn, kb = k / bk;
   int64_t t = 0;
   row_ptr[0] = 0;
   for (int32_t r = 0; r < np; ++r) {
     for (int32_t j = 0; j < kb; ++j) {
       if (mask[(int64_t)r * kb + j] == 0) continue;
       col_idx[t] = j;
-      for (int32_t c = 0; c < b; ++c)
-        for (int32_t kk = 0; kk < b; ++kk)
-          blocks[(t * b + c) * b + kk] = W[(int64_t)(r * b + c) * k + (int64_t)j * b + kk];
+      for (int32_t c = 0; c < bn; ++c)
+        for (int32_t kk = 0; kk < bk; ++kk)
+          blocks[(t * bn + c) * bk + kk] = W[(int64_t)(r * bn + c) * k + (int64_t)j * bk + kk];
       ++t;
     }
     row_ptr[r + 1] = (int32_t)t;
@@ -113,7 +115,7 @@ typedef struct {
   int64_t m0, m1, ldx;
   const uint16_t *W;
   const uint8_t *mask;
-  int32_t n, k, b;
+  int32_t n, k, bn, bk;
   const float *bias;
   int gelu;
   double *Y;
@@ -121,13 +123,13 @@ typedef struct {
 } linear_job;
 
 static void linear_rows(const linear_job *J) {
-  const int32_t kb = J->k / J->b;
+  const int32_t kb = J->k / J->bk;
   for (int64_t m = J->m0; m < J->m1; ++m) {
     for (int32_t o = 0; o < J->n; ++o) {
       double acc = 0.0;
       for (int32_t i = 0; i < J->k; ++i) {
         /* W~ = W (.) M: a removed weight is zero, its stored bits are not used */
-        const int keep = J->mask[(int64_t)(o / J->b) * kb + i / J->b] != 0;
+        const int keep = J->mask[(int64_t)(o / J->bn) * kb + i / J->bk] != 0;
         const double w = keep ? lpvit_oracle_bf16_to_f64(J->W[(int64_t)o * J->k + i]) : 0.0;
         acc += lpvit_oracle_bf16_to_f64(J->X[m * J->ldx + i]) * w;
       }
@@ -144,20 +146,20 @@ static void *linear_thread(void *arg) {
 }
 
 /* Y[m][n] (double) = [gelu](X (W (.) M)^T + bias). X is [m][ldx] bf16 bits, W [n][k] bf16 bits,
- * mask [n/b][k/b] bytes, bias float[n] or NULL. Rows are split across nthreads POSIX threads;
+ * mask [n/bn][k/bk] bytes, bias float[n] or NULL. Rows are split across nthreads POSIX threads;
  * each output element is computed by exactly one thread in the same order, so the result does
  * not depend on nthreads. Returns 0, or -1 on bad arguments. */
 int lpvit_oracle_linear(const uint16_t *X, int64_t m, int64_t ldx, const uint16_t *W, const uint8_t *mask,
-                        int32_t n, int32_t k, int32_t b, const float *bias, int gelu, double *Y, int64_t ldy,
-                        int nthreads) {
-  if (b <= 0 || n % b != 0 || k % b != 0 || m < 0 || ldx < k || ldy < n) return -1;
+                        int32_t n, int32_t k, int32_t bn, int32_t bk, const float *bias, int gelu, double *Y,
+                        int64_t ldy, int nthreads) {
+  if (bn <= 0 || bk <= 0 || n % bn != 0 || k % bk != 0 || m < 0 || ldx < k || ldy < n) return -1;
   if (nthreads < 1) nthreads = 1;
   if (nthreads > 256) nthreads = 256;
   if ((int64_t)nthreads > m) nthreads = (int)(m > 0 ? m : 1);
   linear_job jobs[256];
   pthread_t th[256];
   for (int t = 0; t < nthreads; ++t) {
-    linear_job J = {X, m * t / nthreads, m * (t + 1) / nthreads, ldx, W, mask, n, k, b, bias, gelu, Y, ldy};
+    linear_job J = {X, m * t / nthreads, m * (t + 1) / nthreads, ldx, W, mask, n, k, bn, bk, bias, gelu, Y, ldy};
     jobs[t] = J;
   }
   if (nthreads == 1) {
@@ -179,22 +181,23 @@ void lpvit_oracle_round_bf16_array(const double *y, uint16_t *out, int64_t count
   for (int64_t i = 0; i < count; ++i) out[i] = lpvit_oracle_round_bf16(y[i]);
 }
 
-/* Sec. 3.1: block score S'[r][j] = average over the block of |W[i][l] * G[i][l]|, summed in
- * row-major order within the block, in double. W: bf16 bits [n][k]; G: float32 [n][k];
- * out: [n/b][k/b]. Returns 0, or -1 for a shape that is not a multiple of b. */
-int lpvit_oracle_block_scores(const uint16_t *W, const float *G, int32_t n, int32_t k, int32_t b, double *out) {
-  if (b <= 0 || n % b || k % b) return -1;
-  const int32_t np = n / b, kb = k / b;
+/* Sec. 3.1: block score S'[r][j] = average over the bn x bk block of |W[i][l] * G[i][l]|,
+ * summed in row-major order within the block, in double. W: bf16 bits [n][k]; G: float32
+ * [n][k]; out: [n/bn][k/bk]. Returns 0, or -1 for a shape that is not a multiple of the block. */
+int lpvit_oracle_block_scores(const uint16_t *W, const float *G, int32_t n, int32_t k, int32_t bn, int32_t bk,
+                              double *out) {
+  if (bn <= 0 || bk <= 0 || n % bn || k % bk) return -1;
+  const int32_t np = n / bn, kb = k / bk;
   for (int32_t r = 0; r < np; ++r) {
     for (int32_t j = 0; j < kb; ++j) {
       double sum = 0.0;
-      for (int32_t i = 0; i < b; ++i) {
-        for (int32_t l = 0; l < b; ++l) {
-          const int64_t e = (int64_t)(r * b + i) * k + (int64_t)j * b + l;
+      for (int32_t i = 0; i < bn; ++i) {
+        for (int32_t l = 0; l < bk; ++l) {
+          const int64_t e = (int64_t)(r * bn + i) * k + (int64_t)j * bk + l;
           sum += fabs(lpvit_oracle_bf16_to_f64(W[e]) * (double)G[e]);
         }
       }
-      out[(int64_t)r * kb + j] = sum / ((double)b * (double)b);
+      out[(int64_t)r * kb + j] = sum / ((double)bn * (double)bk);
     }
   }
   return 0;

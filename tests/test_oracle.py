@@ -47,7 +47,8 @@ def _bits(a):
 
 
 def _expand(mask, b):
-    return np.kron(mask.astype(np.float64), np.ones((b, b)))
+    bn, bk = oracle.block_shape(b)
+    return np.kron(mask.astype(np.float64), np.ones((bn, bk)))
 
 
 def _rand_case(rng, m, n, k, b, density=0.5, int_valued=False):
@@ -61,7 +62,8 @@ def _rand_case(rng, m, n, k, b, density=0.5, int_valued=False):
         bias = (0.02 * rng.standard_normal(n)).astype(np.float32)
     Xb = inputs.bf16_bits(torch.tensor(X).to(torch.bfloat16))
     Wb = inputs.bf16_bits(torch.tensor(W).to(torch.bfloat16))
-    mask = (rng.random((n // b, k // b)) < density).astype(np.uint8)
+    bn, bk = oracle.block_shape(b)
+    mask = (rng.random((n // bn, k // bk)) < density).astype(np.uint8)
     return Xb, Wb, mask, bias
 
 
@@ -102,7 +104,9 @@ def test_gelu_matches_scipy_ndtr():
 
 # --------------------------------------------------------------------------- brute force
 
-@pytest.mark.parametrize("m,n,k,b", [(3, 8, 12, 4), (5, 32, 16, 8), (8, 64, 32, 16), (4, 32, 64, 32), (2, 6, 4, 2)])
+@pytest.mark.parametrize("m,n,k,b", [(3, 8, 12, 4), (5, 32, 16, 8), (8, 64, 32, 16), (4, 32, 64, 32), (2, 6, 4, 2),
+                                     (4, 128, 64, (64, 32)), (3, 32, 96, (16, 32)), (2, 12, 8, (3, 2)),
+                                     (3, 64, 64, (32, 16))])
 def test_linear_matches_numpy_dense_masked_product(m, n, k, b):
     rng = np.random.default_rng(1000 + m * 7 + n)
     Xb, Wb, mask, bias = _rand_case(rng, m, n, k, b)
@@ -123,6 +127,30 @@ def test_non_square_mask_orientation():
     X, W = oracle.bf16_to_f64(Xb), oracle.bf16_to_f64(Wb)
     ref = X @ (W * _expand(mask, b)).T + bias
     assert np.allclose(oracle.linear(Xb, Wb, mask, b, bias), ref, rtol=1e-12, atol=1e-14)
+
+
+def test_non_square_blocks_are_rows_by_columns():
+    """A (bn, bk) block is bn output rows by bk input columns: one kept block at (r, j) lets exactly
+    W[r*bn:(r+1)*bn, j*bk:(j+1)*bk] through, and swapping the sides gives a different layer."""
+    rng = np.random.default_rng(11)
+    m, n, k = 3, 64, 64
+    Xb, Wb, _, bias = _rand_case(rng, m, n, k, 8)
+    X, W = oracle.bf16_to_f64(Xb), oracle.bf16_to_f64(Wb)
+    mask = np.zeros((n // 32, k // 16), np.uint8)
+    mask[1, 2] = 1
+    got = oracle.linear(Xb, Wb, mask, (32, 16), None)
+    want = np.zeros((m, n))
+    want[:, 32:64] = X[:, 32:48] @ W[32:64, 32:48].T
+    assert np.allclose(got, want, rtol=1e-13, atol=1e-15)
+    mask2 = np.zeros((n // 16, k // 32), np.uint8)  # the sides swapped: rows 32..47, columns 32..63
+    mask2[2, 1] = 1
+    swapped = oracle.linear(Xb, Wb, mask2, (16, 32), None)
+    want2 = np.zeros((m, n))
+    want2[:, 32:48] = X[:, 32:64] @ W[32:48, 32:64].T
+    assert np.allclose(swapped, want2, rtol=1e-13, atol=1e-15)
+    assert not np.allclose(got, swapped)
+    with pytest.raises(ValueError):
+        oracle.linear(Xb, Wb, mask, (16, 32), None)  # mask shape is for (32, 16) blocks
 
 
 def test_zero_sparsity_equals_dense_torch_matmul_on_config_shapes():
@@ -212,25 +240,27 @@ def test_row_strided_input_view():
 
 # --------------------------------------------------------------------------- pack
 
-@pytest.mark.parametrize("n,k,b", [(64, 32, 16), (96, 192, 32), (128, 64, 64), (32, 32, 16)])
+@pytest.mark.parametrize("n,k,b", [(128, 64, (64, 32)), (64, 96, (16, 32)), (48, 32, (8, 16)), (64, 32, 16), (96, 192, 32), (128, 64, 64), (32, 32, 16)])
 def test_pack_invariants_and_round_trip(n, k, b):
-    rng = np.random.default_rng(n + k + b)
+    rng = np.random.default_rng(n + k + sum(oracle.block_shape(b)))
     _, Wb, mask, _ = _rand_case(rng, 1, n, k, b, density=0.45)
     mask[0, :] = 0  # an empty panel
+    bn, bk = oracle.block_shape(b)
     row_ptr, col_idx, blocks = oracle.pack(Wb, mask, b)
+    assert blocks.shape[1:] == (bn, bk)
     assert row_ptr[0] == 0 and np.all(np.diff(row_ptr) >= 0)
     assert row_ptr[-1] == int(mask.astype(bool).sum()) == len(col_idx)
-    for r in range(n // b):
+    for r in range(n // bn):
         cs = col_idx[row_ptr[r]:row_ptr[r + 1]]
         assert np.all(np.diff(cs) > 0)
         assert cs.tolist() == np.nonzero(mask[r])[0].tolist()
     # unpack(pack(W, M)) == W (.) expand(M), bitwise
     un = np.zeros_like(Wb)
-    for r in range(n // b):
+    for r in range(n // bn):
         for t in range(row_ptr[r], row_ptr[r + 1]):
             j = col_idx[t]
-            un[r * b:(r + 1) * b, j * b:(j + 1) * b] = blocks[t]
-    keep = np.kron(mask, np.ones((b, b), dtype=np.uint8)).astype(bool)
+            un[r * bn:(r + 1) * bn, j * bk:(j + 1) * bk] = blocks[t]
+    keep = np.kron(mask, np.ones((bn, bk), dtype=np.uint8)).astype(bool)
     assert np.array_equal(un, np.where(keep, Wb, 0))
 
 
@@ -342,12 +372,13 @@ def test_taylor_scores_are_local_and_scale_exactly():
 
 def test_taylor_scores_brute_force_and_mask_order():
     rng = np.random.default_rng(6)
-    for b in (16, 32):
-        W = (rng.standard_normal((4 * b, 3 * b)) * 0.02).astype(np.float32)
-        G = rng.standard_normal((4 * b, 3 * b)).astype(np.float32)
+    for b in (16, 32, (64, 32), (16, 32)):
+        bn, bk = oracle.block_shape(b)
+        W = (rng.standard_normal((4 * bn, 3 * bk)) * 0.02).astype(np.float32)
+        G = rng.standard_normal((4 * bn, 3 * bk)).astype(np.float32)
         Wb = _bits(W)
         Wd = oracle.bf16_to_f64(Wb)
-        want = np.abs(Wd * G.astype(np.float64)).reshape(4, b, 3, b).sum(axis=(1, 3)) / (b * b)
+        want = np.abs(Wd * G.astype(np.float64)).reshape(4, bn, 3, bk).sum(axis=(1, 3)) / (bn * bk)
         s = oracle.block_scores(Wb, G, b)
         assert np.allclose(s, want, rtol=1e-13, atol=0)
         for alpha in (0.0, 0.25, 0.5, 0.75, 1.0):
