@@ -445,8 +445,9 @@ def run_case(args, local):
     lp.check(ws)
     ms = sum(a.elapsed_time(b_) for a, b_ in ev) / len(ev)
     nnzb = int((g["mask"] != 0).sum())
-    flops = 2 * m * nnzb * b * b
-    byts = 2 * m * k + 2 * m * n + 2 * nnzb * b * b + 4 * nnzb + 4 * (n // b + 1) + 4 * n
+    bn, bk = inputs.block_sides(b)
+    flops = 2 * m * nnzb * bn * bk
+    byts = 2 * m * k + 2 * m * n + 2 * nnzb * bn * bk + 4 * nnzb + 4 * (n // bn + 1) + 4 * n
     peaks, src = load_peaks()
     print(json.dumps({"case": args.case, "m": m, "k": k, "n": n, "b": b, "sparsity": sp, "gelu": gelu,
                       "linear_ms": ms, "eff_tflops": flops / ms / 1e9, "gbs": byts / ms / 1e6,
@@ -457,7 +458,10 @@ def run_case(args, local):
 
 def run_calibrate(args, local):
     """Cost-model calibration (Sec. 3.3, Eq. for P: p_m (M/B_m) ceil((1 - alpha) N K / (B_n B_k))):
-    time each DeiT GEMM shape over a block-density sweep and fit, per shape, the least-squares line
+    time each DeiT GEMM shape, with the block sizes of Table 2 (DeiT-B 32x32 and 64x32, DeiT-S
+    16x16 and 16x32, "a x b" read as B_n x B_k of Sec. 3.3: a input columns by b output rows, i.e.
+    (bn, bk) = (b, a); the transposed reading is timed too), over a block-density sweep and fit, per
+    shape, the least-squares line
     T = a + p * tiles * nnzb (tiles = ceil(M / 256), the kernel's token tile; nnzb = kept blocks).
     Prints one JSON line per shape with a, p (ns per block-tile), R^2 and the largest relative
     residual, and a final line with the fit over all shapes of each block size."""
@@ -469,13 +473,17 @@ def run_calibrate(args, local):
     __graft_entry__.build()
     import paper_2407_02068_gb300 as lp
     from paper_2407_02068_gb300 import inputs
-    shapes = [("deit_b_fc1", 50432, 768, 3072, 32, True), ("deit_b_fc2", 50432, 3072, 768, 32, False),
-              ("deit_b_qkv", 50432, 768, 2304, 32, False), ("deit_b_proj", 50432, 768, 768, 32, False),
-              ("deit_s_fc1", 12608, 384, 1536, 16, True), ("deit_s_fc2", 12608, 1536, 384, 16, False)]
+    shapes = []
+    for blk in (32, (32, 64), (64, 32)):
+        shapes += [("deit_b_fc1", 50432, 768, 3072, blk, True), ("deit_b_fc2", 50432, 3072, 768, blk, False),
+                   ("deit_b_qkv", 50432, 768, 2304, blk, False), ("deit_b_proj", 50432, 768, 768, blk, False)]
+    for blk in (16, (32, 16), (16, 32)):
+        shapes += [("deit_s_fc1", 12608, 384, 1536, blk, True), ("deit_s_fc2", 12608, 1536, 384, blk, False)]
     densities = [1.0, 0.7, 0.5, 0.3, 0.2]
     reps = max(args.steps, 5)
     pooled = {}
     for si, (name, m, k, n, b, gelu) in enumerate(shapes):
+        bn, bk = inputs.block_sides(b)
         X = inputs.activations(m, k, inputs.seed(6, si, "X"), dev)
         W = inputs.weight(n, k, inputs.seed(6, si, "W"), dev)
         bias = inputs.bias(n, inputs.seed(6, si, "bias"), dev)
@@ -503,10 +511,11 @@ def run_calibrate(args, local):
         (a, p_), *_ = np.linalg.lstsq(A, ts_a, rcond=None)
         pred = a + p_ * xs_a
         r2 = 1 - np.sum((ts_a - pred) ** 2) / np.sum((ts_a - ts_a.mean()) ** 2)
-        print(json.dumps({"shape": name, "m": m, "k": k, "n": n, "b": b, "gelu": gelu, "densities": densities,
+        print(json.dumps({"shape": name, "m": m, "k": k, "n": n, "block": f"{bn}x{bk}", "gelu": gelu,
+                          "densities": densities,
                           "block_tiles": xs, "median_ns": ts, "a_ns": a, "p_ns_per_block_tile": p_, "r2": r2,
                           "max_rel_residual": float(np.max(np.abs(ts_a - pred) / ts_a))}), flush=True)
-        pooled.setdefault(b, []).extend(zip(xs, ts))
+        pooled.setdefault(f"{bn}x{bk}", []).extend(zip(xs, ts))
     for b, pts in pooled.items():
         xs_a = np.array([x for x, _ in pts], dtype=np.float64)
         ts_a = np.array([t for _, t in pts])
@@ -514,7 +523,7 @@ def run_calibrate(args, local):
         (a, p_), *_ = np.linalg.lstsq(A, ts_a, rcond=None)
         pred = a + p_ * xs_a
         r2 = 1 - np.sum((ts_a - pred) ** 2) / np.sum((ts_a - ts_a.mean()) ** 2)
-        print(json.dumps({"pooled_over_shapes_b": b, "a_ns": a, "p_ns_per_block_tile": p_, "r2": r2,
+        print(json.dumps({"pooled_over_shapes_block": b, "a_ns": a, "p_ns_per_block_tile": p_, "r2": r2,
                           "max_rel_residual": float(np.max(np.abs(ts_a - pred) / ts_a))}), flush=True)
 
 

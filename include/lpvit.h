@@ -6,10 +6,12 @@
  * The operation (Sec. 3.1, block-structured pruning; Sec. 3.3, block-sparse matmul):
  *
  *     Y[m][o] = act( sum_i X[m][i] * W~[o][i] + bias[o] ),
- *     W~[o][i] = W[o][i] if mask[o/b][i/b] != 0, else 0,
+ *     W~[o][i] = W[o][i] if mask[o/bn][i/bk] != 0, else 0,
  *
- * with W stored [n = out features][k = in features] (PyTorch Linear layout), b x b blocks
- * (b in {16, 32, 64}), act = identity (lpvit_bsr_linear) or the exact GELU
+ * with W stored [n = out features][k = in features] (PyTorch Linear layout), blocks of bn
+ * output rows by bk input columns (B_n x B_k of Eq. for P; bn, bk in {16, 32, 64}, so the
+ * square 16x16, 32x32, 64x64 and the paper's 64x32 and 16x32 of Table 2 are all covered),
+ * act = identity (lpvit_bsr_linear) or the exact GELU
  * 0.5*y*(1+erf(y/sqrt 2)) (lpvit_bsr_linear_gelu, the DeiT fc1 activation). Only the kept
  * blocks are stored and multiplied: the work is proportional to the number of kept blocks,
  * as in the power model of Sec. 3.3 (Eq. for P).
@@ -38,7 +40,7 @@ extern "C" {
 typedef enum {
   LPVIT_OK = 0,
   LPVIT_ERR_INVALID_ARG = 1, /* bad shape, null pointer, misaligned pointer or stride      */
-  LPVIT_ERR_UNSUPPORTED = 2, /* b not in {16,32,64}, or not an sm_103 device               */
+  LPVIT_ERR_UNSUPPORTED = 2, /* bn or bk not in {16,32,64}, or not an sm_103 device       */
   LPVIT_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed                          */
   LPVIT_ERR_TIMEOUT = 4,     /* a device-side bounded wait ran out (see lpvit_check)       */
   LPVIT_ERR_WORKSPACE = 5    /* workspace or schedule buffer smaller than required          */
@@ -47,16 +49,19 @@ typedef enum {
 typedef enum { LPVIT_BF16 = 0, LPVIT_F32 = 1 } lpvit_dtype;
 
 /* Block-sparse (BSR) weight, filled by lpvit_pack_bsr. Every pointer is caller-owned device
- * memory of the size stated; the struct itself is a plain host value.
- *   row panel r = output rows [r*b, (r+1)*b);  n/b panels.
- *   row_ptr [n/b + 1]          int32   exclusive prefix sum of kept blocks per panel
+ * memory of the size stated; the struct itself is a plain host value. A block is bn output rows
+ * by bk input columns.
+ *   row panel r = output rows [r*bn, (r+1)*bn);  n/bn panels;  block column j = inputs
+ *   [j*bk, (j+1)*bk);  k/bk block columns.
+ *   row_ptr [n/bn + 1]         int32   exclusive prefix sum of kept blocks per panel
  *   col_idx [nnzb_capacity]    int32   kept block columns of each panel, ascending
- *   blocks  [nnzb_capacity][b][b] bf16 kept tiles of W, row-major inside the tile, bits unchanged
+ *   blocks  [nnzb_capacity][bn][bk] bf16 kept tiles of W, row-major inside the tile, bits unchanged
  *   sched   [sched_bytes]      bytes   work list for lpvit_bsr_linear (layout private to the
  *                                      library; see lpvit_sched_bytes)
- * nnzb_capacity must be >= the number of kept blocks; (n/b)*(k/b) always suffices. */
+ * nnzb_capacity must be >= the number of kept blocks; (n/bn)*(k/bk) always suffices. */
 typedef struct {
-  int32_t n, k, b;
+  int32_t n, k;
+  int32_t bn, bk;
   int32_t nnzb_capacity;
   int32_t *row_ptr;
   int32_t *col_idx;
@@ -65,25 +70,25 @@ typedef struct {
   size_t sched_bytes;
 } lpvit_bsr;
 
-/* Bytes of the `sched` buffer needed for an n x k weight with b x b blocks (0 if the shape is
+/* Bytes of the `sched` buffer needed for an n x k weight with bn x bk blocks (0 if the shape is
  * invalid). The work list groups the row panels into 128-feature groups and lists, per group,
  * the block columns where any panel of the group keeps a block (Sec. 3.3: one block matmul per
  * kept block and token tile). It also holds a second copy of the kept weights, arranged entry
  * by entry as the GEMM's tensor-core tiles, so that the GEMM reads `sched` and never `blocks`;
  * that copy is sized for a dense weight: about 2*k*ceil(n/128)*128 bytes plus the list. */
-size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t b);
+size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t bn, int32_t bk);
 
-/* Pack W (bf16 [n][k], row-major, 16-byte aligned) under the block mask (uint8 [n/b][k/b],
+/* Pack W (bf16 [n][k], row-major, 16-byte aligned) under the block mask (uint8 [n/bn][k/bk],
  * nonzero = kept; Sec. 3.1 M_alpha) into bsr->row_ptr / col_idx / blocks and build the work
- * list in bsr->sched. bsr->n, k, b, nnzb_capacity and all its pointers must be set by the
+ * list in bsr->sched. bsr->n, k, bn, bk, nnzb_capacity and all its pointers must be set by the
  * caller. The contents of W inside removed blocks are never read.
  * If nnzb_host is not NULL the call synchronises `stream` and stores the number of kept
  * blocks there. If the mask keeps more blocks than nnzb_capacity, nothing beyond the capacity
  * is written, the work list is marked invalid (linear calls on it then compute nothing and
  * lpvit_check() reports LPVIT_ERR_WORKSPACE), and, when nnzb_host is given, this call returns
- * LPVIT_ERR_WORKSPACE. A capacity of (n/b)*(k/b) never overflows.
+ * LPVIT_ERR_WORKSPACE. A capacity of (n/bn)*(k/bk) never overflows.
  * Errors: LPVIT_ERR_INVALID_ARG (shape, null or misaligned pointer), LPVIT_ERR_UNSUPPORTED
- * (b), LPVIT_ERR_WORKSPACE (sched_bytes too small), LPVIT_ERR_CUDA. */
+ * (bn or bk), LPVIT_ERR_WORKSPACE (sched_bytes too small), LPVIT_ERR_CUDA. */
 lpvit_status lpvit_pack_bsr(const void *W, const uint8_t *mask, lpvit_bsr *bsr, int32_t *nnzb_host,
                             void *stream);
 
@@ -100,20 +105,20 @@ lpvit_status lpvit_pack_bsr_many(int32_t count, const void *const *W, const uint
                                  void *stream);
 
 /* The block mask of Sec. 3.1 ("Block-structured Pruning within layer") from first-order Taylor
- * scores: the neuron score |W . grad W|, a 2D average pooling with the b x b block as window and
- * stride, and the bottom-ranked blocks eliminated at pruning ratio `prune_ratio` (alpha).
+ * scores: the neuron score |W . grad W|, a 2D average pooling with the bn x bk block as window
+ * and stride, and the bottom-ranked blocks eliminated at pruning ratio `prune_ratio` (alpha).
  *   W       bf16 [n][k] row-major, 16-byte aligned (the weight, as for lpvit_pack_bsr)
  *   G       float32 [n][k] row-major, 16-byte aligned (the gradient of the loss with respect to W)
- *   scores  out: double [n/b][k/b], 8-byte aligned: the block scores. Each is the sum of |w * g|
- *           over the block in row-major order in double (every product is exact), divided by b*b,
- *           so it is bit-identical to that sequential sum.
- *   mask    out: uint8 [n/b][k/b], 1 = kept, 0 = eliminated; it can be passed to lpvit_pack_bsr.
+ *   scores  out: double [n/bn][k/bk], 8-byte aligned: the block scores. Each is the sum of |w * g|
+ *           over the block in row-major order in double (every product is exact), divided by
+ *           bn*bk, so it is bit-identical to that sequential sum.
+ *   mask    out: uint8 [n/bn][k/bk], 1 = kept, 0 = eliminated; it can be passed to lpvit_pack_bsr.
  * Exactly round(alpha * blocks), half away from zero, blocks are eliminated: those ranked lowest,
- * where blocks rank by score and equal scores by linear block index r*(k/b)+j, the lower first
+ * where blocks rank by score and equal scores by linear block index r*(k/bk)+j, the lower first
  * (kept first). W and G must hold finite values. Asynchronous on `stream`; allocates nothing.
- * Errors: LPVIT_ERR_UNSUPPORTED (b not in {16,32,64}, more than 2^20 blocks), LPVIT_ERR_INVALID_ARG
- * (shape, alpha outside [0, 1], null or misaligned pointer), LPVIT_ERR_CUDA. */
-lpvit_status lpvit_taylor_block_mask(const void *W, const float *G, int32_t n, int32_t k, int32_t b,
+ * Errors: LPVIT_ERR_UNSUPPORTED (bn or bk not in {16,32,64}, more than 2^20 blocks),
+ * LPVIT_ERR_INVALID_ARG (shape, alpha outside [0, 1], null or misaligned pointer), LPVIT_ERR_CUDA. */
+lpvit_status lpvit_taylor_block_mask(const void *W, const float *G, int32_t n, int32_t k, int32_t bn, int32_t bk,
                                      double prune_ratio, double *scores, uint8_t *mask, void *stream);
 
 /* Bytes of device workspace lpvit_bsr_linear[_gelu] needs for m tokens. The workspace holds

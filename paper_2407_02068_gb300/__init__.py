@@ -1,8 +1,10 @@
 """Block-sparse linear layers for LPViT-pruned vision transformers on GB300 (sm_103a).
 
-LPViT (arXiv 2407.02068) prunes each linear weight of a ViT in b x b blocks (Sec. 3.1) so that
-the layer becomes a block-sparse matmul whose work is proportional to the kept blocks
-(Sec. 3.3). This package wraps the C library ``liblpvit.so`` (include/lpvit.h):
+LPViT (arXiv 2407.02068) prunes each linear weight of a ViT in blocks (Sec. 3.1) so that the
+layer becomes a block-sparse matmul whose work is proportional to the kept blocks (Sec. 3.3). A
+block ``b`` is an int (b x b) or a pair (bn, bk): bn output rows by bk input columns, each 16, 32
+or 64 (Table 2 uses 32x32, 64x32, 16x32 and 16x16). This package wraps the C library
+``liblpvit.so`` (include/lpvit.h):
 
 * ``taylor_block_mask(W, G, b, alpha)`` -- the block mask from first-order Taylor scores (Sec. 3.1)
 * ``pack_bsr(W, mask, b)``  -- mask -> BSR pack + work list, on the GPU
@@ -25,6 +27,15 @@ __all__ = ["BsrWeight", "alloc_bsr", "pack_bsr", "pack_bsr_into", "pack_bsr_many
 LpvitError = _lib.LpvitError
 
 
+def block_sides(b) -> tuple[int, int]:
+    """(bn, bk) of a block given as b (square) or (bn, bk)."""
+    if isinstance(b, (tuple, list)):
+        if len(b) != 2:
+            raise ValueError("a block is b or (bn, bk)")
+        return int(b[0]), int(b[1])
+    return int(b), int(b)
+
+
 def _stream_handle(stream) -> int:
     s = stream if stream is not None else torch.cuda.current_stream()
     return int(s.cuda_stream)
@@ -32,38 +43,47 @@ def _stream_handle(stream) -> int:
 
 @dataclass
 class BsrWeight:
-    """A packed block-sparse weight: device tensors owned by this object."""
+    """A packed block-sparse weight (blocks of bn rows by bk columns): device tensors owned by
+    this object."""
     n: int
     k: int
-    b: int
+    bn: int
+    bk: int
     capacity: int
-    row_ptr: torch.Tensor   # int32 [n/b + 1]
+    row_ptr: torch.Tensor   # int32 [n/bn + 1]
     col_idx: torch.Tensor   # int32 [capacity]
-    blocks: torch.Tensor    # bf16 [capacity, b, b]
+    blocks: torch.Tensor    # bf16 [capacity, bn, bk]
     sched: torch.Tensor     # uint8 [sched_bytes]
     nnzb: int | None = None
 
+    @property
+    def b(self):
+        """The block as given to alloc_bsr: an int when square, else (bn, bk)."""
+        return self.bn if self.bn == self.bk else (self.bn, self.bk)
+
     def struct(self) -> _lib.lpvit_bsr:
-        return _lib.lpvit_bsr(self.n, self.k, self.b, self.capacity, self.row_ptr.data_ptr(),
+        return _lib.lpvit_bsr(self.n, self.k, self.bn, self.bk, self.capacity, self.row_ptr.data_ptr(),
                               self.col_idx.data_ptr(), self.blocks.data_ptr(), self.sched.data_ptr(),
                               self.sched.numel())
 
 
-def alloc_bsr(n: int, k: int, b: int, capacity: int | None = None, device="cuda") -> BsrWeight:
-    """Device buffers for a packed n x k weight with b x b blocks (capacity defaults to every block)."""
+def alloc_bsr(n: int, k: int, b, capacity: int | None = None, device="cuda") -> BsrWeight:
+    """Device buffers for a packed n x k weight with blocks b (int or (bn, bk)); the capacity
+    defaults to every block."""
+    bn, bk = block_sides(b)
     if capacity is None:
-        capacity = (n // b) * (k // b) if b > 0 and n % b == 0 and k % b == 0 else 0
-    sb = _lib.lpvit_sched_bytes(n, k, b)
-    return BsrWeight(n, k, b, capacity,
-                     torch.empty(max(n // max(b, 1), 0) + 1, dtype=torch.int32, device=device),
+        capacity = (n // bn) * (k // bk) if bn > 0 and bk > 0 and n % bn == 0 and k % bk == 0 else 0
+    sb = _lib.lpvit_sched_bytes(n, k, bn, bk)
+    return BsrWeight(n, k, bn, bk, capacity,
+                     torch.empty(max(n // max(bn, 1), 0) + 1, dtype=torch.int32, device=device),
                      torch.empty(max(capacity, 1), dtype=torch.int32, device=device),
-                     torch.empty((max(capacity, 1), max(b, 1), max(b, 1)), dtype=torch.bfloat16, device=device),
+                     torch.empty((max(capacity, 1), max(bn, 1), max(bk, 1)), dtype=torch.bfloat16, device=device),
                      torch.empty(max(sb, 16), dtype=torch.uint8, device=device))
 
 
 def pack_bsr_into(w: BsrWeight, W: torch.Tensor, mask: torch.Tensor, count: bool = False, stream=None) -> BsrWeight:
-    """Pack W (bf16 [n, k], contiguous CUDA) under the block mask (uint8 [n/b, k/b], contiguous CUDA,
-    nonzero = kept) into the buffers of ``w``; asynchronous unless ``count``."""
+    """Pack W (bf16 [n, k], contiguous CUDA) under the block mask (uint8 [n/bn, k/bk], contiguous
+    CUDA, nonzero = kept) into the buffers of ``w``; asynchronous unless ``count``."""
     if W.dtype != torch.bfloat16 or not W.is_cuda or W.dim() != 2 or not W.is_contiguous():
         raise ValueError("W must be a contiguous 2-D bf16 CUDA tensor")
     if mask.dtype != torch.uint8 or not mask.is_contiguous() or mask.device != W.device:
@@ -75,20 +95,22 @@ def pack_bsr_into(w: BsrWeight, W: torch.Tensor, mask: torch.Tensor, count: bool
     return w
 
 
-def taylor_block_mask(W: torch.Tensor, G: torch.Tensor, b: int, prune_ratio: float, stream=None):
+def taylor_block_mask(W: torch.Tensor, G: torch.Tensor, b, prune_ratio: float, stream=None):
     """Block mask of Sec. 3.1 from first-order Taylor scores: W bf16 [n, k], G (the gradient)
-    float32 [n, k], both contiguous CUDA. Returns (mask uint8 [n/b, k/b], 1 = kept; scores float64
-    [n/b, k/b]); round(prune_ratio * blocks) of the lowest-scored blocks are eliminated."""
+    float32 [n, k], both contiguous CUDA; b = int or (bn, bk). Returns (mask uint8 [n/bn, k/bk],
+    1 = kept; scores float64 [n/bn, k/bk]); round(prune_ratio * blocks) of the lowest-scored
+    blocks are eliminated."""
     if W.dtype != torch.bfloat16 or not W.is_cuda or W.dim() != 2 or not W.is_contiguous():
         raise ValueError("W must be a contiguous 2-D bf16 CUDA tensor")
     if G.dtype != torch.float32 or G.shape != W.shape or not G.is_contiguous() or G.device != W.device:
         raise ValueError("G must be a contiguous float32 tensor shaped like W on W's device")
     n, k = W.shape
-    if b <= 0 or n % b or k % b:
-        raise ValueError("n and k must be multiples of b")
-    scores = torch.empty((n // b, k // b), dtype=torch.float64, device=W.device)
-    mask = torch.empty((n // b, k // b), dtype=torch.uint8, device=W.device)
-    st = _lib.lpvit_taylor_block_mask(W.data_ptr(), G.data_ptr(), n, k, b, prune_ratio, scores.data_ptr(),
+    bn, bk = block_sides(b)
+    if bn <= 0 or bk <= 0 or n % bn or k % bk:
+        raise ValueError("n and k must be multiples of the block sides")
+    scores = torch.empty((n // bn, k // bk), dtype=torch.float64, device=W.device)
+    mask = torch.empty((n // bn, k // bk), dtype=torch.uint8, device=W.device)
+    st = _lib.lpvit_taylor_block_mask(W.data_ptr(), G.data_ptr(), n, k, bn, bk, prune_ratio, scores.data_ptr(),
                                       mask.data_ptr(), _stream_handle(stream))
     if st != _lib.LPVIT_OK:
         raise LpvitError(st, "lpvit_taylor_block_mask")
@@ -112,9 +134,10 @@ def pack_bsr_many_into(ws: list, Ws: list, masks: list, stream=None) -> list:
     return ws
 
 
-def pack_bsr(W: torch.Tensor, mask: torch.Tensor, b: int, capacity: int | None = None, count: bool = False,
+def pack_bsr(W: torch.Tensor, mask: torch.Tensor, b, capacity: int | None = None, count: bool = False,
              stream=None) -> BsrWeight:
-    """Pack W (bf16 [n, k], CUDA) under the block mask (uint8 [n/b, k/b], nonzero = kept)."""
+    """Pack W (bf16 [n, k], CUDA) under the block mask (uint8 [n/bn, k/bk], nonzero = kept);
+    b = int (square) or (bn, bk)."""
     if W.dtype != torch.bfloat16 or not W.is_cuda or W.dim() != 2:
         raise ValueError("W must be a 2-D bf16 CUDA tensor")
     W = W.contiguous()

@@ -29,7 +29,7 @@ LPVIT_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 class lpvit_bsr(ctypes.Structure):
     _fields_ = [
-        ("n", ctypes.c_int32), ("k", ctypes.c_int32), ("b", ctypes.c_int32),
+        ("n", ctypes.c_int32), ("k", ctypes.c_int32), ("bn", ctypes.c_int32), ("bk", ctypes.c_int32),
         ("nnzb_capacity", ctypes.c_int32),
         ("row_ptr", ctypes.c_void_p), ("col_idx", ctypes.c_void_p), ("blocks", ctypes.c_void_p),
         ("sched", ctypes.c_void_p), ("sched_bytes", ctypes.c_size_t),
@@ -60,11 +60,11 @@ def load(path: str | None = None):
         V, I32, I64, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
         BP = ctypes.POINTER(lpvit_bsr)
         lib.lpvit_sched_bytes.restype = SZ
-        lib.lpvit_sched_bytes.argtypes = [I32, I32, I32]
+        lib.lpvit_sched_bytes.argtypes = [I32, I32, I32, I32]
         lib.lpvit_pack_bsr.restype = ctypes.c_int
         lib.lpvit_pack_bsr.argtypes = [V, V, BP, ctypes.POINTER(I32), V]
         lib.lpvit_taylor_block_mask.restype = ctypes.c_int
-        lib.lpvit_taylor_block_mask.argtypes = [V, V, I32, I32, I32, ctypes.c_double, V, V, V]
+        lib.lpvit_taylor_block_mask.argtypes = [V, V, I32, I32, I32, I32, ctypes.c_double, V, V, V]
         lib.lpvit_pack_bsr_many.restype = ctypes.c_int
         lib.lpvit_pack_bsr_many.argtypes = [I32, ctypes.POINTER(V), ctypes.POINTER(V), BP, V]
         lib.lpvit_workspace_bytes.restype = SZ
@@ -89,8 +89,8 @@ def status_string(status: int) -> str:
     return load().lpvit_status_string(int(status)).decode()
 
 
-def lpvit_sched_bytes(n: int, k: int, b: int) -> int:
-    return int(load().lpvit_sched_bytes(n, k, b))
+def lpvit_sched_bytes(n: int, k: int, bn: int, bk: int) -> int:
+    return int(load().lpvit_sched_bytes(n, k, bn, bk))
 
 
 def lpvit_pack_bsr(W_ptr: int, mask_ptr: int, bsr: lpvit_bsr, want_count: bool, stream: int):
@@ -114,8 +114,9 @@ def lpvit_pack_bsr_many(W_ptrs, mask_ptrs, bsrs, stream: int) -> int:
     return load().lpvit_pack_bsr_many(n, Wa, Ma, bsrs, stream)
 
 
-def lpvit_taylor_block_mask(W_ptr, G_ptr, n, k, b, prune_ratio, scores_ptr, mask_ptr, stream) -> int:
-    return load().lpvit_taylor_block_mask(W_ptr, G_ptr, n, k, b, float(prune_ratio), scores_ptr, mask_ptr, stream)
+def lpvit_taylor_block_mask(W_ptr, G_ptr, n, k, bn, bk, prune_ratio, scores_ptr, mask_ptr, stream) -> int:
+    return load().lpvit_taylor_block_mask(W_ptr, G_ptr, n, k, bn, bk, float(prune_ratio), scores_ptr, mask_ptr,
+                                          stream)
 
 
 def lpvit_workspace_bytes(bsr: lpvit_bsr, m: int) -> int:

@@ -70,10 +70,12 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-bool valid_b(int b) { return b == 16 || b == 32 || b == 64; }
+// Block sides: bn output rows, bk input columns, each 16, 32 or 64.
+bool valid_side(int s) { return s == 16 || s == 32 || s == 64; }
 
-bool shape_ok(int n, int k, int b) {
-  return valid_b(b) && n > 0 && k > 0 && n <= MAX_DIM && k <= MAX_DIM && n % b == 0 && k % b == 0;
+bool shape_ok(int n, int k, int bn, int bk) {
+  return valid_side(bn) && valid_side(bk) && n > 0 && k > 0 && n <= MAX_DIM && k <= MAX_DIM && n % bn == 0 &&
+         k % bk == 0;
 }
 
 int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
@@ -92,11 +94,11 @@ struct WsLayout {
   size_t tickets_off, partials_off, total;
 };
 
-WsLayout ws_layout(int64_t m, int n, int k, int b, int sms) {
+WsLayout ws_layout(int64_t m, int n, int k, int bk, int sms) {
   WsLayout L;
   const int64_t n_tt = ceil_div(m, TOKENS_PER_TILE);
   const int ng = (int)ceil_div(n, GROUP_FEATURES);
-  const int kb = k / b;
+  const int kb = k / bk;
   const int S = choose_slice(n_tt, ng, kb, sms);
   L.tickets_off = sizeof(Control);
   size_t off = L.tickets_off + (size_t)ceil_div(n_tt * ng * 4, 256) * 256;
@@ -113,9 +115,9 @@ bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) %
 lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias, void *Y,
                         int64_t ldy, lpvit_dtype y_dtype, void *workspace, size_t ws_bytes, void *stream, int gelu) {
   if (!bsr) return LPVIT_ERR_INVALID_ARG;
-  const int n = bsr->n, k = bsr->k, b = bsr->b;
-  if (!valid_b(b)) return LPVIT_ERR_UNSUPPORTED;
-  if (!shape_ok(n, k, b)) return LPVIT_ERR_INVALID_ARG;
+  const int n = bsr->n, k = bsr->k, bn = bsr->bn, bk = bsr->bk;
+  if (!valid_side(bn) || !valid_side(bk)) return LPVIT_ERR_UNSUPPORTED;
+  if (!shape_ok(n, k, bn, bk)) return LPVIT_ERR_INVALID_ARG;
   if (m < 0) return LPVIT_ERR_INVALID_ARG;
   if (y_dtype != LPVIT_BF16 && y_dtype != LPVIT_F32) return LPVIT_ERR_INVALID_ARG;
   if (m == 0) return LPVIT_OK;
@@ -133,22 +135,22 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
     const uintptr_t y0 = reinterpret_cast<uintptr_t>(Y), y1 = y0 + (size_t)((m - 1) * ldy + n) * ysz;
     if (x0 < y1 && y0 < x1) return LPVIT_ERR_INVALID_ARG;
   }
-  if (bsr->sched_bytes < lpvit_sched_bytes(n, k, b)) return LPVIT_ERR_WORKSPACE;
+  if (bsr->sched_bytes < lpvit_sched_bytes(n, k, bn, bk)) return LPVIT_ERR_WORKSPACE;
   int sms = 0;
   lpvit_status st = LPVIT_OK;
   if (!device_info(&sms, &st)) return st;
-  const WsLayout W = ws_layout(m, n, k, b, sms);
+  const WsLayout W = ws_layout(m, n, k, bk, sms);
   if (ws_bytes < W.total) return LPVIT_ERR_WORKSPACE;
   EncodeTiledFn enc = encode_fn();
   if (!enc) return LPVIT_ERR_CUDA;
 
   const CUtensorMapSwizzle swz =
-      b == 16 ? CU_TENSOR_MAP_SWIZZLE_32B : (b == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
+      bk == 16 ? CU_TENSOR_MAP_SWIZZLE_32B : (bk == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
   CUtensorMap tmX;
   {
     cuuint64_t dims[2] = {(cuuint64_t)k, (cuuint64_t)m};
     cuuint64_t strides[1] = {(cuuint64_t)ldx * 2};
-    cuuint32_t box[2] = {(cuuint32_t)b, (cuuint32_t)TOKENS_PER_TILE};
+    cuuint32_t box[2] = {(cuuint32_t)bk, (cuuint32_t)TOKENS_PER_TILE};
     cuuint32_t es[2] = {1, 1};
     if (enc(&tmX, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(X), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -158,8 +160,8 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   LinearParams P;
   const int ng = (int)ceil_div(n, GROUP_FEATURES);
   P.sched = static_cast<const int32_t *>(bsr->sched);
-  P.wstream = static_cast<const uint8_t *>(bsr->sched) + sched_stream_offset_bytes(ng, k / b);
-  P.stream_tiles = sched_stream_tiles(ng, k / b, b);
+  P.wstream = static_cast<const uint8_t *>(bsr->sched) + sched_stream_offset_bytes(ng, k / bk);
+  P.stream_tiles = sched_stream_tiles(ng, k / bk);
   P.bias = bias;
   P.Y = Y;
   P.ldy = ldy;
@@ -168,7 +170,7 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.k = k;
   P.n_tt = (int)ceil_div(m, TOKENS_PER_TILE);
   P.n_groups = ng;
-  P.S = choose_slice(P.n_tt, P.n_groups, k / b, sms);
+  P.S = choose_slice(P.n_tt, P.n_groups, k / bk, sms);
   P.y_f32 = y_dtype == LPVIT_F32;
   P.gelu = gelu;
   P.y_vec16 = (aligned(Y, 16) && ldy % 8 == 0) ? 1 : 0;
@@ -177,23 +179,23 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.tickets = reinterpret_cast<int32_t *>(ws + W.tickets_off);
   P.partials = reinterpret_cast<float *>(ws + W.partials_off);
   P.timeout_ns = TIMEOUT_NS;
-  const int64_t units_max = (int64_t)P.n_tt * P.n_groups * ceil_div(k / b, P.S);
+  const int64_t units_max = (int64_t)P.n_tt * P.n_groups * ceil_div(k / bk, P.S);
   const int grid = (int)(units_max < sms ? units_max : sms);
-  return cuda_status(launch_linear(b, tmX, P, grid, static_cast<cudaStream_t>(stream)));
+  return cuda_status(launch_linear(bk, tmX, P, grid, static_cast<cudaStream_t>(stream)));
 }
 
 // The checks lpvit_pack_bsr applies to one weight.
 lpvit_status check_pack_args(const void *W, const uint8_t *mask, const lpvit_bsr *bsr) {
   if (!bsr) return LPVIT_ERR_INVALID_ARG;
-  const int n = bsr->n, k = bsr->k, b = bsr->b;
-  if (!valid_b(b)) return LPVIT_ERR_UNSUPPORTED;
-  if (!shape_ok(n, k, b)) return LPVIT_ERR_INVALID_ARG;
+  const int n = bsr->n, k = bsr->k, bn = bsr->bn, bk = bsr->bk;
+  if (!valid_side(bn) || !valid_side(bk)) return LPVIT_ERR_UNSUPPORTED;
+  if (!shape_ok(n, k, bn, bk)) return LPVIT_ERR_INVALID_ARG;
   if (!W || !mask || !bsr->row_ptr || !bsr->sched || bsr->nnzb_capacity < 0) return LPVIT_ERR_INVALID_ARG;
   if (bsr->nnzb_capacity > 0 && (!bsr->col_idx || !bsr->blocks)) return LPVIT_ERR_INVALID_ARG;
   if (!aligned(W, 16) || (bsr->blocks && !aligned(bsr->blocks, 16)) || !aligned(bsr->sched, 16) ||
       !aligned(bsr->row_ptr, 4) || (bsr->col_idx && !aligned(bsr->col_idx, 4)))
     return LPVIT_ERR_INVALID_ARG;
-  if (bsr->sched_bytes < lpvit_sched_bytes(n, k, b)) return LPVIT_ERR_WORKSPACE;
+  if (bsr->sched_bytes < lpvit_sched_bytes(n, k, bn, bk)) return LPVIT_ERR_WORKSPACE;
   return LPVIT_OK;
 }
 
@@ -204,27 +206,27 @@ using namespace lpvit;
 
 extern "C" {
 
-size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t b) {
-  if (!shape_ok(n, k, b)) return 0;
+size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t bn, int32_t bk) {
+  if (!shape_ok(n, k, bn, bk)) return 0;
   const int ng = (int)ceil_div(n, GROUP_FEATURES);
-  return (size_t)sched_stream_offset_bytes(ng, k / b) + (size_t)sched_stream_tiles(ng, k / b, b) * stream_tile_bytes(b);
+  return (size_t)sched_stream_offset_bytes(ng, k / bk) + (size_t)sched_stream_tiles(ng, k / bk) * stream_tile_bytes(bk);
 }
 
 
 lpvit_status lpvit_pack_bsr(const void *W, const uint8_t *mask, lpvit_bsr *bsr, int32_t *nnzb_host, void *stream) {
   const lpvit_status chk = check_pack_args(W, mask, bsr);
   if (chk != LPVIT_OK) return chk;
-  const int n = bsr->n, k = bsr->k, b = bsr->b;
+  const int n = bsr->n, k = bsr->k, bn = bsr->bn, bk = bsr->bk;
   int sms = 0;
   lpvit_status st = LPVIT_OK;
   if (!device_info(&sms, &st)) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cudaError_t e = launch_pack(W, mask, n, k, b, bsr->row_ptr, bsr->col_idx, bsr->nnzb_capacity, bsr->blocks,
+  cudaError_t e = launch_pack(W, mask, n, k, bn, bk, bsr->row_ptr, bsr->col_idx, bsr->nnzb_capacity, bsr->blocks,
                               static_cast<int32_t *>(bsr->sched), sms, s);
   if (e != cudaSuccess) return LPVIT_ERR_CUDA;
   if (nnzb_host) {
     int32_t v = 0;
-    e = cudaMemcpyAsync(&v, bsr->row_ptr + n / b, sizeof(v), cudaMemcpyDeviceToHost, s);
+    e = cudaMemcpyAsync(&v, bsr->row_ptr + n / bn, sizeof(v), cudaMemcpyDeviceToHost, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return LPVIT_ERR_CUDA;
     *nnzb_host = v;
@@ -256,18 +258,19 @@ lpvit_status lpvit_pack_bsr_many(int32_t count, const void *const *W, const uint
     j.sched = static_cast<int32_t *>(bsr[i].sched);
     j.n = bsr[i].n;
     j.k = bsr[i].k;
-    j.b = bsr[i].b;
+    j.bn = bsr[i].bn;
+    j.bk = bsr[i].bk;
     j.cap = bsr[i].nnzb_capacity;
   }
   return cuda_status(launch_pack_many(jobs.data(), count, sms, static_cast<cudaStream_t>(stream)));
 }
 
 size_t lpvit_workspace_bytes(const lpvit_bsr *bsr, int64_t m) {
-  if (!bsr || !shape_ok(bsr->n, bsr->k, bsr->b) || m < 0) return 0;
+  if (!bsr || !shape_ok(bsr->n, bsr->k, bsr->bn, bsr->bk) || m < 0) return 0;
   int sms = 0;
   lpvit_status st = LPVIT_OK;
   if (!device_info(&sms, &st)) sms = 152;  // sizing only; the call itself reports the device error
-  return ws_layout(m > 0 ? m : 1, bsr->n, bsr->k, bsr->b, sms).total;
+  return ws_layout(m > 0 ? m : 1, bsr->n, bsr->k, bsr->bk, sms).total;
 }
 
 lpvit_status lpvit_bsr_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias,
@@ -301,7 +304,7 @@ const char *lpvit_status_string(lpvit_status status) {
   switch (status) {
     case LPVIT_OK: return "ok";
     case LPVIT_ERR_INVALID_ARG: return "invalid argument (shape, null or misaligned pointer or stride)";
-    case LPVIT_ERR_UNSUPPORTED: return "unsupported (block size not 16/32/64, or device is not sm_103)";
+    case LPVIT_ERR_UNSUPPORTED: return "unsupported (a block side not 16/32/64, or device is not sm_103)";
     case LPVIT_ERR_CUDA: return "CUDA runtime or driver error";
     case LPVIT_ERR_TIMEOUT: return "a device-side bounded wait ran out; the output is incomplete";
     case LPVIT_ERR_WORKSPACE: return "workspace, schedule buffer or block capacity too small";

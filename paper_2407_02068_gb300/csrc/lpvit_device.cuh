@@ -8,18 +8,19 @@
 
 namespace lpvit {
 
-// Layout of the work list ("sched") shared by the pack and the GEMM.
-// header (16 int32): [0] nnzb, [1] n_groups, [2] total entries, [3] overflow flag, [4] n, [5] k, [6] b
+// Layout of the work list ("sched") shared by the pack and the GEMM, for blocks of bn output rows
+// by bk input columns.
+// header (16 int32): [0] nnzb, [1] n_groups, [2] total entries, [3] overflow flag, [4] n, [5] k,
+// [6] bn, [7] bk
 // then gent_ptr[n_groups + 1] (int32, entries of group g are [gent_ptr[g], gent_ptr[g+1]))
 // then entries, ENTRY_INTS int32 each: [0] = j | (row-panel mask << 16), [1 + p] = block index of
-// the group's p-th row panel at block column j, or -1 (p < GROUP_FEATURES / b <= 8),
-// [ENTRY_TILE_WORD] = index of the entry's first tile in the weight stream;
+// the group's p-th row panel at block column j, or -1 (p < GROUP_FEATURES / bn <= 8),
+// [ENTRY_TILE_WORD] = index of the entry's tile in the weight stream (the entry's own index);
 // then, at sched_stream_offset_bytes (1024-byte aligned), the weight stream: for every entry in
-// order, one tile per MMA panel of the group that keeps a block at column j (ascending panel
-// order; with MP = 128 that is exactly one tile per entry). A tile is W[g*128 + q*MP + r][j*b + c]
-// for r < MP, c < b (MP = mma_panel_rows(b)), with the rows of removed row panels zero, stored as
-// MP rows of 2b bytes whose 16-byte chunks are permuted by stream_chunk_swizzle: the arrangement
-// the MMA's shared-memory descriptor reads, so that one bulk copy moves all of an entry's weights.
+// order, the group's tile at column j: W[g*128 + r][j*bk + c] for r < 128, c < bk, with the rows of
+// the row panels that keep no block there zero, stored as 128 rows of 2*bk bytes whose 16-byte
+// chunks are permuted by stream_chunk_swizzle: the arrangement the MMA's shared-memory descriptor
+// reads, so that one bulk copy moves an entry's weights.
 constexpr int SCHED_HDR_INTS = 16;
 constexpr int ENTRY_INTS = 12;
 constexpr int ENTRY_TILE_WORD = 9;
@@ -35,32 +36,18 @@ __host__ __device__ inline int64_t sched_stream_offset_bytes(int n_groups, int k
   const int64_t end = 4 * (sched_entries_offset_ints(n_groups) + (int64_t)n_groups * kb * ENTRY_INTS);
   return (end + 1023) / 1024 * 1024;
 }
-// Output features per MMA (its M): the whole 128-feature group, so that one MMA per 16-wide k step
-// covers every row panel of the group (those without a block at the column contribute zero rows)
-// and the X chunk it reads from shared memory serves all 128 features.
-__host__ __device__ constexpr int mma_panel_rows(int b) { return b > 0 ? GROUP_FEATURES : 0; }
-__host__ __device__ constexpr int stream_tile_bytes(int b) { return mma_panel_rows(b) * b * 2; }
-// Tiles the stream region holds: every MMA panel of every group at every block column.
-__host__ __device__ inline int64_t sched_stream_tiles(int n_groups, int kb, int b) {
-  return (int64_t)n_groups * kb * (GROUP_FEATURES / mma_panel_rows(b));
-}
+// One MMA's M is the whole 128-feature group: one MMA per 16-wide k step covers every row panel of
+// the group (those without a block at the column contribute zero rows), and the X chunk it reads
+// from shared memory serves all 128 features. A stream tile is that group's rows at one column.
+__host__ __device__ constexpr int stream_tile_bytes(int bk) { return GROUP_FEATURES * bk * 2; }
+// Tiles the stream region holds: one per group and block column (the most entries there can be).
+__host__ __device__ inline int64_t sched_stream_tiles(int n_groups, int kb) { return (int64_t)n_groups * kb; }
 // Position of 16-byte chunk c in tile row r (rows of row_bytes = 32, 64 or 128 bytes): c XOR the
 // row's address bits 7.. above the chunk bits, i.e. the 32/64/128-byte TMA swizzle of a tile
 // placed at a 1024-byte aligned shared-memory address.
 __host__ __device__ constexpr int stream_chunk_swizzle(int r, int row_bytes) {
   return ((r * row_bytes) >> 7) & (row_bytes / 16 - 1);
 }
-// MMA-panel mask of an entry from its row-panel mask (MMA panel q covers row panels
-// [q*PPM, (q+1)*PPM), PPM = mma_panel_rows(b) / b).
-__host__ __device__ inline uint32_t mma_panel_mask(uint32_t pm, int b) {
-  const int ppm = mma_panel_rows(b) / b;
-  if (ppm == 1) return pm;
-  const uint32_t pair = (1u << ppm) - 1u;
-  uint32_t mm = 0;
-  for (int q = 0; q * ppm < MAX_GROUP_PANELS; ++q) mm |= ((pm >> (ppm * q)) & pair) ? (1u << q) : 0u;
-  return mm;
-}
-
 static_assert(GROUP_FEATURES / 16 <= MAX_GROUP_PANELS, "entry holds every row panel of a group");
 static_assert(1 + MAX_GROUP_PANELS <= ENTRY_TILE_WORD && ENTRY_TILE_WORD < ENTRY_INTS, "entry size");
 
@@ -107,8 +94,8 @@ enum ErrBits : unsigned int {
 };
 
 // Launchers (host side, defined next to their kernels).
-cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int b, int32_t *row_ptr, int32_t *col_idx,
-                        int cap, void *blocks, int32_t *sched, int num_sms, cudaStream_t s);
+cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int bn, int bk, int32_t *row_ptr,
+                        int32_t *col_idx, int cap, void *blocks, int32_t *sched, int num_sms, cudaStream_t s);
 
 // One weight of a batched pack; the whole table travels in the kernel parameters.
 struct PackJob {
@@ -118,7 +105,7 @@ struct PackJob {
   int32_t *col_idx;
   uint16_t *blocks;
   int32_t *sched;
-  int n, k, b, cap;
+  int n, k, bn, bk, cap;
 };
 constexpr int PACK_MAX_JOBS = 96;  // jobs per launch (6 KB of parameters)
 struct PackJobs {
@@ -126,7 +113,7 @@ struct PackJobs {
   PackJob job[PACK_MAX_JOBS];
 };
 cudaError_t launch_pack_many(const PackJob *jobs, int count, int num_sms, cudaStream_t s);
-cudaError_t launch_linear(int b, const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s);
+cudaError_t launch_linear(int bk, const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s);
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 

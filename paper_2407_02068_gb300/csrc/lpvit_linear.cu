@@ -1,11 +1,12 @@
 // Block-sparse linear Y = act(X W~^T + bias) on sm_103a (Sec. 3.1 block mask, Sec. 3.3
 // block-sparse matmul: one block matmul per kept block and token tile, nothing for removed
-// blocks).
+// blocks). The kernel is compiled per block width BK (input columns of a block: 16, 32 or 64);
+// the block height only decides which rows of a group tile the pack left zero.
 //
 // Work unit = 256 tokens x one 128-feature group of row panels (x one slice of the group's block
 // columns when the problem is too small to fill the GPU). Per CTA (one per SM, persistent):
 //   warp 0      producer: takes units from a global atomic queue, walks the unit's work-list
-//               entries and, per entry (one block column j), loads the X tile [256 tokens x b]
+//               entries and, per entry (one block column j), loads the X tile [256 tokens x bk]
 //               (TMA tensor copy) and the entry's weight tiles, one per MMA panel keeping a block
 //               at column j, stored back to back in the work list's weight stream (one bulk copy).
 //   warp 1      MMA issuer: per entry and per 16-wide k step, one tcgen05 MMA (M = 128, N = 256,
@@ -27,16 +28,15 @@
 
 namespace lpvit {
 
-template <int B>
+template <int BK>
 struct Cfg {
-  static constexpr int MP = mma_panel_rows(B);              // MMA M: the group's 128 features
-  static constexpr int PPM = MP / B;                        // BSR row panels per MMA tile
-  static constexpr int KSTEPS = B / 16;                     // 16-wide k steps per block column
-  static constexpr int ROW_BYTES = B * 2;                   // bytes of one tile row (bf16)
+  static constexpr int MP = GROUP_FEATURES;                 // MMA M: the group's 128 features
+  static constexpr int KSTEPS = BK / 16;                    // 16-wide k steps per block column
+  static constexpr int ROW_BYTES = BK * 2;                  // bytes of one tile row (bf16)
   static constexpr int TT = TOKENS_PER_TILE;                // MMA N: tokens per unit
   static constexpr int BUF_COLS = TT;                       // TMEM columns per accumulator buffer
-  static constexpr int X_BYTES = TT * ROW_BYTES;            // X tile [256 x b]
-  static constexpr int A_BYTES = MP * ROW_BYTES;            // W tile [128 x b]
+  static constexpr int X_BYTES = TT * ROW_BYTES;            // X tile [256 x bk]
+  static constexpr int A_BYTES = MP * ROW_BYTES;            // W tile [128 x bk]
   static constexpr int STAGE_BYTES = X_BYTES + A_BYTES;
   static constexpr int NSTAGES = 196608 / STAGE_BYTES;      // 192 KB of stages
   static constexpr int UR = 4;                              // unit-info ring depth
@@ -44,7 +44,7 @@ struct Cfg {
   static constexpr int OPS = 2;                             // lane slots per entry: X tile, W tile
   static constexpr int NBMAX = BATCH < 32 / OPS ? BATCH : 32 / OPS;  // entries per batch
   static constexpr uint32_t IDESC = idesc_bf16(MP, TT);
-  static_assert(MP == GROUP_FEATURES && A_BYTES == stream_tile_bytes(B), "weight-stream tile geometry");
+  static_assert(A_BYTES == stream_tile_bytes(BK), "weight-stream tile geometry");
   static_assert(2 * BUF_COLS == 512, "two accumulator buffers fill the 512 TMEM columns");
   static_assert(NSTAGES >= 4, "pipeline depth");
   static_assert(X_BYTES % 1024 == 0 && A_BYTES % 1024 == 0, "tiles stay on their swizzle alignment");
@@ -62,11 +62,11 @@ struct UnitInfo {
 };
 
 
-template <int B>
+template <int BK>
 struct Smem {
   // stages first (1024-byte aligned), then the control area
-  static constexpr int CTRL_OFF = Cfg<B>::NSTAGES * Cfg<B>::STAGE_BYTES;
-  static constexpr int NS = Cfg<B>::NSTAGES, UR = Cfg<B>::UR;
+  static constexpr int CTRL_OFF = Cfg<BK>::NSTAGES * Cfg<BK>::STAGE_BYTES;
+  static constexpr int NS = Cfg<BK>::NSTAGES, UR = Cfg<BK>::UR;
   static constexpr int BAR_OFF = CTRL_OFF;
   // barriers: full[NS], empty[NS], accf[2], acce[2], unitf[UR], unite[UR], drain, episync
   static constexpr int NBARS = 2 * NS + 4 + 2 * UR + 2;
@@ -144,9 +144,9 @@ __device__ __forceinline__ void emit32(float (&y)[32], int f0, int64_t tok_base,
 
 // The MMAs of one work-list entry, issued by one elected thread: for every 16-wide k step,
 // D[128 x 256] (+)= W_tile[128 x 16] * X_tile[256 x 16]^T, both tiles in the stage (X first).
-template <int B>
+template <int BK>
 __device__ __forceinline__ void issue_entry(uint32_t st_u32, uint32_t dbase, uint32_t accumulate) {
-  using C = Cfg<B>;
+  using C = Cfg<BK>;
 #pragma unroll
   for (int kk = 0; kk < C::KSTEPS; ++kk) {
     const uint64_t bdesc = smem_desc<C::ROW_BYTES>(st_u32 + kk * 32);
@@ -155,11 +155,11 @@ __device__ __forceinline__ void issue_entry(uint32_t st_u32, uint32_t dbase, uin
   }
 }
 
-template <int B>
+template <int BK>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
 bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P) {
-  using C = Cfg<B>;
-  using L = Smem<B>;
+  using C = Cfg<BK>;
+  using L = Smem<BK>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t smem_base = smem_u32(smem);
@@ -212,7 +212,9 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0 && lane == 0) prefetch_tensormap(&tmX);
-  const bool sched_ok = P.sched[3] == 0 && P.sched[1] == P.n_groups;
+  // the work list must be this weight's plan: group count, shape and block width
+  const bool sched_ok = P.sched[3] == 0 && P.sched[1] == P.n_groups && P.sched[4] == P.n && P.sched[5] == P.k &&
+                        P.sched[7] == BK;
   if (warp == 2) {
     // slices per group = max(1, ceil(entries / S)); exclusive prefix into slice_ptr
     int run = 0;
@@ -314,7 +316,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
           const int src = min(i + k2, 31);
           const int wk = __shfl_sync(0xffffffffu, w0, src);
           const int tk = __shfl_sync(0xffffffffu, toff, src);
-          uint32_t mm = mma_panel_mask((uint32_t)wk >> 16, B) & 1u;
+          uint32_t mm = ((uint32_t)wk >> 16) != 0u ? 1u : 0u;  // the entry keeps a block of the group
           // a tile range outside the stream region means a corrupt work list: flag it, load no weights
           const bool tiles_ok = tk >= 0 && (int64_t)tk + __popc(mm) <= P.stream_tiles;
           if (!tiles_ok) mm = 0;
@@ -328,7 +330,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
           __syncwarp();
           if (k2 < nb) {
             if ((lane & 1) == 0)
-              tma_load_2d(st_u32, &tmX, (wk & 0xffff) * B, tt * C::TT, full_bar(stk));
+              tma_load_2d(st_u32, &tmX, (wk & 0xffff) * BK, tt * C::TT, full_bar(stk));
             else if (mm)
               bulk_load(st_u32 + C::X_BYTES, P.wstream + (int64_t)tk * C::A_BYTES, __popc(mm) * C::A_BYTES,
                         full_bar(stk));
@@ -390,7 +392,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
         const uint32_t st_u32 = smem_base + stage * C::STAGE_BYTES;
         if (mm) {
           if (elect_one()) {
-            issue_entry<B>(st_u32, dbase, touched);
+            issue_entry<BK>(st_u32, dbase, touched);
             tc_commit(empty_bar(stage));
           }
         } else {
@@ -530,26 +532,26 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
 
 // ------------------------------------------------------------------------------------ host side
 
-template <int B>
-int smem_bytes() { return Smem<B>::BYTES; }
+template <int BK>
+int smem_bytes() { return Smem<BK>::BYTES; }
 
-template <int B>
+template <int BK>
 cudaError_t launch_linear_t(const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s) {
   static bool attr_done[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(bsr_linear_kernel<B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         Smem<B>::BYTES);
+    cudaError_t e = cudaFuncSetAttribute(bsr_linear_kernel<BK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         Smem<BK>::BYTES);
     if (e != cudaSuccess) return e;
     attr_done[dev] = true;
   }
-  bsr_linear_kernel<B><<<grid, NUM_THREADS, Smem<B>::BYTES, s>>>(tmX, P);
+  bsr_linear_kernel<BK><<<grid, NUM_THREADS, Smem<BK>::BYTES, s>>>(tmX, P);
   return cudaGetLastError();
 }
 
-cudaError_t launch_linear(int b, const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s) {
-  switch (b) {
+cudaError_t launch_linear(int bk, const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s) {
+  switch (bk) {
     case 16: return launch_linear_t<16>(tmX, P, grid, s);
     case 32: return launch_linear_t<32>(tmX, P, grid, s);
     case 64: return launch_linear_t<64>(tmX, P, grid, s);

@@ -1,16 +1,16 @@
 // Mask -> BSR pack and work-list build (Sec. 3.1 block mask; Sec. 1 / Sec. 3.3: only the kept
 // blocks are stored, moved and multiplied).
 //
-// plan kernel (one CTA): per row panel r, cnt[r] = number of kept blocks (warp reductions);
-//   row_ptr = exclusive prefix sum of cnt (warp-shuffle scan + a scan of warp totals);
-//   col_idx = kept block columns of each panel in ascending order (ballot compaction);
+// Blocks are bn output rows by bk input columns (Sec. 3.1 mask over B_n x B_k blocks).
+// plan kernel (one CTA): per row panel r (bn rows), cnt[r] = number of kept blocks (warp
+//   reductions); row_ptr = exclusive prefix sum of cnt (warp-shuffle scan + a scan of warp
+//   totals); col_idx = kept block columns of each panel in ascending order (ballot compaction);
 //   work list: panels are grouped 128 output features at a time; for every group, one entry per
 //   block column where any panel of the group keeps a block, with that column's block index in
-//   each panel (or -1) and the index of its first tile in the weight stream (an exclusive scan of
-//   the entries' MMA-panel counts). The GEMM walks these entries.
-// copy kernel (grid-stride): blocks[t] = W[r*b:(r+1)*b, j*b:(j+1)*b], 16-byte vector copies, bits
-//   unchanged; then the weight stream, the same bits once more, entry by entry in the tiles the
-//   GEMM's MMAs read (rows of removed row panels zero, 16-byte chunks swizzled).
+//   each panel (or -1). The GEMM walks these entries.
+// copy kernel (grid-stride): blocks[t] = W[r*bn:(r+1)*bn, j*bk:(j+1)*bk], 16-byte vector copies,
+//   bits unchanged; then the weight stream, the same bits once more, entry by entry as the 128-row
+//   group tiles the GEMM's MMAs read (rows of removed row panels zero, 16-byte chunks swizzled).
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -61,17 +61,15 @@ __device__ int block_exclusive_scan(int *v, int count, int *warp_tot) {
 }
 
 // The plan of one weight, computed by one CTA of PLAN_THREADS threads (plan_smem: plan_smem_bytes).
-__device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int n, int k, int b,
+__device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int n, int k, int bn, int bk,
                                           int32_t *__restrict__ row_ptr, int32_t *__restrict__ col_idx, int cap,
                                           int32_t *__restrict__ sched, int *plan_smem) {
-  const int np = n / b, kb = k / b;
-  const int gb = GROUP_FEATURES / b;  // row panels per group
+  const int np = n / bn, kb = k / bk;
+  const int gb = GROUP_FEATURES / bn;  // row panels per group
   const int ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
-  const int ppm = mma_panel_rows(b) / b;  // row panels per MMA panel
   int *cnt = plan_smem;            // [np + 1]
   int *gcnt = cnt + np + 1;        // [ng + 1]
-  int *gtile = gcnt + ng + 1;      // [ng + 1]
-  int *warp_tot = gtile + ng + 1;  // [33]
+  int *warp_tot = gcnt + ng + 1;   // [33]
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const unsigned lt = (1u << lane) - 1u;
 
@@ -106,34 +104,23 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
       run += __popc(bal);
     }
   }
-  // 4a. entries per group (block columns where any panel of the group keeps a block) and stream
-  //     tiles per group (MMA panels keeping a block, summed over those columns)
+  // 4a. entries per group: block columns where any panel of the group keeps a block
   for (int g = warp; g < ng; g += PLAN_WARPS) {
-    int c = 0, t = 0;
+    int c = 0;
     for (int base = 0; base < kb; base += 32) {
       const int j = base + lane;
-      unsigned any = 0, qany = 0;
+      unsigned any = 0;
       for (int p = 0; p < gb; ++p) {
         const int r = g * gb + p;
         const bool keep = r < np && j < kb && mask[(int64_t)r * kb + j] != 0;
-        const unsigned bal = __ballot_sync(0xffffffffu, keep);
-        any |= bal;
-        qany |= bal;
-        if (p % ppm == ppm - 1) {
-          t += __popc(qany);
-          qany = 0;
-        }
+        any |= __ballot_sync(0xffffffffu, keep);
       }
       c += __popc(any);
     }
-    if (lane == 0) {
-      gcnt[g] = c;
-      gtile[g] = t;
-    }
+    if (lane == 0) gcnt[g] = c;
   }
   __syncthreads();
   const int total_entries = block_exclusive_scan(gcnt, ng, warp_tot);
-  block_exclusive_scan(gtile, ng, warp_tot);
   int32_t *gent = sched + SCHED_HDR_INTS;
   int32_t *entries = sched + sched_entries_offset_ints(ng);
   for (int g = tid; g < ng; g += PLAN_THREADS) gent[g] = gcnt[g];
@@ -145,14 +132,14 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
     sched[3] = nnzb > cap ? 1 : 0;
     sched[4] = n;
     sched[5] = k;
-    sched[6] = b;
-    for (int i = 7; i < SCHED_HDR_INTS; ++i) sched[i] = 0;
+    sched[6] = bn;
+    sched[7] = bk;
+    for (int i = 8; i < SCHED_HDR_INTS; ++i) sched[i] = 0;
   }
   // 4b. entries: j | (panel mask << 16), then the block index of each panel of the group (or -1),
-  //     then the first stream tile
+  //     then the entry's stream tile (its own index)
   for (int g = warp; g < ng; g += PLAN_WARPS) {
     int e_run = gcnt[g];
-    int t_run = gtile[g];
     int p_run[MAX_GROUP_PANELS];
 #pragma unroll
     for (int p = 0; p < MAX_GROUP_PANELS; ++p) p_run[p] = (p < gb && g * gb + p < np) ? cnt[g * gb + p] : 0;
@@ -170,16 +157,9 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
       unsigned pm = 0;
 #pragma unroll
       for (int p = 0; p < MAX_GROUP_PANELS; ++p) pm |= ((bal[p] >> lane) & 1u) << p;
-      // this lane's stream tiles, and the exclusive prefix over the lanes before it
-      const int tc = __popc(mma_panel_mask(pm, b));
-      int tincl = tc;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int v = __shfl_up_sync(0xffffffffu, tincl, o);
-        if (lane >= o) tincl += v;
-      }
       if ((any >> lane) & 1u) {
-        int32_t *e = entries + (int64_t)(e_run + __popc(any & lt)) * ENTRY_INTS;
+        const int ei = e_run + __popc(any & lt);
+        int32_t *e = entries + (int64_t)ei * ENTRY_INTS;
 #pragma unroll
         for (int p = 0; p < MAX_GROUP_PANELS; ++p) {
           const bool keep = (bal[p] >> lane) & 1u;
@@ -188,10 +168,9 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
         e[0] = (int32_t)((unsigned)j | (pm << 16));
 #pragma unroll
         for (int q = 1 + MAX_GROUP_PANELS; q < ENTRY_INTS; ++q) e[q] = 0;
-        e[ENTRY_TILE_WORD] = t_run + tincl - tc;
+        e[ENTRY_TILE_WORD] = ei;
       }
       e_run += __popc(any);
-      t_run += __shfl_sync(0xffffffffu, tincl, 31);
 #pragma unroll
       for (int p = 0; p < MAX_GROUP_PANELS; ++p) p_run[p] += __popc(bal[p]);
     }
@@ -199,27 +178,27 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
 }
 
 __global__ void __launch_bounds__(PLAN_THREADS, 1)
-plan_kernel(const uint8_t *__restrict__ mask, int n, int k, int b, int32_t *__restrict__ row_ptr,
+plan_kernel(const uint8_t *__restrict__ mask, int n, int k, int bn, int bk, int32_t *__restrict__ row_ptr,
             int32_t *__restrict__ col_idx, int cap, int32_t *__restrict__ sched) {
   extern __shared__ int plan_smem[];
-  plan_body(mask, n, k, b, row_ptr, col_idx, cap, sched, plan_smem);
+  plan_body(mask, n, k, bn, bk, row_ptr, col_idx, cap, sched, plan_smem);
 }
 
 // Several weights at once: CTA j plans job j.
 __global__ void __launch_bounds__(PLAN_THREADS, 1) plan_many_kernel(const __grid_constant__ PackJobs J) {
   extern __shared__ int plan_smem[];
   const PackJob &w = J.job[blockIdx.x];
-  plan_body(w.mask, w.n, w.k, w.b, w.row_ptr, w.col_idx, w.cap, w.sched, plan_smem);
+  plan_body(w.mask, w.n, w.k, w.bn, w.bk, w.row_ptr, w.col_idx, w.cap, w.sched, plan_smem);
 }
 
 // Kept blocks t = cta, cta + ncta, ... of one weight.
-__device__ __forceinline__ void copy_body(const uint16_t *__restrict__ W, int n, int k, int b,
+__device__ __forceinline__ void copy_body(const uint16_t *__restrict__ W, int n, int k, int bn, int bk,
                                           const int32_t *__restrict__ row_ptr, const int32_t *__restrict__ col_idx,
                                           int cap, uint16_t *__restrict__ blocks, int cta, int ncta) {
-  const int np = n / b;
+  const int np = n / bn;
   const int nnzb = min(row_ptr[np], cap);
-  const int vec_per_row = b / 8;  // 16-byte vectors per block row
-  const int vecs = b * vec_per_row;
+  const int vec_per_row = bk / 8;  // 16-byte vectors per block row
+  const int vecs = bn * vec_per_row;
   for (int t = cta; t < nnzb; t += ncta) {
     int lo = 0, hi = np - 1;  // largest r with row_ptr[r] <= t (that panel holds block t)
     while (lo < hi) {
@@ -230,22 +209,22 @@ __device__ __forceinline__ void copy_body(const uint16_t *__restrict__ W, int n,
     const int r = lo, j = col_idx[t];
     for (int v = threadIdx.x; v < vecs; v += blockDim.x) {
       const int c = v / vec_per_row, cv = v - c * vec_per_row;
-      const int4 *src = reinterpret_cast<const int4 *>(W + ((int64_t)r * b + c) * k + (int64_t)j * b + cv * 8);
-      int4 *dst = reinterpret_cast<int4 *>(blocks + ((int64_t)t * b + c) * b + cv * 8);
+      const int4 *src = reinterpret_cast<const int4 *>(W + ((int64_t)r * bn + c) * k + (int64_t)j * bk + cv * 8);
+      int4 *dst = reinterpret_cast<int4 *>(blocks + ((int64_t)t * bn + c) * bk + cv * 8);
       *dst = __ldg(src);
     }
   }
 }
 
 // Weight-stream tiles of entries e = cta, cta + ncta, ... of one weight (after its plan).
-__device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int n, int k, int b,
+__device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int n, int k, int bn, int bk,
                                             const int32_t *__restrict__ sched, int cta, int ncta) {
-  const int kb = k / b, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
+  const int kb = k / bk, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
   if (sched[1] != ng || sched[3] != 0) return;  // not this shape's plan, or blocks overflowed
   const int total = sched[2];
-  const int mp = mma_panel_rows(b), row_bytes = 2 * b, cpr = row_bytes / 16, chunks = mp * cpr;
-  const int tile_bytes = stream_tile_bytes(b);
-  const int64_t max_tiles = sched_stream_tiles(ng, kb, b);
+  const int row_bytes = 2 * bk, cpr = row_bytes / 16, chunks = GROUP_FEATURES * cpr;
+  const int tile_bytes = stream_tile_bytes(bk);
+  const int64_t max_tiles = sched_stream_tiles(ng, kb);
   const int32_t *gent = sched + SCHED_HDR_INTS;
   const int32_t *ent = sched + sched_entries_offset_ints(ng);
   uint8_t *stream = reinterpret_cast<uint8_t *>(const_cast<int32_t *>(sched)) + sched_stream_offset_bytes(ng, kb);
@@ -260,59 +239,53 @@ __device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int 
     const int32_t *ep = ent + (int64_t)e * ENTRY_INTS;
     const int j = ep[0] & 0xffff;
     const uint32_t pm = (uint32_t)ep[0] >> 16;
-    const int toff = ep[ENTRY_TILE_WORD];
-    const uint32_t mm = mma_panel_mask(pm, b);
-    const int nt = __popc(mm);
-    if (j >= kb || toff < 0 || (int64_t)toff + nt > max_tiles) continue;
-    for (int v = threadIdx.x; v < nt * chunks; v += blockDim.x) {
-      const int i = v / chunks, ch = v - i * chunks;
-      uint32_t rest = mm;  // the i-th present MMA panel
-      for (int s2 = 0; s2 < i; ++s2) rest &= rest - 1u;
-      const int q = __ffs(rest) - 1;
-      const int r = ch / cpr, c = ch - r * cpr;
-      const int row = g * GROUP_FEATURES + q * mp + r;
+    const int t = ep[ENTRY_TILE_WORD];
+    if (j >= kb || t < 0 || (int64_t)t >= max_tiles) continue;
+    uint8_t *tile = stream + (int64_t)t * tile_bytes;
+    for (int v = threadIdx.x; v < chunks; v += blockDim.x) {
+      const int r = v / cpr, c = v - r * cpr;
+      const int row = g * GROUP_FEATURES + r;
       int4 val = make_int4(0, 0, 0, 0);
-      if (((pm >> ((q * mp + r) / b)) & 1u) && row < n)
-        val = __ldg(reinterpret_cast<const int4 *>(W + (int64_t)row * k + (int64_t)j * b + c * 8));
-      int4 *dst = reinterpret_cast<int4 *>(stream + (int64_t)(toff + i) * tile_bytes + r * row_bytes) +
-                  (c ^ stream_chunk_swizzle(r, row_bytes));
-      *dst = val;
+      if (((pm >> (r / bn)) & 1u) && row < n)
+        val = __ldg(reinterpret_cast<const int4 *>(W + (int64_t)row * k + (int64_t)j * bk + c * 8));
+      reinterpret_cast<int4 *>(tile + r * row_bytes)[c ^ stream_chunk_swizzle(r, row_bytes)] = val;
     }
   }
 }
 
 __global__ void __launch_bounds__(128)
-copy_blocks_kernel(const uint16_t *__restrict__ W, int n, int k, int b, const int32_t *__restrict__ row_ptr,
-                   const int32_t *__restrict__ col_idx, int cap, uint16_t *__restrict__ blocks,
-                   const int32_t *__restrict__ sched) {
-  copy_body(W, n, k, b, row_ptr, col_idx, cap, blocks, blockIdx.x, gridDim.x);
-  stream_body(W, n, k, b, sched, blockIdx.x, gridDim.x);
+copy_blocks_kernel(const uint16_t *__restrict__ W, int n, int k, int bn, int bk,
+                   const int32_t *__restrict__ row_ptr, const int32_t *__restrict__ col_idx, int cap,
+                   uint16_t *__restrict__ blocks, const int32_t *__restrict__ sched) {
+  copy_body(W, n, k, bn, bk, row_ptr, col_idx, cap, blocks, blockIdx.x, gridDim.x);
+  stream_body(W, n, k, bn, bk, sched, blockIdx.x, gridDim.x);
 }
 
 // Several weights at once: every CTA takes its share of every job's kept blocks and stream tiles.
 __global__ void __launch_bounds__(128) copy_many_kernel(const __grid_constant__ PackJobs J) {
   for (int j = 0; j < J.count; ++j) {
     const PackJob &w = J.job[j];
-    if (w.cap > 0) copy_body(w.W, w.n, w.k, w.b, w.row_ptr, w.col_idx, w.cap, w.blocks, blockIdx.x, gridDim.x);
-    stream_body(w.W, w.n, w.k, w.b, w.sched, blockIdx.x, gridDim.x);
+    if (w.cap > 0)
+      copy_body(w.W, w.n, w.k, w.bn, w.bk, w.row_ptr, w.col_idx, w.cap, w.blocks, blockIdx.x, gridDim.x);
+    stream_body(w.W, w.n, w.k, w.bn, w.bk, w.sched, blockIdx.x, gridDim.x);
   }
 }
 
-size_t plan_smem_bytes(int n, int b) {
-  const int np = n / b, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
-  return sizeof(int) * (size_t)(np + 1 + 2 * (ng + 1) + 33);
+size_t plan_smem_bytes(int n, int bn) {
+  const int np = n / bn, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
+  return sizeof(int) * (size_t)(np + 1 + ng + 1 + 33);
 }
 
-cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int b, int32_t *row_ptr, int32_t *col_idx,
-                        int cap, void *blocks, int32_t *sched, int num_sms, cudaStream_t s) {
-  const size_t smem = plan_smem_bytes(n, b);
-  plan_kernel<<<1, PLAN_THREADS, smem, s>>>(mask, n, k, b, row_ptr, col_idx, cap, sched);
+cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int bn, int bk, int32_t *row_ptr,
+                        int32_t *col_idx, int cap, void *blocks, int32_t *sched, int num_sms, cudaStream_t s) {
+  const size_t smem = plan_smem_bytes(n, bn);
+  plan_kernel<<<1, PLAN_THREADS, smem, s>>>(mask, n, k, bn, bk, row_ptr, col_idx, cap, sched);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const int max_blocks = (n / b) * (k / b);
+  const int max_blocks = (n / bn) * (k / bk);
   int grid = max_blocks < num_sms * 16 ? max_blocks : num_sms * 16;
   if (grid < 1) grid = 1;
-  copy_blocks_kernel<<<grid, 128, 0, s>>>(static_cast<const uint16_t *>(W), n, k, b, row_ptr, col_idx, cap,
+  copy_blocks_kernel<<<grid, 128, 0, s>>>(static_cast<const uint16_t *>(W), n, k, bn, bk, row_ptr, col_idx, cap,
                                          static_cast<uint16_t *>(blocks), sched);
   return cudaGetLastError();
 }
@@ -326,9 +299,9 @@ cudaError_t launch_pack_many(const PackJob *jobs, int count, int num_sms, cudaSt
     int64_t blocks_max = 0;
     for (int j = 0; j < J.count; ++j) {
       J.job[j] = jobs[first + j];
-      const size_t sj = plan_smem_bytes(J.job[j].n, J.job[j].b);
+      const size_t sj = plan_smem_bytes(J.job[j].n, J.job[j].bn);
       smem = sj > smem ? sj : smem;
-      blocks_max += (int64_t)(J.job[j].n / J.job[j].b) * (J.job[j].k / J.job[j].b);
+      blocks_max += (int64_t)(J.job[j].n / J.job[j].bn) * (J.job[j].k / J.job[j].bk);
     }
     if (smem > 48 * 1024) {
       int dev = 0;

@@ -66,9 +66,16 @@ def bias(n: int, s: int, device="cpu") -> torch.Tensor:
     return torch.randn(n, generator=_gen(s, device), device=device, dtype=torch.float32) * 0.02
 
 
-def uniform_mask(n: int, k: int, b: int, sparsity: float, s: int) -> torch.Tensor:
-    """[n/b, k/b] uint8 mask with exactly round(sparsity * nblocks) zero (pruned) blocks."""
-    nb, kb = n // b, k // b
+def block_sides(b) -> tuple[int, int]:
+    """A block given as b (b x b) or (bn, bk): bn output rows by bk input columns."""
+    return (int(b[0]), int(b[1])) if isinstance(b, (tuple, list)) else (int(b), int(b))
+
+
+def uniform_mask(n: int, k: int, b, sparsity: float, s: int) -> torch.Tensor:
+    """[n/bn, k/bk] uint8 mask with exactly round(sparsity * nblocks) zero (pruned) blocks
+    (b = int or (bn, bk))."""
+    bn, bk = block_sides(b)
+    nb, kb = n // bn, k // bk
     total = nb * kb
     npruned = min(total, max(0, round_half_away(sparsity * total)))
     perm = torch.randperm(total, generator=_gen(s))
@@ -109,10 +116,11 @@ def zipf_counts(panels: int, kb: int, keep_total: int, exponent: float, s: int) 
     return counts
 
 
-def zipf_mask(n: int, k: int, b: int, sparsity: float, s: int, exponent: float = 1.2) -> torch.Tensor:
-    """[n/b, k/b] uint8 mask whose per-panel kept-block counts follow ``zipf_counts``; each panel's
+def zipf_mask(n: int, k: int, b, sparsity: float, s: int, exponent: float = 1.2) -> torch.Tensor:
+    """[n/bn, k/bk] uint8 mask whose per-panel kept-block counts follow ``zipf_counts``; each panel's
     kept columns are a seeded random subset."""
-    nb, kb = n // b, k // b
+    bn, bk = block_sides(b)
+    nb, kb = n // bn, k // bk
     keep_total = round_half_away((1.0 - sparsity) * nb * kb)
     counts = zipf_counts(nb, kb, keep_total, exponent, s)
     g = _gen(s + 7919)
@@ -151,10 +159,10 @@ def deit_gemms(model: dict):
     return [("qkv", d, 3 * d, False), ("proj", d, d, False), ("fc1", d, h, True), ("fc2", h, d, False)]
 
 
-def make_gemm(config: int, gemm: int, m: int, k: int, n: int, b: int, sparsity: float, mask_kind="uniform",
+def make_gemm(config: int, gemm: int, m: int, k: int, n: int, b, sparsity: float, mask_kind="uniform",
               device="cpu", with_x: bool = True):
     """One seeded block-sparse linear: dict with X (bf16 [m,k] or None), W (bf16 [n,k]),
-    bias (fp32 [n]) and mask (uint8 [n/b, k/b])."""
+    bias (fp32 [n]) and mask (uint8 [n/bn, k/bk]); b = int (square) or (bn, bk)."""
     out = {
         "W": weight(n, k, seed(config, gemm, "W"), device),
         "bias": bias(n, seed(config, gemm, "bias"), device),

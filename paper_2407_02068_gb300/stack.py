@@ -60,16 +60,16 @@ class DeitLinearStack:
 
     # ------------------------------------------------------------------ accounting
     def effective_flops(self, rows: int | None = None) -> int:
-        """2 * rows * sum over GEMMs of (kept blocks) * b^2 (bias and GELU not counted)."""
+        """2 * rows * sum over GEMMs of (kept blocks) * bn * bk (bias and GELU not counted)."""
         r = self.m if rows is None else rows
-        return sum(2 * r * G["nnzb"] * G["w"].b ** 2 for G in self.gemms)
+        return sum(2 * r * G["nnzb"] * G["w"].bn * G["w"].bk for G in self.gemms)
 
     def algorithmic_bytes(self) -> int:
         """Per step of the linears: X read once, Y written once (bf16), kept blocks + indices + bias."""
         tot = 0
         for G in self.gemms:
-            n, k, b = G["w"].n, G["w"].k, G["w"].b
-            tot += 2 * self.m * k + 2 * self.m * n + 2 * G["nnzb"] * b * b + 4 * G["nnzb"] + 4 * (n // b + 1) + 4 * n
+            n, k, bn, bk = G["w"].n, G["w"].k, G["w"].bn, G["w"].bk
+            tot += 2 * self.m * k + 2 * self.m * n + 2 * G["nnzb"] * bn * bk + 4 * G["nnzb"] + 4 * (n // bn + 1) + 4 * n
         return tot
 
     def launches_per_step(self) -> int:
@@ -160,8 +160,8 @@ class DeitLinearStack:
         if not hasattr(self, "_dense"):
             self._dense = []
             for G in self.gemms:
-                b = G["w"].b
-                keep = G["mask"].repeat_interleave(b, 0).repeat_interleave(b, 1).bool()
+                bn, bk = G["w"].bn, G["w"].bk
+                keep = G["mask"].repeat_interleave(bn, 0).repeat_interleave(bk, 1).bool()
                 self._dense.append(torch.where(keep, G["W"], torch.zeros_like(G["W"])))
         F = torch.nn.functional
         h = h0

@@ -32,20 +32,28 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_sched_bytes_and_status_strings(lib):
-    assert lib.lpvit_sched_bytes(1152, 384, 32) > 0
-    assert lib.lpvit_sched_bytes(1152, 384, 24) == 0      # unsupported block size
-    assert lib.lpvit_sched_bytes(1000, 384, 32) == 0      # n not a multiple of b
+    assert lib.lpvit_sched_bytes(1152, 384, 32, 32) > 0
+    assert lib.lpvit_sched_bytes(1152, 384, 64, 32) > 0   # 64 rows x 32 columns
+    assert lib.lpvit_sched_bytes(1152, 384, 16, 32) == lib.lpvit_sched_bytes(1152, 384, 64, 32)  # bn: list only
+    assert lib.lpvit_sched_bytes(1152, 384, 24, 32) == 0  # unsupported block height
+    assert lib.lpvit_sched_bytes(1152, 384, 32, 24) == 0  # unsupported block width
+    assert lib.lpvit_sched_bytes(1000, 384, 32, 32) == 0  # n not a multiple of bn
+    assert lib.lpvit_sched_bytes(1152, 400, 64, 32) == 0  # k not a multiple of bk
     for st in range(6):
         assert lib.status_string(st)
 
 
 def test_bad_arguments_are_rejected_without_a_gpu(lib):
-    bsr = lib.lpvit_bsr(1152, 384, 32, 432, None, None, None, None, 0)
+    bsr = lib.lpvit_bsr(1152, 384, 32, 32, 432, None, None, None, None, 0)
     st, _ = lib.lpvit_pack_bsr(None, None, bsr, False, None)
     assert st == lib.LPVIT_ERR_INVALID_ARG
-    bad_b = lib.lpvit_bsr(1152, 384, 24, 432, None, None, None, None, 0)
+    bad_b = lib.lpvit_bsr(1152, 384, 24, 24, 432, None, None, None, None, 0)
     st, _ = lib.lpvit_pack_bsr(None, None, bad_b, False, None)
     assert st == lib.LPVIT_ERR_UNSUPPORTED
+    for bn, bk in ((64, 24), (8, 32), (128, 32)):
+        st, _ = lib.lpvit_pack_bsr(None, None, lib.lpvit_bsr(1152, 384, bn, bk, 432, None, None, None, None, 0),
+                                   False, None)
+        assert st == lib.LPVIT_ERR_UNSUPPORTED, (bn, bk)
     assert lib.lpvit_bsr_linear(bsr, None, 197, 384, None, None, 1152, 0, None, 0, None) == lib.LPVIT_ERR_INVALID_ARG
     assert lib.lpvit_bsr_linear(bsr, None, -1, 384, None, None, 1152, 0, None, 0, None) == lib.LPVIT_ERR_INVALID_ARG
     assert lib.lpvit_bsr_linear(bsr, None, 0, 384, None, None, 1152, 0, None, 0, None) == lib.LPVIT_OK  # empty
@@ -66,13 +74,16 @@ def test_bad_arguments_are_rejected_without_a_gpu(lib):
     assert lib.lpvit_pack_bsr_many([0x1000, 0], [0x2000, 0x2000], [bsr, bsr], None) == lib.LPVIT_ERR_INVALID_ARG
     # the Taylor block mask validates before launching anything
     tm = lib.lpvit_taylor_block_mask
-    assert tm(0x1000, 0x2000, 64, 64, 24, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_UNSUPPORTED
-    assert tm(0x1000, 0x2000, 64, 48, 32, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG   # k % b
+    assert tm(0x1000, 0x2000, 64, 64, 24, 24, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_UNSUPPORTED
+    assert tm(0x1000, 0x2000, 64, 64, 32, 24, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_UNSUPPORTED
+    assert tm(0x1000, 0x2000, 64, 48, 32, 32, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG   # k % bk
+    assert tm(0x1000, 0x2000, 96, 64, 64, 32, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG   # n % bn
     for bad_alpha in (-0.1, 1.5, float("nan")):
-        assert tm(0x1000, 0x2000, 64, 64, 32, bad_alpha, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG
-    assert tm(0, 0x2000, 64, 64, 32, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG
-    assert tm(0x1008, 0x2000, 64, 64, 32, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG     # W alignment
-    assert tm(0x1000, 0x2000, 65536, 65536, 16, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_UNSUPPORTED  # > 2^20
+        assert tm(0x1000, 0x2000, 64, 64, 32, 32, bad_alpha, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert tm(0, 0x2000, 64, 64, 32, 32, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert tm(0x1008, 0x2000, 64, 64, 32, 32, 0.5, 0x3000, 0x4000, None) == lib.LPVIT_ERR_INVALID_ARG  # W alignment
+    assert tm(0x1000, 0x2000, 65536, 65536, 16, 16, 0.5, 0x3000, 0x4000, None) == \
+        lib.LPVIT_ERR_UNSUPPORTED  # > 2^20 blocks
     # the wait self-test validates before launching anything
     assert lib.lpvit_selftest_wait(0, 10 ** 6, 0, None) == lib.LPVIT_ERR_INVALID_ARG          # no workspace
     assert lib.lpvit_selftest_wait(0x100010, 10 ** 6, 0, None) == lib.LPVIT_ERR_INVALID_ARG   # misaligned

@@ -6,6 +6,10 @@ test_gpu_stack.py): the CUDA path against the fp64 oracle on the same seeded inp
   3  DeiT-B fc1 + GELU and fc2 at batch 256 (M = 50432), 32x32 blocks, sparsity 0/30/50/70/80%.
   5  Zipf(1.2) row-panel imbalance at 60% on DeiT-B fc1 + GELU and fc2, 16x16 and 64x64 blocks,
      at batch 1024 (M = 201728) and batch 1 (M = 197).
+  7  The non-square blocks of Table 2, read in Sec. 3.3's notation (weight [N in x K out], block
+     B_n x B_k, so "64x32" spans 64 input columns and 32 output rows): DeiT-B fc1 + GELU, fc2, qkv
+     and proj at batch 256 with 32x64 (rows x columns) blocks, 61.5% sparse (38.5% of the FLOPs
+     remain), and the DeiT-S layer at batch 64 with "16x32" = 32x16 blocks, 28.7% sparse.
 
 Large cases are checked on a seeded sample of token rows plus the first and last token tiles;
 the gate is max|y - y_ref| / rms(y_ref) <= 1e-4 on fp32 output (the stated 1e-2 with margin).
@@ -61,7 +65,8 @@ def _run_and_check(lp, config, gemm, m, k, n, b, sparsity, gelu, mask_kind="unif
         gb = Yb[rows_t].float().cpu().double().numpy()
         # one bf16 ulp of the exact value plus the fp32 accumulation bound (k * 2^-24 * sum|x w|)
         Xd = oracle.bf16_to_f64(Xs)
-        Wd = oracle.bf16_to_f64(inputs.bf16_bits(g["W"])) * np.repeat(np.repeat(g["mask"].numpy(), b, 0), b, 1)
+        bn, bk = inputs.block_sides(b)
+        Wd = oracle.bf16_to_f64(inputs.bf16_bits(g["W"])) * np.repeat(np.repeat(g["mask"].numpy(), bn, 0), bk, 1)
         acc = k * 2.0 ** -24 * (np.abs(Xd) @ np.abs(Wd).T + np.abs(g["bias"].cpu().numpy()))
         ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.abs(ref), 2.0 ** -126))) - 7)
         assert np.all(np.abs(gb - ref) <= ulp + (1.13 if gelu else 1.0) * acc)
@@ -92,3 +97,15 @@ def test_config5_zipf_imbalance(lp, m, b, t):
     k, n, gelu = (768, 3072, True) if t == 0 else (3072, 768, False)
     gemm = t + 2 * (b == 64) + 4 * (m == 197)
     _run_and_check(lp, 5, gemm, m, k, n, b, 0.6, gelu, mask_kind="zipf")
+
+
+@pytest.mark.parametrize("gemm", [0, 1, 2, 3])
+def test_config7_table2_non_square_deit_b_64x32(lp, gemm):
+    name, k, n, gelu = inputs.deit_gemms(inputs.DEIT_B)[gemm]
+    _run_and_check(lp, 7, gemm, 256 * 197, k, n, (32, 64), 0.615, gelu)
+
+
+@pytest.mark.parametrize("gemm", [0, 1, 2, 3])
+def test_config7_table2_non_square_deit_s_16x32(lp, gemm):
+    name, k, n, gelu = inputs.deit_gemms(inputs.DEIT_S)[gemm]
+    _run_and_check(lp, 7, 4 + gemm, 64 * 197, k, n, (32, 16), 0.287, gelu, bf16_too=(gemm == 2))

@@ -16,6 +16,20 @@ pytestmark = pytest.mark.gpu
 NORM_TOL = 1e-2      # max|y - y_ref| / rms(y_ref), fp32 output
 TIGHT_TOL = 1e-4
 
+# blocks: b (square) or (bn rows, bk columns); Table 2 uses 32x32, 64x32, 16x32 and 16x16
+BLOCKS = [16, 32, 64, (64, 32), (16, 32)]
+BLOCKS_ALL = BLOCKS + [(32, 16), (32, 64), (16, 64), (64, 16)]
+
+
+def _sides(b):
+    return inputs.block_sides(b)
+
+
+def _sid(b):
+    """A seed offset per block (square blocks keep their historic b)."""
+    bn, bk = _sides(b)
+    return bn if bn == bk else 100 * bn + bk
+
 
 @pytest.fixture(scope="module")
 def lp():
@@ -49,7 +63,8 @@ def _ulp_bf16(x):
 
 def _acc_bound(X, W, mask, b, bias):
     """Bound on the fp32 accumulation error of any summation order: k * 2^-24 * sum_k |x w~|."""
-    keep = mask.repeat_interleave(b, 0).repeat_interleave(b, 1).bool()
+    bn, bk = _sides(b)
+    keep = mask.repeat_interleave(bn, 0).repeat_interleave(bk, 1).bool()
     Wa = torch.where(keep, W, torch.zeros_like(W)).double().abs().cpu()
     S = X.double().abs().cpu() @ Wa.T + bias.double().abs().cpu()
     return (W.shape[1] * 2.0 ** -24 * S).numpy()
@@ -82,7 +97,9 @@ def _case(m, n, k, b, sp, seed, device="cuda", int_valued=False, mask_kind="unif
 # ------------------------------------------------------------------------------------- pack
 
 @pytest.mark.parametrize("n,k,b,sp", [(1152, 384, 32, 0.5), (384, 1536, 16, 0.5), (768, 3072, 64, 0.3),
-                                      (3072, 768, 32, 0.0), (256, 256, 16, 1.0), (64, 48, 16, 0.4)])
+                                      (3072, 768, 32, 0.0), (256, 256, 16, 1.0), (64, 48, 16, 0.4),
+                                      (768, 3072, (64, 32), 0.6), (384, 1536, (16, 32), 0.3),
+                                      (192, 128, (32, 64), 0.5), (64, 96, (64, 16), 0.4)])
 def test_pack_bit_exact(lp, n, k, b, sp):
     X, W, bias, mask = _case(4, n, k, b, sp, 11)
     mask[0] = 0  # an empty panel
@@ -104,12 +121,15 @@ def _decode_sched(w):
     return raw[:16], gent, ent
 
 
-@pytest.mark.parametrize("n,k,b", [(1152, 384, 32), (384, 1536, 16), (768, 3072, 64), (200 * 16, 64, 16)])
+@pytest.mark.parametrize("n,k,b", [(1152, 384, 32), (384, 1536, 16), (768, 3072, 64), (200 * 16, 64, 16),
+                                   (768, 768, (64, 32)), (208, 384, (16, 32)), (320, 128, (64, 16))])
 def test_work_list_covers_every_kept_block_once(lp, n, k, b):
     X, W, bias, mask = _case(4, n, k, b, 0.55, 12)
     w = lp.pack_bsr(W, mask, b, count=True)
     hdr, gent, ent = _decode_sched(w)
-    gb = 128 // b
+    bn, bk = _sides(b)
+    assert (int(hdr[4]), int(hdr[5]), int(hdr[6]), int(hdr[7])) == (n, k, bn, bk)
+    gb = 128 // bn
     M = mask.cpu().numpy()
     rp, ci, _ = oracle.pack(_bits(W), M, b)
     seen = set()
@@ -122,10 +142,10 @@ def test_work_list_covers_every_kept_block_once(lp, n, k, b):
                 r = g * gb + p
                 if (pm >> p) & 1:
                     t = int(e[1 + p])
-                    assert r < n // b and M[r, j] and ci[t] == j and rp[r] <= t < rp[r + 1]
+                    assert r < n // bn and M[r, j] and ci[t] == j and rp[r] <= t < rp[r + 1]
                     seen.add(t)
                 else:
-                    assert e[1 + p] == -1 and (r >= n // b or not M[r, j])
+                    assert e[1 + p] == -1 and (r >= n // bn or not M[r, j])
         assert js == sorted(set(js))
         want = sorted(set(np.nonzero(M[g * gb:(g + 1) * gb].any(axis=0))[0].tolist()))
         assert js == want
@@ -136,11 +156,11 @@ def _check_weight_stream(w, W, mask):
     """The work list's weight stream: entry by entry, the 128-row tile of the entry's group at its
     block column (W's rows there, removed row panels zero), tiles contiguous in entry order,
     16-byte chunk c of tile row r stored at chunk c ^ ((r * rowbytes >> 7) & (rowbytes / 16 - 1))."""
-    n, k, b = w.n, w.k, w.b
+    n, k, bn, bk = w.n, w.k, w.bn, w.bk
     hdr, gent, ent = _decode_sched(w)
-    ng, kb = int(hdr[1]), k // b
+    ng, kb = int(hdr[1]), k // bk
     mp = 128
-    rb, cpr = 2 * b, 2 * b // 16
+    rb, cpr = 2 * bk, 2 * bk // 16
     raw = w.sched.cpu().numpy().view(np.uint8)
     ent_end = 4 * ((16 + ng + 1 + 3) // 4 * 4 + ng * kb * 12)
     stream = raw[(ent_end + 1023) // 1024 * 1024:]
@@ -151,22 +171,23 @@ def _check_weight_stream(w, W, mask):
         for e in ent[gent[g]:gent[g + 1]]:
             j, pm = int(e[0]) & 0xFFFF, (int(e[0]) >> 16) & 0xFFFF
             assert int(e[9]) == t_next
-            panels = [q for q in range(128 // mp) if any((pm >> ((q * mp + r) // b)) & 1 for r in range(0, mp, b))]
+            panels = [q for q in range(128 // mp) if any((pm >> ((q * mp + r) // bn)) & 1 for r in range(0, mp, bn))]
             for i, q in enumerate(panels):
                 tile = stream[(t_next + i) * mp * rb:(t_next + i + 1) * mp * rb].reshape(mp, cpr, 16)
                 for r in range(mp):
                     row = g * 128 + q * mp + r
-                    kept = (pm >> ((q * mp + r) // b)) & 1
-                    want = Wb[row, j * b:(j + 1) * b] if kept else np.zeros(b, np.uint16)
+                    kept = (pm >> ((q * mp + r) // bn)) & 1
+                    want = Wb[row, j * bk:(j + 1) * bk] if kept else np.zeros(bk, np.uint16)
                     if kept:
-                        assert M[row // b, j]
+                        assert M[row // bn, j]
                     sw = ((r * rb) >> 7) & (cpr - 1)
                     got = np.concatenate([tile[r, c ^ sw] for c in range(cpr)]).view(np.uint16)
                     assert np.array_equal(got, want), (g, j, q, r)
             t_next += len(panels)
 
 
-@pytest.mark.parametrize("n,k,b", [(384, 256, 32), (208, 128, 16), (384, 192, 64), (96, 64, 32)])
+@pytest.mark.parametrize("n,k,b", [(384, 256, 32), (208, 128, 16), (384, 192, 64), (96, 64, 32), (384, 128, (64, 32)),
+                                   (208, 128, (16, 32)), (192, 192, (32, 64))])
 def test_weight_stream_holds_every_entry_tile(lp, n, k, b):
     X, W, bias, mask = _case(4, n, k, b, 0.5, 31)
     w = lp.pack_bsr(W, mask, b, count=True)
@@ -206,11 +227,11 @@ def test_pack_many_matches_single_packs(lp, count):
 
 # ------------------------------------------------------------------------------------- GEMM
 
-@pytest.mark.parametrize("b", [16, 32, 64])
+@pytest.mark.parametrize("b", BLOCKS_ALL)
 @pytest.mark.parametrize("m", [1, 197, 300, 777])
 def test_linear_fp32_out(lp, b, m):
     n, k = 384, 256
-    X, W, bias, mask = _case(m, n, k, b, 0.5, 100 + b + m)
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 100 + _sid(b) + m)
     w = lp.pack_bsr(W, mask, b)
     Y = lp.bsr_linear(w, X, bias, out_dtype=torch.float32)
     ws = lp.workspace_for(w, m)
@@ -221,20 +242,20 @@ def test_linear_fp32_out(lp, b, m):
     assert err <= TIGHT_TOL
 
 
-@pytest.mark.parametrize("b", [16, 32, 64])
+@pytest.mark.parametrize("b", BLOCKS)
 def test_linear_integer_inputs_bit_exact(lp, b):
     m, n, k = 520, 256, 512
-    X, W, bias, mask = _case(m, n, k, b, 0.5, 200 + b, int_valued=True)
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 200 + _sid(b), int_valued=True)
     w = lp.pack_bsr(W, mask, b)
     Y = lp.bsr_linear(w, X, bias, out_dtype=torch.float32)
     ref = _oracle(X, W, mask, b, bias)
     assert np.array_equal(Y.cpu().double().numpy(), ref)
 
 
-@pytest.mark.parametrize("b", [16, 32, 64])
+@pytest.mark.parametrize("b", BLOCKS)
 def test_linear_bf16_out_within_one_ulp(lp, b):
     m, n, k = 600, 512, 384
-    X, W, bias, mask = _case(m, n, k, b, 0.5, 300 + b)
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 300 + _sid(b))
     w = lp.pack_bsr(W, mask, b)
     Y = lp.bsr_linear(w, X, bias)
     ref = _oracle(X, W, mask, b, bias)
@@ -242,10 +263,10 @@ def test_linear_bf16_out_within_one_ulp(lp, b):
     assert np.all(np.abs(y - ref) <= _bf16_tol(ref, X, W, mask, b, bias))
 
 
-@pytest.mark.parametrize("b", [16, 32, 64])
+@pytest.mark.parametrize("b", BLOCKS)
 def test_linear_gelu(lp, b):
     m, n, k = 333, 256, 256
-    X, W, bias, mask = _case(m, n, k, b, 0.4, 400 + b)
+    X, W, bias, mask = _case(m, n, k, b, 0.4, 400 + _sid(b))
     w = lp.pack_bsr(W, mask, b)
     Y = lp.bsr_linear(w, X, bias, gelu=True, out_dtype=torch.float32)
     ref = _oracle(X, W, mask, b, bias, gelu=True)
@@ -254,11 +275,12 @@ def test_linear_gelu(lp, b):
     assert np.all(np.abs(Yb.float().cpu().double().numpy() - ref) <= _bf16_tol(ref, X, W, mask, b, bias, gelu=True))
 
 
-@pytest.mark.parametrize("b", [16, 32, 64])
+@pytest.mark.parametrize("b", BLOCKS)
 def test_all_zero_mask_is_bias(lp, b):
     m, n, k = 260, 256, 128
-    X, W, bias, _ = _case(m, n, k, b, 0.5, 500 + b)
-    mask = torch.zeros(n // b, k // b, dtype=torch.uint8, device="cuda")
+    X, W, bias, _ = _case(m, n, k, b, 0.5, 500 + _sid(b))
+    bn, bk = _sides(b)
+    mask = torch.zeros(n // bn, k // bk, dtype=torch.uint8, device="cuda")
     w = lp.pack_bsr(W, mask, b)
     Y = lp.bsr_linear(w, X, bias, out_dtype=torch.float32)
     assert torch.equal(Y, bias.expand(m, n))
@@ -269,11 +291,12 @@ def test_all_zero_mask_is_bias(lp, b):
     assert torch.count_nonzero(Yn) == 0
 
 
-@pytest.mark.parametrize("b", [16, 32, 64])
+@pytest.mark.parametrize("b", BLOCKS)
 def test_pruned_blocks_never_read(lp, b):
     m, n, k = 300, 256, 256
-    X, W, bias, mask = _case(m, n, k, b, 0.5, 600 + b)
-    keep = mask.repeat_interleave(b, 0).repeat_interleave(b, 1).bool()
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 600 + _sid(b))
+    bn, bk = _sides(b)
+    keep = mask.repeat_interleave(bn, 0).repeat_interleave(bk, 1).bool()
     Wp = W.clone()
     Wp[~keep] = float("nan")
     Wz = W.clone()
@@ -309,9 +332,10 @@ def test_strided_input_output_and_guard_band(lp):
     assert torch.all(Yw[m:] == canary) and torch.all(Yw[:, :16] == canary) and torch.all(Yw[:, 16 + n:] == canary)
 
 
-def test_deterministic_repeats(lp):
-    m, n, k, b = 197, 768, 3072, 32   # small m: split slices + fix-up path
-    X, W, bias, mask = _case(m, n, k, b, 0.5, 900)
+@pytest.mark.parametrize("b", [32, (64, 32), (16, 32)])
+def test_deterministic_repeats(lp, b):
+    m, n, k = 197, 768, 3072   # small m: split slices + fix-up path
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 900 + (0 if b == 32 else _sid(b)))
     w = lp.pack_bsr(W, mask, b)
     ws = lp.workspace_for(w, m)
     Y1 = lp.bsr_linear(w, X, bias, out_dtype=torch.float32, workspace=ws)
@@ -322,10 +346,10 @@ def test_deterministic_repeats(lp):
     assert _norm_err(Y1.cpu().double().numpy(), ref) <= TIGHT_TOL
 
 
-@pytest.mark.parametrize("b", [16, 64])
+@pytest.mark.parametrize("b", [16, 64, (16, 32)])
 def test_zipf_imbalanced_masks(lp, b):
     m, n, k = 513, 768, 3072
-    X, W, bias, mask = _case(m, n, k, b, 0.6, 1000 + b, mask_kind="zipf")
+    X, W, bias, mask = _case(m, n, k, b, 0.6, 1000 + _sid(b), mask_kind="zipf")
     w = lp.pack_bsr(W, mask, b)
     Y = lp.bsr_linear(w, X, bias, gelu=True, out_dtype=torch.float32)
     ref = _oracle(X, W, mask, b, bias, gelu=True)

@@ -35,15 +35,18 @@ def _oracle(W, G, b, alpha):
 
 
 @pytest.mark.parametrize("n,k,b", [(384, 256, 32), (208, 1536, 16), (768, 3072, 64), (3072, 768, 32),
-                                   (768, 3072, 32), (1152, 384, 16)])
+                                   (768, 3072, 32), (1152, 384, 16), (768, 3072, (64, 32)), (384, 1536, (16, 32)),
+                                   (192, 320, (32, 16))])
 @pytest.mark.parametrize("alpha", [0.0, 0.3, 0.5, 0.8, 1.0])
 def test_scores_and_mask_bit_exact(lp, n, k, b, alpha):
-    W, G = _wg(n, k, 4000 + n + k + b)
+    bn, bk = inputs.block_sides(b)
+    W, G = _wg(n, k, 4000 + n + k + (bn if bn == bk else 100 * bn + bk))
     mask, scores = lp.taylor_block_mask(W, G, b, alpha)
     s_ref, m_ref = _oracle(W, G, b, alpha)
+    assert scores.shape == (n // bn, k // bk)
     assert np.array_equal(scores.cpu().numpy(), s_ref)
     assert np.array_equal(mask.cpu().numpy(), m_ref)
-    assert int(mask.sum()) == (n // b) * (k // b) - oracle.prune_count(alpha, (n // b) * (k // b))
+    assert int(mask.sum()) == (n // bn) * (k // bk) - oracle.prune_count(alpha, (n // bn) * (k // bk))
 
 
 @pytest.mark.parametrize("b", [16, 32, 64])
