@@ -459,9 +459,8 @@ def run_case(args, local):
 def run_calibrate(args, local):
     """Cost-model calibration (Sec. 3.3, Eq. for P: p_m (M/B_m) ceil((1 - alpha) N K / (B_n B_k))):
     time each DeiT GEMM shape, with the block sizes of Table 2 (DeiT-B 32x32 and 64x32, DeiT-S
-    16x16 and 16x32, "a x b" read as B_n x B_k of Sec. 3.3: a input columns by b output rows, i.e.
-    (bn, bk) = (b, a); the transposed reading is timed too), over a block-density sweep and fit, per
-    shape, the least-squares line
+    16x16 and 16x32, printed output rows x input columns as Table 4's "BK x BN"; the transposed
+    shapes are timed too), over a block-density sweep and fit, per shape, the least-squares line
     T = a + p * tiles * nnzb (tiles = ceil(M / 256), the kernel's token tile; nnzb = kept blocks).
     Prints one JSON line per shape with a, p (ns per block-tile), R^2 and the largest relative
     residual, and a final line with the fit over all shapes of each block size."""
@@ -474,10 +473,10 @@ def run_calibrate(args, local):
     import paper_2407_02068_gb300 as lp
     from paper_2407_02068_gb300 import inputs
     shapes = []
-    for blk in (32, (32, 64), (64, 32)):
+    for blk in (32, (64, 32), (32, 64)):
         shapes += [("deit_b_fc1", 50432, 768, 3072, blk, True), ("deit_b_fc2", 50432, 3072, 768, blk, False),
                    ("deit_b_qkv", 50432, 768, 2304, blk, False), ("deit_b_proj", 50432, 768, 768, blk, False)]
-    for blk in (16, (32, 16), (16, 32)):
+    for blk in (16, (16, 32), (32, 16)):
         shapes += [("deit_s_fc1", 12608, 384, 1536, blk, True), ("deit_s_fc2", 12608, 1536, 384, blk, False)]
     densities = [1.0, 0.7, 0.5, 0.3, 0.2]
     reps = max(args.steps, 5)

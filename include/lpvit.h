@@ -9,12 +9,15 @@
  *     W~[o][i] = W[o][i] if mask[o/bn][i/bk] != 0, else 0,
  *
  * with W stored [n = out features][k = in features] (PyTorch Linear layout), blocks of bn
- * output rows by bk input columns (B_n x B_k of Eq. for P; bn, bk in {16, 32, 64}, so the
+ * output rows by bk input columns (B_k x B_n in Eq. for P, whose weight is [N in x K out], and the
+ * order Table 4 prints, "BK x BN"; bn, bk in {16, 32, 64}, so the
  * square 16x16, 32x32, 64x64 and the paper's 64x32 and 16x32 of Table 2 are all covered),
  * act = identity (lpvit_bsr_linear) or the exact GELU
  * 0.5*y*(1+erf(y/sqrt 2)) (lpvit_bsr_linear_gelu, the DeiT fc1 activation). Only the kept
- * blocks are stored and multiplied: the work is proportional to the number of kept blocks,
- * as in the power model of Sec. 3.3 (Eq. for P).
+ * blocks are stored, and removed blocks are never read. The GEMM multiplies, per 128-output group,
+ * only the block columns where the group keeps a block (rows of removed blocks there enter as
+ * zeros), so its work follows those group columns rather than exactly the kept blocks that the
+ * power model of Sec. 3.3 (Eq. for P) counts.
  *
  * Conventions for every call:
  *  - All pointers except nnzb_host are DEVICE pointers owned by the caller; the library never

@@ -11,8 +11,9 @@
  *      W~[i][j] = W[i][j] (.) M[ceil(i/B_h)][ceil(j/B_w)]
  *    The paper indexes blocks 1-based with a ceiling; with 0-based indices the block of
  *    element (i, j) is (floor(i/bn), floor(j/bk)), a block being bn output rows by bk input
- *    columns (B_n x B_k in Eq. for P; Table 2 uses 32x32, 64x32, 16x32 and 16x16, and a
- *    square b x b block is bn = bk = b). A nonzero mask byte keeps the block; a
+ *    columns. Eq. for P writes the weight as [N inputs x K outputs] with B_n x B_k blocks, so
+ *    bn x bk here is B_k x B_n there, the order Table 4 prints ("BK x BN"); Table 2 uses 32x32,
+ *    64x32, 16x32 and 16x16, and a square b x b block is bn = bk = b. A nonzero mask byte keeps the block; a
  *    zero byte removes it, and a removed weight is exactly zero whatever W holds there
  *    (the pruned value is never multiplied, so NaN or Inf in a pruned block has no effect).
  *

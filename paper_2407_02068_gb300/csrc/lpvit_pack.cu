@@ -1,7 +1,8 @@
 // Mask -> BSR pack and work-list build (Sec. 3.1 block mask; Sec. 1 / Sec. 3.3: only the kept
 // blocks are stored, moved and multiplied).
 //
-// Blocks are bn output rows by bk input columns (Sec. 3.1 mask over B_n x B_k blocks).
+// Blocks are bn output rows by bk input columns (Sec. 3.1 block mask; B_k x B_n in the notation of
+// Sec. 3.3, whose weight is [N inputs x K outputs]).
 // plan kernel (one CTA): per row panel r (bn rows), cnt[r] = number of kept blocks (warp
 //   reductions); row_ptr = exclusive prefix sum of cnt (warp-shuffle scan + a scan of warp
 //   totals); col_idx = kept block columns of each panel in ascending order (ballot compaction);
