@@ -7,8 +7,9 @@ definitions, slow on purpose.
 What it computes:
 
 * ``mean_gradient(G)`` -- the first-order gradient grad_W f as the average of N per-sample
-  gradients, summed over the samples in order in float64 and rounded to float32 (the gradient the
-  Taylor block scores of Sec. 3.1 take).
+  gradients, in float32 like the gradients themselves: summed over the samples in order with
+  float32 additions, then divided by N (IEEE float32; the gradient the Taylor block scores of
+  Sec. 3.1 take).
 * ``delta_curve`` -- the per-layer curve of Sec. 3.4 / 3.5: for alpha_k = k / steps, k = 0..steps,
       delta(alpha_k) = g . dW_k + 1/2 dW_k^T H dW_k,
   where dW_k = -W on the blocks pruned at alpha_k (the bottom prune_count(alpha_k, blocks) blocks
@@ -35,12 +36,12 @@ from . import bf16_to_f64, block_scores, block_shape, taylor_mask
 
 
 def mean_gradient(G: np.ndarray) -> np.ndarray:
-    """float32 [n, k]: the samples of G (float32 [N, n, k]) summed in order in float64, / N."""
+    """float32 [n, k]: the samples of G (float32 [N, n, k]) summed in order in float32, / N."""
     G = np.asarray(G, dtype=np.float32)
-    acc = np.zeros(G.shape[1:], dtype=np.float64)
+    acc = np.zeros(G.shape[1:], dtype=np.float32)
     for i in range(G.shape[0]):
-        acc += G[i].astype(np.float64)
-    return (acc / G.shape[0]).astype(np.float32)
+        acc = acc + G[i]
+    return acc / np.float32(G.shape[0])
 
 
 def pruned_delta_w(W_bits: np.ndarray, g32: np.ndarray, b, alpha: float) -> np.ndarray:

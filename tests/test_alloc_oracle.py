@@ -48,11 +48,15 @@ def _case(n, k, b, N, seed, scale=1e-2):
     return Wb, G
 
 
-def test_mean_gradient_sums_in_double_then_rounds():
-    G = np.array([[[1e8]], [[1.0]], [[-1e8]]], dtype=np.float32)  # float32 sum order would lose the 1
-    assert alloc.mean_gradient(G)[0, 0] == np.float32(1.0 / 3.0)
+def test_mean_gradient_sums_in_float32_in_sample_order():
+    G = np.array([[[1e8]], [[1.0]], [[-1e8]]], dtype=np.float32)
+    assert alloc.mean_gradient(G)[0, 0] == 0.0                    # 1e8 + 1 rounds back to 1e8 in float32
+    G2 = np.array([[[1.0]], [[1e8]], [[-1e8]]], dtype=np.float32)
+    assert alloc.mean_gradient(G2)[0, 0] == 0.0
+    G3 = np.array([[[1e8]], [[-1e8]], [[1.0]]], dtype=np.float32)
+    assert alloc.mean_gradient(G3)[0, 0] == np.float32(1.0) / np.float32(3.0)  # order decides
     G = (np.arange(24, dtype=np.float32).reshape(3, 2, 4) / 8)
-    assert np.array_equal(alloc.mean_gradient(G), G.mean(axis=0))  # exact dyadic values
+    assert np.array_equal(alloc.mean_gradient(G), (G[0] + G[1] + G[2]) / np.float32(3))
 
 
 def test_no_pruning_gives_zero_and_zero_gradients_give_the_kappa_closed_form():
