@@ -370,6 +370,21 @@ def test_taylor_scores_are_local_and_scale_exactly():
     assert changed[1, 0] and changed.sum() == 1
 
 
+def test_taylor_scores_sum_rows_then_blocks_in_float32():
+    """One 2 x 32 block: row 0 holds 1 and 31 products of 2^-25, row 1 holds 32 products of 2^-25.
+    In float32 each 2^-25 added to 1 is lost (below half an ulp of 1), while row 1's products add
+    exactly among themselves to 2^-20, which survives the addition of the row sums: the score is
+    (1 + 2^-20) / 64. A double sum, or one float32 sum over the whole block, gives other values."""
+    W = np.full((2, 32), 2.0 ** -8, dtype=np.float32)
+    W[0, 0] = 1.0
+    G = np.full((2, 32), 2.0 ** -17, dtype=np.float32)
+    G[0, 0] = 1.0
+    s = oracle.block_scores(_bits(W), G, (2, 32))
+    assert s[0, 0] == (1.0 + 2.0 ** -20) / 64
+    assert s[0, 0] != (1.0 + 63 * 2.0 ** -25) / 64   # the double sum
+    assert s[0, 0] != 1.0 / 64                        # one float32 sum over the block
+
+
 def test_taylor_scores_brute_force_and_mask_order():
     rng = np.random.default_rng(6)
     for b in (16, 32, (64, 32), (16, 32)):
@@ -380,7 +395,9 @@ def test_taylor_scores_brute_force_and_mask_order():
         Wd = oracle.bf16_to_f64(Wb)
         want = np.abs(Wd * G.astype(np.float64)).reshape(4, bn, 3, bk).sum(axis=(1, 3)) / (bn * bk)
         s = oracle.block_scores(Wb, G, b)
-        assert np.allclose(s, want, rtol=1e-13, atol=0)
+        # float32 products and two levels of float32 sums of non-negative terms: relative error at
+        # most (1 + (bk - 1) + (bn - 1)) 2^-24 of the exact average
+        assert np.allclose(s, want, rtol=(bn + bk) * 2.0 ** -24, atol=0)
         for alpha in (0.0, 0.25, 0.5, 0.75, 1.0):
             m = oracle.taylor_mask(s, alpha)
             kept, pruned = s[m == 1], s[m == 0]
