@@ -59,6 +59,9 @@ def parse_args():
                    help="stack (the benchmarked workload) or one GEMM of it, for profiling")
     p.add_argument("--calibrate", action="store_true",
                    help="fit measured GEMM time to the block-tile count of the paper's power model")
+    p.add_argument("--alloc", action="store_true",
+                   help="pruning-ratio allocation: distortion curves of the 48 DeiT-B weights + lambda search")
+    p.add_argument("--alloc-samples", type=int, default=16, help="per-sample gradients per layer (--alloc)")
     return p.parse_args()
 
 
@@ -526,6 +529,83 @@ def run_calibrate(args, local):
                           "max_rel_residual": float(np.max(np.abs(ts_a - pred) / ts_a))}), flush=True)
 
 
+def run_alloc(args, local):
+    """Pruning-ratio allocation (Sec. 3.4-3.5) for the 12-layer DeiT-B linear stack, 32x32 blocks:
+    the distortion curve of each of the 48 weights from N seeded per-sample gradients (20 ratio
+    steps, kappa 1e-3), timed with CUDA events layer by layer (gradients are generated on the device
+    outside the timed region), then the host lambda search at a 50% FLOPs target. One JSON line:
+    throughput in GB/s of algorithmic bytes (the gradients and the weight read once), against the
+    measured HBM copy bandwidth; the oracle is timed on one qkv weight."""
+    import torch
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2407_02068_gb300 as lp
+    from paper_2407_02068_gb300 import inputs
+    N, steps, kappa, b, m = args.alloc_samples, 20, 1e-3, 32, M_TOKENS
+    shapes = [(gi, k, n) for l in range(12) for gi, (_, k, n, _) in
+              ((4 * l + t, g) for t, g in enumerate(inputs.deit_gemms(inputs.DEIT_B)))]
+    Ws = [inputs.weight(n, k, inputs.seed(8, gi, "W"), dev) for gi, k, n in shapes]
+    gen = torch.Generator(device=dev)
+    ws_bytes = max(lp._lib.lpvit_delta_curve_workspace_bytes(N, n, k, b, b, steps) for _, k, n in shapes)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    G = torch.empty(N * max(n * k for _, k, n in shapes), dtype=torch.float32, device=dev)
+
+    def grads(gi, k, n):
+        gen.manual_seed(inputs.seed(8, gi, "X"))
+        Gv = G[:N * n * k].view(N, n, k)
+        Gv.normal_(0.0, 1e-2, generator=gen)
+        return Gv
+
+    lp.delta_curve(Ws[0], grads(*shapes[0]), b, steps, kappa, workspace=ws)  # warm-up
+    torch.cuda.synchronize()
+    clk = ClockSampler(local)
+    clk.start()
+    curves, total_ms, algo = [], 0.0, 0
+    for (gi, k, n), W in zip(shapes, Ws):
+        Gv = grads(gi, k, n)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        d = lp.delta_curve(W, Gv, b, steps, kappa, workspace=ws)
+        e1.record()
+        e1.synchronize()
+        total_ms += e0.elapsed_time(e1)
+        algo += 4 * N * n * k + 2 * n * k
+        curves.append(d.cpu().numpy())
+    clocks = clk.stop()
+    F = [float(m * n * k) for _, k, n in shapes]
+    c = [float(m * n * k) / (b * b) for _, k, n in shapes]
+    t0 = time.perf_counter()
+    ks, lam, ratio = lp.lambda_search(curves, steps, F, c, 1e-12, 0.5)
+    search_ms = (time.perf_counter() - t0) * 1e3
+    peaks, src = load_peaks()
+    achieved = algo / (total_ms / 1e3) / 1e9
+    line = {"metric": "pruning-ratio allocation: distortion-curve throughput (per-sample gradients + weights)",
+            "value": achieved, "unit": "GB/s", "n_gpus": 1, "higher_is_better": True, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": "deit_b_12layer_allocation", "weights": 48, "block": b,
+                                            "samples": N, "ratio_steps": steps, "kappa": kappa,
+                                            "flops_target": 0.5, "beta": 1e-12},
+            "ms_total": total_ms, "lambda_search_ms": search_ms, "allocated_k": ks, "flops_remained": ratio,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": float(peaks.get("hbm_gbs", 6800.0)),
+                         "unit": "GB/s", "frac": achieved / float(peaks.get("hbm_gbs", 6800.0)), "traffic": None,
+                         "peak_source": src + " hbm_gbs (STREAM-style copy)"},
+            "gpu_launches": 5 * len(shapes), "clocks": clocks}
+    if not args.no_cpu_baseline:
+        import oracle.alloc as oalloc
+        gi, k, n = shapes[0]
+        Wb = inputs.bf16_bits(Ws[0])
+        Gh = grads(gi, k, n).cpu().numpy()
+        t0 = time.perf_counter()
+        oalloc.delta_curve(Wb, Gh, b, steps, kappa)
+        cpu_s = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": (4 * N * n * k + 2 * n * k) / cpu_s / 1e9, "unit": "GB/s",
+                                "cores": os.cpu_count(), "kind": "oracle",
+                                "sample": f"one qkv weight ({n}x{k}), {N} samples, {steps + 1} ratios, numpy fp64 "
+                                          f"with its default BLAS threading, {cpu_s:.1f} s"}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     world, rank, local = dist_setup(args)
@@ -534,6 +614,9 @@ def main():
         return
     if args.calibrate:
         run_calibrate(args, local)
+        return
+    if args.alloc:
+        run_alloc(args, local)
         return
     if args.case != "stack":
         run_case(args, local)

@@ -112,9 +112,10 @@ lpvit_status lpvit_pack_bsr_many(int32_t count, const void *const *W, const uint
  * and stride, and the bottom-ranked blocks eliminated at pruning ratio `prune_ratio` (alpha).
  *   W       bf16 [n][k] row-major, 16-byte aligned (the weight, as for lpvit_pack_bsr)
  *   G       float32 [n][k] row-major, 16-byte aligned (the gradient of the loss with respect to W)
- *   scores  out: double [n/bn][k/bk], 8-byte aligned: the block scores. Each is the sum of |w * g|
- *           over the block in row-major order in double (every product is exact), divided by
- *           bn*bk, so it is bit-identical to that sequential sum.
+ *   scores  out: double [n/bn][k/bk], 8-byte aligned: the block scores, in float32 (the
+ *           gradient's precision) with a fixed order: each |w * g| rounded to float32, each block
+ *           row summed in order, the row sums summed in row order; that total widened to double
+ *           and divided by bn*bk. Bit-identical to a plain loop doing the same operations.
  *   mask    out: uint8 [n/bn][k/bk], 1 = kept, 0 = eliminated; it can be passed to lpvit_pack_bsr.
  * Exactly round(alpha * blocks), half away from zero, blocks are eliminated: those ranked lowest,
  * where blocks rank by score and equal scores by linear block index r*(k/bk)+j, the lower first
@@ -123,6 +124,55 @@ lpvit_status lpvit_pack_bsr_many(int32_t count, const void *const *W, const uint
  * LPVIT_ERR_INVALID_ARG (shape, alpha outside [0, 1], null or misaligned pointer), LPVIT_ERR_CUDA. */
 lpvit_status lpvit_taylor_block_mask(const void *W, const float *G, int32_t n, int32_t k, int32_t bn, int32_t bk,
                                      double prune_ratio, double *scores, uint8_t *mask, void *stream);
+
+/* The first-order gradient of Sec. 3.1 / 3.5 as the mean of N per-sample gradients:
+ * g[e] = (sum_i G[i][e]) / N in float32, the sum in sample order (IEEE float32 additions and
+ * division: the precision of the gradients themselves).
+ * G float32 [nsamples][count], g float32 [count] (device, 4-byte aligned), 1 <= nsamples <= 1024.
+ * This is the gradient lpvit_delta_curve ranks blocks by; pass it to lpvit_taylor_block_mask to
+ * get the masks the allocated ratios stand for. Asynchronous on `stream`.
+ * Errors: LPVIT_ERR_INVALID_ARG, LPVIT_ERR_CUDA. */
+lpvit_status lpvit_mean_gradient(const float *G, int32_t nsamples, int64_t count, float *g, void *stream);
+
+/* Pruning-ratio allocation, Sec. 3.4-3.5. For one layer (weight W, bf16 [n][k], 16-byte aligned)
+ * and N per-sample gradients G (float32 [nsamples][n][k], 16-byte aligned), the curve
+ *     delta[s] = g . dW_s + 1/2 dW_s^T H dW_s,   s = 0..steps, alpha_s = s / steps,
+ * where g = (sum_i G[i]) / N (as lpvit_mean_gradient computes it), dW_s = -W on
+ * the blocks (bn rows by bk columns) that the Taylor ranking of Sec. 3.1 under gradient g
+ * eliminates at alpha_s (exactly as lpvit_taylor_block_mask would at that ratio) and 0 elsewhere,
+ * and H = kappa I + (1/N) sum_i G[i] G[i]^T is the empirical Fisher of Sec. 3.5. It is computed by
+ * the incremental update of Eq. update with H in low-rank form (per-block sums of G[i] * W with
+ * exact products and float-pair accumulation, about 2^-43 of the block's sum of magnitudes; steps
+ * in double; no D x D matrix), delta[0] = 0.
+ *   delta     out: double [steps + 1] on the device, 8-byte aligned
+ *   workspace device, 256-byte aligned, >= lpvit_delta_curve_workspace_bytes(...) bytes
+ * 1 <= nsamples <= 1024, 1 <= steps <= 4096, kappa >= 0 and finite, at most 2^20 blocks.
+ * Asynchronous on `stream`; allocates nothing.
+ * Errors: LPVIT_ERR_UNSUPPORTED (bn or bk not in {16,32,64}, more than 2^20 blocks),
+ * LPVIT_ERR_INVALID_ARG (shape, nsamples, steps, kappa, null or misaligned pointer),
+ * LPVIT_ERR_WORKSPACE, LPVIT_ERR_CUDA. */
+size_t lpvit_delta_curve_workspace_bytes(int32_t nsamples, int32_t n, int32_t k, int32_t bn, int32_t bk,
+                                         int32_t steps);
+lpvit_status lpvit_delta_curve(const void *W, const float *G, int32_t nsamples, int32_t n, int32_t k, int32_t bn,
+                               int32_t bk, double kappa, int32_t steps, double *delta, void *workspace,
+                               size_t ws_bytes, void *stream);
+
+/* The lambda search of Sec. 3.4 (Eq. langrangian2) over per-layer curves; HOST memory, host code,
+ * synchronous, no GPU. delta: [layers][steps + 1] (lpvit_delta_curve's output per layer); the
+ * distortion of layer i at alpha_s is D_i[s] = delta_i[s]^2 (Eq. obj_f). flops[i] > 0: the layer's
+ * dense FLOPs (M N K); power_coef[i] = M N K / (B_n B_k), its power term per unit of (1 - alpha).
+ * For a multiplier lambda, layer i takes the largest k such that every slope
+ * (D_i[j] - D_i[j-1]) * steps, j = 1..k, is at most lambda + beta * power_coef[i]. Lambda runs
+ * over every value at which some layer's k changes (and minus infinity); the result is the
+ * smallest such lambda whose FLOPs-remained ratio sum_i (1 - k_i/steps) flops[i] / sum flops is
+ * at most flops_ratio (the least pruning that meets the target), else the most pruning.
+ *   k_out      out: int32 [layers], alpha_i = k_out[i] / steps
+ *   lambda_out, ratio_out   out (may be NULL): the multiplier and the FLOPs-remained ratio
+ * Errors: LPVIT_ERR_INVALID_ARG (counts, null pointers, non-finite or non-positive flops,
+ * non-finite power_coef or beta, NaN in delta or flops_ratio). */
+lpvit_status lpvit_lambda_search(int32_t layers, int32_t steps, const double *delta, const double *flops,
+                                 const double *power_coef, double beta, double flops_ratio, int32_t *k_out,
+                                 double *lambda_out, double *ratio_out);
 
 /* Bytes of device workspace lpvit_bsr_linear[_gelu] needs for m tokens. The workspace holds
  * scheduler counters, the device error word and, for small m, fp32 partial sums of split

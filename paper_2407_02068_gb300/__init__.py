@@ -10,6 +10,8 @@ or 64 (Table 2 uses 32x32, 64x32, 16x32 and 16x16). This package wraps the C lib
 * ``pack_bsr(W, mask, b)``  -- mask -> BSR pack + work list, on the GPU
 * ``pack_bsr_many_into(ws, Ws, masks)`` -- the same for a list of weights in two launches
 * ``bsr_linear(w, X, bias, gelu=...)`` -- Y = act(X (W (.) M)^T + bias)
+* ``delta_curve(W, G, b, steps, kappa)`` / ``lambda_search(...)`` -- the layer-wise pruning-ratio
+  allocation of Sec. 3.4-3.5 (empirical-Fisher distortion curves, Lagrangian slope matching)
 
 PyTorch provides device memory and streams only; every step runs in the library's kernels.
 """
@@ -22,7 +24,7 @@ import torch
 from . import _lib
 
 __all__ = ["BsrWeight", "alloc_bsr", "pack_bsr", "pack_bsr_into", "pack_bsr_many_into", "taylor_block_mask",
-           "workspace_for", "bsr_linear", "check", "LpvitError"]
+           "workspace_for", "bsr_linear", "check", "LpvitError", "delta_curve", "lambda_search", "mean_gradient"]
 
 LpvitError = _lib.LpvitError
 
@@ -115,6 +117,52 @@ def taylor_block_mask(W: torch.Tensor, G: torch.Tensor, b, prune_ratio: float, s
     if st != _lib.LPVIT_OK:
         raise LpvitError(st, "lpvit_taylor_block_mask")
     return mask, scores
+
+
+def delta_curve(W: torch.Tensor, G: torch.Tensor, b, steps: int, kappa: float, workspace: torch.Tensor | None = None,
+                stream=None) -> torch.Tensor:
+    """Sec. 3.4-3.5 distortion curve of one layer: W bf16 [n, k], G float32 per-sample gradients
+    [N, n, k], both contiguous CUDA. Returns float64 [steps + 1] on the device: delta at
+    alpha = s / steps (see lpvit_delta_curve)."""
+    if W.dtype != torch.bfloat16 or not W.is_cuda or W.dim() != 2 or not W.is_contiguous():
+        raise ValueError("W must be a contiguous 2-D bf16 CUDA tensor")
+    if G.dtype != torch.float32 or G.dim() != 3 or tuple(G.shape[1:]) != tuple(W.shape) or not G.is_contiguous() \
+            or G.device != W.device:
+        raise ValueError("G must be a contiguous float32 [N, n, k] tensor on W's device")
+    n, k = W.shape
+    bn, bk = block_sides(b)
+    N = G.shape[0]
+    need = _lib.lpvit_delta_curve_workspace_bytes(N, n, k, bn, bk, steps)
+    if workspace is None:
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=W.device)
+    out = torch.empty(steps + 1, dtype=torch.float64, device=W.device)
+    st = _lib.lpvit_delta_curve(W.data_ptr(), G.data_ptr(), N, n, k, bn, bk, kappa, steps, out.data_ptr(),
+                                workspace.data_ptr(), workspace.numel(), _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_delta_curve")
+    return out
+
+
+def mean_gradient(G: torch.Tensor, stream=None) -> torch.Tensor:
+    """float32 [n, k]: the mean over the first axis of G (float32 [N, n, k], contiguous CUDA), summed in
+    float32 in sample order (the gradient lpvit_delta_curve and the Taylor mask rank blocks by)."""
+    if G.dtype != torch.float32 or not G.is_cuda or G.dim() < 2 or not G.is_contiguous():
+        raise ValueError("G must be a contiguous float32 CUDA tensor [N, ...]")
+    g = torch.empty(G.shape[1:], dtype=torch.float32, device=G.device)
+    st = _lib.lpvit_mean_gradient(G.data_ptr(), G.shape[0], g.numel(), g.data_ptr(), _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_mean_gradient")
+    return g
+
+
+def lambda_search(deltas, steps: int, flops, power_coef, beta: float, flops_ratio: float):
+    """Sec. 3.4 lambda search (host): deltas = per-layer curves of steps + 1 values. Returns
+    (k list with alpha_i = k_i / steps, lambda, FLOPs-remained ratio)."""
+    rows = [d.tolist() if hasattr(d, "tolist") else list(d) for d in deltas]
+    st, ks, lam, ratio = _lib.lpvit_lambda_search(rows, steps, flops, power_coef, beta, flops_ratio)
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_lambda_search")
+    return ks, lam, ratio
 
 
 def pack_bsr_many_into(ws: list, Ws: list, masks: list, stream=None) -> list:

@@ -23,7 +23,8 @@ LPVIT_F32 = 1
 
 EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_workspace_bytes", "lpvit_bsr_linear",
            "lpvit_bsr_linear_gelu", "lpvit_bsr_linear_noalloc", "lpvit_check", "lpvit_status_string",
-           "lpvit_selftest_wait", "lpvit_pack_bsr_many", "lpvit_taylor_block_mask")
+           "lpvit_selftest_wait", "lpvit_pack_bsr_many", "lpvit_taylor_block_mask",
+           "lpvit_delta_curve_workspace_bytes", "lpvit_delta_curve", "lpvit_lambda_search", "lpvit_mean_gradient")
 LPVIT_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 
@@ -65,6 +66,14 @@ def load(path: str | None = None):
         lib.lpvit_pack_bsr.argtypes = [V, V, BP, ctypes.POINTER(I32), V]
         lib.lpvit_taylor_block_mask.restype = ctypes.c_int
         lib.lpvit_taylor_block_mask.argtypes = [V, V, I32, I32, I32, I32, ctypes.c_double, V, V, V]
+        lib.lpvit_delta_curve_workspace_bytes.restype = SZ
+        lib.lpvit_delta_curve_workspace_bytes.argtypes = [I32, I32, I32, I32, I32, I32]
+        lib.lpvit_delta_curve.restype = ctypes.c_int
+        lib.lpvit_delta_curve.argtypes = [V, V, I32, I32, I32, I32, I32, ctypes.c_double, I32, V, V, SZ, V]
+        lib.lpvit_mean_gradient.restype = ctypes.c_int
+        lib.lpvit_mean_gradient.argtypes = [V, I32, I64, V, V]
+        lib.lpvit_lambda_search.restype = ctypes.c_int
+        lib.lpvit_lambda_search.argtypes = [I32, I32, V, V, V, ctypes.c_double, ctypes.c_double, V, V, V]
         lib.lpvit_pack_bsr_many.restype = ctypes.c_int
         lib.lpvit_pack_bsr_many.argtypes = [I32, ctypes.POINTER(V), ctypes.POINTER(V), BP, V]
         lib.lpvit_workspace_bytes.restype = SZ
@@ -117,6 +126,34 @@ def lpvit_pack_bsr_many(W_ptrs, mask_ptrs, bsrs, stream: int) -> int:
 def lpvit_taylor_block_mask(W_ptr, G_ptr, n, k, bn, bk, prune_ratio, scores_ptr, mask_ptr, stream) -> int:
     return load().lpvit_taylor_block_mask(W_ptr, G_ptr, n, k, bn, bk, float(prune_ratio), scores_ptr, mask_ptr,
                                           stream)
+
+
+def lpvit_delta_curve_workspace_bytes(nsamples: int, n: int, k: int, bn: int, bk: int, steps: int) -> int:
+    return int(load().lpvit_delta_curve_workspace_bytes(nsamples, n, k, bn, bk, steps))
+
+
+def lpvit_delta_curve(W_ptr, G_ptr, nsamples, n, k, bn, bk, kappa, steps, delta_ptr, ws_ptr, ws_bytes,
+                      stream) -> int:
+    return load().lpvit_delta_curve(W_ptr, G_ptr, nsamples, n, k, bn, bk, float(kappa), steps, delta_ptr, ws_ptr,
+                                    ws_bytes, stream)
+
+
+def lpvit_mean_gradient(G_ptr, nsamples, count, g_ptr, stream) -> int:
+    return load().lpvit_mean_gradient(G_ptr, nsamples, count, g_ptr, stream)
+
+
+def lpvit_lambda_search(delta_rows, steps: int, flops, power_coef, beta: float, flops_ratio: float):
+    """Host call. delta_rows: sequence of per-layer sequences of steps + 1 floats. Returns
+    (status, [k_i], lambda, ratio)."""
+    L = len(delta_rows)
+    D = (ctypes.c_double * (L * (steps + 1)))(*[float(v) for row in delta_rows for v in row])
+    F = (ctypes.c_double * L)(*[float(v) for v in flops])
+    C = (ctypes.c_double * L)(*[float(v) for v in power_coef])
+    K = (ctypes.c_int32 * L)()
+    lam, ratio = ctypes.c_double(0.0), ctypes.c_double(0.0)
+    st = load().lpvit_lambda_search(L, steps, D, F, C, float(beta), float(flops_ratio), K, ctypes.byref(lam),
+                                    ctypes.byref(ratio))
+    return st, list(K), lam.value, ratio.value
 
 
 def lpvit_workspace_bytes(bsr: lpvit_bsr, m: int) -> int:

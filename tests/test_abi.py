@@ -90,3 +90,54 @@ def test_bad_arguments_are_rejected_without_a_gpu(lib):
     assert lib.lpvit_selftest_wait(0x100000, 0, 0, None) == lib.LPVIT_ERR_INVALID_ARG         # no limit
     assert lib.lpvit_selftest_wait(0x100000, 11 * 10 ** 9, 0, None) == lib.LPVIT_ERR_INVALID_ARG  # > 10 s
     assert lib.lpvit_selftest_wait(0x100000, 10 ** 6, 10 ** 6, None) == lib.LPVIT_ERR_INVALID_ARG  # abort >= limit
+
+
+def test_lambda_search_host_matches_the_oracle(lib):
+    """lpvit_lambda_search is host code: it runs here, without a GPU, against the oracle."""
+    import math
+    import numpy as np
+    from oracle import alloc
+    # the hand-worked example, given as delta curves (D = delta^2)
+    d1 = [math.sqrt(v) for v in (0, 1, 3, 7)]
+    d2 = [math.sqrt(v) for v in (0, 2, 4, 6)]
+    for beta, R in ((0, 0.5), (0, 0.95), (2, 0.5), (2, 0.1), (0, 1.0)):
+        st, ks, lam, ratio = lib.lpvit_lambda_search([d1, d2], 3, [1, 3], [1, 2], beta, R)
+        want = alloc.lambda_search([alloc.distortion(d1), alloc.distortion(d2)], 3, [1, 3], [1, 2], beta, R)
+        assert st == lib.LPVIT_OK and (lam, ks, ratio) == (want[0], want[1], want[2]), (beta, R)
+    rng = np.random.default_rng(9)
+    for trial in range(20):
+        L, steps = int(rng.integers(1, 30)), int(rng.integers(1, 25))
+        deltas = [np.concatenate([[0.0], np.cumsum(rng.standard_normal(steps))]) for _ in range(L)]
+        F = rng.uniform(0.5, 4.0, L)
+        c = rng.uniform(0.0, 3.0, L)
+        beta, R = float(rng.uniform(0, 2)), float(rng.uniform(-0.1, 1.1))
+        st, ks, lam, ratio = lib.lpvit_lambda_search(deltas, steps, F, c, beta, R)
+        want = alloc.lambda_search([alloc.distortion(d) for d in deltas], steps, F, c, beta, R)
+        assert st == lib.LPVIT_OK and ks == want[1] and lam == want[0] and ratio == want[2], trial
+
+
+def test_allocation_arguments_are_checked_without_a_gpu(lib):
+    L = lib.load()
+    assert lib.lpvit_delta_curve_workspace_bytes(8, 768, 3072, 32, 32, 20) > 8 * 768 * 3072 // 1024 * 8
+    assert lib.lpvit_delta_curve_workspace_bytes(0, 768, 3072, 32, 32, 20) == 0
+    assert lib.lpvit_delta_curve_workspace_bytes(8, 768, 3000, 32, 32, 20) == 0
+    assert lib.lpvit_delta_curve_workspace_bytes(8, 768, 3072, 32, 32, 0) == 0
+    dc = lib.lpvit_delta_curve
+    ok = dict(W_ptr=0x1000, G_ptr=0x2000, nsamples=8, n=256, k=256, bn=32, bk=32, kappa=0.1, steps=10,
+              delta_ptr=0x3000, ws_ptr=0x100000, ws_bytes=1 << 30, stream=None)
+    def call(**kw):
+        a = dict(ok, **kw)
+        return dc(a["W_ptr"], a["G_ptr"], a["nsamples"], a["n"], a["k"], a["bn"], a["bk"], a["kappa"], a["steps"],
+                  a["delta_ptr"], a["ws_ptr"], a["ws_bytes"], a["stream"])
+    assert call(bn=24) == lib.LPVIT_ERR_UNSUPPORTED
+    assert call(n=65536, k=65536, bn=16, bk=16) == lib.LPVIT_ERR_UNSUPPORTED  # > 2^20 blocks
+    for bad in (dict(nsamples=0), dict(nsamples=1025), dict(steps=0), dict(steps=5000), dict(kappa=-1.0),
+                dict(kappa=float("inf")), dict(kappa=float("nan")), dict(W_ptr=0), dict(G_ptr=0x2004),
+                dict(delta_ptr=0x3004), dict(ws_ptr=0x100010), dict(k=250)):
+        assert call(**bad) == lib.LPVIT_ERR_INVALID_ARG, bad
+    assert call(ws_bytes=16) == lib.LPVIT_ERR_WORKSPACE
+    st, *_ = lib.lpvit_lambda_search([[0.0, 1.0]], 1, [0.0], [1.0], 0.0, 0.5)   # flops must be > 0
+    assert st == lib.LPVIT_ERR_INVALID_ARG
+    st, *_ = lib.lpvit_lambda_search([[0.0, float("nan")]], 1, [1.0], [1.0], 0.0, 0.5)
+    assert st == lib.LPVIT_ERR_INVALID_ARG
+    assert L.lpvit_lambda_search(0, 1, None, None, None, 0.0, 0.5, None, None, None) == lib.LPVIT_ERR_INVALID_ARG

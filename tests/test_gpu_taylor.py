@@ -1,6 +1,6 @@
 """The block mask of Sec. 3.1 from first-order Taylor scores on the GPU (lpvit_taylor_block_mask)
-against the oracle: block scores bit for bit (both sum the exact products in row-major order in
-double) and masks bit for bit (rank by score, ties to the lower block index, round(alpha * blocks)
+against the oracle: block scores bit for bit (both take the same float32 operations in the same
+order: products, row sums, the sum of the row sums) and masks bit for bit (rank by score, ties to the lower block index, round(alpha * blocks)
 eliminated); then the mask drives the pack and the linear."""
 import numpy as np
 import pytest
