@@ -65,14 +65,6 @@ __device__ __forceinline__ void pair_add(float &hi, float &lo, float x) {
   lo = __fadd_rn(lo, err);
 }
 
-__device__ __forceinline__ double warp_sum(double v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
-// Warp w handles block t = w / (N + 1) and row u = w % (N + 1): u < N gives s[u][t] (sample u),
-// u == N gives gw[t] and w2[t].
 // (hi, lo) += (bh, bl): two-sum of the high parts, the low parts and the error added.
 __device__ __forceinline__ void pair_add2(float &hi, float &lo, float bh, float bl) {
   pair_add(hi, lo, bh);
@@ -87,47 +79,81 @@ __device__ __forceinline__ void warp_pair_sum(float &hi, float &lo) {
   }
 }
 
+__device__ __forceinline__ double warp_sum(double v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Warp w handles block t and sample group u (samples [u*SPW, u*SPW + SPW) of N; the last group,
+// u == groups - 1, gives gw[t] and w2[t] from g instead). Lane l takes the block's 4-element chunks
+// l, l + 32, ... in row-major order (a chunk stays inside one block row: bk is a multiple of 4),
+// loading 4 weights and, per sample, 4 gradients as vectors.
+constexpr int SPW = 4;  // samples per warp
+
 template <int BK>
 __global__ void __launch_bounds__(ALLOC_THREADS)
 block_sums_kernel(const uint16_t *__restrict__ W, const float *__restrict__ G, const float *__restrict__ g,
                   int nsamples, int n, int k, int bn, float2 *__restrict__ s, float2 *__restrict__ gw,
                   float2 *__restrict__ w2) {
   const int lane = threadIdx.x & 31;
-  constexpr int bk = BK;
-  const int kb = k / bk;
+  constexpr int CPR = BK / 4;  // chunks per block row
+  const int kb = k / BK;
   const int64_t T = (int64_t)(n / bn) * kb;
   const int64_t D = (int64_t)n * k;
+  const int groups = (nsamples + SPW - 1) / SPW + 1;
+  const int chunks = bn * CPR;
   const int64_t warps = (int64_t)gridDim.x * (blockDim.x / 32);
-  for (int64_t w = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); w < T * (nsamples + 1);
-       w += warps) {
-    const int64_t t = w / (nsamples + 1);
-    const int u = (int)(w - t * (nsamples + 1));
+  for (int64_t w = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); w < T * groups; w += warps) {
+    const int64_t t = w / groups;
+    const int u = (int)(w - t * groups);
+    const bool last = u == groups - 1;
+    const int n0 = u * SPW;
+    const int ns = last ? 1 : min(SPW, nsamples - n0);
     const int r = (int)(t / kb), j = (int)(t - (int64_t)r * kb);
-    const float *src = u < nsamples ? G + (int64_t)u * D : g;
-    float ah = 0.f, al = 0.f, bh = 0.f, bl = 0.f;
-    for (int v = lane; v < bn * bk; v += 32) {
-      const int i = v / bk, l = v - i * bk;
-      const int64_t e = (int64_t)(r * bn + i) * k + (int64_t)j * bk + l;
-      const float wv = __uint_as_float((uint32_t)__ldg(W + e) << 16);
-      const float gv = __ldg(src + e);
-      const float p = __fmul_rn(wv, gv);
-      const float pe = __fmaf_rn(wv, gv, -p);  // w * g = p + pe exactly
-      pair_add(ah, al, p);
-      al = __fadd_rn(al, pe);
-      if (u == nsamples) {
-        const float q = __fmul_rn(wv, wv);  // a bf16 square has at most 16 bits: exact
-        pair_add(bh, bl, q);
+    float ah[SPW], al[SPW];
+#pragma unroll
+    for (int q = 0; q < SPW; ++q) ah[q] = al[q] = 0.f;
+    float bh = 0.f, bl = 0.f;
+    for (int c = lane; c < chunks; c += 32) {
+      const int i = c / CPR, l = 4 * (c - i * CPR);
+      const int64_t e = (int64_t)(r * bn + i) * k + (int64_t)j * BK + l;
+      const uint2 wr = __ldg(reinterpret_cast<const uint2 *>(W + e));
+      const float wv[4] = {__uint_as_float(wr.x << 16), __uint_as_float(wr.x & 0xffff0000u),
+                           __uint_as_float(wr.y << 16), __uint_as_float(wr.y & 0xffff0000u)};
+#pragma unroll
+      for (int q = 0; q < SPW; ++q) {
+        if (q < ns) {
+          const float *src = last ? g : G + (int64_t)(n0 + q) * D;
+          const float4 gv4 = __ldg(reinterpret_cast<const float4 *>(src + e));
+          const float gv[4] = {gv4.x, gv4.y, gv4.z, gv4.w};
+#pragma unroll
+          for (int x = 0; x < 4; ++x) {
+            const float p = __fmul_rn(wv[x], gv[x]);
+            const float pe = __fmaf_rn(wv[x], gv[x], -p);  // w * g = p + pe exactly
+            pair_add(ah[q], al[q], p);
+            al[q] = __fadd_rn(al[q], pe);
+          }
+        }
+      }
+      if (last) {
+#pragma unroll
+        for (int x = 0; x < 4; ++x) pair_add(bh, bl, __fmul_rn(wv[x], wv[x]));  // a bf16 square is exact
       }
     }
-    warp_pair_sum(ah, al);
-    if (u < nsamples) {
-      if (lane == 0) s[(int64_t)u * T + t] = make_float2(ah, al);
-    } else {
-      warp_pair_sum(bh, bl);
-      if (lane == 0) {
-        gw[t] = make_float2(ah, al);
-        w2[t] = make_float2(bh, bl);
+#pragma unroll
+    for (int q = 0; q < SPW; ++q) {
+      if (q < ns) {
+        warp_pair_sum(ah[q], al[q]);
+        if (lane == 0) {
+          if (last) gw[t] = make_float2(ah[q], al[q]);
+          else s[(int64_t)(n0 + q) * T + t] = make_float2(ah[q], al[q]);
+        }
       }
+    }
+    if (last) {
+      warp_pair_sum(bh, bl);
+      if (lane == 0) w2[t] = make_float2(bh, bl);
     }
   }
 }
@@ -301,7 +327,7 @@ lpvit_status lpvit_delta_curve(const void *W, const float *G, int32_t nsamples, 
   grid = (T + ALLOC_THREADS - 1) / ALLOC_THREADS;
   order_kernel<<<(int)(grid < 152 * 8 ? grid : 152 * 8), ALLOC_THREADS, 0, st>>>(rank, T, order);
   if (cudaGetLastError() != cudaSuccess) return LPVIT_ERR_CUDA;
-  const int64_t warps = T * (nsamples + 1);
+  const int64_t warps = T * ((nsamples + SPW - 1) / SPW + 1);
   grid = (warps + ALLOC_THREADS / 32 - 1) / (ALLOC_THREADS / 32);
   const int bgrid = (int)(grid < 152 * 64 ? grid : 152 * 64);
   switch (bk) {
