@@ -174,6 +174,27 @@ lpvit_status lpvit_lambda_search(int32_t layers, int32_t steps, const double *de
                                  const double *power_coef, double beta, double flops_ratio, int32_t *k_out,
                                  double *lambda_out, double *ratio_out);
 
+/* The non-linear parts of a pre-norm ViT (DeiT) encoder block, so that a whole encoder forward
+ * around the block-sparse linears runs in this library (the pruned ViTs of Sec. 4).
+ *
+ * Residual add + LayerNorm over rows of D features (bf16 [rows][D], row-major, 16-byte aligned):
+ *   s = bf16(x + r)  (r may be NULL: s = x),   y = (s - mean) / sqrt(var + eps) * gamma + beta,
+ * mean and biased variance over the row in float32; y rounded to bf16 into norm_out, s stored into
+ * sum_out when r is given. gamma, beta float32 [D], 16-byte aligned. 8 <= D <= 1024, D % 8 == 0,
+ * eps > 0. Asynchronous on `stream`. Errors: LPVIT_ERR_INVALID_ARG, LPVIT_ERR_CUDA. */
+lpvit_status lpvit_add_layernorm(const void *x, const void *r, const float *gamma, const float *beta, int64_t rows,
+                                 int32_t D, double eps, void *sum_out, void *norm_out, void *stream);
+
+/* Multi-head softmax self-attention per image: qkv bf16 [images * tokens][3 * heads * head_dim]
+ * (columns ordered q, k, v, each split into heads of head_dim), out bf16 [images * tokens]
+ * [heads * head_dim] = softmax(q k^T / sqrt(head_dim)) v per image and head, heads concatenated.
+ * bf16 tensor-core products with fp32 accumulation; the softmax weights are rounded to bf16 for
+ * the product with v. head_dim == 64 and 1 <= tokens <= 208 (DeiT: 197) else
+ * LPVIT_ERR_UNSUPPORTED; both pointers 16-byte aligned. Asynchronous on `stream`.
+ * Errors: LPVIT_ERR_UNSUPPORTED, LPVIT_ERR_INVALID_ARG, LPVIT_ERR_CUDA. */
+lpvit_status lpvit_attention(const void *qkv, int64_t images, int32_t tokens, int32_t heads, int32_t head_dim,
+                             void *out, void *stream);
+
 /* Bytes of device workspace lpvit_bsr_linear[_gelu] needs for m tokens. The workspace holds
  * scheduler counters, the device error word and, for small m, fp32 partial sums of split
  * work units. It must be zero-filled once before its first use (cudaMemset); every call

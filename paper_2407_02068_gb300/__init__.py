@@ -12,6 +12,8 @@ or 64 (Table 2 uses 32x32, 64x32, 16x32 and 16x16). This package wraps the C lib
 * ``bsr_linear(w, X, bias, gelu=...)`` -- Y = act(X (W (.) M)^T + bias)
 * ``delta_curve(W, G, b, steps, kappa)`` / ``lambda_search(...)`` -- the layer-wise pruning-ratio
   allocation of Sec. 3.4-3.5 (empirical-Fisher distortion curves, Lagrangian slope matching)
+* ``add_layernorm`` / ``attention`` -- the rest of a pre-norm ViT block; ``encoder.SparseEncoder``
+  runs a whole DeiT encoder forward on them and the block-sparse linears
 
 PyTorch provides device memory and streams only; every step runs in the library's kernels.
 """
@@ -24,7 +26,8 @@ import torch
 from . import _lib
 
 __all__ = ["BsrWeight", "alloc_bsr", "pack_bsr", "pack_bsr_into", "pack_bsr_many_into", "taylor_block_mask",
-           "workspace_for", "bsr_linear", "check", "LpvitError", "delta_curve", "lambda_search", "mean_gradient"]
+           "workspace_for", "bsr_linear", "check", "LpvitError", "delta_curve", "lambda_search", "mean_gradient",
+           "add_layernorm", "attention"]
 
 LpvitError = _lib.LpvitError
 
@@ -141,6 +144,48 @@ def delta_curve(W: torch.Tensor, G: torch.Tensor, b, steps: int, kappa: float, w
     if st != _lib.LPVIT_OK:
         raise LpvitError(st, "lpvit_delta_curve")
     return out
+
+
+def add_layernorm(x: torch.Tensor, r: torch.Tensor | None, gamma: torch.Tensor, beta: torch.Tensor,
+                  eps: float = 1e-6, norm_out: torch.Tensor | None = None, sum_out: torch.Tensor | None = None,
+                  stream=None):
+    """s = bf16(x + r) (r may be None: s = x) and y = LayerNorm(s) * gamma + beta over the last axis.
+    x, r: contiguous bf16 CUDA [rows, D]; gamma, beta: float32 [D]. Returns y, or (s, y) when r is
+    given."""
+    if x.dtype != torch.bfloat16 or not x.is_cuda or x.dim() != 2 or not x.is_contiguous():
+        raise ValueError("x must be a contiguous 2-D bf16 CUDA tensor")
+    rows, D = x.shape
+    if r is not None and (r.shape != x.shape or r.dtype != x.dtype or not r.is_contiguous()):
+        raise ValueError("r must match x")
+    if gamma.dtype != torch.float32 or beta.dtype != torch.float32 or gamma.numel() != D or beta.numel() != D:
+        raise ValueError("gamma and beta must be float32 [D]")
+    y = norm_out if norm_out is not None else torch.empty_like(x)
+    sm = None
+    if r is not None:
+        sm = sum_out if sum_out is not None else torch.empty_like(x)
+    st = _lib.lpvit_add_layernorm(x.data_ptr(), 0 if r is None else r.data_ptr(), gamma.data_ptr(), beta.data_ptr(),
+                                  rows, D, eps, 0 if sm is None else sm.data_ptr(), y.data_ptr(),
+                                  _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_add_layernorm")
+    return y if r is None else (sm, y)
+
+
+def attention(qkv: torch.Tensor, tokens: int, heads: int, out: torch.Tensor | None = None, stream=None):
+    """softmax(q k^T / sqrt(head_dim)) v per image and head: qkv bf16 [images * tokens, 3 * heads * 64],
+    contiguous CUDA; returns bf16 [images * tokens, heads * 64]."""
+    if qkv.dtype != torch.bfloat16 or not qkv.is_cuda or qkv.dim() != 2 or not qkv.is_contiguous():
+        raise ValueError("qkv must be a contiguous 2-D bf16 CUDA tensor")
+    M, C = qkv.shape
+    if M % tokens or C % (3 * heads):
+        raise ValueError("qkv shape does not match tokens and heads")
+    head_dim = C // (3 * heads)
+    o = out if out is not None else torch.empty((M, C // 3), dtype=torch.bfloat16, device=qkv.device)
+    st = _lib.lpvit_attention(qkv.data_ptr(), M // tokens, tokens, heads, head_dim, o.data_ptr(),
+                              _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_attention")
+    return o
 
 
 def mean_gradient(G: torch.Tensor, stream=None) -> torch.Tensor:

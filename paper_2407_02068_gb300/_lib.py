@@ -24,7 +24,8 @@ LPVIT_F32 = 1
 EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_workspace_bytes", "lpvit_bsr_linear",
            "lpvit_bsr_linear_gelu", "lpvit_bsr_linear_noalloc", "lpvit_check", "lpvit_status_string",
            "lpvit_selftest_wait", "lpvit_pack_bsr_many", "lpvit_taylor_block_mask",
-           "lpvit_delta_curve_workspace_bytes", "lpvit_delta_curve", "lpvit_lambda_search", "lpvit_mean_gradient")
+           "lpvit_delta_curve_workspace_bytes", "lpvit_delta_curve", "lpvit_lambda_search", "lpvit_mean_gradient",
+           "lpvit_add_layernorm", "lpvit_attention")
 LPVIT_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 
@@ -70,6 +71,10 @@ def load(path: str | None = None):
         lib.lpvit_delta_curve_workspace_bytes.argtypes = [I32, I32, I32, I32, I32, I32]
         lib.lpvit_delta_curve.restype = ctypes.c_int
         lib.lpvit_delta_curve.argtypes = [V, V, I32, I32, I32, I32, I32, ctypes.c_double, I32, V, V, SZ, V]
+        lib.lpvit_add_layernorm.restype = ctypes.c_int
+        lib.lpvit_add_layernorm.argtypes = [V, V, V, V, I64, I32, ctypes.c_double, V, V, V]
+        lib.lpvit_attention.restype = ctypes.c_int
+        lib.lpvit_attention.argtypes = [V, I64, I32, I32, I32, V, V]
         lib.lpvit_mean_gradient.restype = ctypes.c_int
         lib.lpvit_mean_gradient.argtypes = [V, I32, I64, V, V]
         lib.lpvit_lambda_search.restype = ctypes.c_int
@@ -136,6 +141,14 @@ def lpvit_delta_curve(W_ptr, G_ptr, nsamples, n, k, bn, bk, kappa, steps, delta_
                       stream) -> int:
     return load().lpvit_delta_curve(W_ptr, G_ptr, nsamples, n, k, bn, bk, float(kappa), steps, delta_ptr, ws_ptr,
                                     ws_bytes, stream)
+
+
+def lpvit_add_layernorm(x_ptr, r_ptr, gamma_ptr, beta_ptr, rows, D, eps, sum_ptr, norm_ptr, stream) -> int:
+    return load().lpvit_add_layernorm(x_ptr, r_ptr, gamma_ptr, beta_ptr, rows, D, float(eps), sum_ptr, norm_ptr, stream)
+
+
+def lpvit_attention(qkv_ptr, images, tokens, heads, head_dim, out_ptr, stream) -> int:
+    return load().lpvit_attention(qkv_ptr, images, tokens, heads, head_dim, out_ptr, stream)
 
 
 def lpvit_mean_gradient(G_ptr, nsamples, count, g_ptr, stream) -> int:

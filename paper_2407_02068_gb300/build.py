@@ -20,7 +20,7 @@ BUILD = os.path.join(PKG, "_build")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(BUILD, "liblpvit.so")
 SOURCES = ["lpvit_pack.cu", "lpvit_linear.cu", "lpvit_api.cu", "lpvit_noalloc.cu", "lpvit_selftest.cu",
-           "lpvit_mask.cu", "lpvit_alloc.cu"]
+           "lpvit_mask.cu", "lpvit_alloc.cu", "lpvit_encoder.cu"]
 HEADERS = ["lpvit_device.cuh", "lpvit_taylor.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

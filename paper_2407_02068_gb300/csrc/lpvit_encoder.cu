@@ -1,0 +1,281 @@
+// The non-linear parts of a pre-norm ViT (DeiT) encoder block around the block-sparse linears, so
+// that a whole encoder forward runs in this library's kernels: residual add + LayerNorm, and
+// multi-head softmax attention.
+//
+// add_layernorm_kernel (one warp per token row, 16-byte vectors): s = bf16(x + r) (x alone when r
+//   is null), then y = (s - mean) / sqrt(var + eps) * gamma + beta over the row in float32 (biased
+//   variance, two passes over the row held in registers), stored as bf16; s is stored too when r
+//   is given (the new residual stream).
+// attention_kernel (one CTA of 4 warps per image and head; head_dim 64, at most 208 tokens): Q, K
+//   and V of the head are staged in shared memory (rows padded to 144 bytes: ldmatrix rows fall in
+//   distinct banks), each warp takes 16-query tiles: S = Q K^T with bf16 tensor-core MMAs
+//   (mma.sync m16n8k16, fp32 accumulation) for all keys at once in registers, scaled by
+//   1/sqrt(64) = 1/8, padded keys masked, row max and sum over the four lanes sharing a row, P =
+//   exp(S - max) rounded to bf16 as the A operand of O = P V (V fragments by ldmatrix.trans),
+//   O / sum stored as bf16. Attention is under 1% of a DeiT forward's FLOPs, so these legacy
+//   warp-level MMAs are used rather than tcgen05.
+#include <cmath>
+#include <cstdint>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "lpvit.h"
+
+namespace lpvit {
+
+namespace {
+
+constexpr int LN_THREADS = 256;
+constexpr int LN_MAX_D = 1024;
+constexpr int LN_VPL = LN_MAX_D / 8 / 32;  // 16-byte vectors per lane at most
+
+constexpr int ATT_WARPS = 4;
+constexpr int HD = 64;                   // head dimension
+constexpr int MAX_TOKENS = 208;          // 13 tiles of 16
+constexpr int NT = MAX_TOKENS / 8;       // key tiles of 8
+constexpr int ROW = HD + 8;              // shared-memory row in bf16 (144 bytes)
+constexpr int ATT_SMEM = 3 * MAX_TOKENS * ROW * 2;
+
+__device__ __forceinline__ float warp_sum_f(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__global__ void __launch_bounds__(LN_THREADS)
+add_layernorm_kernel(const __nv_bfloat16 *__restrict__ x, const __nv_bfloat16 *__restrict__ r,
+                     const float *__restrict__ gamma, const float *__restrict__ beta, int64_t rows, int D, float eps,
+                     __nv_bfloat16 *__restrict__ sum_out, __nv_bfloat16 *__restrict__ norm_out) {
+  const int lane = threadIdx.x & 31;
+  const int nv = D / 8;
+  const int64_t warps = (int64_t)gridDim.x * (blockDim.x / 32);
+  for (int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5); row < rows; row += warps) {
+    const int64_t base = row * D;
+    float v[LN_VPL][8];
+    float s1 = 0.f;
+#pragma unroll
+    for (int i = 0; i < LN_VPL; ++i) {
+      const int c = lane + 32 * i;
+      if (c < nv) {
+        const uint4 xv = __ldg(reinterpret_cast<const uint4 *>(x + base) + c);
+        const __nv_bfloat16 *xb = reinterpret_cast<const __nv_bfloat16 *>(&xv);
+        uint4 sv = xv;
+        if (r) {
+          const uint4 rv = __ldg(reinterpret_cast<const uint4 *>(r + base) + c);
+          const __nv_bfloat16 *rb = reinterpret_cast<const __nv_bfloat16 *>(&rv);
+          __nv_bfloat16 *sb = reinterpret_cast<__nv_bfloat16 *>(&sv);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) sb[e] = __float2bfloat16_rn(__bfloat162float(xb[e]) + __bfloat162float(rb[e]));
+          reinterpret_cast<uint4 *>(sum_out + base)[c] = sv;
+        }
+        const __nv_bfloat16 *sb = reinterpret_cast<const __nv_bfloat16 *>(&sv);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          v[i][e] = __bfloat162float(sb[e]);
+          s1 += v[i][e];
+        }
+      }
+    }
+    const float mean = warp_sum_f(s1) / (float)D;
+    float s2 = 0.f;
+#pragma unroll
+    for (int i = 0; i < LN_VPL; ++i)
+      if (lane + 32 * i < nv) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float d = v[i][e] - mean;
+          s2 += d * d;
+        }
+      }
+    const float rstd = rsqrtf(warp_sum_f(s2) / (float)D + eps);
+#pragma unroll
+    for (int i = 0; i < LN_VPL; ++i) {
+      const int c = lane + 32 * i;
+      if (c < nv) {
+        uint4 ov;
+        __nv_bfloat16 *ob = reinterpret_cast<__nv_bfloat16 *>(&ov);
+        const float4 g0 = __ldg(reinterpret_cast<const float4 *>(gamma) + 2 * c);
+        const float4 g1 = __ldg(reinterpret_cast<const float4 *>(gamma) + 2 * c + 1);
+        const float4 b0 = __ldg(reinterpret_cast<const float4 *>(beta) + 2 * c);
+        const float4 b1 = __ldg(reinterpret_cast<const float4 *>(beta) + 2 * c + 1);
+        const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+        const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) ob[e] = __float2bfloat16_rn((v[i][e] - mean) * rstd * gg[e] + bb[e]);
+        reinterpret_cast<uint4 *>(norm_out + base)[c] = ov;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &a0, uint32_t &a1, uint32_t &a2, uint32_t &a3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(a0), "=r"(a1), "=r"(a2), "=r"(a3) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t &b0, uint32_t &b1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];" : "=r"(b0), "=r"(b1) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2_trans(uint32_t addr, uint32_t &b0, uint32_t &b1) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0,%1}, [%2];" : "=r"(b0), "=r"(b1) : "r"(addr));
+}
+// D (16x8 fp32) += A (16x16 bf16, row) * B (16x8 bf16, col)
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+  asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+               "{%0,%1,%2,%3};"
+               : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+               : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t *>(&p);
+}
+
+__global__ void __launch_bounds__(32 * ATT_WARPS)
+attention_kernel(const __nv_bfloat16 *__restrict__ qkv, int tokens, int heads, __nv_bfloat16 *__restrict__ out) {
+  extern __shared__ __align__(16) __nv_bfloat16 att_smem[];
+  __nv_bfloat16 *Qs = att_smem, *Ks = Qs + MAX_TOKENS * ROW, *Vs = Ks + MAX_TOKENS * ROW;
+  const int img = blockIdx.x / heads, h = blockIdx.x - img * heads;
+  const int D = heads * HD;
+  const int tp = (tokens + 15) / 16 * 16;  // padded token count
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // stage Q, K, V of this head (8 vectors of 16 bytes per row each); padded rows are zero
+  for (int idx = threadIdx.x; idx < tp * 8 * 3; idx += blockDim.x) {
+    const int m = idx / (tp * 8), rem = idx - m * tp * 8, row = rem >> 3, c = rem & 7;
+    uint4 val = make_uint4(0, 0, 0, 0);
+    if (row < tokens)
+      val = __ldg(reinterpret_cast<const uint4 *>(qkv + ((int64_t)img * tokens + row) * 3 * D + m * D + h * HD) + c);
+    reinterpret_cast<uint4 *>(att_smem + (m * MAX_TOKENS + row) * ROW)[c] = val;
+  }
+  __syncthreads();
+  const int ntiles = tp / 8, kq = lane & 3, rq = lane >> 2;
+  for (int mt = warp; mt < tp / 16; mt += ATT_WARPS) {
+    uint32_t qa[HD / 16][4];
+#pragma unroll
+    for (int ks = 0; ks < HD / 16; ++ks)
+      ldsm_x4(smem_addr(Qs + (16 * mt + (lane & 15)) * ROW + 16 * ks + (lane >> 4) * 8), qa[ks][0], qa[ks][1],
+              qa[ks][2], qa[ks][3]);
+    float s[NT][4];
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+      if (nt < ntiles) {
+#pragma unroll
+        for (int ks = 0; ks < HD / 16; ++ks) {
+          uint32_t b0, b1;
+          ldsm_x2(smem_addr(Ks + (8 * nt + (lane & 7)) * ROW + 16 * ks + ((lane >> 3) & 1) * 8), b0, b1);
+          mma_bf16(s[nt], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
+        }
+      }
+    }
+    // scale, mask, row max (rows rq and rq + 8 of the tile; columns 8 nt + 2 kq + {0, 1})
+    float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int col = 8 * nt + 2 * kq + (e & 1);
+        s[nt][e] = (nt < ntiles && col < tokens) ? s[nt][e] * 0.125f : -INFINITY;
+      }
+      mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]));
+      mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]));
+    }
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+    float sum0 = 0.f, sum1 = 0.f;
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      s[nt][0] = expf(s[nt][0] - mx0);
+      s[nt][1] = expf(s[nt][1] - mx0);
+      s[nt][2] = expf(s[nt][2] - mx1);
+      s[nt][3] = expf(s[nt][3] - mx1);
+      sum0 += s[nt][0] + s[nt][1];
+      sum1 += s[nt][2] + s[nt][3];
+    }
+    sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
+    sum0 += __shfl_xor_sync(0xffffffffu, sum0, 2);
+    sum1 += __shfl_xor_sync(0xffffffffu, sum1, 1);
+    sum1 += __shfl_xor_sync(0xffffffffu, sum1, 2);
+    // O = P V
+    float o[HD / 8][4];
+#pragma unroll
+    for (int nd = 0; nd < HD / 8; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
+#pragma unroll
+    for (int kt = 0; kt < NT / 2; ++kt) {
+      if (2 * kt < ntiles) {
+        const uint32_t a0 = pack_bf16(s[2 * kt][0], s[2 * kt][1]), a1 = pack_bf16(s[2 * kt][2], s[2 * kt][3]);
+        const uint32_t a2 = pack_bf16(s[2 * kt + 1][0], s[2 * kt + 1][1]);
+        const uint32_t a3 = pack_bf16(s[2 * kt + 1][2], s[2 * kt + 1][3]);
+#pragma unroll
+        for (int nd = 0; nd < HD / 8; ++nd) {
+          uint32_t b0, b1;
+          ldsm_x2_trans(smem_addr(Vs + (16 * kt + (lane & 15)) * ROW + 8 * nd), b0, b1);
+          mma_bf16(o[nd], a0, a1, a2, a3, b0, b1);
+        }
+      }
+    }
+    const float inv0 = 1.f / sum0, inv1 = 1.f / sum1;
+    const int r0 = 16 * mt + rq, r1 = r0 + 8;
+#pragma unroll
+    for (int nd = 0; nd < HD / 8; ++nd) {
+      const int col = h * HD + 8 * nd + 2 * kq;
+      if (r0 < tokens)
+        *reinterpret_cast<uint32_t *>(out + ((int64_t)img * tokens + r0) * D + col) =
+            pack_bf16(o[nd][0] * inv0, o[nd][1] * inv0);
+      if (r1 < tokens)
+        *reinterpret_cast<uint32_t *>(out + ((int64_t)img * tokens + r1) * D + col) =
+            pack_bf16(o[nd][2] * inv1, o[nd][3] * inv1);
+    }
+  }
+}
+
+bool aligned_to(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+}  // namespace
+}  // namespace lpvit
+
+using namespace lpvit;
+
+extern "C" {
+
+lpvit_status lpvit_add_layernorm(const void *x, const void *r, const float *gamma, const float *beta, int64_t rows,
+                                 int32_t D, double eps, void *sum_out, void *norm_out, void *stream) {
+  if (rows < 0 || D < 8 || D > LN_MAX_D || D % 8 || !(eps > 0.0) || !std::isfinite(eps)) return LPVIT_ERR_INVALID_ARG;
+  if (rows == 0) return LPVIT_OK;
+  if (!x || !gamma || !beta || !norm_out || (r && !sum_out)) return LPVIT_ERR_INVALID_ARG;
+  if (!aligned_to(x, 16) || !aligned_to(gamma, 16) || !aligned_to(beta, 16) || !aligned_to(norm_out, 16) ||
+      (r && (!aligned_to(r, 16) || !aligned_to(sum_out, 16))))
+    return LPVIT_ERR_INVALID_ARG;
+  const int64_t want = (rows + LN_THREADS / 32 - 1) / (LN_THREADS / 32);
+  const int grid = (int)(want < 152 * 32 ? want : 152 * 32);
+  add_layernorm_kernel<<<grid, LN_THREADS, 0, static_cast<cudaStream_t>(stream)>>>(
+      static_cast<const __nv_bfloat16 *>(x), static_cast<const __nv_bfloat16 *>(r), gamma, beta, rows, D, (float)eps,
+      static_cast<__nv_bfloat16 *>(sum_out), static_cast<__nv_bfloat16 *>(norm_out));
+  return cudaGetLastError() == cudaSuccess ? LPVIT_OK : LPVIT_ERR_CUDA;
+}
+
+lpvit_status lpvit_attention(const void *qkv, int64_t images, int32_t tokens, int32_t heads, int32_t head_dim,
+                             void *out, void *stream) {
+  if (head_dim != HD || tokens < 1 || tokens > MAX_TOKENS) return LPVIT_ERR_UNSUPPORTED;
+  if (images < 0 || heads < 1 || heads > 64) return LPVIT_ERR_INVALID_ARG;
+  if (images == 0) return LPVIT_OK;
+  if (images * heads > 0x7fffffffLL) return LPVIT_ERR_INVALID_ARG;
+  if (!qkv || !out || !aligned_to(qkv, 16) || !aligned_to(out, 16)) return LPVIT_ERR_INVALID_ARG;
+  static bool attr_done[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+    if (cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, ATT_SMEM) != cudaSuccess)
+      return LPVIT_ERR_CUDA;
+    attr_done[dev] = true;
+  }
+  attention_kernel<<<(int)(images * heads), 32 * ATT_WARPS, ATT_SMEM, static_cast<cudaStream_t>(stream)>>>(
+      static_cast<const __nv_bfloat16 *>(qkv), tokens, heads, static_cast<__nv_bfloat16 *>(out));
+  return cudaGetLastError() == cudaSuccess ? LPVIT_OK : LPVIT_ERR_CUDA;
+}
+
+}  // extern "C"

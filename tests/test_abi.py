@@ -141,3 +141,21 @@ def test_allocation_arguments_are_checked_without_a_gpu(lib):
     st, *_ = lib.lpvit_lambda_search([[0.0, float("nan")]], 1, [1.0], [1.0], 0.0, 0.5)
     assert st == lib.LPVIT_ERR_INVALID_ARG
     assert L.lpvit_lambda_search(0, 1, None, None, None, 0.0, 0.5, None, None, None) == lib.LPVIT_ERR_INVALID_ARG
+
+
+def test_encoder_kernel_arguments_are_checked_without_a_gpu(lib):
+    ln = lib.lpvit_add_layernorm
+    assert ln(0x1000, None, 0x2000, 0x3000, 0, 384, 1e-6, None, 0x4000, None) == lib.LPVIT_OK   # no rows
+    for bad in ((0x1000, None, 0x2000, 0x3000, 4, 1028, 1e-6, None, 0x4000),     # D > 1024
+                (0x1000, None, 0x2000, 0x3000, 4, 100, 1e-6, None, 0x4000),      # D % 8
+                (0x1000, None, 0x2000, 0x3000, 4, 384, 0.0, None, 0x4000),       # eps
+                (0x1000, 0x5000, 0x2000, 0x3000, 4, 384, 1e-6, None, 0x4000),    # r without sum_out
+                (0x1008, None, 0x2000, 0x3000, 4, 384, 1e-6, None, 0x4000),      # alignment
+                (0, None, 0x2000, 0x3000, 4, 384, 1e-6, None, 0x4000)):
+        assert ln(*bad, None) == lib.LPVIT_ERR_INVALID_ARG, bad
+    at = lib.lpvit_attention
+    assert at(0x1000, 2, 197, 6, 32, 0x2000, None) == lib.LPVIT_ERR_UNSUPPORTED    # head_dim
+    assert at(0x1000, 2, 209, 6, 64, 0x2000, None) == lib.LPVIT_ERR_UNSUPPORTED    # tokens
+    assert at(0x1000, 0, 197, 6, 64, 0x2000, None) == lib.LPVIT_OK                 # no images
+    assert at(0x1008, 2, 197, 6, 64, 0x2000, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert at(0x1000, 2, 197, 0, 64, 0x2000, None) == lib.LPVIT_ERR_INVALID_ARG
