@@ -62,6 +62,9 @@ def parse_args():
     p.add_argument("--alloc", action="store_true",
                    help="pruning-ratio allocation: distortion curves of the 48 DeiT-B weights + lambda search")
     p.add_argument("--alloc-samples", type=int, default=16, help="per-sample gradients per layer (--alloc)")
+    p.add_argument("--encoder", choices=["deit_b", "deit_s"], default=None,
+                   help="end-to-end encoder forward (LayerNorm, attention, block-sparse linears) against dense")
+    p.add_argument("--images", type=int, default=256, help="batch of 197-token images (--encoder)")
     return p.parse_args()
 
 
@@ -606,6 +609,105 @@ def run_alloc(args, local):
     print(json.dumps(line), flush=True)
 
 
+def run_encoder(args, local):
+    """End-to-end pre-norm encoder forward (the pruned ViTs of Sec. 4): DeiT-B (12 layers, 768 wide,
+    12 heads) or DeiT-S (12 layers, 384 wide, 6 heads), 32x32 blocks with the stack's per-GEMM
+    sparsities (U[0.30, 0.70], mean 50%), seeded random weights, masks, biases and LayerNorm
+    parameters, 197-token images. Times the library's forward (every step in liblpvit.so: 2
+    add+LayerNorms, 4 block-sparse linears and attention per layer, a final LayerNorm) and the same
+    model on torch's dense bf16 operations, with CUDA events; the speedup over dense is the measure
+    the paper reports end to end on its A100. e2e adds the host->device copy of the images and the
+    device->host copy of the output every step."""
+    import torch
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2407_02068_gb300 import inputs
+    from paper_2407_02068_gb300.encoder import SparseEncoder
+    model = inputs.DEIT_B if args.encoder == "deit_b" else inputs.DEIT_S
+    D, hidden, heads, T, b = model["dim"], model["hidden"], model["dim"] // 64, 197, 32
+    config = 9
+    sp = inputs.stack_sparsities(config)
+    gen = torch.Generator(device=dev).manual_seed(inputs.seed(config, 0, "bias"))
+    layers = []
+    for l in range(12):
+        lay = {"ln1": ((1 + 0.1 * torch.randn(D, generator=gen, device=dev)).contiguous(),
+                       (0.1 * torch.randn(D, generator=gen, device=dev)).contiguous()),
+               "ln2": ((1 + 0.1 * torch.randn(D, generator=gen, device=dev)).contiguous(),
+                       (0.1 * torch.randn(D, generator=gen, device=dev)).contiguous())}
+        for t, (name, k, n, _) in enumerate(inputs.deit_gemms(model)):
+            gi = 4 * l + t
+            lay[name] = (inputs.weight(n, k, inputs.seed(config, gi, "W"), dev),
+                         inputs.uniform_mask(n, k, b, sp[l][t], inputs.seed(config, gi, "mask")).to(dev),
+                         inputs.bias(n, inputs.seed(config, gi, "bias"), dev))
+        layers.append(lay)
+    final = ((1 + 0.1 * torch.randn(D, generator=gen, device=dev)).contiguous(),
+             (0.1 * torch.randn(D, generator=gen, device=dev)).contiguous())
+    enc = SparseEncoder(layers, final, heads, T, b)
+    M = args.images * T
+    x = inputs.activations(M, D, inputs.seed(config, 0, "X"), dev)
+    steps, warm = max(args.steps // 20, 5), max(args.warmup, 3)
+
+    def timed(fn):
+        for _ in range(warm):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(steps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / steps
+
+    clk = ClockSampler(local)
+    clk.start()
+    ms_sparse = timed(lambda: enc.forward(x))
+    clocks = clk.stop()
+    ms_dense = timed(lambda: enc.dense_forward(x))
+    # end to end: pinned host images in, output back, every step
+    xh = x.cpu().pin_memory()
+    yh = torch.empty((M, D), dtype=torch.bfloat16).pin_memory()
+    xd = torch.empty_like(x)
+
+    def e2e_step():
+        xd.copy_(xh, non_blocking=True)
+        yh.copy_(enc.forward(xd), non_blocking=True)
+    ms_e2e = timed(e2e_step)
+    dense_flops = sum(2 * M * k * n for l in range(12) for (_, k, n, _) in inputs.deit_gemms(model))
+    eff_flops = sum(2 * M * int((L[name][1] != 0).sum()) * b * b for L in layers for name in ("qkv", "proj", "fc1", "fc2"))
+    line = {"metric": f"end-to-end {args.encoder} encoder forward throughput", "value": args.images / (ms_sparse / 1e3),
+            "unit": "images/s", "n_gpus": 1, "steps": steps, "warmup": warm, "ms_per_step": ms_sparse,
+            "higher_is_better": True, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": f"{args.encoder}_12layer_encoder_batch{args.images}", "images": args.images,
+                       "tokens": T, "block": b, "sparsity": "per-GEMM U[0.30,0.70], antithetic layer pairs, mean 0.50",
+                       "flops_remained_linears": eff_flops / dense_flops},
+            "dense_torch_ms_per_step": ms_dense, "speedup_vs_dense": ms_dense / ms_sparse,
+            "e2e": {"value": args.images / (ms_e2e / 1e3), "unit": "images/s", "h2d_bytes_per_step": 2 * M * D,
+                    "d2h_bytes_per_step": 2 * M * D},
+            "gpu_launches": steps * enc.launches(), "clocks": clocks}
+    if not args.no_cpu_baseline:
+        import numpy as np
+        import oracle
+        from oracle import encoder as oenc
+        ol = []
+        for L in layers:
+            d = {"ln1": tuple(v.cpu().double().numpy() for v in L["ln1"]),
+                 "ln2": tuple(v.cpu().double().numpy() for v in L["ln2"])}
+            for name in ("qkv", "proj", "fc1", "fc2"):
+                W, Mk, bias = L[name]
+                d[name] = (inputs.bf16_bits(W), Mk.cpu().numpy(), bias.cpu().numpy(), b)
+            ol.append(d)
+        of = tuple(v.cpu().double().numpy() for v in final)
+        t0 = time.perf_counter()
+        oenc.encoder_forward(inputs.bf16_bits(x[:T]), ol, of, T, heads)
+        cpu_s = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": 1.0 / cpu_s, "unit": "images/s", "cores": os.cpu_count(), "kind": "oracle",
+                                "sample": f"one image through the 12-layer encoder, fp64 C/numpy oracle, {cpu_s:.1f} s"}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     world, rank, local = dist_setup(args)
@@ -617,6 +719,9 @@ def main():
         return
     if args.alloc:
         run_alloc(args, local)
+        return
+    if args.encoder:
+        run_encoder(args, local)
         return
     if args.case != "stack":
         run_case(args, local)
