@@ -7,8 +7,8 @@
 //   variance, two passes over the row held in registers), stored as bf16; s is stored too when r
 //   is given (the new residual stream).
 // attention_kernel (one CTA of 4 warps per image and head; head_dim 64, at most 208 tokens): Q, K
-//   and V of the head are staged in shared memory (rows padded to 144 bytes: ldmatrix rows fall in
-//   distinct banks), each warp takes 16-query tiles: S = Q K^T with bf16 tensor-core MMAs
+//   and V of the head are staged in shared memory by asynchronous 16-byte copies (rows padded to
+//   144 bytes: ldmatrix rows fall in distinct banks), each warp takes 16-query tiles: S = Q K^T with bf16 tensor-core MMAs
 //   (mma.sync m16n8k16, fp32 accumulation) for all keys at once in registers, scaled by
 //   1/sqrt(64) = 1/8, padded keys masked, row max and sum over the four lanes sharing a row, P =
 //   exp(S - max) rounded to bf16 as the A operand of O = P V (V fragments by ldmatrix.trans),
@@ -141,14 +141,20 @@ attention_kernel(const __nv_bfloat16 *__restrict__ qkv, int tokens, int heads, _
   const int D = heads * HD;
   const int tp = (tokens + 15) / 16 * 16;  // padded token count
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // stage Q, K, V of this head (8 vectors of 16 bytes per row each); padded rows are zero
+  // stage Q, K, V of this head (8 vectors of 16 bytes per row each) with asynchronous copies, all
+  // in flight together; padded rows are zero
   for (int idx = threadIdx.x; idx < tp * 8 * 3; idx += blockDim.x) {
     const int m = idx / (tp * 8), rem = idx - m * tp * 8, row = rem >> 3, c = rem & 7;
-    uint4 val = make_uint4(0, 0, 0, 0);
-    if (row < tokens)
-      val = __ldg(reinterpret_cast<const uint4 *>(qkv + ((int64_t)img * tokens + row) * 3 * D + m * D + h * HD) + c);
-    reinterpret_cast<uint4 *>(att_smem + (m * MAX_TOKENS + row) * ROW)[c] = val;
+    uint4 *dst = reinterpret_cast<uint4 *>(att_smem + (m * MAX_TOKENS + row) * ROW) + c;
+    if (row < tokens) {
+      const uint4 *src =
+          reinterpret_cast<const uint4 *>(qkv + ((int64_t)img * tokens + row) * 3 * D + m * D + h * HD) + c;
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" :: "r"(smem_addr(dst)), "l"(src) : "memory");
+    } else {
+      *dst = make_uint4(0, 0, 0, 0);
+    }
   }
+  asm volatile("cp.async.wait_all;" ::: "memory");
   __syncthreads();
   const int ntiles = tp / 8, kq = lane & 3, rq = lane >> 2;
   for (int mt = warp; mt < tp / 16; mt += ATT_WARPS) {
