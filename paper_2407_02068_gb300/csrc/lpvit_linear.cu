@@ -248,12 +248,15 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
 
   if (warp == 0) {
     // ============================================================== producer
+    // The next unit is taken from the queue one unit ahead, and the next 32 entry records are
+    // loaded while the current ones are issued, so neither global round trip sits on the path.
     uint32_t it = 0, ui = 0;
     bool ok = true;
+    uint32_t u_next = 0;
+    if (lane == 0) u_next = atomicAdd(&P.ctl->next_unit, 1u);
     while (true) {
-      uint32_t u = 0;
-      if (lane == 0) u = atomicAdd(&P.ctl->next_unit, 1u);
-      u = __shfl_sync(0xffffffffu, u, 0);
+      const uint32_t u = __shfl_sync(0xffffffffu, u_next, 0);
+      if (lane == 0 && u < total_units) u_next = atomicAdd(&P.ctl->next_unit, 1u);
       const uint32_t slot = ui % L::UR, uph = (ui / L::UR) & 1u;
       if (!mbar_wait(unite_bar(slot), uph ^ 1u, abort_flag, tmo)) {
         ok = false;
@@ -278,11 +281,8 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
       const int g = lo, s = rr - slice_ptr[g], nsl = slice_ptr[g + 1] - slice_ptr[g];
       const int ge0 = gent[g], ge1 = gent[g + 1];
       const int e0 = min(ge0 + s * P.S, ge1), e1 = min(e0 + P.S, ge1);
-      // whether any entry of this unit keeps a block (else the accumulator is never written)
-      unsigned touched = 0;
-      for (int e = e0 + lane; e < e1; e += 32) touched |= (unsigned)entries[(int64_t)e * ENTRY_INTS] >> 16;
-      touched = __reduce_or_sync(0xffffffffu, touched);
-      const unsigned tmask = touched ? 1u : 0u;
+      // every entry keeps a block of the group, so the accumulator is written iff there is one
+      const unsigned tmask = e1 > e0 ? 1u : 0u;
       if (lane == 0) {
         UnitInfo inf;
         inf.tt = tt; inf.g = g; inf.s = s; inf.nsl = nsl; inf.e0 = e0; inf.e1 = e1; inf.touched = (int)tmask;
@@ -290,13 +290,20 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
         ring[slot] = inf;
         mbar_arrive(unitf_bar(slot));
       }
+      int w0n = 0, toffn = -1;  // records of entries base + lane, loaded one chunk ahead
+      if (e0 + lane < e1) {
+        const int32_t *ep = entries + (int64_t)(e0 + lane) * ENTRY_INTS;
+        w0n = ep[0];
+        toffn = ep[ENTRY_TILE_WORD];
+      }
       for (int base = e0; base < e1 && ok; base += 32) {
-        const int e = base + lane;
-        int w0 = 0, toff = -1;
-        if (e < e1) {
-          const int32_t *ep = entries + (int64_t)e * ENTRY_INTS;
-          w0 = ep[0];
-          toff = ep[ENTRY_TILE_WORD];
+        const int w0 = w0n, toff = toffn;
+        w0n = 0;
+        toffn = -1;
+        if (base + 32 + lane < e1) {
+          const int32_t *ep = entries + (int64_t)(base + 32 + lane) * ENTRY_INTS;
+          w0n = ep[0];
+          toffn = ep[ENTRY_TILE_WORD];
         }
         const int cnt = min(32, e1 - base);
         for (int i = 0; i < cnt && ok;) {
