@@ -75,7 +75,8 @@ struct Smem {
   static constexpr int META_OFF = BAR_OFF + 8 * NBARS;
   static constexpr int RING_OFF = (META_OFF + 4 * NS + 31) / 32 * 32;
   static constexpr int SLICE_OFF = RING_OFF + (int)sizeof(UnitInfo) * UR;
-  static constexpr int MISC_OFF = SLICE_OFF + 4 * (MAX_GROUPS + 1);
+  static constexpr int GENT_OFF = SLICE_OFF + 4 * (MAX_GROUPS + 1);  // the group entry table, staged
+  static constexpr int MISC_OFF = GENT_OFF + 4 * (MAX_GROUPS + 1);
   static constexpr int EPI_OFF = (MISC_OFF + 64 + 127) / 128 * 128;
   static constexpr int EPI_TILE = 16 * 80;  // per epilogue warp: 16 token rows x 32 bf16, rows padded to 80 B
   static constexpr int END = EPI_OFF + EPI_WARPS * EPI_TILE;
@@ -179,6 +180,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
   volatile int *meta = reinterpret_cast<volatile int *>(smem + L::META_OFF);
   UnitInfo *ring = reinterpret_cast<UnitInfo *>(smem + L::RING_OFF);
   int *slice_ptr = reinterpret_cast<int *>(smem + L::SLICE_OFF);
+  int *gent_s = reinterpret_cast<int *>(smem + L::GENT_OFF);
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + L::MISC_OFF);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 4);
   volatile int *last_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 8);
@@ -237,6 +239,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
       run += __shfl_sync(0xffffffffu, incl, 31);
     }
     if (lane == 0) slice_ptr[P.n_groups] = run;
+    for (int g = lane; g <= P.n_groups; g += 32) gent_s[g] = gent[g];
   }
   tc_fence_before();
   __syncthreads();
@@ -248,15 +251,53 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
 
   if (warp == 0) {
     // ============================================================== producer
-    // The next unit is taken from the queue one unit ahead, and the next 32 entry records are
-    // loaded while the current ones are issued, so neither global round trip sits on the path.
+    // Unit i is decoded (shared-memory tables) and its first 32 entry records are loaded while unit
+    // i - 1 is issued, and the queue index of unit i + 1 is fetched then; within a unit the next 32
+    // records are loaded while the current ones are issued. No global round trip sits on the path.
     uint32_t it = 0, ui = 0;
     bool ok = true;
-    uint32_t u_next = 0;
-    if (lane == 0) u_next = atomicAdd(&P.ctl->next_unit, 1u);
+    struct Unit {
+      int tt, g, s, nsl, e0, e1;
+    };
+    auto decode = [&](uint32_t u) {  // shared-memory tables only
+      Unit d;
+      d.tt = (int)(u / (uint32_t)total_slices);
+      const int rr = (int)(u % (uint32_t)total_slices);
+      int lo = 0, hi = P.n_groups - 1;  // group g with slice_ptr[g] <= rr < slice_ptr[g+1]
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (slice_ptr[mid] <= rr) lo = mid;
+        else hi = mid - 1;
+      }
+      d.g = lo;
+      d.s = rr - slice_ptr[lo];
+      d.nsl = slice_ptr[lo + 1] - slice_ptr[lo];
+      const int ge0 = gent_s[lo], ge1 = gent_s[lo + 1];
+      d.e0 = min(ge0 + d.s * P.S, ge1);
+      d.e1 = min(d.e0 + P.S, ge1);
+      return d;
+    };
+    auto first_records = [&](const Unit &d, int &w, int &t) {
+      w = 0;
+      t = -1;
+      if (d.e0 + lane < d.e1) {
+        const int32_t *ep = entries + (int64_t)(d.e0 + lane) * ENTRY_INTS;
+        w = ep[0];
+        t = ep[ENTRY_TILE_WORD];
+      }
+    };
+    uint32_t fetched = 0;
+    if (lane == 0) fetched = atomicAdd(&P.ctl->next_unit, 1u);
+    uint32_t u_cur = __shfl_sync(0xffffffffu, fetched, 0);
+    Unit cur = {0, 0, 0, 1, 0, 0};
+    int w0c = 0, toffc = -1;
+    if (u_cur < total_units) {
+      cur = decode(u_cur);
+      first_records(cur, w0c, toffc);
+      if (lane == 0) fetched = atomicAdd(&P.ctl->next_unit, 1u);
+    }
     while (true) {
-      const uint32_t u = __shfl_sync(0xffffffffu, u_next, 0);
-      if (lane == 0 && u < total_units) u_next = atomicAdd(&P.ctl->next_unit, 1u);
+      const uint32_t u = u_cur;
       const uint32_t slot = ui % L::UR, uph = (ui / L::UR) & 1u;
       if (!mbar_wait(unite_bar(slot), uph ^ 1u, abort_flag, tmo)) {
         ok = false;
@@ -270,32 +311,27 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
         }
         break;
       }
-      const int tt = (int)(u / (uint32_t)total_slices);
-      const int rr = (int)(u % (uint32_t)total_slices);
-      int lo = 0, hi = P.n_groups - 1;  // group g with slice_ptr[g] <= rr < slice_ptr[g+1]
-      while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (slice_ptr[mid] <= rr) lo = mid;
-        else hi = mid - 1;
-      }
-      const int g = lo, s = rr - slice_ptr[g], nsl = slice_ptr[g + 1] - slice_ptr[g];
-      const int ge0 = gent[g], ge1 = gent[g + 1];
-      const int e0 = min(ge0 + s * P.S, ge1), e1 = min(e0 + P.S, ge1);
+      const int tt = cur.tt, e0 = cur.e0, e1 = cur.e1;
       // every entry keeps a block of the group, so the accumulator is written iff there is one
       const unsigned tmask = e1 > e0 ? 1u : 0u;
       if (lane == 0) {
         UnitInfo inf;
-        inf.tt = tt; inf.g = g; inf.s = s; inf.nsl = nsl; inf.e0 = e0; inf.e1 = e1; inf.touched = (int)tmask;
+        inf.tt = tt; inf.g = cur.g; inf.s = cur.s; inf.nsl = cur.nsl; inf.e0 = e0; inf.e1 = e1;
+        inf.touched = (int)tmask;
         inf.pad = 0;
         ring[slot] = inf;
         mbar_arrive(unitf_bar(slot));
       }
-      int w0n = 0, toffn = -1;  // records of entries base + lane, loaded one chunk ahead
-      if (e0 + lane < e1) {
-        const int32_t *ep = entries + (int64_t)(e0 + lane) * ENTRY_INTS;
-        w0n = ep[0];
-        toffn = ep[ENTRY_TILE_WORD];
+      // the next unit: decode it, start loading its first records, fetch the one after
+      const uint32_t u_nx = __shfl_sync(0xffffffffu, fetched, 0);
+      Unit nxt = {0, 0, 0, 1, 0, 0};
+      int w0x = 0, toffx = -1;
+      if (u_nx < total_units) {
+        nxt = decode(u_nx);
+        first_records(nxt, w0x, toffx);
+        if (lane == 0) fetched = atomicAdd(&P.ctl->next_unit, 1u);
       }
+      int w0n = w0c, toffn = toffc;  // records of entries base + lane, loaded one chunk ahead
       for (int base = e0; base < e1 && ok; base += 32) {
         const int w0 = w0n, toff = toffn;
         w0n = 0;
@@ -351,6 +387,10 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
       }
       if (!ok) break;
       ++ui;
+      u_cur = u_nx;
+      cur = nxt;
+      w0c = w0x;
+      toffc = toffx;
     }
     if (!ok && lane == 0) *abort_flag = 1;
     // queue bookkeeping: the last CTA to leave resets the counters for the next launch
