@@ -23,7 +23,9 @@
  *    with W stored [out=n][in=k]. The sum runs over k in ascending order in double.
  *
  *  - GELU after fc1 (the DeiT MLP activation; the paper does not state its form, the exact
- *    erf form is used): gelu(y) = 0.5 * y * (1 + erf(y / sqrt(2))).
+ *    erf form is used): gelu(y) = y * Phi(y) = 0.5 * y * (1 + erf(y / sqrt(2))), evaluated as
+ *    0.5 * y * erfc(-y / sqrt(2)) (the same function; 1 + erf cancels where erf is near -1, erfc
+ *    keeps the relative accuracy there).
  *
  *  - Block-sparse packing of the surviving blocks (BSR), Sec. 1 and Sec. 3.3 (only the
  *    surviving blocks are stored and moved): for each row panel r (bn consecutive output
@@ -88,7 +90,7 @@ uint16_t lpvit_oracle_round_bf16(double y) {
   return (uint16_t)(sign | (uint16_t)((u >> 16) & 0x7FFF));
 }
 
-double lpvit_oracle_gelu(double y) { return 0.5 * y * (1.0 + erf(y / sqrt(2.0))); }
+double lpvit_oracle_gelu(double y) { return 0.5 * y * erfc(-y / sqrt(2.0)); }
 
 /* BSR pack by the definition above, bn x bk blocks. col_idx and blocks must hold
  * (n/bn)*(k/bk) entries. Returns nnzb, or -1 on bad arguments. */
