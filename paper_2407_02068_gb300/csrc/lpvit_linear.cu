@@ -85,24 +85,24 @@ struct Smem {
 };
 
 // Epilogue of one 32 x 32 block held by a warp: y[i] = accumulator of token tok_base + i for feature
-// f0 + lane (turned into the output in place). Adds the bias, applies GELU, rounds, and stores rows [tok_base, min(tok_base + 32, m)).
+// f0 + lane (turned into the output in place), bb = that feature's bias (0 without one). Adds the
+// bias, applies GELU, rounds, and stores rows [tok_base, min(tok_base + 32, m)).
 // bf16 output is staged through this warp's shared tile (rows padded to 80 bytes, conflict-free) so
 // that every token row leaves as 16-byte vector stores; fp32 output is stored directly (a warp
 // writes 128 contiguous bytes per token).
-__device__ __forceinline__ void emit32(float (&y)[32], int f0, int64_t tok_base, const LinearParams &P,
-                                       uint8_t *tile) {
+__device__ __forceinline__ void emit32(float (&y)[32], float bb, int f0, int64_t tok_base,
+                                       const LinearParams &P, uint8_t *tile) {
   const int lane = threadIdx.x & 31;
   const int f = f0 + lane;
   const bool fvalid = f < P.n;
-  const float bb = (P.bias != nullptr && fvalid) ? __ldg(P.bias + f) : 0.f;
   const int64_t left = P.m - tok_base;
   const int rows = left >= 32 ? 32 : (left > 0 ? (int)left : 0);
   if (P.gelu) {
-    const float kInvSqrt2 = 0.70710678118654752440f;
 #pragma unroll
     for (int i = 0; i < 32; ++i) {
+      // exact GELU, t * Phi(t); where 1 + erf cancels (t < -3) the error is a few ulps of 1 times t / 2
       const float t = y[i] + bb;
-      y[i] = 0.5f * t * (1.f + erff(t * kInvSqrt2));
+      y[i] = 0.5f * t * (1.f + erff(t * 0.70710678118654752440f));
     }
   } else {
 #pragma unroll
@@ -483,6 +483,9 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
       }
       const UnitInfo inf = ring[slot];
       if (inf.tt < 0) break;
+      const int f0 = inf.g * GROUP_FEATURES + 32 * q;  // first feature of this warp's blocks
+      // the bias of this lane's feature, loaded while the accumulator is still being computed
+      const float bb = (P.bias != nullptr && f0 + lane < P.n) ? __ldg(P.bias + f0 + lane) : 0.f;
       const uint32_t buf = ui & 1u, aph = (ui >> 1) & 1u;
       if (!mbar_wait(accf_bar(buf), aph, abort_flag, tmo)) {
         if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_ACC); *abort_flag = 1; }
@@ -493,7 +496,6 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
       float *part = nullptr;
       if (split)
         part = P.partials + ((int64_t)inf.tt * total_slices + slice_ptr[inf.g] + inf.s) * (int64_t)(C::TT * 128);
-      const int f0 = inf.g * GROUP_FEATURES + 32 * q;  // first feature of this warp's blocks
 #pragma unroll 1
       for (int j = wq; j < QBLK; j += EPI_WARPS / 4) {
         const int tok0 = 32 * j;  // first token of the block (its accumulator column)
@@ -510,7 +512,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
 #pragma unroll
           for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
         } else {
-          emit32(v, f0, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
+          emit32(v, bb, f0, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
         }
       }
       // accumulator buffer and unit slot are free again
@@ -564,7 +566,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
                 v[4 * i] += t.x; v[4 * i + 1] += t.y; v[4 * i + 2] += t.z; v[4 * i + 3] += t.w;
               }
             }
-            emit32(v, f0, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
+            emit32(v, bb, f0, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
           }
         }
       }

@@ -275,6 +275,34 @@ def test_linear_gelu(lp, b):
     assert np.all(np.abs(Yb.float().cpu().double().numpy() - ref) <= _bf16_tol(ref, X, W, mask, b, bias, gelu=True))
 
 
+def test_gelu_epilogue_over_the_float32_range(lp):
+    """All-zero mask: the output is GELU(bias). Biases sweep [-14, 14], tiny, huge and signed-zero
+    values, against the oracle's exact GELU: float32 output within 5e-4 relative plus 2^-21 |t|
+    (the epilogue forms 1 + erf(t / sqrt 2) in float32, which cancels for t < -3), bf16 output
+    within one bf16 ulp plus that."""
+    f32 = np.float32
+    special = [0.0, -0.0, 1e-30, -1e-30, 1e-6, -1e-6, 20.0, -20.0, 1e4, -1e4, 3.0, -3.0]
+    sweep = np.linspace(-14.0, 14.0, 4096 - len(special))
+    t = np.concatenate([np.array(special, np.float64), sweep]).astype(np.float32)
+    n, k, m = t.size, 32, 40
+    bias = torch.from_numpy(t).cuda()
+    W = torch.zeros(n, k, dtype=torch.bfloat16, device="cuda")
+    X = torch.zeros(m, k, dtype=torch.bfloat16, device="cuda")
+    mask = torch.zeros(n // 32, k // 32, dtype=torch.uint8, device="cuda")
+    w = lp.pack_bsr(W, mask, 32)
+    ref = oracle.gelu(t.astype(np.float64))
+    Y = lp.bsr_linear(w, X, bias, gelu=True, out_dtype=torch.float32).cpu().double().numpy()
+    assert np.all(Y == Y[0])
+    y = Y[0]
+    tol = 5e-4 * np.abs(ref) + 2.0 ** -21 * np.abs(t)
+    assert np.all(np.abs(y - ref) <= tol)
+    core = (t > -3) & (np.abs(ref) > 1e-36)
+    assert np.all(np.abs(y[core] - ref[core]) <= 5e-4 * np.abs(ref[core]))   # relative where no cancellation
+    assert y[0] == 0.0 and y[special.index(20.0)] == 20.0 and y[special.index(1e4)] == f32(1e4)
+    Yb = lp.bsr_linear(w, X, bias, gelu=True).float().cpu().double().numpy()[0]
+    assert np.all(np.abs(Yb - ref) <= _ulp_bf16(ref) + tol)
+
+
 @pytest.mark.parametrize("b", BLOCKS)
 def test_all_zero_mask_is_bias(lp, b):
     m, n, k = 260, 256, 128
