@@ -360,6 +360,26 @@ def test_strided_input_output_and_guard_band(lp):
     assert torch.all(Yw[m:] == canary) and torch.all(Yw[:, :16] == canary) and torch.all(Yw[:, 16 + n:] == canary)
 
 
+@pytest.mark.parametrize("col0,extra", [(1, 33), (2, 34)])
+def test_bf16_output_offsets_and_row_strides(lp, col0, extra):
+    """bf16 output inside a larger buffer, with bases and row strides that rule out 16-byte stores
+    (element stores instead); the canary around the output region survives and the values are
+    those of a contiguous output."""
+    m, n, k, b = 301, 256, 128, 32
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 850 + col0)
+    canary = torch.tensor(-777.0, dtype=torch.bfloat16)
+    Yw = torch.full((m + 3, n + extra), canary.item(), dtype=torch.bfloat16, device="cuda")
+    w = lp.pack_bsr(W, mask, b)
+    for gelu in (False, True):
+        lp.bsr_linear(w, X, bias, gelu=gelu, out=Yw[:m, col0:col0 + n])
+        Yc = lp.bsr_linear(w, X, bias, gelu=gelu)
+        assert torch.equal(Yw[:m, col0:col0 + n], Yc)
+        assert torch.all(Yw[m:] == canary) and torch.all(Yw[:, :col0] == canary)
+        assert torch.all(Yw[:, col0 + n:] == canary)
+    ref = _oracle(X, W, mask, b, bias, gelu=True)
+    assert np.all(np.abs(Yc.float().cpu().double().numpy() - ref) <= _bf16_tol(ref, X, W, mask, b, bias, gelu=True))
+
+
 @pytest.mark.parametrize("b", [32, (64, 32), (16, 32)])
 def test_deterministic_repeats(lp, b):
     m, n, k = 197, 768, 3072   # small m: split slices + fix-up path
