@@ -168,6 +168,7 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.m = m;
   P.n = n;
   P.k = k;
+  P.bn = bn;
   P.n_tt = (int)ceil_div(m, TOKENS_PER_TILE);
   P.n_groups = ng;
   P.S = choose_slice(P.n_tt, P.n_groups, k / bk, sms);

@@ -13,12 +13,16 @@ namespace lpvit {
 // header (16 int32): [0] nnzb, [1] n_groups, [2] total entries, [3] overflow flag, [4] n, [5] k,
 // [6] bn, [7] bk
 // then gent_ptr[n_groups + 1] (int32, entries of group g are [gent_ptr[g], gent_ptr[g+1]))
-// then entries, ENTRY_INTS int32 each: [0] = j | (row-panel mask << 16), [1 + p] = block index of
-// the group's p-th row panel at block column j, or -1 (p < GROUP_FEATURES / bn <= 8),
+// then gpan[n_groups][MAX_GROUP_PANELS] (int32): the row panel in slot p of group g, or -1. A group
+// is GROUP_FEATURES / bn row panels, not necessarily consecutive: the plan picks panels whose kept
+// block columns overlap, so that a group has fewer entries; group row r is panel gpan[g][r / bn],
+// row r % bn, i.e. output feature gpan[g][r / bn] * bn + r % bn.
+// then entries, ENTRY_INTS int32 each: [0] = j | (slot mask << 16), [1 + p] = block index of
+// the panel in slot p at block column j, or -1 (p < GROUP_FEATURES / bn <= 8),
 // [ENTRY_TILE_WORD] = index of the entry's tile in the weight stream (the entry's own index);
 // then, at sched_stream_offset_bytes (1024-byte aligned), the weight stream: for every entry in
-// order, the group's tile at column j: W[g*128 + r][j*bk + c] for r < 128, c < bk, with the rows of
-// the row panels that keep no block there zero, stored as 128 rows of 2*bk bytes whose 16-byte
+// order, the group's tile at column j: row r < 128 holds W[feature of group row r][j*bk + c] for
+// c < bk, zero for the slots that keep no block there, stored as 128 rows of 2*bk bytes whose 16-byte
 // chunks are permuted by stream_chunk_swizzle: the arrangement the MMA's shared-memory descriptor
 // reads, so that one bulk copy moves an entry's weights.
 constexpr int SCHED_HDR_INTS = 16;
@@ -29,8 +33,9 @@ constexpr int MAX_GROUP_PANELS = GROUP_FEATURES / 16;
 constexpr int TOKENS_PER_TILE = 256;  // tokens covered by one work unit (the .ws MMA N)
 
 __host__ __device__ inline int sched_gent_offset_ints() { return SCHED_HDR_INTS; }
+__host__ __device__ inline int64_t sched_gpan_offset_ints(int n_groups) { return (int64_t)SCHED_HDR_INTS + n_groups + 1; }
 __host__ __device__ inline int64_t sched_entries_offset_ints(int n_groups) {
-  return ((int64_t)SCHED_HDR_INTS + n_groups + 1 + 3) / 4 * 4;  // 16-byte aligned entries
+  return (sched_gpan_offset_ints(n_groups) + (int64_t)n_groups * MAX_GROUP_PANELS + 3) / 4 * 4;  // 16-byte aligned
 }
 __host__ __device__ inline int64_t sched_stream_offset_bytes(int n_groups, int kb) {
   const int64_t end = 4 * (sched_entries_offset_ints(n_groups) + (int64_t)n_groups * kb * ENTRY_INTS);
@@ -71,6 +76,7 @@ struct LinearParams {
   int64_t ldy;
   int64_t m;
   int n, k;
+  int bn;                  // block height: a group holds GROUP_FEATURES / bn row panels
   int n_tt, n_groups, S;   // token tiles, 128-feature groups, max entries per slice
   int y_f32, gelu;
   int y_vec16;             // bf16 output rows may take 16-byte stores (Y 16-byte aligned, ldy % 8 == 0)

@@ -3,7 +3,8 @@
 // blocks). The kernel is compiled per block width BK (input columns of a block: 16, 32 or 64);
 // the block height only decides which rows of a group tile the pack left zero.
 //
-// Work unit = 256 tokens x one 128-feature group of row panels (x one slice of the group's block
+// Work unit = 256 tokens x one 128-feature group of row panels (the work list's group table names
+// the panels of each group; the epilogue maps a group row to its output feature through it) (x one slice of the group's block
 // columns when the problem is too small to fill the GPU). Per CTA (one per SM, persistent):
 //   warp 0      producer: takes units from a global atomic queue, walks the unit's work-list
 //               entries and, per entry (one block column j), loads the X tile [256 tokens x bk]
@@ -84,17 +85,18 @@ struct Smem {
   static_assert(BYTES <= 227 * 1024, "shared memory per CTA");
 };
 
-// Epilogue of one 32 x 32 block held by a warp: y[i] = accumulator of token tok_base + i for feature
-// f0 + lane (turned into the output in place), bb = that feature's bias (0 without one). Adds the
-// bias, applies GELU, rounds, and stores rows [tok_base, min(tok_base + 32, m)).
+// Epilogue of one 32 x 32 block held by a warp: y[i] = accumulator of token tok_base + i for the
+// lane's output feature fl (-1: a group row without a panel; turned into the output in place), bb =
+// that feature's bias (0 without one). Lanes 8c .. 8c + 7 hold consecutive features of one row panel.
+// Adds the bias, applies GELU, rounds, and stores rows [tok_base, min(tok_base + 32, m)).
 // bf16 output is staged through this warp's shared tile (rows padded to 80 bytes, conflict-free) so
 // that every token row leaves as 16-byte vector stores; fp32 output is stored directly (a warp
 // writes 128 contiguous bytes per token).
-__device__ __forceinline__ void emit32(float (&y)[32], float bb, int f0, int64_t tok_base,
+__device__ __forceinline__ void emit32(float (&y)[32], float bb, int fl, int64_t tok_base,
                                        const LinearParams &P, uint8_t *tile) {
   const int lane = threadIdx.x & 31;
-  const int f = f0 + lane;
-  const bool fvalid = f < P.n;
+  const int f = fl;
+  const bool fvalid = fl >= 0;
   const int64_t left = P.m - tok_base;
   const int rows = left >= 32 ? 32 : (left > 0 ? (int)left : 0);
   if (P.gelu) {
@@ -119,7 +121,8 @@ __device__ __forceinline__ void emit32(float (&y)[32], float bb, int f0, int64_t
   }
   __nv_bfloat16 *t = reinterpret_cast<__nv_bfloat16 *>(tile);
   const int ch = lane & 3;
-  const bool cvalid = f0 + ch * 8 < P.n;
+  const int fch = __shfl_sync(0xffffffffu, fl, 8 * ch);  // first feature of the lane's 8-feature chunk
+  const bool cvalid = fch >= 0;
 #pragma unroll
   for (int half = 0; half < 2; ++half) {  // 16 token rows at a time through the warp's tile
 #pragma unroll
@@ -130,7 +133,7 @@ __device__ __forceinline__ void emit32(float (&y)[32], float bb, int f0, int64_t
       const int rt = 8 * it + (lane >> 2), row = 16 * half + rt;
       const int4 val = *reinterpret_cast<const int4 *>(tile + rt * 80 + ch * 16);
       if (row < rows && cvalid) {
-        __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(P.Y) + (tok_base + row) * P.ldy + f0 + ch * 8;
+        __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(P.Y) + (tok_base + row) * P.ldy + fch;
         if (P.y_vec16) {
           *reinterpret_cast<int4 *>(dst) = val;
         } else {
@@ -188,6 +191,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
 
   const int32_t *gent = P.sched + SCHED_HDR_INTS;
   const int32_t *entries = P.sched + sched_entries_offset_ints(P.n_groups);
+  const int32_t *gpan = P.sched + sched_gpan_offset_ints(P.n_groups);
   const uint64_t tmo = P.timeout_ns;
 
   // ---------------------------------------------------------------- prologue
@@ -218,7 +222,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
   if (warp == 0 && lane == 0) prefetch_tensormap(&tmX);
   // the work list must be this weight's plan: group count, shape and block width
   const bool sched_ok = P.sched[3] == 0 && P.sched[1] == P.n_groups && P.sched[4] == P.n && P.sched[5] == P.k &&
-                        P.sched[7] == BK;
+                        P.sched[6] == P.bn && P.sched[7] == BK;
   if (warp == 2) {
     // slices per group = max(1, ceil(entries / S)); exclusive prefix into slice_ptr
     int run = 0;
@@ -483,9 +487,12 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
       }
       const UnitInfo inf = ring[slot];
       if (inf.tt < 0) break;
-      const int f0 = inf.g * GROUP_FEATURES + 32 * q;  // first feature of this warp's blocks
-      // the bias of this lane's feature, loaded while the accumulator is still being computed
-      const float bb = (P.bias != nullptr && f0 + lane < P.n) ? __ldg(P.bias + f0 + lane) : 0.f;
+      // this lane's group row 32 q + lane is row (32 q + lane) % bn of the panel in slot (32 q + lane) / bn;
+      // its feature and bias are loaded while the accumulator is still being computed
+      const int grow = 32 * q + lane;
+      const int panel = __ldg(gpan + (int64_t)inf.g * MAX_GROUP_PANELS + grow / P.bn);
+      const int fl = panel >= 0 ? panel * P.bn + grow % P.bn : -1;
+      const float bb = (P.bias != nullptr && fl >= 0) ? __ldg(P.bias + fl) : 0.f;
       const uint32_t buf = ui & 1u, aph = (ui >> 1) & 1u;
       if (!mbar_wait(accf_bar(buf), aph, abort_flag, tmo)) {
         if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_ACC); *abort_flag = 1; }
@@ -512,7 +519,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
 #pragma unroll
           for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
         } else {
-          emit32(v, bb, f0, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
+          emit32(v, bb, fl, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
         }
       }
       // accumulator buffer and unit slot are free again
@@ -566,7 +573,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
                 v[4 * i] += t.x; v[4 * i + 1] += t.y; v[4 * i + 2] += t.z; v[4 * i + 3] += t.w;
               }
             }
-            emit32(v, bb, f0, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
+            emit32(v, bb, fl, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
           }
         }
       }

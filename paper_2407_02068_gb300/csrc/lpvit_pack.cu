@@ -6,9 +6,10 @@
 // plan kernel (one CTA): per row panel r (bn rows), cnt[r] = number of kept blocks (warp
 //   reductions); row_ptr = exclusive prefix sum of cnt (warp-shuffle scan + a scan of warp
 //   totals); col_idx = kept block columns of each panel in ascending order (ballot compaction);
-//   work list: panels are grouped 128 output features at a time; for every group, one entry per
-//   block column where any panel of the group keeps a block, with that column's block index in
-//   each panel (or -1). The GEMM walks these entries.
+//   work list: panels are grouped 128 output features (128 / bn panels) at a time, greedily by
+//   overlap of their kept block columns (one warp; consecutive panels when that is not better);
+//   for every group, one entry per block column where any panel of the group keeps a block, with
+//   that column's block index in each panel (or -1). The GEMM walks these entries.
 // copy kernel (grid-stride): blocks[t] = W[r*bn:(r+1)*bn, j*bk:(j+1)*bk], 16-byte vector copies,
 //   bits unchanged; then the weight stream, the same bits once more, entry by entry as the 128-row
 //   group tiles the GEMM's MMAs read (rows of removed row panels zero, 16-byte chunks swizzled).
@@ -61,6 +62,90 @@ __device__ int block_exclusive_scan(int *v, int count, int *warp_tot) {
   return total;
 }
 
+// Panel grouping runs when its bitmaps fit the plan's shared memory: at most GROUPING_MAX_PANELS
+// row panels and GROUPING_MAX_WORDS words of per-panel column bitmaps.
+constexpr int GROUPING_MAX_PANELS = 1024;
+constexpr int GROUPING_MAX_WORDS = 8192;
+__host__ __device__ inline bool grouping_on(int np, int kb, int gb) {
+  const int W = (kb + 31) / 32;
+  return gb >= 2 && np <= GROUPING_MAX_PANELS && (int64_t)np * W <= GROUPING_MAX_WORDS;
+}
+
+__device__ __forceinline__ int warp_sum(int v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Group the row panels, one warp. A group starts with the unassigned panel keeping the most blocks
+// and then takes, gb - 1 times, the unassigned panel that adds the fewest block columns to the
+// group's union (ties to the lower panel index). The work list has one entry per block column of
+// the union, so overlapping panels make fewer entries. The grouping is kept only if it gives fewer
+// entries than consecutive panels; gpan is written either way.
+__device__ void group_panels(const unsigned *__restrict__ bits, int W, const int *__restrict__ kcnt, int np,
+                             int gb, int ng, unsigned *U, int *asg, int32_t *__restrict__ gpan) {
+  const int lane = threadIdx.x & 31;
+  for (int p = lane; p < np; p += 32) asg[p] = 0;
+  int id_e = 0;  // entries of consecutive groups
+  for (int g = lane; g < ng; g += 32)
+    for (int w = 0; w < W; ++w) {
+      unsigned u = 0;
+      for (int p = 0; p < gb; ++p)
+        if (g * gb + p < np) u |= bits[(g * gb + p) * W + w];
+      id_e += __popc(u);
+    }
+  id_e = warp_sum(id_e);
+  __syncwarp();
+  int gr_e = 0;
+  for (int g = 0; g < ng; ++g) {
+    for (int sl = 0; sl < gb; ++sl) {
+      int best = 0x7fffffff, bi = 0x7fffffff;
+      for (int p = lane; p < np; p += 32) {
+        if (asg[p]) continue;
+        int sc = 0;
+        if (sl == 0) {
+          sc = -kcnt[p];
+        } else {
+          for (int w = 0; w < W; ++w) sc += __popc(bits[p * W + w] & ~U[w]);
+        }
+        if (sc < best || (sc == best && p < bi)) {
+          best = sc;
+          bi = p;
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const int ob = __shfl_xor_sync(0xffffffffu, best, o), oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        if (ob < best || (ob == best && oi < bi)) {
+          best = ob;
+          bi = oi;
+        }
+      }
+      const int pick = bi == 0x7fffffff ? -1 : bi;
+      if (lane == 0) {
+        gpan[g * MAX_GROUP_PANELS + sl] = pick;
+        if (pick >= 0) asg[pick] = 1;
+      }
+      for (int w = lane; w < W; w += 32) {
+        const unsigned add = pick >= 0 ? bits[pick * W + w] : 0u;
+        U[w] = (sl == 0 ? 0u : U[w]) | add;
+      }
+      __syncwarp();
+    }
+    if (lane >= gb && lane < MAX_GROUP_PANELS) gpan[g * MAX_GROUP_PANELS + lane] = -1;
+    int c = 0;
+    for (int w = lane; w < W; w += 32) c += __popc(U[w]);
+    gr_e += warp_sum(c);
+    __syncwarp();
+  }
+  if (gr_e >= id_e) {
+    for (int i = lane; i < ng * MAX_GROUP_PANELS; i += 32) {
+      const int g = i / MAX_GROUP_PANELS, sl = i - g * MAX_GROUP_PANELS, r = g * gb + sl;
+      gpan[i] = (sl < gb && r < np) ? r : -1;
+    }
+  }
+}
+
 // The plan of one weight, computed by one CTA of PLAN_THREADS threads (plan_smem: plan_smem_bytes).
 __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int n, int k, int bn, int bk,
                                           int32_t *__restrict__ row_ptr, int32_t *__restrict__ col_idx, int cap,
@@ -68,9 +153,16 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
   const int np = n / bn, kb = k / bk;
   const int gb = GROUP_FEATURES / bn;  // row panels per group
   const int ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
+  const int W = (kb + 31) / 32;    // words of a panel's column bitmap
+  const bool grouping = grouping_on(np, kb, gb);
   int *cnt = plan_smem;            // [np + 1]
   int *gcnt = cnt + np + 1;        // [ng + 1]
   int *warp_tot = gcnt + ng + 1;   // [33]
+  int *kcnt = warp_tot + 33;       // [np] kept blocks per panel
+  unsigned *bits = reinterpret_cast<unsigned *>(kcnt + np);  // grouping: [np][W] column bitmaps
+  unsigned *U = bits + (grouping ? np * W : 0);              // grouping: [W] union of a group
+  int *asg = reinterpret_cast<int *>(U + (grouping ? W : 0));  // grouping: [np] assigned flags
+  int32_t *gpan = sched + sched_gpan_offset_ints(ng);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const unsigned lt = (1u << lane) - 1u;
 
@@ -80,7 +172,16 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
     for (int j = lane; j < kb; j += 32) c += mask[(int64_t)r * kb + j] != 0;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
-    if (lane == 0) cnt[r] = c;
+    if (lane == 0) {
+      cnt[r] = c;
+      kcnt[r] = c;
+    }
+    if (grouping)
+      for (int base = 0; base < kb; base += 32) {
+        const int j = base + lane;
+        const unsigned bal = __ballot_sync(0xffffffffu, j < kb && mask[(int64_t)r * kb + j] != 0);
+        if (lane == 0) bits[r * W + base / 32] = bal;
+      }
   }
   __syncthreads();
   // 2. row_ptr = exclusive scan
@@ -105,6 +206,16 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
       run += __popc(bal);
     }
   }
+  // 3b. group table: overlapping panels (one warp), or consecutive panels
+  if (grouping) {
+    if (warp == 0) group_panels(bits, W, kcnt, np, gb, ng, U, asg, gpan);
+  } else {
+    for (int i = tid; i < ng * MAX_GROUP_PANELS; i += PLAN_THREADS) {
+      const int g = i / MAX_GROUP_PANELS, sl = i - g * MAX_GROUP_PANELS, r = g * gb + sl;
+      gpan[i] = (sl < gb && r < np) ? r : -1;
+    }
+  }
+  __syncthreads();
   // 4a. entries per group: block columns where any panel of the group keeps a block
   for (int g = warp; g < ng; g += PLAN_WARPS) {
     int c = 0;
@@ -112,8 +223,8 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
       const int j = base + lane;
       unsigned any = 0;
       for (int p = 0; p < gb; ++p) {
-        const int r = g * gb + p;
-        const bool keep = r < np && j < kb && mask[(int64_t)r * kb + j] != 0;
+        const int r = gpan[g * MAX_GROUP_PANELS + p];
+        const bool keep = r >= 0 && j < kb && mask[(int64_t)r * kb + j] != 0;
         any |= __ballot_sync(0xffffffffu, keep);
       }
       c += __popc(any);
@@ -142,16 +253,20 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
   for (int g = warp; g < ng; g += PLAN_WARPS) {
     int e_run = gcnt[g];
     int p_run[MAX_GROUP_PANELS];
+    int rr[MAX_GROUP_PANELS];  // the panel of each slot, or -1
 #pragma unroll
-    for (int p = 0; p < MAX_GROUP_PANELS; ++p) p_run[p] = (p < gb && g * gb + p < np) ? cnt[g * gb + p] : 0;
+    for (int p = 0; p < MAX_GROUP_PANELS; ++p) {
+      rr[p] = p < gb ? gpan[g * MAX_GROUP_PANELS + p] : -1;
+      p_run[p] = rr[p] >= 0 ? cnt[rr[p]] : 0;
+    }
     for (int base = 0; base < kb; base += 32) {
       const int j = base + lane;
       unsigned bal[MAX_GROUP_PANELS];
       unsigned any = 0;
 #pragma unroll
       for (int p = 0; p < MAX_GROUP_PANELS; ++p) {
-        const int r = g * gb + p;
-        const bool keep = p < gb && r < np && j < kb && mask[(int64_t)r * kb + j] != 0;
+        const int r = rr[p];
+        const bool keep = r >= 0 && j < kb && mask[(int64_t)r * kb + j] != 0;
         bal[p] = __ballot_sync(0xffffffffu, keep);
         any |= bal[p];
       }
@@ -227,6 +342,7 @@ __device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int 
   const int tile_bytes = stream_tile_bytes(bk);
   const int64_t max_tiles = sched_stream_tiles(ng, kb);
   const int32_t *gent = sched + SCHED_HDR_INTS;
+  const int32_t *gpan = sched + sched_gpan_offset_ints(ng);
   const int32_t *ent = sched + sched_entries_offset_ints(ng);
   uint8_t *stream = reinterpret_cast<uint8_t *>(const_cast<int32_t *>(sched)) + sched_stream_offset_bytes(ng, kb);
   for (int e = cta; e < total; e += ncta) {
@@ -245,9 +361,10 @@ __device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int 
     uint8_t *tile = stream + (int64_t)t * tile_bytes;
     for (int v = threadIdx.x; v < chunks; v += blockDim.x) {
       const int r = v / cpr, c = v - r * cpr;
-      const int row = g * GROUP_FEATURES + r;
+      const int panel = gpan[g * MAX_GROUP_PANELS + r / bn];
+      const int row = panel * bn + r % bn;  // the output feature of group row r
       int4 val = make_int4(0, 0, 0, 0);
-      if (((pm >> (r / bn)) & 1u) && row < n)
+      if (((pm >> (r / bn)) & 1u) && panel >= 0 && row < n)
         val = __ldg(reinterpret_cast<const int4 *>(W + (int64_t)row * k + (int64_t)j * bk + c * 8));
       reinterpret_cast<int4 *>(tile + r * row_bytes)[c ^ stream_chunk_swizzle(r, row_bytes)] = val;
     }
@@ -272,14 +389,17 @@ __global__ void __launch_bounds__(128) copy_many_kernel(const __grid_constant__ 
   }
 }
 
-size_t plan_smem_bytes(int n, int bn) {
-  const int np = n / bn, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
-  return sizeof(int) * (size_t)(np + 1 + ng + 1 + 33);
+size_t plan_smem_bytes(int n, int k, int bn, int bk) {
+  const int np = n / bn, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES, kb = k / bk;
+  const int W = (kb + 31) / 32;
+  size_t words = (size_t)np + 1 + ng + 1 + 33 + np;
+  if (grouping_on(np, kb, GROUP_FEATURES / bn)) words += (size_t)np * W + W + np;
+  return sizeof(int) * words;
 }
 
 cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int bn, int bk, int32_t *row_ptr,
                         int32_t *col_idx, int cap, void *blocks, int32_t *sched, int num_sms, cudaStream_t s) {
-  const size_t smem = plan_smem_bytes(n, bn);
+  const size_t smem = plan_smem_bytes(n, k, bn, bk);
   plan_kernel<<<1, PLAN_THREADS, smem, s>>>(mask, n, k, bn, bk, row_ptr, col_idx, cap, sched);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
@@ -300,7 +420,7 @@ cudaError_t launch_pack_many(const PackJob *jobs, int count, int num_sms, cudaSt
     int64_t blocks_max = 0;
     for (int j = 0; j < J.count; ++j) {
       J.job[j] = jobs[first + j];
-      const size_t sj = plan_smem_bytes(J.job[j].n, J.job[j].bn);
+      const size_t sj = plan_smem_bytes(J.job[j].n, J.job[j].k, J.job[j].bn, J.job[j].bk);
       smem = sj > smem ? sj : smem;
       blocks_max += (int64_t)(J.job[j].n / J.job[j].bn) * (J.job[j].k / J.job[j].bk);
     }

@@ -113,12 +113,49 @@ def test_pack_bit_exact(lp, n, k, b, sp):
 
 
 def _decode_sched(w):
+    """Header, group entry pointers, entries and the group table (row panel of every slot, or -1)."""
     raw = w.sched.cpu().numpy().view(np.int32)
     ng = int(raw[1])
     gent = raw[16:16 + ng + 1]
-    off = (16 + ng + 1 + 3) // 4 * 4
+    gpan = raw[16 + ng + 1:16 + ng + 1 + 8 * ng].reshape(ng, 8)
+    off = _entries_offset(ng)
     ent = raw[off:off + int(gent[-1]) * 12].reshape(-1, 12)
-    return raw[:16], gent, ent
+    return raw[:16], gent, ent, gpan
+
+
+def _entries_offset(ng):
+    return (16 + ng + 1 + 8 * ng + 3) // 4 * 4
+
+
+def _grouping(M, bn):
+    """The plan's grouping rule restated: a group starts with the unassigned panel keeping the most
+    blocks, then takes the unassigned panel adding the fewest block columns to the group's union
+    (ties to the lower index); kept only if it has fewer entries than consecutive panels, and only
+    for up to 1024 panels and 8192 bitmap words."""
+    npan, kb = M.shape
+    gb = 128 // bn
+    ng = -(-npan // gb)
+    ident = [[g * gb + p if p < gb and g * gb + p < npan else -1 for p in range(8)] for g in range(ng)]
+    if not (gb >= 2 and npan <= 1024 and npan * ((kb + 31) // 32) <= 8192):
+        return ident
+    rows = [set(np.nonzero(M[r])[0].tolist()) for r in range(npan)]
+    asg, table = [False] * npan, []
+    for g in range(ng):
+        t, U = [], set()
+        for sl in range(gb):
+            cand = [p for p in range(npan) if not asg[p]]
+            if not cand:
+                t.append(-1)
+                continue
+            pick = min(cand, key=(lambda p: (-len(rows[p]), p)) if sl == 0 else (lambda p: (len(rows[p] - U), p)))
+            asg[pick] = True
+            t.append(pick)
+            U |= rows[pick]
+        table.append(t + [-1] * (8 - gb))
+
+    def entries(tab):
+        return sum(len(set().union(*[rows[r] for r in t if r >= 0])) for t in tab)
+    return table if entries(table) < entries(ident) else ident
 
 
 @pytest.mark.parametrize("n,k,b", [(1152, 384, 32), (384, 1536, 16), (768, 3072, 64), (200 * 16, 64, 16),
@@ -126,11 +163,15 @@ def _decode_sched(w):
 def test_work_list_covers_every_kept_block_once(lp, n, k, b):
     X, W, bias, mask = _case(4, n, k, b, 0.55, 12)
     w = lp.pack_bsr(W, mask, b, count=True)
-    hdr, gent, ent = _decode_sched(w)
+    hdr, gent, ent, gpan = _decode_sched(w)
     bn, bk = _sides(b)
     assert (int(hdr[4]), int(hdr[5]), int(hdr[6]), int(hdr[7])) == (n, k, bn, bk)
     gb = 128 // bn
     M = mask.cpu().numpy()
+    # the group table: every row panel in exactly one slot, as the grouping rule picks them
+    used = sorted(int(r) for r in gpan.ravel() if r >= 0)
+    assert used == list(range(n // bn)) and np.all(gpan[:, gb:] == -1)
+    assert gpan.tolist() == _grouping(M, bn)
     rp, ci, _ = oracle.pack(_bits(W), M, b)
     seen = set()
     for g in range(int(hdr[1])):
@@ -139,15 +180,16 @@ def test_work_list_covers_every_kept_block_once(lp, n, k, b):
             j, pm = int(e[0]) & 0xFFFF, (int(e[0]) >> 16) & 0xFFFF
             js.append(j)
             for p in range(gb):
-                r = g * gb + p
+                r = int(gpan[g, p])
                 if (pm >> p) & 1:
                     t = int(e[1 + p])
-                    assert r < n // bn and M[r, j] and ci[t] == j and rp[r] <= t < rp[r + 1]
+                    assert r >= 0 and M[r, j] and ci[t] == j and rp[r] <= t < rp[r + 1]
                     seen.add(t)
                 else:
-                    assert e[1 + p] == -1 and (r >= n // bn or not M[r, j])
+                    assert e[1 + p] == -1 and (r < 0 or not M[r, j])
         assert js == sorted(set(js))
-        want = sorted(set(np.nonzero(M[g * gb:(g + 1) * gb].any(axis=0))[0].tolist()))
+        panels = [int(r) for r in gpan[g, :gb] if r >= 0]
+        want = sorted(set(np.nonzero(M[panels].any(axis=0))[0].tolist())) if panels else []
         assert js == want
     assert seen == set(range(len(ci)))
 
@@ -157,12 +199,12 @@ def _check_weight_stream(w, W, mask):
     block column (W's rows there, removed row panels zero), tiles contiguous in entry order,
     16-byte chunk c of tile row r stored at chunk c ^ ((r * rowbytes >> 7) & (rowbytes / 16 - 1))."""
     n, k, bn, bk = w.n, w.k, w.bn, w.bk
-    hdr, gent, ent = _decode_sched(w)
+    hdr, gent, ent, gpan = _decode_sched(w)
     ng, kb = int(hdr[1]), k // bk
     mp = 128
     rb, cpr = 2 * bk, 2 * bk // 16
     raw = w.sched.cpu().numpy().view(np.uint8)
-    ent_end = 4 * ((16 + ng + 1 + 3) // 4 * 4 + ng * kb * 12)
+    ent_end = 4 * (_entries_offset(ng) + ng * kb * 12)
     stream = raw[(ent_end + 1023) // 1024 * 1024:]
     Wb = _bits(W).reshape(n, k)
     M = mask.cpu().numpy()
@@ -175,7 +217,8 @@ def _check_weight_stream(w, W, mask):
             for i, q in enumerate(panels):
                 tile = stream[(t_next + i) * mp * rb:(t_next + i + 1) * mp * rb].reshape(mp, cpr, 16)
                 for r in range(mp):
-                    row = g * 128 + q * mp + r
+                    panel = int(gpan[g, (q * mp + r) // bn])
+                    row = panel * bn + (q * mp + r) % bn   # the output feature of group row r
                     kept = (pm >> ((q * mp + r) // bn)) & 1
                     want = Wb[row, j * bk:(j + 1) * bk] if kept else np.zeros(bk, np.uint16)
                     if kept:
@@ -219,6 +262,7 @@ def test_pack_many_matches_single_packs(lp, count):
         # header, group pointers and entries (the words padding the entries to 16 bytes are not defined)
         ha, hs, ea, es = _decode_sched(a)[0], _decode_sched(s1)[0], _decode_sched(a), _decode_sched(s1)
         assert np.array_equal(ha, hs) and np.array_equal(ea[1], es[1]) and np.array_equal(ea[2], es[2])
+        assert np.array_equal(ea[3], es[3])
         if i < 5:
             _check_weight_stream(a, Ws[i], masks[i])
         rp, ci, bl = oracle.pack(_bits(Ws[i]), masks[i].cpu().numpy(), b)
