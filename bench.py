@@ -62,6 +62,8 @@ def parse_args():
     p.add_argument("--alloc", action="store_true",
                    help="pruning-ratio allocation: distortion curves of the 48 DeiT-B weights + lambda search")
     p.add_argument("--alloc-samples", type=int, default=16, help="per-sample gradients per layer (--alloc)")
+    p.add_argument("--alloc-streams", type=int, default=8,
+                   help="CUDA streams the 48 independent weights are spread over (--alloc)")
     p.add_argument("--encoder", choices=["deit_b", "deit_s"], default=None,
                    help="end-to-end encoder forward (LayerNorm, attention, block-sparse linears) against dense")
     p.add_argument("--images", type=int, default=256, help="batch of 197-token images (--encoder)")
@@ -535,8 +537,9 @@ def run_calibrate(args, local):
 def run_alloc(args, local):
     """Pruning-ratio allocation (Sec. 3.4-3.5) for the 12-layer DeiT-B linear stack, 32x32 blocks:
     the distortion curve of each of the 48 weights from N seeded per-sample gradients (20 ratio
-    steps, kappa 1e-3), timed with CUDA events layer by layer (gradients are generated on the device
-    outside the timed region), then the host lambda search at a 50% FLOPs target. One JSON line:
+    steps, kappa 1e-3; the weights are independent and go round-robin to --alloc-streams CUDA streams,
+    each with its own workspace; every weight's gradients are generated on the device before the
+    timed region), then the host lambda search at a 50% FLOPs target. One JSON line:
     throughput in GB/s of algorithmic bytes (the gradients and the weight read once), against the
     measured HBM copy bandwidth; the oracle is timed on one qkv weight."""
     import torch
@@ -552,31 +555,45 @@ def run_alloc(args, local):
     Ws = [inputs.weight(n, k, inputs.seed(8, gi, "W"), dev) for gi, k, n in shapes]
     gen = torch.Generator(device=dev)
     ws_bytes = max(lp._lib.lpvit_delta_curve_workspace_bytes(N, n, k, b, b, steps) for _, k, n in shapes)
-    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
-    G = torch.empty(N * max(n * k for _, k, n in shapes), dtype=torch.float32, device=dev)
+    ns = max(1, args.alloc_streams)
+    wss = [torch.empty(ws_bytes, dtype=torch.uint8, device=dev) for _ in range(ns)]
 
     def grads(gi, k, n):
         gen.manual_seed(inputs.seed(8, gi, "X"))
-        Gv = G[:N * n * k].view(N, n, k)
+        Gv = torch.empty(N, n, k, dtype=torch.float32, device=dev)
         Gv.normal_(0.0, 1e-2, generator=gen)
         return Gv
 
-    lp.delta_curve(Ws[0], grads(*shapes[0]), b, steps, kappa, workspace=ws)  # warm-up
+    Gs = [grads(gi, k, n) for gi, k, n in shapes]  # all resident (N x 85 M floats) before timing
+    streams = [torch.cuda.Stream(dev) for _ in range(ns)]
+    main = torch.cuda.current_stream(dev)
+
+    def one_pass():
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(main)
+        for st in streams:
+            st.wait_event(e0)
+        ds = []
+        for i, ((gi, k, n), W) in enumerate(zip(shapes, Ws)):
+            st = streams[i % ns]
+            with torch.cuda.stream(st):
+                ds.append(lp.delta_curve(W, Gs[i], b, steps, kappa, workspace=wss[i % ns], stream=st))
+        for st in streams:
+            ev = torch.cuda.Event()
+            ev.record(st)
+            main.wait_event(ev)
+        e1.record(main)
+        e1.synchronize()
+        return e0.elapsed_time(e1), ds
+
+    one_pass()  # warm-up
     torch.cuda.synchronize()
     clk = ClockSampler(local)
     clk.start()
-    curves, total_ms, algo = [], 0.0, 0
-    for (gi, k, n), W in zip(shapes, Ws):
-        Gv = grads(gi, k, n)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        d = lp.delta_curve(W, Gv, b, steps, kappa, workspace=ws)
-        e1.record()
-        e1.synchronize()
-        total_ms += e0.elapsed_time(e1)
-        algo += 4 * N * n * k + 2 * n * k
-        curves.append(d.cpu().numpy())
+    total_ms, ds = one_pass()
     clocks = clk.stop()
+    curves = [d.cpu().numpy() for d in ds]
+    algo = sum(4 * N * n * k + 2 * n * k for _, k, n in shapes)
     F = [float(m * n * k) for _, k, n in shapes]
     c = [float(m * n * k) / (b * b) for _, k, n in shapes]
     t0 = time.perf_counter()
@@ -587,18 +604,18 @@ def run_alloc(args, local):
     line = {"metric": "pruning-ratio allocation: distortion-curve throughput (per-sample gradients + weights)",
             "value": achieved, "unit": "GB/s", "n_gpus": 1, "higher_is_better": True, "dtype": "f64",
             "data": "synthetic", "config": {"workload": "deit_b_12layer_allocation", "weights": 48, "block": b,
-                                            "samples": N, "ratio_steps": steps, "kappa": kappa,
+                                            "samples": N, "ratio_steps": steps, "kappa": kappa, "streams": ns,
                                             "flops_target": 0.5, "beta": 1e-12},
             "ms_total": total_ms, "lambda_search_ms": search_ms, "allocated_k": ks, "flops_remained": ratio,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": float(peaks.get("hbm_gbs", 6800.0)),
                          "unit": "GB/s", "frac": achieved / float(peaks.get("hbm_gbs", 6800.0)), "traffic": None,
                          "peak_source": src + " hbm_gbs (STREAM-style copy)"},
-            "gpu_launches": 5 * len(shapes), "clocks": clocks}
+            "gpu_launches": 8 * len(shapes), "clocks": clocks}
     if not args.no_cpu_baseline:
         import oracle.alloc as oalloc
         gi, k, n = shapes[0]
         Wb = inputs.bf16_bits(Ws[0])
-        Gh = grads(gi, k, n).cpu().numpy()
+        Gh = Gs[0].cpu().numpy()
         t0 = time.perf_counter()
         oalloc.delta_curve(Wb, Gh, b, steps, kappa)
         cpu_s = time.perf_counter() - t0
