@@ -29,7 +29,8 @@ constexpr int LN_THREADS = 256;
 constexpr int LN_MAX_D = 1024;
 constexpr int LN_VPL = LN_MAX_D / 8 / 32;  // 16-byte vectors per lane at most
 
-constexpr int ATT_WARPS = 4;
+constexpr int ATT_WARPS = 7;             // 13 query tiles of 16 in two rounds
+constexpr int KCHUNK = 8;                // key tiles of 8 per online-softmax chunk (64 keys)
 constexpr int HD = 64;                   // head dimension
 constexpr int MAX_TOKENS = 208;          // 13 tiles of 16
 constexpr int NT = MAX_TOKENS / 8;       // key tiles of 8
@@ -133,7 +134,12 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   return *reinterpret_cast<uint32_t *>(&p);
 }
 
-__global__ void __launch_bounds__(32 * ATT_WARPS)
+// One CTA per (image, head): Q, K, V of the head staged in shared memory by asynchronous copies;
+// each warp takes 16-query tiles and streams the keys in chunks of 64 with an online softmax
+// (running row max and sum, rescaling the partial output when the max grows), so a chunk's scores
+// stay in 32 registers per thread. Scores and exponentials in float32 (base 2, the 1/sqrt(64) scale
+// folded into log2 e), P rounded to bf16 for the P V products, fp32 accumulation.
+__global__ void __launch_bounds__(32 * ATT_WARPS, 2)
 attention_kernel(const __nv_bfloat16 *__restrict__ qkv, int tokens, int heads, __nv_bfloat16 *__restrict__ out) {
   extern __shared__ __align__(16) __nv_bfloat16 att_smem[];
   __nv_bfloat16 *Qs = att_smem, *Ks = Qs + MAX_TOKENS * ROW, *Vs = Ks + MAX_TOKENS * ROW;
@@ -156,6 +162,7 @@ attention_kernel(const __nv_bfloat16 *__restrict__ qkv, int tokens, int heads, _
   }
   asm volatile("cp.async.wait_all;" ::: "memory");
   __syncthreads();
+  constexpr float kScaleLog2 = 0.125f * 1.4426950408889634f;  // 1/sqrt(64) * log2(e)
   const int ntiles = tp / 8, kq = lane & 3, rq = lane >> 2;
   for (int mt = warp; mt < tp / 16; mt += ATT_WARPS) {
     uint32_t qa[HD / 16][4];
@@ -163,68 +170,84 @@ attention_kernel(const __nv_bfloat16 *__restrict__ qkv, int tokens, int heads, _
     for (int ks = 0; ks < HD / 16; ++ks)
       ldsm_x4(smem_addr(Qs + (16 * mt + (lane & 15)) * ROW + 16 * ks + (lane >> 4) * 8), qa[ks][0], qa[ks][1],
               qa[ks][2], qa[ks][3]);
-    float s[NT][4];
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-      s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-      if (nt < ntiles) {
-#pragma unroll
-        for (int ks = 0; ks < HD / 16; ++ks) {
-          uint32_t b0, b1;
-          ldsm_x2(smem_addr(Ks + (8 * nt + (lane & 7)) * ROW + 16 * ks + ((lane >> 3) & 1) * 8), b0, b1);
-          mma_bf16(s[nt], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
-        }
-      }
-    }
-    // scale, mask, row max (rows rq and rq + 8 of the tile; columns 8 nt + 2 kq + {0, 1})
-    float mx0 = -INFINITY, mx1 = -INFINITY;
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int col = 8 * nt + 2 * kq + (e & 1);
-        s[nt][e] = (nt < ntiles && col < tokens) ? s[nt][e] * 0.125f : -INFINITY;
-      }
-      mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]));
-      mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]));
-    }
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-    float sum0 = 0.f, sum1 = 0.f;
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-      s[nt][0] = expf(s[nt][0] - mx0);
-      s[nt][1] = expf(s[nt][1] - mx0);
-      s[nt][2] = expf(s[nt][2] - mx1);
-      s[nt][3] = expf(s[nt][3] - mx1);
-      sum0 += s[nt][0] + s[nt][1];
-      sum1 += s[nt][2] + s[nt][3];
-    }
-    sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
-    sum0 += __shfl_xor_sync(0xffffffffu, sum0, 2);
-    sum1 += __shfl_xor_sync(0xffffffffu, sum1, 1);
-    sum1 += __shfl_xor_sync(0xffffffffu, sum1, 2);
-    // O = P V
     float o[HD / 8][4];
 #pragma unroll
     for (int nd = 0; nd < HD / 8; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;  // rows rq and rq + 8 of the tile
+    for (int kc = 0; kc < ntiles; kc += KCHUNK) {
+      // S = Q K^T for keys 8 kc .. 8 (kc + KCHUNK)
+      float s[KCHUNK][4];
 #pragma unroll
-    for (int kt = 0; kt < NT / 2; ++kt) {
-      if (2 * kt < ntiles) {
-        const uint32_t a0 = pack_bf16(s[2 * kt][0], s[2 * kt][1]), a1 = pack_bf16(s[2 * kt][2], s[2 * kt][3]);
-        const uint32_t a2 = pack_bf16(s[2 * kt + 1][0], s[2 * kt + 1][1]);
-        const uint32_t a3 = pack_bf16(s[2 * kt + 1][2], s[2 * kt + 1][3]);
+      for (int nt = 0; nt < KCHUNK; ++nt) {
+        s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+        if (kc + nt < ntiles) {
 #pragma unroll
-        for (int nd = 0; nd < HD / 8; ++nd) {
-          uint32_t b0, b1;
-          ldsm_x2_trans(smem_addr(Vs + (16 * kt + (lane & 15)) * ROW + 8 * nd), b0, b1);
-          mma_bf16(o[nd], a0, a1, a2, a3, b0, b1);
+          for (int ks = 0; ks < HD / 16; ++ks) {
+            uint32_t b0, b1;
+            ldsm_x2(smem_addr(Ks + (8 * (kc + nt) + (lane & 7)) * ROW + 16 * ks + ((lane >> 3) & 1) * 8), b0, b1);
+            mma_bf16(s[nt], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
+          }
+        }
+      }
+      float cm0 = -INFINITY, cm1 = -INFINITY;
+#pragma unroll
+      for (int nt = 0; nt < KCHUNK; ++nt) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int col = 8 * (kc + nt) + 2 * kq + (e & 1);
+          s[nt][e] = col < tokens ? s[nt][e] * kScaleLog2 : -INFINITY;
+        }
+        cm0 = fmaxf(cm0, fmaxf(s[nt][0], s[nt][1]));
+        cm1 = fmaxf(cm1, fmaxf(s[nt][2], s[nt][3]));
+      }
+      cm0 = fmaxf(cm0, __shfl_xor_sync(0xffffffffu, cm0, 1));
+      cm0 = fmaxf(cm0, __shfl_xor_sync(0xffffffffu, cm0, 2));
+      cm1 = fmaxf(cm1, __shfl_xor_sync(0xffffffffu, cm1, 1));
+      cm1 = fmaxf(cm1, __shfl_xor_sync(0xffffffffu, cm1, 2));
+      // the first chunk always holds key 0, so the running max is finite from here on
+      const float n0 = fmaxf(m0, cm0), n1 = fmaxf(m1, cm1);
+      const float a0 = exp2f(m0 - n0), a1 = exp2f(m1 - n1);  // 0 on the first chunk
+      m0 = n0;
+      m1 = n1;
+      l0 *= a0;
+      l1 *= a1;
+#pragma unroll
+      for (int nd = 0; nd < HD / 8; ++nd) {
+        o[nd][0] *= a0;
+        o[nd][1] *= a0;
+        o[nd][2] *= a1;
+        o[nd][3] *= a1;
+      }
+#pragma unroll
+      for (int nt = 0; nt < KCHUNK; ++nt) {
+        s[nt][0] = exp2f(s[nt][0] - n0);
+        s[nt][1] = exp2f(s[nt][1] - n0);
+        s[nt][2] = exp2f(s[nt][2] - n1);
+        s[nt][3] = exp2f(s[nt][3] - n1);
+        l0 += s[nt][0] + s[nt][1];
+        l1 += s[nt][2] + s[nt][3];
+      }
+      // O += P V over the chunk's keys, 16 at a time (ntiles is even)
+#pragma unroll
+      for (int kt = 0; kt < KCHUNK / 2; ++kt) {
+        if (kc + 2 * kt < ntiles) {
+          const uint32_t p0 = pack_bf16(s[2 * kt][0], s[2 * kt][1]), p1 = pack_bf16(s[2 * kt][2], s[2 * kt][3]);
+          const uint32_t p2 = pack_bf16(s[2 * kt + 1][0], s[2 * kt + 1][1]);
+          const uint32_t p3 = pack_bf16(s[2 * kt + 1][2], s[2 * kt + 1][3]);
+#pragma unroll
+          for (int nd = 0; nd < HD / 8; ++nd) {
+            uint32_t b0, b1;
+            ldsm_x2_trans(smem_addr(Vs + (8 * kc + 16 * kt + (lane & 15)) * ROW + 8 * nd), b0, b1);
+            mma_bf16(o[nd], p0, p1, p2, p3, b0, b1);
+          }
         }
       }
     }
-    const float inv0 = 1.f / sum0, inv1 = 1.f / sum1;
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+    l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+    const float inv0 = 1.f / l0, inv1 = 1.f / l1;
     const int r0 = 16 * mt + rq, r1 = r0 + 8;
 #pragma unroll
     for (int nd = 0; nd < HD / 8; ++nd) {
