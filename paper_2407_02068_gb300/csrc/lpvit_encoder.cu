@@ -33,7 +33,6 @@ constexpr int ATT_WARPS = 7;             // 13 query tiles of 16 in two rounds
 constexpr int KCHUNK = 8;                // key tiles of 8 per online-softmax chunk (64 keys)
 constexpr int HD = 64;                   // head dimension
 constexpr int MAX_TOKENS = 208;          // 13 tiles of 16
-constexpr int NT = MAX_TOKENS / 8;       // key tiles of 8
 constexpr int ROW = HD + 8;              // shared-memory row in bf16 (144 bytes)
 constexpr int ATT_SMEM = 3 * MAX_TOKENS * ROW * 2;
 

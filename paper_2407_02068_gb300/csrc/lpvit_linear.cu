@@ -3,9 +3,10 @@
 // blocks). The kernel is compiled per block width BK (input columns of a block: 16, 32 or 64);
 // the block height only decides which rows of a group tile the pack left zero.
 //
-// Work unit = 256 tokens x one 128-feature group of row panels (the work list's group table names
-// the panels of each group; the epilogue maps a group row to its output feature through it) (x one slice of the group's block
-// columns when the problem is too small to fill the GPU). Per CTA (one per SM, persistent):
+// Work unit = 256 tokens x one 128-feature group of row panels (x one slice of the group's block
+// columns when the problem is too small to fill the GPU); the work list's group table names the
+// panels of each group and the epilogue maps a group row to its output feature through it.
+// Per CTA (one per SM, persistent):
 //   warp 0      producer: takes units from a global atomic queue, walks the unit's work-list
 //               entries and, per entry (one block column j), loads the X tile [256 tokens x bk]
 //               (TMA tensor copy) and the entry's weight tiles, one per MMA panel keeping a block
@@ -180,7 +181,6 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
   auto unite_bar = [&](int u) { return bar0 + 8u * (2 * L::NS + 4 + L::UR + u); };
   const uint32_t drain_bar = bar0 + 8u * (2 * L::NS + 4 + 2 * L::UR);
   const uint32_t episync_bar = drain_bar + 8u;
-  volatile int *meta = reinterpret_cast<volatile int *>(smem + L::META_OFF);
   UnitInfo *ring = reinterpret_cast<UnitInfo *>(smem + L::RING_OFF);
   int *slice_ptr = reinterpret_cast<int *>(smem + L::SLICE_OFF);
   int *gent_s = reinterpret_cast<int *>(smem + L::GENT_OFF);
@@ -373,7 +373,6 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
           const uint32_t st_u32 = smem_base + stk * C::STAGE_BYTES;
           if (k2 < nb && (lane & 1) == 0) {
             if (!tiles_ok) atomicOr(&P.ctl->err, ERR_BAD_SCHED);
-            meta[stk] = (int)mm;
             mbar_arrive_expect_tx(full_bar(stk), C::X_BYTES + __popc(mm) * C::A_BYTES);
           }
           __syncwarp();
@@ -441,18 +440,15 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
           break;
         }
         tc_fence_after();
-        const uint32_t mm = (uint32_t)meta[stage];  // 1: the stage holds this entry's W tile
+        // every entry keeps a block of its group, so every stage holds a W tile (a work list whose
+        // tile range is corrupt has its error bit set and its stage's weights left stale)
         const uint32_t st_u32 = smem_base + stage * C::STAGE_BYTES;
-        if (mm) {
-          if (elect_one()) {
-            issue_entry<BK>(st_u32, dbase, touched);
-            tc_commit(empty_bar(stage));
-          }
-        } else {
-          if (elect_one()) mbar_arrive(empty_bar(stage));
+        if (elect_one()) {
+          issue_entry<BK>(st_u32, dbase, touched);
+          tc_commit(empty_bar(stage));
         }
         __syncwarp();
-        touched |= mm;
+        touched = 1;
         ++it;
       }
       if (!ok) break;

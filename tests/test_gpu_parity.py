@@ -194,6 +194,37 @@ def test_work_list_covers_every_kept_block_once(lp, n, k, b):
     assert seen == set(range(len(ci)))
 
 
+@pytest.mark.parametrize("b", [32, 16, (64, 32)])
+def test_grouping_pairs_panels_with_the_same_columns(lp, b):
+    """Row panels of two kinds keep blocks in two disjoint sets of block columns (even panels in
+    A, odd panels in B). Consecutive groups would mix the kinds and need |A u B| entries each; the
+    plan's grouping puts panels of one kind together, so each group needs |A| or |B| entries. The
+    linear on that work list still matches the oracle."""
+    bn, bk = _sides(b)
+    n, k = 1024, 512
+    npan, kb = n // bn, k // bk
+    rng = np.random.default_rng(77)
+    cols = rng.permutation(kb)
+    A, B = np.sort(cols[:kb // 3]), np.sort(cols[kb // 3:kb // 3 + kb // 4])
+    M = np.zeros((npan, kb), np.uint8)
+    M[0::2, A] = 1
+    M[1::2, B] = 1
+    X, W, bias, _ = _case(300, n, k, b, 0.5, 1234)
+    mask = torch.from_numpy(M).cuda()
+    w = lp.pack_bsr(W, mask, b, count=True)
+    hdr, gent, ent, gpan = _decode_sched(w)
+    gb = 128 // bn
+    assert gpan.tolist() == _grouping(M, bn)
+    for g in range(int(hdr[1])):
+        kinds = {int(r) % 2 for r in gpan[g, :gb] if r >= 0}
+        assert len(kinds) == 1                       # one kind of panel per group
+    ng = npan // gb
+    assert int(gent[-1]) == (ng // 2) * (len(A) + len(B))
+    Y = lp.bsr_linear(w, X, bias, out_dtype=torch.float32)
+    ref = _oracle(X, W, mask, b, bias)
+    assert _norm_err(Y.cpu().double().numpy(), ref) <= TIGHT_TOL
+
+
 def _check_weight_stream(w, W, mask):
     """The work list's weight stream: entry by entry, the 128-row tile of the entry's group at its
     block column (W's rows there, removed row panels zero), tiles contiguous in entry order,
