@@ -220,6 +220,20 @@ lpvit_status lpvit_bsr_linear_gelu(const lpvit_bsr *bsr, const void *X, int64_t 
                                    const float *bias, void *Y, int64_t ldy, lpvit_dtype y_dtype, void *workspace,
                                    size_t ws_bytes, void *stream);
 
+/* Y = round_bf16(round_bf16(act(X W~^T + bias)) + R): lpvit_bsr_linear (gelu == 0) or
+ * lpvit_bsr_linear_gelu (gelu == 1) with bf16 output, followed by the residual addition of a
+ * pre-norm transformer block (x + sublayer(x), the DeiT blocks whose linears Sec. 4 prunes), done in
+ * the GEMM's epilogue instead of a separate pass over the activations. Each sum is formed in float32
+ * from the two bf16 values and rounded to nearest even, as a separate bf16 addition would round it.
+ *   R    bf16 [m][ldr] device, ldr >= n, ldr % 8 == 0, 16-byte aligned; read only. R may be Y itself
+ *        (R == Y and ldr == ldy: Y += the layer, in place); otherwise it must not overlap Y.
+ *   gelu 0 or 1.
+ * Other arguments, ownership, asynchrony and errors as for lpvit_bsr_linear (y_dtype is bf16).
+ * Returns LPVIT_ERR_INVALID_ARG for a null R, a bad ldr or alignment, or a partial overlap of R and Y. */
+lpvit_status lpvit_bsr_linear_residual(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx,
+                                       const float *bias, int32_t gelu, const void *R, int64_t ldr, void *Y,
+                                       int64_t ldy, void *workspace, size_t ws_bytes, void *stream);
+
 /* Size of the library-held scratch array used by lpvit_bsr_linear_noalloc (8 MiB). */
 #define LPVIT_NOALLOC_SCRATCH_BYTES (8 * 1024 * 1024)
 

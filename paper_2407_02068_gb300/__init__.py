@@ -248,9 +248,11 @@ def workspace_for(w: BsrWeight, m: int, device=None) -> torch.Tensor:
 
 def bsr_linear(w: BsrWeight, X: torch.Tensor, bias: torch.Tensor | None = None, gelu: bool = False,
                out: torch.Tensor | None = None, out_dtype=torch.bfloat16, workspace: torch.Tensor | None = None,
-               stream=None) -> torch.Tensor:
+               stream=None, residual: torch.Tensor | None = None) -> torch.Tensor:
     """Y = act(X W~^T + bias). X: bf16 [m, k] CUDA (a row-strided view with unit column stride is
-    fine); bias: fp32 [n] or None. Returns Y [m, n] (or writes ``out``)."""
+    fine); bias: fp32 [n] or None. Returns Y [m, n] (or writes ``out``). With ``residual`` (bf16
+    [m, n], 16-byte rows; may be ``out`` itself) Y = round(round(act(...)) + residual), bf16
+    (lpvit_bsr_linear_residual)."""
     if X.dtype != torch.bfloat16 or X.dim() != 2 or X.stride(1) != 1:
         raise ValueError("X must be a 2-D bf16 tensor with unit column stride")
     m = X.shape[0]
@@ -263,6 +265,17 @@ def bsr_linear(w: BsrWeight, X: torch.Tensor, bias: torch.Tensor | None = None, 
             raise ValueError("bias must be a contiguous fp32 tensor")
     if workspace is None:
         workspace = workspace_for(w, m, X.device)
+    if residual is not None:
+        if residual.dtype != torch.bfloat16 or residual.dim() != 2 or residual.stride(1) != 1 \
+                or tuple(residual.shape) != (m, w.n) or out.dtype != torch.bfloat16:
+            raise ValueError("residual must be a bf16 [m, n] tensor with unit column stride, out bf16")
+        st = _lib.lpvit_bsr_linear_residual(w.struct(), X.data_ptr(), m, X.stride(0),
+                                            bias.data_ptr() if bias is not None else None, gelu,
+                                            residual.data_ptr(), residual.stride(0), out.data_ptr(), out.stride(0),
+                                            workspace.data_ptr(), workspace.numel(), _stream_handle(stream))
+        if st != _lib.LPVIT_OK:
+            raise LpvitError(st, "lpvit_bsr_linear_residual")
+        return out
     fn = _lib.lpvit_bsr_linear_gelu if gelu else _lib.lpvit_bsr_linear
     st = fn(w.struct(), X.data_ptr(), m, X.stride(0), bias.data_ptr() if bias is not None else None,
             out.data_ptr(), out.stride(0), _lib.LPVIT_F32 if out.dtype == torch.float32 else _lib.LPVIT_BF16,

@@ -25,7 +25,7 @@ EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_workspace_bytes", "lpvi
            "lpvit_bsr_linear_gelu", "lpvit_bsr_linear_noalloc", "lpvit_check", "lpvit_status_string",
            "lpvit_selftest_wait", "lpvit_pack_bsr_many", "lpvit_taylor_block_mask",
            "lpvit_delta_curve_workspace_bytes", "lpvit_delta_curve", "lpvit_lambda_search", "lpvit_mean_gradient",
-           "lpvit_add_layernorm", "lpvit_attention")
+           "lpvit_add_layernorm", "lpvit_attention", "lpvit_bsr_linear_residual")
 LPVIT_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 
@@ -87,6 +87,8 @@ def load(path: str | None = None):
             f = getattr(lib, name)
             f.restype = ctypes.c_int
             f.argtypes = [BP, V, I64, I64, V, V, I64, ctypes.c_int, V, SZ, V]
+        lib.lpvit_bsr_linear_residual.restype = ctypes.c_int
+        lib.lpvit_bsr_linear_residual.argtypes = [BP, V, I64, I64, V, ctypes.c_int32, V, I64, V, I64, V, SZ, V]
         lib.lpvit_bsr_linear_noalloc.restype = ctypes.c_int
         lib.lpvit_bsr_linear_noalloc.argtypes = [BP, V, I64, I64, V, V, I64, ctypes.c_int, ctypes.c_int, V]
         lib.lpvit_check.restype = ctypes.c_int
@@ -181,6 +183,12 @@ def lpvit_bsr_linear(bsr, X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, ws_ptr, 
 def lpvit_bsr_linear_gelu(bsr, X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, ws_ptr, ws_bytes, stream) -> int:
     return load().lpvit_bsr_linear_gelu(ctypes.byref(bsr), X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, ws_ptr,
                                         ws_bytes, stream)
+
+
+def lpvit_bsr_linear_residual(bsr, X_ptr, m, ldx, bias_ptr, gelu, R_ptr, ldr, Y_ptr, ldy, ws_ptr, ws_bytes,
+                              stream) -> int:
+    return load().lpvit_bsr_linear_residual(ctypes.byref(bsr), X_ptr, m, ldx, bias_ptr, int(gelu), R_ptr,
+                                            ldr, Y_ptr, ldy, ws_ptr, ws_bytes, stream)
 
 
 def lpvit_bsr_linear_noalloc(bsr, X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, gelu, stream) -> int:

@@ -113,7 +113,8 @@ lpvit_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LPVIT_OK : L
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias, void *Y,
-                        int64_t ldy, lpvit_dtype y_dtype, void *workspace, size_t ws_bytes, void *stream, int gelu) {
+                        int64_t ldy, lpvit_dtype y_dtype, void *workspace, size_t ws_bytes, void *stream, int gelu,
+                        const void *R = nullptr, int64_t ldr = 0) {
   if (!bsr) return LPVIT_ERR_INVALID_ARG;
   const int n = bsr->n, k = bsr->k, bn = bsr->bn, bk = bsr->bk;
   if (!valid_side(bn) || !valid_side(bk)) return LPVIT_ERR_UNSUPPORTED;
@@ -130,10 +131,18 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   if (bias && !aligned(bias, 4)) return LPVIT_ERR_INVALID_ARG;
   if (m > (int64_t)0x7fffff00) return LPVIT_ERR_INVALID_ARG;
   // X and Y must not overlap
+  const uintptr_t y0 = reinterpret_cast<uintptr_t>(Y), y1 = y0 + (size_t)((m - 1) * ldy + n) * ysz;
   {
     const uintptr_t x0 = reinterpret_cast<uintptr_t>(X), x1 = x0 + (size_t)((m - 1) * ldx + k) * 2;
-    const uintptr_t y0 = reinterpret_cast<uintptr_t>(Y), y1 = y0 + (size_t)((m - 1) * ldy + n) * ysz;
     if (x0 < y1 && y0 < x1) return LPVIT_ERR_INVALID_ARG;
+  }
+  // the residual: bf16, 16-byte rows like X; either Y itself (in place) or clear of Y
+  if (R) {
+    if (y_dtype != LPVIT_BF16) return LPVIT_ERR_UNSUPPORTED;
+    if (ldr < n || ldr % 8 != 0 || !aligned(R, 16)) return LPVIT_ERR_INVALID_ARG;
+    const uintptr_t r0 = reinterpret_cast<uintptr_t>(R), r1 = r0 + (size_t)((m - 1) * ldr + n) * 2;
+    const bool in_place = R == Y && ldr == ldy;
+    if (!in_place && r0 < y1 && y0 < r1) return LPVIT_ERR_INVALID_ARG;
   }
   if (bsr->sched_bytes < lpvit_sched_bytes(n, k, bn, bk)) return LPVIT_ERR_WORKSPACE;
   int sms = 0;
@@ -175,6 +184,8 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.y_f32 = y_dtype == LPVIT_F32;
   P.gelu = gelu;
   P.y_vec16 = (aligned(Y, 16) && ldy % 8 == 0) ? 1 : 0;
+  P.R = static_cast<const uint16_t *>(R);
+  P.ldr = R ? ldr : 0;
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   P.ctl = reinterpret_cast<Control *>(ws);
   P.tickets = reinterpret_cast<int32_t *>(ws + W.tickets_off);
@@ -284,6 +295,13 @@ lpvit_status lpvit_bsr_linear_gelu(const lpvit_bsr *bsr, const void *X, int64_t 
                                    const float *bias, void *Y, int64_t ldy, lpvit_dtype y_dtype, void *workspace,
                                    size_t ws_bytes, void *stream) {
   return run_linear(bsr, X, m, ldx, bias, Y, ldy, y_dtype, workspace, ws_bytes, stream, 1);
+}
+
+lpvit_status lpvit_bsr_linear_residual(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx,
+                                       const float *bias, int32_t gelu, const void *R, int64_t ldr, void *Y,
+                                       int64_t ldy, void *workspace, size_t ws_bytes, void *stream) {
+  if (!R || (gelu != 0 && gelu != 1)) return LPVIT_ERR_INVALID_ARG;
+  return run_linear(bsr, X, m, ldx, bias, Y, ldy, LPVIT_BF16, workspace, ws_bytes, stream, gelu, R, ldr);
 }
 
 lpvit_status lpvit_check(void *workspace, void *stream) {

@@ -80,6 +80,8 @@ struct LinearParams {
   int n_tt, n_groups, S;   // token tiles, 128-feature groups, max entries per slice
   int y_f32, gelu;
   int y_vec16;             // bf16 output rows may take 16-byte stores (Y 16-byte aligned, ldy % 8 == 0)
+  const uint16_t *R;       // bf16 residual [m][ldr] added after rounding (bf16 output only), or nullptr
+  int64_t ldr;
   Control *ctl;
   int32_t *tickets;        // [n_tt * n_groups] arrival tickets of split units
   float *partials;         // [slots][128 features][256 tokens] fp32 partial sums of split units

@@ -89,7 +89,8 @@ struct Smem {
 // Epilogue of one 32 x 32 block held by a warp: y[i] = accumulator of token tok_base + i for the
 // lane's output feature fl (-1: a group row without a panel; turned into the output in place), bb =
 // that feature's bias (0 without one). Lanes 8c .. 8c + 7 hold consecutive features of one row panel.
-// Adds the bias, applies GELU, rounds, and stores rows [tok_base, min(tok_base + 32, m)).
+// Adds the bias, applies GELU, rounds, adds the bf16 residual if there is one (rounding again), and
+// stores rows [tok_base, min(tok_base + 32, m)).
 // bf16 output is staged through this warp's shared tile (rows padded to 80 bytes, conflict-free) so
 // that every token row leaves as 16-byte vector stores; fp32 output is stored directly (a warp
 // writes 128 contiguous bytes per token).
@@ -132,8 +133,17 @@ __device__ __forceinline__ void emit32(float (&y)[32], float bb, int fl, int64_t
 #pragma unroll
     for (int it = 0; it < 2; ++it) {
       const int rt = 8 * it + (lane >> 2), row = 16 * half + rt;
-      const int4 val = *reinterpret_cast<const int4 *>(tile + rt * 80 + ch * 16);
+      int4 val = *reinterpret_cast<const int4 *>(tile + rt * 80 + ch * 16);
       if (row < rows && cvalid) {
+        if (P.R != nullptr) {
+          // + the residual, each sum rounded to bf16 (a plain load: R may be Y itself, read and then
+          // written by this thread only)
+          const int4 rv = *reinterpret_cast<const int4 *>(P.R + (tok_base + row) * P.ldr + fch);
+          __nv_bfloat16 *a = reinterpret_cast<__nv_bfloat16 *>(&val);
+          const __nv_bfloat16 *b = reinterpret_cast<const __nv_bfloat16 *>(&rv);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) a[e] = __float2bfloat16_rn(__bfloat162float(a[e]) + __bfloat162float(b[e]));
+        }
         __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(P.Y) + (tok_base + row) * P.ldy + fch;
         if (P.y_vec16) {
           *reinterpret_cast<int4 *>(dst) = val;

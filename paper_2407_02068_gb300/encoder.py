@@ -55,7 +55,7 @@ class SparseEncoder:
             for name in NAMES:
                 if self.layers:
                     ws[name] = workspace_for(self.w[0][name], M, dev)
-            self._bufs[M] = dict(h=e(D), qkv=e(3 * D), a=e(D), p=e(D), f=e(hid), o=e(D), s0=e(D), s1=e(D),
+            self._bufs[M] = dict(h=e(D), qkv=e(3 * D), a=e(D), f=e(hid), s0=e(D), s1=e(D),
                                  out=e(D), ws=ws)
         return self._bufs[M]
 
@@ -64,29 +64,25 @@ class SparseEncoder:
         (a buffer reused by the next call with the same shape)."""
         M = x.shape[0]
         B = self._buffers(M, x.device)
+        # the residual stream ping-pongs between s0 and s1 (x itself is never written); proj and fc2
+        # add it in their epilogues, so every LayerNorm reads the finished sum
         s_cur, s_next = x, B["s0"]
-        for i, (L, W) in enumerate(zip(self.layers, self.w)):
-            if i == 0:
-                add_layernorm(x, None, *L["ln1"], eps=self.eps, norm_out=B["h"])
-            else:
-                add_layernorm(s_cur, B["o"], *L["ln1"], eps=self.eps, norm_out=B["h"], sum_out=s_next)
-                s_cur, s_next = s_next, (B["s1"] if s_next is B["s0"] else B["s0"])
+        for L, W in zip(self.layers, self.w):
+            add_layernorm(s_cur, None, *L["ln1"], eps=self.eps, norm_out=B["h"])
             bsr_linear(W["qkv"], B["h"], L["qkv"][2], out=B["qkv"], workspace=B["ws"]["qkv"])
             attention(B["qkv"], self.tokens, self.heads, out=B["a"])
-            bsr_linear(W["proj"], B["a"], L["proj"][2], out=B["p"], workspace=B["ws"]["proj"])
-            add_layernorm(s_cur, B["p"], *L["ln2"], eps=self.eps, norm_out=B["h"], sum_out=s_next)
+            bsr_linear(W["proj"], B["a"], L["proj"][2], out=s_next, workspace=B["ws"]["proj"], residual=s_cur)
             s_cur, s_next = s_next, (B["s1"] if s_next is B["s0"] else B["s0"])
+            add_layernorm(s_cur, None, *L["ln2"], eps=self.eps, norm_out=B["h"])
             bsr_linear(W["fc1"], B["h"], L["fc1"][2], gelu=True, out=B["f"], workspace=B["ws"]["fc1"])
-            bsr_linear(W["fc2"], B["f"], L["fc2"][2], out=B["o"], workspace=B["ws"]["fc2"])
-        if self.layers:
-            add_layernorm(s_cur, B["o"], *self.final, eps=self.eps, norm_out=B["out"], sum_out=s_next)
-        else:
-            add_layernorm(x, None, *self.final, eps=self.eps, norm_out=B["out"])
+            bsr_linear(W["fc2"], B["f"], L["fc2"][2], out=s_next, workspace=B["ws"]["fc2"], residual=s_cur)
+            s_cur, s_next = s_next, (B["s1"] if s_next is B["s0"] else B["s0"])
+        add_layernorm(s_cur, None, *self.final, eps=self.eps, norm_out=B["out"])
         return B["out"]
 
     def launches(self) -> int:
-        """Library kernel launches per forward: per layer 2 add-LayerNorms, 4 linears, 1 attention;
-        plus the final LayerNorm."""
+        """Library kernel launches per forward: per layer 2 LayerNorms, 4 linears (proj and fc2 adding
+        the residual), 1 attention; plus the final LayerNorm."""
         return 7 * len(self.layers) + 1
 
     def dense_forward(self, x: torch.Tensor) -> torch.Tensor:

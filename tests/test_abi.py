@@ -66,6 +66,22 @@ def test_bad_arguments_are_rejected_without_a_gpu(lib):
     assert lib.lpvit_bsr_linear(bsr, fake.value, 4, 388, None, 0x200000, 1152, 0, 0x100000, 1 << 20, None) == \
         lib.LPVIT_ERR_INVALID_ARG
     assert lib.lpvit_check(None, None) == lib.LPVIT_ERR_INVALID_ARG
+    # residual linear: R present, gelu 0/1, R 16-byte aligned with ldr >= n and ldr % 8 == 0, R either
+    # Y itself (then the call proceeds to the work-list size check) or clear of Y
+    rb = lib.lpvit_bsr(1152, 384, 32, 32, 432, None, None, None, 0x400000, 0)
+    X, Y, ws = 0x1000, 0x200000, 0x100000
+
+    def res(R, ldr, gelu=0, ldy=1152):
+        return lib.lpvit_bsr_linear_residual(rb, X, 4, 384, None, gelu, R, ldr, Y, ldy, ws, 1 << 20, None)
+    assert res(None, 1152) == lib.LPVIT_ERR_INVALID_ARG
+    assert res(0x300000, 1152, gelu=2) == lib.LPVIT_ERR_INVALID_ARG
+    assert res(0x300002, 1152) == lib.LPVIT_ERR_INVALID_ARG           # misaligned
+    assert res(0x300000, 1148) == lib.LPVIT_ERR_INVALID_ARG           # ldr < n
+    assert res(0x300000, 1156) == lib.LPVIT_ERR_INVALID_ARG           # ldr % 8
+    assert res(Y + 16, 1152) == lib.LPVIT_ERR_INVALID_ARG             # overlaps Y without being Y
+    assert res(Y, 1160, ldy=1152) == lib.LPVIT_ERR_INVALID_ARG        # Y's rows, another stride
+    assert res(Y, 1152) == lib.LPVIT_ERR_WORKSPACE                    # in place: accepted, no work list
+    assert res(0x300000, 1152) == lib.LPVIT_ERR_WORKSPACE             # clear of Y: accepted
     # the batched pack checks every job before launching anything
     assert lib.load().lpvit_pack_bsr_many(0, None, None, None, None) == lib.LPVIT_OK
     assert lib.load().lpvit_pack_bsr_many(-1, None, None, None, None) == lib.LPVIT_ERR_INVALID_ARG

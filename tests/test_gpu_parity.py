@@ -455,6 +455,24 @@ def test_bf16_output_offsets_and_row_strides(lp, col0, extra):
     assert np.all(np.abs(Yc.float().cpu().double().numpy() - ref) <= _bf16_tol(ref, X, W, mask, b, bias, gelu=True))
 
 
+@pytest.mark.parametrize("b,m,n,k,gelu", [(32, 333, 256, 256, False), (16, 197, 768, 3072, False),
+                                          ((64, 32), 300, 384, 512, True)])
+def test_residual_linear_is_the_bf16_sum(lp, b, m, n, k, gelu):
+    """lpvit_bsr_linear_residual: Y equals, bit for bit, the plain linear's bf16 output plus R
+    rounded to bf16 (the sum formed in float32), into a new tensor and in place (R = Y); the
+    197-row case splits its units (the fix-up path)."""
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 1300 + _sid(b))
+    w = lp.pack_bsr(W, mask, b)
+    R = torch.randn(m, n, generator=torch.Generator().manual_seed(9)).to(torch.bfloat16).cuda()
+    Y0 = lp.bsr_linear(w, X, bias, gelu=gelu)
+    want = (Y0.float() + R.float()).to(torch.bfloat16)
+    Y = lp.bsr_linear(w, X, bias, gelu=gelu, residual=R)
+    assert torch.equal(Y, want)
+    Z = R.clone()
+    lp.bsr_linear(w, X, bias, gelu=gelu, out=Z, residual=Z)
+    assert torch.equal(Z, want)
+
+
 @pytest.mark.parametrize("b", [32, (64, 32), (16, 32)])
 def test_deterministic_repeats(lp, b):
     m, n, k = 197, 768, 3072   # small m: split slices + fix-up path
