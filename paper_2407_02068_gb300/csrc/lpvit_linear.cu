@@ -9,12 +9,12 @@
 // Per CTA (one per SM, persistent):
 //   warp 0      producer: takes units from a global atomic queue, walks the unit's work-list
 //               entries and, per entry (one block column j), loads the X tile [256 tokens x bk]
-//               (TMA tensor copy) and the entry's weight tiles, one per MMA panel keeping a block
-//               at column j, stored back to back in the work list's weight stream (one bulk copy).
+//               (TMA tensor copy) and the entry's 128 x bk group tile from the work list's weight
+//               stream (one bulk copy), for a batch of entries at a time, one lane per copy.
 //   warp 1      MMA issuer: per entry and per 16-wide k step, one tcgen05 MMA (M = 128, N = 256,
-//               K = 16, both operands from shared memory): D[128 features x 256 tokens] +=
+//               K = 16, both operands from shared memory): D[128 group rows x 256 tokens] +=
 //               W_tile * X_tile^T, fp32 in TMEM. The W tile covers the whole group, with zero rows
-//               for the row panels that keep no block at this column.
+//               for the slots whose panel keeps no block at this column.
 //   warps 2..17 epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
 //               type, stores of 64-byte row segments; split slices are summed in slice order
 //               by the last slice to finish (ticket), which makes the result deterministic.
@@ -74,8 +74,7 @@ struct Smem {
   static constexpr int BAR_OFF = CTRL_OFF;
   // barriers: full[NS], empty[NS], accf[2], acce[2], unitf[UR], unite[UR], drain, episync
   static constexpr int NBARS = 2 * NS + 4 + 2 * UR + 2;
-  static constexpr int META_OFF = BAR_OFF + 8 * NBARS;
-  static constexpr int RING_OFF = (META_OFF + 4 * NS + 31) / 32 * 32;
+  static constexpr int RING_OFF = (BAR_OFF + 8 * NBARS + 31) / 32 * 32;
   static constexpr int SLICE_OFF = RING_OFF + (int)sizeof(UnitInfo) * UR;
   static constexpr int GENT_OFF = SLICE_OFF + 4 * (MAX_GROUPS + 1);  // the group entry table, staged
   static constexpr int MISC_OFF = GENT_OFF + 4 * (MAX_GROUPS + 1);
