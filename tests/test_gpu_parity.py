@@ -159,7 +159,10 @@ def _grouping(M, bn):
 
 
 @pytest.mark.parametrize("n,k,b", [(1152, 384, 32), (384, 1536, 16), (768, 3072, 64), (200 * 16, 64, 16),
-                                   (768, 768, (64, 32)), (208, 384, (16, 32)), (320, 128, (64, 16))])
+                                   (768, 768, (64, 32)), (208, 384, (16, 32)), (320, 128, (64, 16)),
+                                   (1024 * 16, 64, 16),      # 1024 panels: the grouping's limit
+                                   (1025 * 16, 64, 16),      # 1025 panels: consecutive groups
+                                   (8192, 8704, 16)])        # 512 panels x 17 bitmap words > 8192
 def test_work_list_covers_every_kept_block_once(lp, n, k, b):
     X, W, bias, mask = _case(4, n, k, b, 0.55, 12)
     w = lp.pack_bsr(W, mask, b, count=True)
