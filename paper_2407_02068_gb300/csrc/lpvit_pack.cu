@@ -313,8 +313,8 @@ __device__ __forceinline__ void copy_body(const uint16_t *__restrict__ W, int n,
                                           int cap, uint16_t *__restrict__ blocks, int cta, int ncta) {
   const int np = n / bn;
   const int nnzb = min(row_ptr[np], cap);
-  const int vec_per_row = bk / 8;  // 16-byte vectors per block row
-  const int vecs = bn * vec_per_row;
+  const int lvpr = __ffs(bk / 8) - 1;  // log2 of the 16-byte vectors per block row (bk is a power of 2)
+  const int vecs = bn << lvpr;
   for (int t = cta; t < nnzb; t += ncta) {
     int lo = 0, hi = np - 1;  // largest r with row_ptr[r] <= t (that panel holds block t)
     while (lo < hi) {
@@ -324,7 +324,7 @@ __device__ __forceinline__ void copy_body(const uint16_t *__restrict__ W, int n,
     }
     const int r = lo, j = col_idx[t];
     for (int v = threadIdx.x; v < vecs; v += blockDim.x) {
-      const int c = v / vec_per_row, cv = v - c * vec_per_row;
+      const int c = v >> lvpr, cv = v & ((1 << lvpr) - 1);
       const int4 *src = reinterpret_cast<const int4 *>(W + ((int64_t)r * bn + c) * k + (int64_t)j * bk + cv * 8);
       int4 *dst = reinterpret_cast<int4 *>(blocks + ((int64_t)t * bn + c) * bk + cv * 8);
       *dst = __ldg(src);
@@ -339,6 +339,7 @@ __device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int 
   if (sched[1] != ng || sched[3] != 0) return;  // not this shape's plan, or blocks overflowed
   const int total = sched[2];
   const int row_bytes = 2 * bk, cpr = row_bytes / 16, chunks = GROUP_FEATURES * cpr;
+  const int lcpr = __ffs(cpr) - 1, lbn = __ffs(bn) - 1;  // bk and bn are powers of 2
   const int tile_bytes = stream_tile_bytes(bk);
   const int64_t max_tiles = sched_stream_tiles(ng, kb);
   const int32_t *gent = sched + SCHED_HDR_INTS;
@@ -360,11 +361,11 @@ __device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int 
     if (j >= kb || t < 0 || (int64_t)t >= max_tiles) continue;
     uint8_t *tile = stream + (int64_t)t * tile_bytes;
     for (int v = threadIdx.x; v < chunks; v += blockDim.x) {
-      const int r = v / cpr, c = v - r * cpr;
-      const int panel = gpan[g * MAX_GROUP_PANELS + r / bn];
-      const int row = panel * bn + r % bn;  // the output feature of group row r
+      const int r = v >> lcpr, c = v & (cpr - 1), slot = r >> lbn;
+      const int panel = gpan[g * MAX_GROUP_PANELS + slot];
+      const int row = (panel << lbn) + (r & (bn - 1));  // the output feature of group row r
       int4 val = make_int4(0, 0, 0, 0);
-      if (((pm >> (r / bn)) & 1u) && panel >= 0 && row < n)
+      if (((pm >> slot) & 1u) && panel >= 0 && row < n)
         val = __ldg(reinterpret_cast<const int4 *>(W + (int64_t)row * k + (int64_t)j * bk + c * 8));
       reinterpret_cast<int4 *>(tile + r * row_bytes)[c ^ stream_chunk_swizzle(r, row_bytes)] = val;
     }
