@@ -9,7 +9,8 @@ or 64 (Table 2 uses 32x32, 64x32, 16x32 and 16x16). This package wraps the C lib
 * ``taylor_block_mask(W, G, b, alpha)`` -- the block mask from first-order Taylor scores (Sec. 3.1)
 * ``pack_bsr(W, mask, b)``  -- mask -> BSR pack + work list, on the GPU
 * ``pack_bsr_many_into(ws, Ws, masks)`` -- the same for a list of weights in two launches
-* ``bsr_linear(w, X, bias, gelu=...)`` -- Y = act(X (W (.) M)^T + bias)
+* ``bsr_linear(w, X, bias, gelu=..., residual=...)`` -- Y = act(X (W (.) M)^T + bias), optionally
+  plus a bf16 residual in the same pass (the x + sublayer(x) of a pre-norm block)
 * ``delta_curve(W, G, b, steps, kappa)`` / ``lambda_search(...)`` -- the layer-wise pruning-ratio
   allocation of Sec. 3.4-3.5 (empirical-Fisher distortion curves, Lagrangian slope matching)
 * ``add_layernorm`` / ``attention`` -- the rest of a pre-norm ViT block; ``encoder.SparseEncoder``
