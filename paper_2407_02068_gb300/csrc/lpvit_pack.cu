@@ -146,6 +146,92 @@ __device__ void group_panels(const unsigned *__restrict__ bits, int W, const int
   }
 }
 
+// group_panels for up to 32 * FAST_NPL panels and FAST_W bitmap words, with the same rule and
+// result: each lane keeps its candidates' bitmaps and kept counts in registers and every lane the
+// group's union, so a step is register arithmetic, the warp argmin and FAST_W shuffles.
+constexpr int FAST_NPL = 4, FAST_W = 4;
+__device__ void group_panels_fast(const unsigned *__restrict__ bits, int W, const int *__restrict__ kcnt, int np,
+                                  int gb, int ng, int32_t *__restrict__ gpan) {
+  const int lane = threadIdx.x & 31;
+  unsigned cb[FAST_NPL][FAST_W];
+  int kc[FAST_NPL];
+  unsigned alive = 0;  // bit i: candidate lane + 32 i is unassigned
+#pragma unroll
+  for (int i = 0; i < FAST_NPL; ++i) {
+    const int p = lane + 32 * i;
+    kc[i] = p < np ? kcnt[p] : 0;
+    if (p < np) alive |= 1u << i;
+#pragma unroll
+    for (int w = 0; w < FAST_W; ++w) cb[i][w] = (p < np && w < W) ? bits[p * W + w] : 0u;
+  }
+  int id_e = 0;  // entries of consecutive groups
+  for (int g = lane; g < ng; g += 32)
+    for (int w = 0; w < W; ++w) {
+      unsigned u = 0;
+      for (int p = 0; p < gb; ++p)
+        if (g * gb + p < np) u |= bits[(g * gb + p) * W + w];
+      id_e += __popc(u);
+    }
+  id_e = warp_sum(id_e);
+  int gr_e = 0;
+  unsigned U[FAST_W];
+  for (int g = 0; g < ng; ++g) {
+#pragma unroll
+    for (int w = 0; w < FAST_W; ++w) U[w] = 0u;
+    for (int sl = 0; sl < gb; ++sl) {
+      int best = 0x7fffffff, bi = 0x7fffffff;
+#pragma unroll
+      for (int i = 0; i < FAST_NPL; ++i) {
+        if ((alive >> i) & 1u) {
+          int sc = 0;
+          if (sl == 0) {
+            sc = -kc[i];
+          } else {
+#pragma unroll
+            for (int w = 0; w < FAST_W; ++w) sc += __popc(cb[i][w] & ~U[w]);
+          }
+          if (sc < best) {  // candidates of a lane come in ascending index order
+            best = sc;
+            bi = lane + 32 * i;
+          }
+        }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const int ob = __shfl_xor_sync(0xffffffffu, best, o), oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        if (ob < best || (ob == best && oi < bi)) {
+          best = ob;
+          bi = oi;
+        }
+      }
+      const int pick = bi == 0x7fffffff ? -1 : bi;
+      if (lane == 0) gpan[g * MAX_GROUP_PANELS + sl] = pick;
+      if (pick >= 0) {
+        const int owner = pick & 31, ip = pick >> 5;
+        if (lane == owner) alive &= ~(1u << ip);
+#pragma unroll
+        for (int w = 0; w < FAST_W; ++w) {
+          unsigned mine = 0;
+#pragma unroll
+          for (int i = 0; i < FAST_NPL; ++i)
+            if (i == ip) mine = cb[i][w];
+          U[w] |= __shfl_sync(0xffffffffu, mine, owner);
+        }
+      }
+    }
+    if (lane >= gb && lane < MAX_GROUP_PANELS) gpan[g * MAX_GROUP_PANELS + lane] = -1;
+#pragma unroll
+    for (int w = 0; w < FAST_W; ++w) gr_e += __popc(U[w]);  // the same in every lane
+  }
+  __syncwarp();
+  if (gr_e >= id_e) {
+    for (int i = lane; i < ng * MAX_GROUP_PANELS; i += 32) {
+      const int g = i / MAX_GROUP_PANELS, sl = i - g * MAX_GROUP_PANELS, r = g * gb + sl;
+      gpan[i] = (sl < gb && r < np) ? r : -1;
+    }
+  }
+}
+
 // The plan of one weight, computed by one CTA of PLAN_THREADS threads (plan_smem: plan_smem_bytes).
 __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int n, int k, int bn, int bk,
                                           int32_t *__restrict__ row_ptr, int32_t *__restrict__ col_idx, int cap,
@@ -208,7 +294,10 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
   }
   // 3b. group table: overlapping panels (one warp), or consecutive panels
   if (grouping) {
-    if (warp == 0) group_panels(bits, W, kcnt, np, gb, ng, U, asg, gpan);
+    if (warp == 0) {
+      if (np <= 32 * FAST_NPL && W <= FAST_W) group_panels_fast(bits, W, kcnt, np, gb, ng, gpan);
+      else group_panels(bits, W, kcnt, np, gb, ng, U, asg, gpan);
+    }
   } else {
     for (int i = tid; i < ng * MAX_GROUP_PANELS; i += PLAN_THREADS) {
       const int g = i / MAX_GROUP_PANELS, sl = i - g * MAX_GROUP_PANELS, r = g * gb + sl;
