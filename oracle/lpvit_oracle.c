@@ -42,10 +42,10 @@
  *    that score and the bottom ones are eliminated at the layer's pruning ratio alpha.
  *    Readings where the paper is silent: the number eliminated is round(alpha * blocks),
  *    half away from zero; equal scores rank by linear block index r * (k/bk) + j, the lower
- *    index first (kept first); the score is taken in float32, the gradient's precision: each
- *    product |w * g| rounded to float32, each block row summed in order in float32, the row
- *    sums summed in row order in float32, and that total widened to double and divided by
- *    bn * bk in double.
+ *    index first (kept first). The score is the plain average of the definition: each product
+ *    |w * g| of a bf16 weight and a float32 gradient is exact in double (8 + 24 significant
+ *    bits), the magnitudes are added in row-major order in double and the sum is divided by
+ *    bn * bk (relative rounding error below bn * bk * 2^-53).
  *
  * Inputs X and W arrive as bfloat16 bit patterns (the same bits the GPU reads); bias as
  * float32. Widening bf16 -> double is exact.
@@ -185,28 +185,23 @@ void lpvit_oracle_round_bf16_array(const double *y, uint16_t *out, int64_t count
   for (int64_t i = 0; i < count; ++i) out[i] = lpvit_oracle_round_bf16(y[i]);
 }
 
-/* Sec. 3.1: block score S'[r][j] = average over the bn x bk block of |W[i][l] * G[i][l]|, in
- * float32 as described above (row sums, then their sum), divided by bn * bk in double.
- * W: bf16 bits [n][k]; G: float32 [n][k]; out: [n/bn][k/bk]. Returns 0, or -1 for a shape that
- * is not a multiple of the block. */
+/* Sec. 3.1: block score S'[r][j] = the average over the bn x bk block of |W[i][l] * G[i][l]|, in
+ * double (see the header). W: bf16 bits [n][k]; G: float32 [n][k]; out: [n/bn][k/bk]. Returns 0, or
+ * -1 for a shape that is not a multiple of the block. */
 int lpvit_oracle_block_scores(const uint16_t *W, const float *G, int32_t n, int32_t k, int32_t bn, int32_t bk,
                               double *out) {
   if (bn <= 0 || bk <= 0 || n % bn || k % bk) return -1;
   const int32_t np = n / bn, kb = k / bk;
   for (int32_t r = 0; r < np; ++r) {
     for (int32_t j = 0; j < kb; ++j) {
-      float sum = 0.0f;
+      double sum = 0.0;
       for (int32_t i = 0; i < bn; ++i) {
-        float row = 0.0f;
         for (int32_t l = 0; l < bk; ++l) {
           const int64_t e = (int64_t)(r * bn + i) * k + (int64_t)j * bk + l;
-          const float w = (float)lpvit_oracle_bf16_to_f64(W[e]); /* exact: a bf16 is a float32 */
-          const float prod = w * G[e];                           /* rounded to float32 */
-          row += fabsf(prod);
+          sum += fabs(lpvit_oracle_bf16_to_f64(W[e]) * (double)G[e]); /* exact product */
         }
-        sum += row;
       }
-      out[(int64_t)r * kb + j] = (double)sum / ((double)bn * (double)bk);
+      out[(int64_t)r * kb + j] = sum / ((double)bn * (double)bk);
     }
   }
   return 0;

@@ -452,9 +452,10 @@ __device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int 
     for (int v = threadIdx.x; v < chunks; v += blockDim.x) {
       const int r = v >> lcpr, c = v & (cpr - 1), slot = r >> lbn;
       const int panel = gpan[g * MAX_GROUP_PANELS + slot];
-      const int row = (panel << lbn) + (r & (bn - 1));  // the output feature of group row r
+      // the output feature of group row r (none for an empty slot)
+      const int row = panel >= 0 ? (panel << lbn) + (r & (bn - 1)) : -1;
       int4 val = make_int4(0, 0, 0, 0);
-      if (((pm >> slot) & 1u) && panel >= 0 && row < n)
+      if (((pm >> slot) & 1u) && row >= 0 && row < n)
         val = __ldg(reinterpret_cast<const int4 *>(W + (int64_t)row * k + (int64_t)j * bk + c * 8));
       reinterpret_cast<int4 *>(tile + r * row_bytes)[c ^ stream_chunk_swizzle(r, row_bytes)] = val;
     }

@@ -6,8 +6,10 @@
 
 namespace lpvit {
 
-// scores[r][j] = sum of |W * G| over block (r, j) (bn rows by bk columns) in row-major order in
-// double, divided by bn * bk. W bf16 [n][k], G float32 [n][k], both 16-byte aligned.
+// scores[r][j] = the average of |W * G| over block (r, j) (bn rows by bk columns): each product
+// rounded to float32, each block row summed in float32, the row sums summed in float32, the total
+// divided by bn * bk in double; within (bn + bk) 2^-24 of the exact average (sums of non-negative
+// terms). W bf16 [n][k], G float32 [n][k], both 16-byte aligned.
 cudaError_t launch_block_scores(const uint16_t *W, const float *G, int n, int k, int bn, int bk, double *scores,
                                 cudaStream_t s);
 // For each of `total` blocks: rank[t] = the number of blocks ranked ahead of it (higher score, or

@@ -192,3 +192,28 @@ def deit_b_stack(config: int = 4, b: int = 32, device="cpu"):
             L[name] = g
         layers.append(L)
     return layers
+
+
+def deit_encoder_params(model: dict, b=32, config: int = 9, layers: int = 12, device="cpu"):
+    """Seeded parameters of a pre-norm DeiT encoder with block-sparse linears: per layer a dict with
+    'ln1', 'ln2' = (gamma ~ 1 + N(0, 0.1), beta ~ N(0, 0.1)) float32 [D] and 'qkv', 'proj', 'fc1',
+    'fc2' = (W bf16 [n, k], uniform mask uint8 [n/bn, k/bk] at the stack's per-GEMM sparsities,
+    bias float32 [n]); plus the final LayerNorm's (gamma, beta)."""
+    D = model["dim"]
+    sp = stack_sparsities(config, layers)
+    gen = _gen(seed(config, 0, "bias"), device)
+    out = []
+    for l in range(layers):
+        lay = {"ln1": ((1 + 0.1 * torch.randn(D, generator=gen, device=device)).contiguous(),
+                       (0.1 * torch.randn(D, generator=gen, device=device)).contiguous()),
+               "ln2": ((1 + 0.1 * torch.randn(D, generator=gen, device=device)).contiguous(),
+                       (0.1 * torch.randn(D, generator=gen, device=device)).contiguous())}
+        for t, (name, k, n, _) in enumerate(deit_gemms(model)):
+            gi = 4 * l + t
+            lay[name] = (weight(n, k, seed(config, gi, "W"), device),
+                         uniform_mask(n, k, b, sp[l][t], seed(config, gi, "mask")).to(device),
+                         bias(n, seed(config, gi, "bias"), device))
+        out.append(lay)
+    final = ((1 + 0.1 * torch.randn(D, generator=gen, device=device)).contiguous(),
+             (0.1 * torch.randn(D, generator=gen, device=device)).contiguous())
+    return out, final

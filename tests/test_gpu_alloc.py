@@ -3,7 +3,12 @@
 curves within 1e-9 of their largest magnitude (the GPU takes exact products, float-pair lane sums of
 at most 128 terms, double beyond, and updates incrementally by Eq. update; the oracle evaluates
 every alpha directly in double), and the whole allocation -- curves, lambda search,
-Taylor masks at the allocated ratios, pack and linear -- on a small stack."""
+Taylor masks at the allocated ratios, pack and linear -- on a small stack.
+
+The GPU ranks blocks by float32 Taylor scores, the oracle by their exact averages (Sec. 3.1). A
+ratio step whose cut-off falls within the float32 bound of two blocks' scores may prune either of
+them (taylor_bounds); such steps are named and left out of the curve comparison, every other step
+is compared."""
 import numpy as np
 import pytest
 import torch
@@ -11,6 +16,7 @@ import torch
 import oracle
 from oracle import alloc
 from paper_2407_02068_gb300 import inputs
+from taylor_bounds import ambiguous_steps, assert_mask_matches_away_from_cutoff
 
 pytestmark = pytest.mark.gpu
 
@@ -51,7 +57,12 @@ def test_delta_curve_matches_the_oracle(lp, n, k, b, N, steps, kappa):
     assert got[0] == 0.0
     scale = np.max(np.abs(want))
     assert scale > 0
-    assert np.max(np.abs(got - want)) <= CURVE_TOL * scale, np.max(np.abs(got - want)) / scale
+    exact = oracle.block_scores(inputs.bf16_bits(W), alloc.mean_gradient(G.cpu().numpy()), b)
+    amb = ambiguous_steps(exact, steps, bn, bk)
+    assert len(amb) <= 1, amb
+    ok = np.ones(steps + 1, dtype=bool)
+    ok[amb] = False
+    assert np.max(np.abs(got - want)[ok]) <= CURVE_TOL * scale, np.max(np.abs(got - want)[ok]) / scale
 
 
 def test_zero_gradients_give_the_kappa_closed_form(lp):
@@ -74,27 +85,39 @@ def test_allocation_feeds_the_masks_and_the_linear(lp):
     layers = [("qkv", 384, 1152), ("proj", 384, 384), ("fc1", 384, 1536), ("fc2", 1536, 384)]
     b, N, steps, kappa, beta, R, m = 32, 6, 8, 1e-3, 2e-9, 0.5, 197
     curves, refs, Ws, Gs = [], [], [], []
+    ambiguous_any = False
     for i, (name, k, n) in enumerate(layers):
         W, G = _wg(n, k, N, 7100 + i)
         Ws.append(W)
         Gs.append(G)
         curves.append(lp.delta_curve(W, G, b, steps, kappa).cpu().numpy())
         refs.append(alloc.delta_curve(inputs.bf16_bits(W), G.cpu().numpy(), b, steps, kappa))
-        assert np.max(np.abs(curves[-1] - refs[-1])) <= CURVE_TOL * np.max(np.abs(refs[-1]))
+        exact = oracle.block_scores(inputs.bf16_bits(W), alloc.mean_gradient(G.cpu().numpy()), b)
+        amb = ambiguous_steps(exact, steps, b, b)
+        assert len(amb) <= 1, (name, amb)
+        ok = np.ones(steps + 1, dtype=bool)
+        ok[amb] = False
+        ambiguous_any = ambiguous_any or bool(amb)
+        assert np.max(np.abs(curves[-1] - refs[-1])[ok]) <= CURVE_TOL * np.max(np.abs(refs[-1]))
     F = [m * n * k for _, k, n in layers]
     c = [m * n * k / (b * b) for _, k, n in layers]
     ks, lam, ratio = lp.lambda_search(curves, steps, F, c, beta, R)
-    want = alloc.lambda_search([alloc.distortion(d) for d in refs], steps, F, c, beta, R)
-    assert ks == want[1] and ratio <= R
+    # the search itself, on the GPU's curves, is the oracle's search
+    assert ks == alloc.lambda_search([alloc.distortion(d) for d in curves], steps, F, c, beta, R)[1]
+    if not ambiguous_any:
+        want = alloc.lambda_search([alloc.distortion(d) for d in refs], steps, F, c, beta, R)
+        assert ks == want[1]
+    assert ratio <= R
     for i, (name, k, n) in enumerate(layers):
         g = lp.mean_gradient(Gs[i])
         mask, _ = lp.taylor_block_mask(Ws[i], g, b, ks[i] / steps)
         g_ref = alloc.mean_gradient(Gs[i].cpu().numpy())
-        m_ref = oracle.taylor_mask(oracle.block_scores(inputs.bf16_bits(Ws[i]), g_ref, b), ks[i] / steps)
-        assert np.array_equal(mask.cpu().numpy(), m_ref)
+        exact = oracle.block_scores(inputs.bf16_bits(Ws[i]), g_ref, b)
+        got_m = mask.cpu().numpy()
+        assert_mask_matches_away_from_cutoff(got_m, exact, ks[i] / steps, b, b)
         X = inputs.activations(m, k, 7200 + i, "cuda")
         w = lp.pack_bsr(Ws[i], mask, b)
         Y = lp.bsr_linear(w, X, None, out_dtype=torch.float32)
-        ref = oracle.linear(inputs.bf16_bits(X), inputs.bf16_bits(Ws[i]), m_ref, b, None)
+        ref = oracle.linear(inputs.bf16_bits(X), inputs.bf16_bits(Ws[i]), got_m, b, None)
         err = np.max(np.abs(Y.cpu().double().numpy() - ref)) / max(np.sqrt(np.mean(ref ** 2)), 1e-30)
         assert err <= 1e-4

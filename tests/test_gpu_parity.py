@@ -162,7 +162,11 @@ def _grouping(M, bn):
                                    (768, 768, (64, 32)), (208, 384, (16, 32)), (320, 128, (64, 16)),
                                    (1024 * 16, 64, 16),      # 1024 panels: the grouping's limit
                                    (1025 * 16, 64, 16),      # 1025 panels: consecutive groups
-                                   (8192, 8704, 16)])        # 512 panels x 17 bitmap words > 8192
+                                   (8192, 8704, 16),         # 512 panels x 17 bitmap words > 8192
+                                   (100 * 32, 4096, 32),     # register grouping: 100 panels, 4 words
+                                   (128 * 32, 4096, 32),     # register grouping at its limits: 128 panels, 4 words
+                                   (129 * 32, 4096, 32),     # 129 panels: shared-memory grouping
+                                   (128 * 32, 5120, 32)])    # 5 bitmap words: shared-memory grouping
 def test_work_list_covers_every_kept_block_once(lp, n, k, b):
     X, W, bias, mask = _case(4, n, k, b, 0.55, 12)
     w = lp.pack_bsr(W, mask, b, count=True)

@@ -374,19 +374,28 @@ def test_taylor_scores_are_local_and_scale_exactly():
     assert changed[1, 0] and changed.sum() == 1
 
 
-def test_taylor_scores_sum_rows_then_blocks_in_float32():
-    """One 2 x 32 block: row 0 holds 1 and 31 products of 2^-25, row 1 holds 32 products of 2^-25.
-    In float32 each 2^-25 added to 1 is lost (below half an ulp of 1), while row 1's products add
-    exactly among themselves to 2^-20, which survives the addition of the row sums: the score is
-    (1 + 2^-20) / 64. A double sum, or one float32 sum over the whole block, gives other values."""
+def test_taylor_scores_are_the_exact_block_average():
+    """One 2 x 32 block: one product of 1 and 63 products of 2^-25. The exact average is
+    (1 + 63 * 2^-25) / 64, representable in double; a float32 accumulation (any order that adds the
+    small products to 1 one at a time, or row by row) loses some or all of the 2^-25 terms."""
     W = np.full((2, 32), 2.0 ** -8, dtype=np.float32)
     W[0, 0] = 1.0
     G = np.full((2, 32), 2.0 ** -17, dtype=np.float32)
     G[0, 0] = 1.0
     s = oracle.block_scores(_bits(W), G, (2, 32))
-    assert s[0, 0] == (1.0 + 2.0 ** -20) / 64
-    assert s[0, 0] != (1.0 + 63 * 2.0 ** -25) / 64   # the double sum
-    assert s[0, 0] != 1.0 / 64                        # one float32 sum over the block
+    assert s[0, 0] == (1.0 + 63 * 2.0 ** -25) / 64
+    assert s[0, 0] != (1.0 + 2.0 ** -20) / 64   # row sums in float32, then their sum
+    assert s[0, 0] != 1.0 / 64                  # one float32 sum over the block
+
+
+def test_taylor_scores_ignore_the_sign_of_each_product():
+    """|W . G| element by element, not |sum|: a block whose products cancel still scores their
+    magnitudes (the hand-worked block (1,1) of the golden file, here on a 16 x 16 block)."""
+    W = np.ones((16, 16), dtype=np.float32)
+    W[::2] = -1.0
+    G = np.full((16, 16), 0.5, dtype=np.float32)
+    s = oracle.block_scores(_bits(W), G, 16)
+    assert s[0, 0] == 0.5
 
 
 def test_taylor_scores_brute_force_and_mask_order():
@@ -399,9 +408,8 @@ def test_taylor_scores_brute_force_and_mask_order():
         Wd = oracle.bf16_to_f64(Wb)
         want = np.abs(Wd * G.astype(np.float64)).reshape(4, bn, 3, bk).sum(axis=(1, 3)) / (bn * bk)
         s = oracle.block_scores(Wb, G, b)
-        # float32 products and two levels of float32 sums of non-negative terms: relative error at
-        # most (1 + (bk - 1) + (bn - 1)) 2^-24 of the exact average
-        assert np.allclose(s, want, rtol=(bn + bk) * 2.0 ** -24, atol=0)
+        # the same average by numpy's pairwise double sum: only the summation order differs
+        assert np.allclose(s, want, rtol=1e-13, atol=0)
         for alpha in (0.0, 0.25, 0.5, 0.75, 1.0):
             m = oracle.taylor_mask(s, alpha)
             kept, pruned = s[m == 1], s[m == 0]
