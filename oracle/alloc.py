@@ -53,6 +53,13 @@ def pruned_delta_w(W_bits: np.ndarray, g32: np.ndarray, b, alpha: float) -> np.n
     return np.where(keep, 0.0, -W)
 
 
+def _delta(dW: np.ndarray, g: np.ndarray, Gd: np.ndarray, kappa: float) -> float:
+    """g . dW + 1/2 (kappa |dW|^2 + (1/N) sum_n (g_n . dW)^2) for flattened float64 operands."""
+    first = float(g @ dW)
+    quad = kappa * float(dW @ dW) + float(np.sum((Gd @ dW) ** 2)) / Gd.shape[0]
+    return first + 0.5 * quad
+
+
 def delta_curve(W_bits: np.ndarray, G: np.ndarray, b, steps: int, kappa: float) -> np.ndarray:
     """delta(alpha_k) for alpha_k = k / steps, k = 0..steps (float64 [steps + 1]).
 
@@ -64,11 +71,20 @@ def delta_curve(W_bits: np.ndarray, G: np.ndarray, b, steps: int, kappa: float) 
     Gd = G.reshape(N, -1).astype(np.float64)
     out = np.empty(steps + 1, dtype=np.float64)
     for kk in range(steps + 1):
-        dW = pruned_delta_w(W_bits, g32, b, kk / steps).ravel()
-        first = float(g @ dW)
-        quad = kappa * float(dW @ dW) + float(np.sum((Gd @ dW) ** 2)) / N
-        out[kk] = first + 0.5 * quad
+        out[kk] = _delta(pruned_delta_w(W_bits, g32, b, kk / steps).ravel(), g, Gd, kappa)
     return out
+
+
+def delta_at_mask(W_bits: np.ndarray, G: np.ndarray, b, mask: np.ndarray, kappa: float) -> float:
+    """delta for a given block mask (1 = kept): dW = -W on the removed blocks, as in delta_curve."""
+    bn, bk = block_shape(b)
+    G = np.asarray(G, dtype=np.float32)
+    N = G.shape[0]
+    g = mean_gradient(G).astype(np.float64).ravel()
+    Gd = G.reshape(N, -1).astype(np.float64)
+    keep = np.kron(np.asarray(mask, dtype=np.uint8), np.ones((bn, bk), dtype=np.uint8)).astype(bool)
+    dW = np.where(keep, 0.0, -bf16_to_f64(W_bits)).ravel()
+    return _delta(dW, g, Gd, kappa)
 
 
 def distortion(delta: np.ndarray) -> np.ndarray:

@@ -80,30 +80,37 @@ bool shape_ok(int n, int k, int bn, int bk) {
 
 int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
-// Entries per slice. With enough (token tile, group) units to fill every SM twice, a unit covers
-// the whole group; otherwise the group's block columns are cut into slices so that about two
-// units per SM exist, and the slices are summed by the fix-up.
-int choose_slice(int64_t n_tt, int n_groups, int kb, int sms) {
+// Entries per slice. With at least half as many (token tile, group) units as CTA pairs, a unit
+// covers the whole group; otherwise the group's chunks are cut into slices so that about one unit
+// per pair exists, and the reduction kernel adds the slices' partial sums.
+int choose_slice(int64_t n_tt, int n_groups, int kc, int pairs) {
   const int64_t units = n_tt * n_groups;
-  if (units >= 2LL * sms) return kb;
-  const int64_t s = ceil_div((int64_t)kb * units, 2LL * sms);
-  return (int)(s < 1 ? 1 : (s > kb ? kb : s));
+  if (2 * units >= pairs) return kc;
+  const int64_t nsl = ceil_div(pairs, units);
+  const int64_t s = ceil_div(kc, nsl);
+  return (int)(s < 1 ? 1 : (s > kc ? kc : s));
 }
 
 struct WsLayout {
-  size_t tickets_off, partials_off, total;
+  size_t partials_off, total;
+  int S, part_rows;
+  bool split;
 };
 
-WsLayout ws_layout(int64_t m, int n, int k, int bk, int sms) {
+// Workspace: the 256-byte control block, then (split launches only) the fp32 partial sums,
+// [token tile][slice][part_rows][GROUP_FEATURES].
+WsLayout ws_layout(int64_t m, int n, int k, int sms) {
   WsLayout L;
   const int64_t n_tt = ceil_div(m, TOKENS_PER_TILE);
   const int ng = (int)ceil_div(n, GROUP_FEATURES);
-  const int kb = k / bk;
-  const int S = choose_slice(n_tt, ng, kb, sms);
-  L.tickets_off = sizeof(Control);
-  size_t off = L.tickets_off + (size_t)ceil_div(n_tt * ng * 4, 256) * 256;
-  L.partials_off = off;
-  if (S < kb) off += (size_t)n_tt * ng * ceil_div(kb, S) * TOKENS_PER_TILE * GROUP_FEATURES * sizeof(float);
+  const int kc = sched_chunks(k);
+  L.S = choose_slice(n_tt, ng, kc, sms / 2);
+  L.split = L.S < kc;
+  L.part_rows = (int)(n_tt == 1 ? m : TOKENS_PER_TILE);
+  L.partials_off = sizeof(Control);
+  size_t off = L.partials_off;
+  if (L.split)
+    off += (size_t)n_tt * ng * ceil_div(kc, L.S) * L.part_rows * GROUP_FEATURES * sizeof(float);
   L.total = off;
   return L;
 }
@@ -148,29 +155,41 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   int sms = 0;
   lpvit_status st = LPVIT_OK;
   if (!device_info(&sms, &st)) return st;
-  const WsLayout W = ws_layout(m, n, k, bk, sms);
+  const WsLayout W = ws_layout(m, n, k, sms);
   if (ws_bytes < W.total) return LPVIT_ERR_WORKSPACE;
   EncodeTiledFn enc = encode_fn();
   if (!enc) return LPVIT_ERR_CUDA;
 
-  const CUtensorMapSwizzle swz =
-      bk == 16 ? CU_TENSOR_MAP_SWIZZLE_32B : (bk == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B);
-  CUtensorMap tmX;
+  const int ng = (int)ceil_div(n, GROUP_FEATURES);
+  const int kc = sched_chunks(k);
+  const int64_t stream_tiles = sched_stream_tiles(ng, kc);
+  cuuint32_t es[2] = {1, 1};
+  // X: [m rows][k columns], boxes of 64 columns x 128 tokens (one CTA's half of a token tile);
+  // rows beyond m and columns beyond k read as zero
+  CUtensorMap tmX, tmW;
   {
     cuuint64_t dims[2] = {(cuuint64_t)k, (cuuint64_t)m};
     cuuint64_t strides[1] = {(cuuint64_t)ldx * 2};
-    cuuint32_t box[2] = {(cuuint32_t)bk, (cuuint32_t)TOKENS_PER_TILE};
-    cuuint32_t es[2] = {1, 1};
+    cuuint32_t box[2] = {(cuuint32_t)CHUNK_COLS, (cuuint32_t)CTA_TOKENS};
     if (enc(&tmX, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(X), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return LPVIT_ERR_INVALID_ARG;
+  }
+  // the weight stream: tiles of 256 rows x 64 columns, boxes of 128 rows (one CTA's half)
+  {
+    void *wstream = static_cast<uint8_t *>(bsr->sched) + sched_stream_offset_bytes(ng, kc);
+    cuuint64_t dims[2] = {(cuuint64_t)CHUNK_COLS, (cuuint64_t)(stream_tiles * GROUP_FEATURES)};
+    cuuint64_t strides[1] = {(cuuint64_t)CHUNK_COLS * 2};
+    cuuint32_t box[2] = {(cuuint32_t)CHUNK_COLS, (cuuint32_t)HALF_FEATURES};
+    if (enc(&tmW, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, wstream, dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return LPVIT_ERR_INVALID_ARG;
   }
   LinearParams P;
-  const int ng = (int)ceil_div(n, GROUP_FEATURES);
   P.sched = static_cast<const int32_t *>(bsr->sched);
-  P.wstream = static_cast<const uint8_t *>(bsr->sched) + sched_stream_offset_bytes(ng, k / bk);
-  P.stream_tiles = sched_stream_tiles(ng, k / bk);
+  P.stream_tiles = stream_tiles;
   P.bias = bias;
   P.Y = Y;
   P.ldy = ldy;
@@ -180,20 +199,42 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.bn = bn;
   P.n_tt = (int)ceil_div(m, TOKENS_PER_TILE);
   P.n_groups = ng;
-  P.S = choose_slice(P.n_tt, P.n_groups, k / bk, sms);
+  P.S = W.S;
   P.y_f32 = y_dtype == LPVIT_F32;
   P.gelu = gelu;
-  P.y_vec16 = (aligned(Y, 16) && ldy % 8 == 0) ? 1 : 0;
+  P.y_vec16 = (aligned(Y, 16) && ((size_t)ldy * ysz) % 16 == 0) ? 1 : 0;
+  P.bias_vec16 = (bias && aligned(bias, 16)) ? 1 : 0;
   P.R = static_cast<const uint16_t *>(R);
   P.ldr = R ? ldr : 0;
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   P.ctl = reinterpret_cast<Control *>(ws);
-  P.tickets = reinterpret_cast<int32_t *>(ws + W.tickets_off);
   P.partials = reinterpret_cast<float *>(ws + W.partials_off);
+  P.part_rows = W.part_rows;
   P.timeout_ns = TIMEOUT_NS;
-  const int64_t units_max = (int64_t)P.n_tt * P.n_groups * ceil_div(k / bk, P.S);
-  const int grid = (int)(units_max < sms ? units_max : sms);
-  return cuda_status(launch_linear(bk, tmX, P, grid, static_cast<cudaStream_t>(stream)));
+  const int pairs = sms / 2;
+  const int64_t units_max = (int64_t)P.n_tt * P.n_groups * ceil_div(kc, P.S);
+  const int grid = 2 * (int)(units_max < pairs ? units_max : pairs);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = launch_linear(tmX, tmW, P, grid, s);
+  if (e != cudaSuccess || !W.split) return cuda_status(e);
+  ReduceParams RP;
+  RP.sched = P.sched;
+  RP.partials = P.partials;
+  RP.bias = bias;
+  RP.Y = Y;
+  RP.ldy = ldy;
+  RP.m = m;
+  RP.n = n;
+  RP.bn = bn;
+  RP.n_tt = P.n_tt;
+  RP.n_groups = ng;
+  RP.S = P.S;
+  RP.part_rows = P.part_rows;
+  RP.y_f32 = P.y_f32;
+  RP.gelu = gelu;
+  RP.R = P.R;
+  RP.ldr = P.ldr;
+  return cuda_status(launch_split_reduce(RP, (int64_t)P.n_tt * ng * P.part_rows * (GROUP_FEATURES / 8), s));
 }
 
 // The checks lpvit_pack_bsr applies to one weight.
@@ -221,7 +262,8 @@ extern "C" {
 size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t bn, int32_t bk) {
   if (!shape_ok(n, k, bn, bk)) return 0;
   const int ng = (int)ceil_div(n, GROUP_FEATURES);
-  return (size_t)sched_stream_offset_bytes(ng, k / bk) + (size_t)sched_stream_tiles(ng, k / bk) * stream_tile_bytes(bk);
+  const int kc = sched_chunks(k);
+  return (size_t)sched_stream_offset_bytes(ng, kc) + (size_t)sched_stream_tiles(ng, kc) * stream_tile_bytes();
 }
 
 
@@ -282,7 +324,7 @@ size_t lpvit_workspace_bytes(const lpvit_bsr *bsr, int64_t m) {
   int sms = 0;
   lpvit_status st = LPVIT_OK;
   if (!device_info(&sms, &st)) sms = 152;  // sizing only; the call itself reports the device error
-  return ws_layout(m > 0 ? m : 1, bsr->n, bsr->k, bsr->bk, sms).total;
+  return ws_layout(m > 0 ? m : 1, bsr->n, bsr->k, sms).total;
 }
 
 lpvit_status lpvit_bsr_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias,

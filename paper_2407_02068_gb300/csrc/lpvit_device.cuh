@@ -9,52 +9,47 @@
 namespace lpvit {
 
 // Layout of the work list ("sched") shared by the pack and the GEMM, for blocks of bn output rows
-// by bk input columns.
+// by bk input columns. The GEMM covers the weight in tiles of GROUP_FEATURES output features by
+// CHUNK_COLS input columns (one pipeline stage of MMAs), and skips the tiles whose blocks are all
+// removed.
 // header (16 int32): [0] nnzb, [1] n_groups, [2] total entries, [3] overflow flag, [4] n, [5] k,
-// [6] bn, [7] bk
+// [6] bn, [7] bk, [8] layout version (SCHED_VERSION)
 // then gent_ptr[n_groups + 1] (int32, entries of group g are [gent_ptr[g], gent_ptr[g+1]))
 // then gpan[n_groups][MAX_GROUP_PANELS] (int32): the row panel in slot p of group g, or -1. A group
 // is GROUP_FEATURES / bn row panels, not necessarily consecutive: the plan picks panels whose kept
-// block columns overlap, so that a group has fewer entries; group row r is panel gpan[g][r / bn],
-// row r % bn, i.e. output feature gpan[g][r / bn] * bn + r % bn.
-// then entries, ENTRY_INTS int32 each: [0] = j | (slot mask << 16), [1 + p] = block index of
-// the panel in slot p at block column j, or -1 (p < GROUP_FEATURES / bn <= 8),
-// [ENTRY_TILE_WORD] = index of the entry's tile in the weight stream (the entry's own index);
-// then, at sched_stream_offset_bytes (1024-byte aligned), the weight stream: for every entry in
-// order, the group's tile at column j: row r < 128 holds W[feature of group row r][j*bk + c] for
-// c < bk, zero for the slots that keep no block there, stored as 128 rows of 2*bk bytes whose 16-byte
-// chunks are permuted by stream_chunk_swizzle: the arrangement the MMA's shared-memory descriptor
-// reads, so that one bulk copy moves an entry's weights.
+// chunks overlap, so that a group has fewer entries; group row r is panel gpan[g][r / bn], row
+// r % bn, i.e. output feature gpan[g][r / bn] * bn + r % bn.
+// then entries, one int32 each: the chunk index c (input columns [c * CHUNK_COLS, (c + 1) *
+// CHUNK_COLS)) of a tile of the group holding at least one kept block; entry e's tile in the
+// weight stream is tile e;
+// then, at sched_stream_offset_bytes (1024-byte aligned), the weight stream: per entry a tile of
+// GROUP_FEATURES rows of CHUNK_COLS bf16, row-major (128-byte rows), row r = group row r:
+// W[feature][c * CHUNK_COLS + col] where its block is kept, zero where it is removed, where the
+// slot has no panel and beyond column k. The GEMM's tensor copies load each 128-row half with the
+// 128-byte swizzle its MMA descriptors read.
 constexpr int SCHED_HDR_INTS = 16;
-constexpr int ENTRY_INTS = 12;
-constexpr int ENTRY_TILE_WORD = 9;
-constexpr int GROUP_FEATURES = 128;   // output features covered by one work unit
+constexpr int SCHED_VERSION = 2;
+constexpr int GROUP_FEATURES = 256;   // output features of one work unit (the pair MMA's N)
+constexpr int HALF_FEATURES = GROUP_FEATURES / 2;  // weight rows one CTA of the pair stages
 constexpr int MAX_GROUP_PANELS = GROUP_FEATURES / 16;
-constexpr int TOKENS_PER_TILE = 256;  // tokens covered by one work unit (the .ws MMA N)
+constexpr int CHUNK_COLS = 64;        // input columns per stage: four 16-wide MMA k steps
+constexpr int TOKENS_PER_TILE = 256;  // tokens of one work unit (the pair MMA's M)
+constexpr int CTA_TOKENS = TOKENS_PER_TILE / 2;
 
+__host__ __device__ inline int sched_chunks(int k) { return (k + CHUNK_COLS - 1) / CHUNK_COLS; }
 __host__ __device__ inline int sched_gent_offset_ints() { return SCHED_HDR_INTS; }
 __host__ __device__ inline int64_t sched_gpan_offset_ints(int n_groups) { return (int64_t)SCHED_HDR_INTS + n_groups + 1; }
 __host__ __device__ inline int64_t sched_entries_offset_ints(int n_groups) {
   return (sched_gpan_offset_ints(n_groups) + (int64_t)n_groups * MAX_GROUP_PANELS + 3) / 4 * 4;  // 16-byte aligned
 }
-__host__ __device__ inline int64_t sched_stream_offset_bytes(int n_groups, int kb) {
-  const int64_t end = 4 * (sched_entries_offset_ints(n_groups) + (int64_t)n_groups * kb * ENTRY_INTS);
+__host__ __device__ inline int64_t sched_stream_offset_bytes(int n_groups, int kc) {
+  const int64_t end = 4 * (sched_entries_offset_ints(n_groups) + (int64_t)n_groups * kc);
   return (end + 1023) / 1024 * 1024;
 }
-// One MMA's M is the whole 128-feature group: one MMA per 16-wide k step covers every row panel of
-// the group (those without a block at the column contribute zero rows), and the X chunk it reads
-// from shared memory serves all 128 features. A stream tile is that group's rows at one column.
-__host__ __device__ constexpr int stream_tile_bytes(int bk) { return GROUP_FEATURES * bk * 2; }
-// Tiles the stream region holds: one per group and block column (the most entries there can be).
-__host__ __device__ inline int64_t sched_stream_tiles(int n_groups, int kb) { return (int64_t)n_groups * kb; }
-// Position of 16-byte chunk c in tile row r (rows of row_bytes = 32, 64 or 128 bytes): c XOR the
-// row's address bits 7.. above the chunk bits, i.e. the 32/64/128-byte TMA swizzle of a tile
-// placed at a 1024-byte aligned shared-memory address.
-__host__ __device__ constexpr int stream_chunk_swizzle(int r, int row_bytes) {
-  return ((r * row_bytes) >> 7) & (row_bytes / 16 - 1);
-}
-static_assert(GROUP_FEATURES / 16 <= MAX_GROUP_PANELS, "entry holds every row panel of a group");
-static_assert(1 + MAX_GROUP_PANELS <= ENTRY_TILE_WORD && ENTRY_TILE_WORD < ENTRY_INTS, "entry size");
+__host__ __device__ constexpr int stream_tile_bytes() { return GROUP_FEATURES * CHUNK_COLS * 2; }
+// Tiles the stream region holds: one per group and chunk (the most entries there can be).
+__host__ __device__ inline int64_t sched_stream_tiles(int n_groups, int kc) { return (int64_t)n_groups * kc; }
+static_assert(MAX_GROUP_PANELS <= 16, "a group's slot mask fits 16 bits");
 
 // Workspace control block (first 256 bytes of the caller's workspace).
 struct Control {
@@ -68,24 +63,40 @@ static_assert(sizeof(Control) == 256, "control block is 256 bytes");
 
 // Parameter block of the linear kernel (host fills it, the kernel reads it by value).
 struct LinearParams {
-  const int32_t *sched;    // work list (header, gent_ptr, entries)
-  const uint8_t *wstream;  // weight stream inside sched (16-byte aligned)
-  int64_t stream_tiles;    // tiles the stream region holds (bound on every entry's tile range)
+  const int32_t *sched;    // work list (header, gent_ptr, gpan, entries)
+  int64_t stream_tiles;    // tiles the stream region holds (bound on every entry's tile)
   const float *bias;       // [n] or nullptr
   void *Y;
   int64_t ldy;
   int64_t m;
   int n, k;
   int bn;                  // block height: a group holds GROUP_FEATURES / bn row panels
-  int n_tt, n_groups, S;   // token tiles, 128-feature groups, max entries per slice
+  int n_tt, n_groups, S;   // token tiles, groups, max entries per slice
   int y_f32, gelu;
-  int y_vec16;             // bf16 output rows may take 16-byte stores (Y 16-byte aligned, ldy % 8 == 0)
+  int y_vec16;             // output rows may take 16-byte stores (Y 16-byte aligned, ldy * size % 16 == 0)
+  int bias_vec16;          // bias is 16-byte aligned
   const uint16_t *R;       // bf16 residual [m][ldr] added after rounding (bf16 output only), or nullptr
   int64_t ldr;
   Control *ctl;
-  int32_t *tickets;        // [n_tt * n_groups] arrival tickets of split units
-  float *partials;         // [slots][128 features][256 tokens] fp32 partial sums of split units
+  float *partials;         // split units: [slice][part_rows][GROUP_FEATURES] fp32 partial sums
+  int part_rows;           // token rows of one partial tile: min(m, TOKENS_PER_TILE)
   uint64_t timeout_ns;     // limit of every device-side wait
+};
+
+// Parameter block of the split-slice reduction (after the linear kernel, same stream).
+struct ReduceParams {
+  const int32_t *sched;
+  const float *partials;
+  const float *bias;
+  void *Y;
+  int64_t ldy;
+  int64_t m;
+  int n, bn;
+  int n_tt, n_groups, S;
+  int part_rows;
+  int y_f32, gelu;
+  const uint16_t *R;
+  int64_t ldr;
 };
 
 enum ErrBits : unsigned int {
@@ -121,7 +132,10 @@ struct PackJobs {
   PackJob job[PACK_MAX_JOBS];
 };
 cudaError_t launch_pack_many(const PackJob *jobs, int count, int num_sms, cudaStream_t s);
-cudaError_t launch_linear(int bk, const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s);
+// grid = 2 * pairs (clusters of two CTAs); a split launch is followed by the reduction.
+cudaError_t launch_linear(const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
+                          cudaStream_t s);
+cudaError_t launch_split_reduce(const ReduceParams &R, int64_t threads, cudaStream_t s);
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
@@ -199,6 +213,65 @@ __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence:
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" :: "r"(bar) : "memory");
+}
+
+// ------------------------------------------------------------------ CTA pairs (cluster of 2)
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// The cluster address of this CTA's shared-memory location `a` in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t mapa_rank(uint32_t a, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(rank));
+  return r;
+}
+// Arrive on an mbarrier of either CTA of the cluster (release at cluster scope: earlier writes of
+// this thread, to either CTA's shared memory, are visible to the waiter).
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" :: "r"(cluster_addr) : "memory");
+}
+__device__ __forceinline__ void st_cluster_v4(uint32_t cluster_addr, int4 v) {
+  asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" :: "r"(cluster_addr), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w) : "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Tensor copy into this CTA's shared memory whose completion is counted on an mbarrier of either
+// CTA of the pair (cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap *map, int32_t x, int32_t y,
+                                                 uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2 "
+      "[%0], [%1, {%2, %3}], [%4];"
+      :: "r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar_cluster) : "memory");
+}
+// TMEM allocation for the pair: one warp of each CTA executes it, both get the same columns.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" :: "r"(dst_smem), "r"(ncols));
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" :: "r"(taddr), "r"(ncols));
+}
+// Arrive once on the mbarrier at shared-memory offset `bar` of every CTA in `mask` when this
+// thread's earlier pair MMAs complete.
+__device__ __forceinline__ void tc_commit_pair(uint32_t bar, uint16_t mask) {
+  asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;"
+               :: "r"(bar), "h"(mask) : "memory");
+}
+// D[256 x N] (+)= A[256 x 16] * B[N x 16]^T over the CTA pair: A rows 0-127 from this CTA's shared
+// memory, 128-255 from the peer's (same offset); B rows 0 .. N/2 - 1 from this CTA, the rest from
+// the peer; D rows 0-127 in this CTA's TMEM, 128-255 in the peer's. Issued by the leader alone.
+__device__ __forceinline__ void umma_f16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                              uint32_t accumulate) {
+  asm volatile("{.reg .pred p; setp.ne.b32 p, %4, 0;\n"
+               "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;}\n"
+               :: "r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
 }
 
 // Shared-memory matrix descriptor for a K-major operand tile whose rows are `row_bytes`

@@ -1,26 +1,31 @@
 // Block-sparse linear Y = act(X W~^T + bias) on sm_103a (Sec. 3.1 block mask, Sec. 3.3
-// block-sparse matmul: one block matmul per kept block and token tile, nothing for removed
-// blocks). The kernel is compiled per block width BK (input columns of a block: 16, 32 or 64);
-// the block height only decides which rows of a group tile the pack left zero.
+// block-sparse matmul: work for the kept blocks; tiles whose blocks are all removed are skipped).
 //
-// Work unit = 256 tokens x one 128-feature group of row panels (x one slice of the group's block
-// columns when the problem is too small to fill the GPU); the work list's group table names the
-// panels of each group and the epilogue maps a group row to its output feature through it.
+// Work unit = 256 tokens x one group of 256 output features (x one slice of the group's entries
+// when the problem is too small to fill the GPU). A unit runs on a CTA pair (cluster of two CTAs on
+// two SMs) with tcgen05 MMAs of cta_group::2: M = 256 tokens (128 per CTA, the A operand), N = 256
+// features (128 weight rows staged per CTA, the B operand), K = 16, fp32 accumulators in TMEM
+// (each CTA holds its 128 tokens x 256 features). Per work-list entry, one chunk of 64 input
+// columns: a stage of two tensor copies per CTA (its 128 x 64 X tile and its 128 x 64 half of the
+// entry's weight-stream tile, 128-byte swizzle), four MMAs.
 // Per CTA (one per SM, persistent):
-//   warp 0      producer: takes units from a global atomic queue, walks the unit's work-list
-//               entries and, per entry (one block column j), loads the X tile [256 tokens x bk]
-//               (TMA tensor copy) and the entry's 128 x bk group tile from the work list's weight
-//               stream (one bulk copy), for a batch of entries at a time, one lane per copy.
-//   warp 1      MMA issuer: per entry and per 16-wide k step, one tcgen05 MMA (M = 128, N = 256,
-//               K = 16, both operands from shared memory): D[128 group rows x 256 tokens] +=
-//               W_tile * X_tile^T, fp32 in TMEM. The W tile covers the whole group, with zero rows
-//               for the slots whose panel keeps no block at this column.
-//   warps 2..17 epilogue: TMEM -> registers, + bias, optional exact GELU, rounding to the output
-//               type, stores of 64-byte row segments; split slices are summed in slice order
-//               by the last slice to finish (ticket), which makes the result deterministic.
-// Accumulators are double-buffered in TMEM (2 x 256 columns) so the epilogue of one unit overlaps
-// the MMAs of the next. Every wait is bounded: on timeout the CTA records an error bit, drains its
-// own copies and MMAs, frees TMEM and returns.
+//   warp 0      X producer: walks each unit's entries and loads its X tiles, two stages per batch,
+//               every copy completing on the leader's full barrier.
+//   warp 18     weight producer: the same walk, loading the weight tiles (a second issuing warp:
+//               a tensor copy keeps its issuing thread for a few hundred cycles).
+//   warp 19     scheduler (leader only): takes units from a global atomic queue and publishes each,
+//               with the chunk indices of its first 32 entries, to both CTAs' unit rings, up to
+//               UR units ahead of the producers.
+//   warp 1      MMA issuer (leader only): per stage four MMAs, the commit multicast to both CTAs'
+//               empty barriers; per unit the commit to both CTAs' accumulator-full barriers.
+//   warps 2..17 epilogue: TMEM -> registers (a lane per token, consecutive features along the
+//               registers), + bias, optional exact GELU, rounding, optional bf16 residual, stores
+//               of whole 16-byte pieces of output rows; split units write fp32 partial sums that
+//               the reduction kernel adds in slice order (deterministic).
+// Accumulators are double-buffered in TMEM (2 x 256 columns), so one unit's epilogue overlaps the
+// next unit's MMAs. Every wait is bounded: on timeout the CTA records an error bit, drains its own
+// copies and MMAs, frees TMEM and returns.
+#include <cstddef>
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -30,209 +35,267 @@
 
 namespace lpvit {
 
-template <int BK>
-struct Cfg {
-  static constexpr int MP = GROUP_FEATURES;                 // MMA M: the group's 128 features
-  static constexpr int KSTEPS = BK / 16;                    // 16-wide k steps per block column
-  static constexpr int ROW_BYTES = BK * 2;                  // bytes of one tile row (bf16)
-  static constexpr int TT = TOKENS_PER_TILE;                // MMA N: tokens per unit
-  static constexpr int BUF_COLS = TT;                       // TMEM columns per accumulator buffer
-  static constexpr int X_BYTES = TT * ROW_BYTES;            // X tile [256 x bk]
-  static constexpr int A_BYTES = MP * ROW_BYTES;            // W tile [128 x bk]
-  static constexpr int STAGE_BYTES = X_BYTES + A_BYTES;
-  static constexpr int NSTAGES = 196608 / STAGE_BYTES;      // 192 KB of stages
-  static constexpr int UR = 4;                              // unit-info ring depth
-  // most entries per lane-parallel copy batch: the producer waits until that many stages are free,
-  // so a batch trades its fixed issue cost against idle stages (measured best: 4 of 16, 3 of 8)
-  static constexpr int BATCH = NSTAGES >= 16 ? 4 : (NSTAGES >= 8 ? 3 : 2);
-  static constexpr int OPS = 2;                             // lane slots per entry: X tile, W tile
-  static constexpr int NBMAX = BATCH < 32 / OPS ? BATCH : 32 / OPS;  // entries per batch
-  static constexpr uint32_t IDESC = idesc_bf16(MP, TT);
-  static_assert(A_BYTES == stream_tile_bytes(BK), "weight-stream tile geometry");
-  static_assert(2 * BUF_COLS == 512, "two accumulator buffers fill the 512 TMEM columns");
-  static_assert(NSTAGES >= 4, "pipeline depth");
-  static_assert(X_BYTES % 1024 == 0 && A_BYTES % 1024 == 0, "tiles stay on their swizzle alignment");
-};
+namespace {
 
-constexpr int MMA_WARPS = 1;       // one MMA issuer
-constexpr int FIRST_EPI = 1 + MMA_WARPS;
-constexpr int EPI_WARPS = 16;      // four per TMEM lane quarter
-static_assert(EPI_WARPS % 4 == 0, "epilogue warps come in whole sets of four lane quarters");
-constexpr int NUM_THREADS = 32 * (FIRST_EPI + EPI_WARPS);   // 576
-constexpr int MAX_GROUPS = 512;    // n <= 65536
+constexpr int NSTAGES = 6;
+constexpr int X_BYTES = CTA_TOKENS * CHUNK_COLS * 2;      // 16 KB: this CTA's tokens x 64 columns
+constexpr int W_BYTES = HALF_FEATURES * CHUNK_COLS * 2;   // 16 KB: this CTA's weight rows x 64 columns
+constexpr int STAGE_BYTES = X_BYTES + W_BYTES;
+constexpr int KSTEPS = CHUNK_COLS / 16;
+constexpr int BUF_COLS = GROUP_FEATURES;                  // TMEM columns of one accumulator
+constexpr int UR = 8;                                     // unit ring depth
+constexpr int BATCH = 2;                                  // stages per producer batch
+static_assert(32 % BATCH == 0, "producer batches tile the 32-entry windows");
+constexpr int FIRST_EPI = 2;
+constexpr int EPI_WARPS = 16;                             // four per TMEM lane quarter
+constexpr int W_WARP = FIRST_EPI + EPI_WARPS;             // the weight-copy producer
+constexpr int SCHED_WARP = W_WARP + 1;                    // the pair's unit scheduler (leader)
+constexpr int NUM_THREADS = 32 * (SCHED_WARP + 1);        // 640
+constexpr int MAX_GROUPS = 256;                           // n <= 65536
+constexpr uint32_t IDESC = idesc_bf16(2 * CTA_TOKENS, GROUP_FEATURES);
+// arrivals that free a unit-ring slot: the leader's MMA warp, both CTAs' epilogue warps and both
+// CTAs' two producers
+constexpr int UNIT_CONSUMERS = 1 + 2 * EPI_WARPS + 4;
+static_assert(2 * BUF_COLS == 512, "two accumulator buffers fill the 512 TMEM columns");
+static_assert(CHUNK_COLS * 2 == 128, "stage rows are 128 bytes (the 128-byte swizzle)");
+static_assert(EPI_WARPS == 16 && GROUP_FEATURES == 4 * 64, "each epilogue warp takes 64 feature columns");
 
 struct UnitInfo {
-  int tt, g, s, nsl, e0, e1, touched, pad;
+  int tt, g, s, nsl, e0, e1, pad0, pad1;
+};
+static_assert(sizeof(UnitInfo) == 32, "unit record is two 16-byte vectors");
+// A unit-ring slot: the unit and the chunk indices of its first 32 entries (0 past its end).
+struct UnitSlot {
+  UnitInfo inf;
+  int win[32];
 };
 
-
-template <int BK>
 struct Smem {
-  // stages first (1024-byte aligned), then the control area
-  static constexpr int CTRL_OFF = Cfg<BK>::NSTAGES * Cfg<BK>::STAGE_BYTES;
-  static constexpr int NS = Cfg<BK>::NSTAGES, UR = Cfg<BK>::UR;
-  static constexpr int BAR_OFF = CTRL_OFF;
-  // barriers: full[NS], empty[NS], accf[2], acce[2], unitf[UR], unite[UR], drain, episync
-  static constexpr int NBARS = 2 * NS + 4 + 2 * UR + 2;
+  static constexpr int BAR_OFF = NSTAGES * STAGE_BYTES;
+  // barriers: full[NS], empty[NS], accf[2], acce[2], unitf[UR], unite[UR], drain
+  static constexpr int NBARS = 2 * NSTAGES + 4 + 2 * UR + 1;
   static constexpr int RING_OFF = (BAR_OFF + 8 * NBARS + 31) / 32 * 32;
-  static constexpr int SLICE_OFF = RING_OFF + (int)sizeof(UnitInfo) * UR;
-  static constexpr int GENT_OFF = SLICE_OFF + 4 * (MAX_GROUPS + 1);  // the group entry table, staged
+  static constexpr int SLICE_OFF = RING_OFF + (int)sizeof(UnitSlot) * UR;
+  static constexpr int GENT_OFF = SLICE_OFF + 4 * (MAX_GROUPS + 1);
   static constexpr int MISC_OFF = GENT_OFF + 4 * (MAX_GROUPS + 1);
-  static constexpr int EPI_OFF = (MISC_OFF + 64 + 127) / 128 * 128;
-  static constexpr int EPI_TILE = 16 * 80;  // per epilogue warp: 16 token rows x 32 bf16, rows padded to 80 B
-  static constexpr int END = EPI_OFF + EPI_WARPS * EPI_TILE;
+  static constexpr int BIAS_OFF = (MISC_OFF + 64 + 15) / 16 * 16;  // per epilogue warp: its 64 features' bias
+  static constexpr int END = BIAS_OFF + EPI_WARPS * 64 * 4;
   static constexpr int BYTES = END + 1024;  // + alignment slack for the dynamic smem base
   static_assert(BYTES <= 227 * 1024, "shared memory per CTA");
 };
 
-// Epilogue of one 32 x 32 block held by a warp: y[i] = accumulator of token tok_base + i for the
-// lane's output feature fl (-1: a group row without a panel; turned into the output in place), bb =
-// that feature's bias (0 without one). Lanes 8c .. 8c + 7 hold consecutive features of one row panel.
-// Adds the bias, applies GELU, rounds, adds the bf16 residual if there is one (rounding again), and
-// stores rows [tok_base, min(tok_base + 32, m)).
-// bf16 output is staged through this warp's shared tile (rows padded to 80 bytes, conflict-free) so
-// that every token row leaves as 16-byte vector stores; fp32 output is stored directly (a warp
-// writes 128 contiguous bytes per token).
-__device__ __forceinline__ void emit32(float (&y)[32], float bb, int fl, int64_t tok_base,
-                                       const LinearParams &P, uint8_t *tile) {
-  const int lane = threadIdx.x & 31;
-  const int f = fl;
-  const bool fvalid = fl >= 0;
-  const int64_t left = P.m - tok_base;
-  const int rows = left >= 32 ? 32 : (left > 0 ? (int)left : 0);
-  if (P.gelu) {
+// Bounded wait whose completion must also make remote (peer CTA) writes visible.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{.reg .pred p; mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p;}"
+      : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, const volatile int *abort_flag,
+                                                  uint64_t limit_ns) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (;;) {
+#pragma unroll 1
+    for (int i = 0; i < 32; ++i)
+      if (mbar_try_wait_cluster(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer_ns() - t0 > limit_ns) return false;
+  }
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+__device__ __forceinline__ float ex2_approx(float x) {
+  float r;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+
+// GELU(t) = t * Phi(t), Phi(t) = erfc(-t / sqrt 2) / 2, with erfc(x) for x >= 0 by Abramowitz &
+// Stegun 7.1.26 (Hastings): erfc(x) = (a1 s + a2 s^2 + a3 s^3 + a4 s^4 + a5 s^5) exp(-x^2),
+// s = 1 / (1 + p x), absolute error below 1.5e-7; for t < 0 the same expression is Phi's tail
+// itself (no 1 - erf cancellation), for t >= 0 Phi = 1 - erfc(x) / 2. Branch-free, two MUFU ops.
+__device__ __forceinline__ float gelu_erf(float t) {
+  const float x = fabsf(t) * 0.70710678118654752440f;
+  const float s = rcp_approx(fmaf(0.3275911f, x, 1.f));
+  float p = 1.061405429f;
+  p = fmaf(p, s, -1.453152027f);
+  p = fmaf(p, s, 1.421413741f);
+  p = fmaf(p, s, -0.284496736f);
+  p = fmaf(p, s, 0.254829592f);
+  const float half_erfc = 0.5f * p * s * ex2_approx(-1.44269504088896340736f * x * x);
+  return t * (t >= 0.f ? 1.f - half_erfc : half_erfc);
+}
+
+// Transpose 16-byte chunks within groups of CPR lanes: lane i of a group holds chunks
+// w[4 j .. 4 j + 3] (j < CPR) of its own row; afterwards it holds chunk i of row j of the group in
+// w[4 j .. 4 j + 3] (butterfly exchange over lane bits 1, 2, 4, ...).
+template <int CPR>
+__device__ __forceinline__ void transpose_chunks(uint32_t (&w)[4 * CPR], int lane) {
+  const int i = lane & (CPR - 1);
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      // exact GELU, t * Phi(t); where 1 + erf cancels (t < -3) the error is a few ulps of 1 times t / 2
-      const float t = y[i] + bb;
-      y[i] = 0.5f * t * (1.f + erff(t * 0.70710678118654752440f));
+  for (int sft = 1; sft < CPR; sft <<= 1) {
+    const bool hi = (i & sft) != 0;
+#pragma unroll
+    for (int j = 0; j < CPR; ++j) {
+      if (j & sft) continue;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const uint32_t send = hi ? w[4 * j + q] : w[4 * (j ^ sft) + q];
+        const uint32_t recv = __shfl_xor_sync(0xffffffffu, send, sft);
+        if (hi) w[4 * j + q] = recv;
+        else w[4 * (j ^ sft) + q] = recv;
+      }
     }
+  }
+}
+
+// The outputs of one run of 16 consecutive group rows (features f0 .. f0 + 15) for the warp's 32
+// tokens (a lane per token, tokens tok0 .. tok0 + 31): y[0..16) are the lane's accumulated sums (or
+// zero), bs the run's bias in shared memory (the same for every lane). Adds the bias, applies GELU,
+// rounds, then exchanges 16-byte chunks between lanes so that each store instruction writes whole
+// 16-feature row segments (32 bytes bf16, 64 bytes fp32) of 32 / CPR tokens; bf16 output may add
+// the residual (each sum rounded, as a separate bf16 addition would). Warp-uniform: every lane
+// calls it.
+template <bool GELU, bool F32>
+__device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, int64_t tok0, const LinearParams &P) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int i = 0; i < 16; i += 4) {
+    float4 b;
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(b.x), "=f"(b.y), "=f"(b.z), "=f"(b.w) : "r"(bs + 4 * i));
+    y[i] += b.x; y[i + 1] += b.y; y[i + 2] += b.z; y[i + 3] += b.w;
+  }
+  if (GELU) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) y[i] = gelu_erf(y[i]);
+  }
+  constexpr int CPR = F32 ? 4 : 2;  // 16-byte chunks per row segment
+  uint32_t w[4 * CPR];
+  if (F32) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) w[i] = __float_as_uint(y[i]);
   } else {
 #pragma unroll
-    for (int i = 0; i < 32; ++i) y[i] += bb;
+    for (int i = 0; i < 8; ++i) w[i] = pack_bf16x2(y[2 * i], y[2 * i + 1]);
   }
-  if (P.y_f32) {
-    float *dst = static_cast<float *>(P.Y) + tok_base * P.ldy + f;
-    if (fvalid) {
+  transpose_chunks<CPR>(w, lane);
+  const int ci = lane & (CPR - 1), grp = lane / CPR;
 #pragma unroll
-      for (int i = 0; i < 32; ++i)
-        if (i < rows) dst[(int64_t)i * P.ldy] = y[i];
-    }
-    return;
-  }
-  __nv_bfloat16 *t = reinterpret_cast<__nv_bfloat16 *>(tile);
-  const int ch = lane & 3;
-  const int fch = __shfl_sync(0xffffffffu, fl, 8 * ch);  // first feature of the lane's 8-feature chunk
-  const bool cvalid = fch >= 0;
+  for (int j = 0; j < CPR; ++j) {
+    const int64_t t = tok0 + grp * CPR + j;
+    if (t >= P.m) continue;
+    uint32_t o[4] = {w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]};
+    if (F32) {
+      float *dst = static_cast<float *>(P.Y) + t * P.ldy + f0 + 4 * ci;
+      if (P.y_vec16) {
+        *reinterpret_cast<int4 *>(dst) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
+      } else {  // row not 16-byte aligned: element by element
 #pragma unroll
-  for (int half = 0; half < 2; ++half) {  // 16 token rows at a time through the warp's tile
+        for (int q = 0; q < 4; ++q) dst[q] = __uint_as_float(o[q]);
+      }
+    } else {
+      if (P.R != nullptr) {
+        // a plain load: R may be Y itself, read and then written by this lane only
+        const int4 rv = *reinterpret_cast<const int4 *>(P.R + t * P.ldr + f0 + 8 * ci);
+        const uint32_t rw[4] = {(uint32_t)rv.x, (uint32_t)rv.y, (uint32_t)rv.z, (uint32_t)rv.w};
 #pragma unroll
-    for (int i = 0; i < 16; ++i) t[i * 40 + lane] = __float2bfloat16_rn(y[16 * half + i]);
-    __syncwarp();
-#pragma unroll
-    for (int it = 0; it < 2; ++it) {
-      const int rt = 8 * it + (lane >> 2), row = 16 * half + rt;
-      int4 val = *reinterpret_cast<const int4 *>(tile + rt * 80 + ch * 16);
-      if (row < rows && cvalid) {
-        if (P.R != nullptr) {
-          // + the residual, each sum rounded to bf16 (a plain load: R may be Y itself, read and then
-          // written by this thread only)
-          const int4 rv = *reinterpret_cast<const int4 *>(P.R + (tok_base + row) * P.ldr + fch);
-          __nv_bfloat16 *a = reinterpret_cast<__nv_bfloat16 *>(&val);
-          const __nv_bfloat16 *b = reinterpret_cast<const __nv_bfloat16 *>(&rv);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) a[e] = __float2bfloat16_rn(__bfloat162float(a[e]) + __bfloat162float(b[e]));
+        for (int q = 0; q < 4; ++q) {
+          const float lo = __uint_as_float(o[q] << 16) + __uint_as_float(rw[q] << 16);
+          const float hi = __uint_as_float(o[q] & 0xffff0000u) + __uint_as_float(rw[q] & 0xffff0000u);
+          o[q] = pack_bf16x2(lo, hi);
         }
-        __nv_bfloat16 *dst = static_cast<__nv_bfloat16 *>(P.Y) + (tok_base + row) * P.ldy + fch;
-        if (P.y_vec16) {
-          *reinterpret_cast<int4 *>(dst) = val;
-        } else {
-          const __nv_bfloat16 *src = reinterpret_cast<const __nv_bfloat16 *>(&val);
+      }
+      uint16_t *dst = static_cast<uint16_t *>(P.Y) + t * P.ldy + f0 + 8 * ci;
+      if (P.y_vec16) {
+        *reinterpret_cast<int4 *>(dst) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
+      } else {  // row not 16-byte aligned: element by element
 #pragma unroll
-          for (int e = 0; e < 8; ++e) dst[e] = src[e];
+        for (int q = 0; q < 4; ++q) {
+          dst[2 * q] = (uint16_t)(o[q] & 0xffffu);
+          dst[2 * q + 1] = (uint16_t)(o[q] >> 16);
         }
       }
     }
-    __syncwarp();
   }
 }
 
-
-// The MMAs of one work-list entry, issued by one elected thread: for every 16-wide k step,
-// D[128 x 256] (+)= W_tile[128 x 16] * X_tile[256 x 16]^T, both tiles in the stage (X first).
-template <int BK>
-__device__ __forceinline__ void issue_entry(uint32_t st_u32, uint32_t dbase, uint32_t accumulate) {
-  using C = Cfg<BK>;
-#pragma unroll
-  for (int kk = 0; kk < C::KSTEPS; ++kk) {
-    const uint64_t bdesc = smem_desc<C::ROW_BYTES>(st_u32 + kk * 32);
-    const uint64_t adesc = smem_desc<C::ROW_BYTES>(st_u32 + C::X_BYTES + kk * 32);
-    umma_f16(dbase, adesc, bdesc, C::IDESC, (kk > 0 || accumulate) ? 1u : 0u);
-  }
-}
-
-template <int BK>
+template <bool GELU, bool F32>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P) {
-  using C = Cfg<BK>;
-  using L = Smem<BK>;
+bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
+                  const LinearParams P) {
+  using L = Smem;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t smem_base = smem_u32(smem);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t rank = cluster_rank();  // 0: the pair's leader (schedules, issues the MMAs), 1: its peer
+  const bool leader = rank == 0;
 
   const uint32_t bar0 = smem_base + L::BAR_OFF;
-  auto full_bar = [&](int s) { return bar0 + 8u * s; };
-  auto empty_bar = [&](int s) { return bar0 + 8u * (L::NS + s); };
-  auto accf_bar = [&](int b) { return bar0 + 8u * (2 * L::NS + b); };
-  auto acce_bar = [&](int b) { return bar0 + 8u * (2 * L::NS + 2 + b); };
-  auto unitf_bar = [&](int u) { return bar0 + 8u * (2 * L::NS + 4 + u); };
-  auto unite_bar = [&](int u) { return bar0 + 8u * (2 * L::NS + 4 + L::UR + u); };
-  const uint32_t drain_bar = bar0 + 8u * (2 * L::NS + 4 + 2 * L::UR);
-  const uint32_t episync_bar = drain_bar + 8u;
-  UnitInfo *ring = reinterpret_cast<UnitInfo *>(smem + L::RING_OFF);
+  auto full_bar = [&](int i) { return bar0 + 8u * i; };
+  auto empty_bar = [&](int i) { return bar0 + 8u * (NSTAGES + i); };
+  constexpr int RB = 2 * NSTAGES;  // first barrier after the stage ring
+  auto accf_bar = [&](int b) { return bar0 + 8u * (RB + b); };
+  auto acce_bar = [&](int b) { return bar0 + 8u * (RB + 2 + b); };
+  auto unitf_bar = [&](int u) { return bar0 + 8u * (RB + 4 + u); };
+  auto unite_bar = [&](int u) { return bar0 + 8u * (RB + 4 + UR + u); };
+  const uint32_t drain_bar = bar0 + 8u * (RB + 4 + 2 * UR);
+  UnitSlot *ring = reinterpret_cast<UnitSlot *>(smem + L::RING_OFF);
   int *slice_ptr = reinterpret_cast<int *>(smem + L::SLICE_OFF);
   int *gent_s = reinterpret_cast<int *>(smem + L::GENT_OFF);
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + L::MISC_OFF);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 4);
-  volatile int *last_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 8);
-  volatile int *never_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 12);  // stays 0
+  volatile int *never_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 8);  // stays 0
 
   const int32_t *gent = P.sched + SCHED_HDR_INTS;
-  const int32_t *entries = P.sched + sched_entries_offset_ints(P.n_groups);
   const int32_t *gpan = P.sched + sched_gpan_offset_ints(P.n_groups);
+  const int32_t *entries = P.sched + sched_entries_offset_ints(P.n_groups);
+  const int kc = sched_chunks(P.k);
   const uint64_t tmo = P.timeout_ns;
 
   // ---------------------------------------------------------------- prologue
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), 512);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_u32(tmem_slot), 512);  // one warp of each CTA, together
+    tmem_relinquish_pair();
   }
   if (tid == 0) {
-    for (int s = 0; s < L::NS; ++s) {
-      mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), MMA_WARPS);
+    for (int i = 0; i < NSTAGES; ++i) {
+      mbar_init(full_bar(i), 1);
+      mbar_init(empty_bar(i), 1);
     }
     for (int b = 0; b < 2; ++b) {
-      mbar_init(accf_bar(b), MMA_WARPS);
-      mbar_init(acce_bar(b), EPI_WARPS);
+      mbar_init(accf_bar(b), 1);
+      mbar_init(acce_bar(b), 2 * EPI_WARPS);
     }
-    for (int u = 0; u < L::UR; ++u) {
+    for (int u = 0; u < UR; ++u) {
       mbar_init(unitf_bar(u), 1);
-      mbar_init(unite_bar(u), EPI_WARPS);
+      mbar_init(unite_bar(u), UNIT_CONSUMERS);
     }
-    mbar_init(drain_bar, MMA_WARPS);
-    mbar_init(episync_bar, EPI_WARPS);
+    mbar_init(drain_bar, 1);
     *abort_flag = 0;
-    *last_flag = 0;
     *never_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 0 && lane == 0) prefetch_tensormap(&tmX);
-  // the work list must be this weight's plan: group count, shape and block width
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmX);
+    prefetch_tensormap(&tmW);
+  }
+  // the work list must be this weight's plan: layout, group count, shape
   const bool sched_ok = P.sched[3] == 0 && P.sched[1] == P.n_groups && P.sched[4] == P.n && P.sched[5] == P.k &&
-                        P.sched[6] == P.bn && P.sched[7] == BK;
-  if (warp == 2) {
+                        P.sched[6] == P.bn && P.sched[8] == SCHED_VERSION && P.n_groups <= MAX_GROUPS;
+  if (warp == 2 && sched_ok) {
     // slices per group = max(1, ceil(entries / S)); exclusive prefix into slice_ptr
     int run = 0;
     for (int base = 0; base < P.n_groups; base += 32) {
@@ -256,331 +319,322 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // both CTAs' barriers are initialised before any signal crosses the pair
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int total_slices = slice_ptr[P.n_groups];
+  const int total_slices = sched_ok ? slice_ptr[P.n_groups] : 0;
   const uint32_t total_units = sched_ok ? (uint32_t)P.n_tt * (uint32_t)total_slices : 0u;
-  if (!sched_ok && tid == 0) atomicOr(&P.ctl->err, P.sched[3] ? ERR_SCHED_OVERFLOW : ERR_BAD_SCHED);
+  if (!sched_ok && tid == 0 && leader) atomicOr(&P.ctl->err, P.sched[3] ? ERR_SCHED_OVERFLOW : ERR_BAD_SCHED);
 
-  if (warp == 0) {
-    // ============================================================== producer
-    // Unit i is decoded (shared-memory tables) and its first 32 entry records are loaded while unit
-    // i - 1 is issued, and the queue index of unit i + 1 is fetched then; within a unit the next 32
-    // records are loaded while the current ones are issued. No global round trip sits on the path.
+  if (warp == 0 || warp == W_WARP) {
+    // ============================================================== producers
+    const bool xrole = warp == 0;           // X tiles (else weight tiles)
     uint32_t it = 0, ui = 0;
     bool ok = true;
-    struct Unit {
-      int tt, g, s, nsl, e0, e1;
-    };
-    auto decode = [&](uint32_t u) {  // shared-memory tables only
-      Unit d;
-      d.tt = (int)(u / (uint32_t)total_slices);
-      const int rr = (int)(u % (uint32_t)total_slices);
-      int lo = 0, hi = P.n_groups - 1;  // group g with slice_ptr[g] <= rr < slice_ptr[g+1]
-      while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (slice_ptr[mid] <= rr) lo = mid;
-        else hi = mid - 1;
-      }
-      d.g = lo;
-      d.s = rr - slice_ptr[lo];
-      d.nsl = slice_ptr[lo + 1] - slice_ptr[lo];
-      const int ge0 = gent_s[lo], ge1 = gent_s[lo + 1];
-      d.e0 = min(ge0 + d.s * P.S, ge1);
-      d.e1 = min(d.e0 + P.S, ge1);
-      return d;
-    };
-    auto first_records = [&](const Unit &d, int &w, int &t) {
-      w = 0;
-      t = -1;
-      if (d.e0 + lane < d.e1) {
-        const int32_t *ep = entries + (int64_t)(d.e0 + lane) * ENTRY_INTS;
-        w = ep[0];
-        t = ep[ENTRY_TILE_WORD];
-      }
-    };
-    uint32_t fetched = 0;
-    if (lane == 0) fetched = atomicAdd(&P.ctl->next_unit, 1u);
-    uint32_t u_cur = __shfl_sync(0xffffffffu, fetched, 0);
-    Unit cur = {0, 0, 0, 1, 0, 0};
-    int w0c = 0, toffc = -1;
-    if (u_cur < total_units) {
-      cur = decode(u_cur);
-      first_records(cur, w0c, toffc);
-      if (lane == 0) fetched = atomicAdd(&P.ctl->next_unit, 1u);
-    }
-    while (true) {
-      const uint32_t u = u_cur;
-      const uint32_t slot = ui % L::UR, uph = (ui / L::UR) & 1u;
-      if (!mbar_wait(unite_bar(slot), uph ^ 1u, abort_flag, tmo)) {
+    while (ok) {
+      const uint32_t slot = ui % UR, uph = (ui / UR) & 1u;
+      if (!mbar_wait_cluster(unitf_bar(slot), uph, abort_flag, tmo)) {
         ok = false;
         if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_UNIT);
         break;
       }
-      if (u >= total_units) {
-        if (lane == 0) {
-          ring[slot].tt = -1;
-          mbar_arrive(unitf_bar(slot));
-        }
-        break;
-      }
-      const int tt = cur.tt, e0 = cur.e0, e1 = cur.e1;
-      // every entry keeps a block of the group, so the accumulator is written iff there is one
-      const unsigned tmask = e1 > e0 ? 1u : 0u;
+      const UnitInfo inf = ring[slot].inf;
+      int cw = ring[slot].win[lane];  // chunk indices of entries win .. win + 31, one per lane
+      __syncwarp();
       if (lane == 0) {
-        UnitInfo inf;
-        inf.tt = tt; inf.g = cur.g; inf.s = cur.s; inf.nsl = cur.nsl; inf.e0 = e0; inf.e1 = e1;
-        inf.touched = (int)tmask;
-        inf.pad = 0;
-        ring[slot] = inf;
-        mbar_arrive(unitf_bar(slot));
+        if (leader) mbar_arrive(unite_bar(slot));
+        else mbar_arrive_cluster(mapa_rank(unite_bar(slot), 0));
       }
-      // the next unit: decode it, start loading its first records, fetch the one after
-      const uint32_t u_nx = __shfl_sync(0xffffffffu, fetched, 0);
-      Unit nxt = {0, 0, 0, 1, 0, 0};
-      int w0x = 0, toffx = -1;
-      if (u_nx < total_units) {
-        nxt = decode(u_nx);
-        first_records(nxt, w0x, toffx);
-        if (lane == 0) fetched = atomicAdd(&P.ctl->next_unit, 1u);
-      }
-      int w0n = w0c, toffn = toffc;  // records of entries base + lane, loaded one chunk ahead
-      for (int base = e0; base < e1 && ok; base += 32) {
-        const int w0 = w0n, toff = toffn;
-        w0n = 0;
-        toffn = -1;
-        if (base + 32 + lane < e1) {
-          const int32_t *ep = entries + (int64_t)(base + 32 + lane) * ENTRY_INTS;
-          w0n = ep[0];
-          toffn = ep[ENTRY_TILE_WORD];
+      if (inf.tt < 0) break;
+      // Stages: a batch of up to BATCH consecutive entries; lane i < nb waits for stage i's empty
+      // barrier, then issues its stage's copy (this warp's kind), completing on the leader's full
+      // barrier; the leader's X producer posts the stage's expected bytes (both kinds, both CTAs).
+      const int ytok = inf.tt * TOKENS_PER_TILE + (int)rank * CTA_TOKENS;
+      int win = inf.e0;
+      int cw_next = xrole && win + 32 + lane < inf.e1 ? __ldg(entries + win + 32 + lane) : 0;
+      for (int base = inf.e0; base < inf.e1 && ok; base += BATCH) {
+        const int nb = min(BATCH, inf.e1 - base);
+        if (base >= win + 32) {  // BATCH divides 32: a batch never straddles two windows
+          win += 32;
+          cw = cw_next;
+          cw_next = xrole && win + 32 + lane < inf.e1 ? __ldg(entries + win + 32 + lane) : 0;
         }
-        const int cnt = min(32, e1 - base);
-        for (int i = 0; i < cnt && ok;) {
-          // One batch = NBMAX consecutive entries. Lanes 2k and 2k+1 issue the two copies of entry k
-          // (its X tile, its weight tiles), all in one instruction: a thread's bulk copies are
-          // processed one after another, copies from different threads overlap.
-          const int nb = min(C::NBMAX, cnt - i);
-          bool wok = true;
-          if (lane < nb) {
-            const uint32_t itk = it + lane;
-            wok = mbar_wait(empty_bar(itk % L::NS), ((itk / L::NS) & 1u) ^ 1u, abort_flag, tmo);
-          }
-          if (!__all_sync(0xffffffffu, wok)) {
-            ok = false;
-            if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_EMPTY);
-            break;
-          }
-          const int k2 = lane >> 1;
-          const int src = min(i + k2, 31);
-          const int wk = __shfl_sync(0xffffffffu, w0, src);
-          const int tk = __shfl_sync(0xffffffffu, toff, src);
-          uint32_t mm = ((uint32_t)wk >> 16) != 0u ? 1u : 0u;  // the entry keeps a block of the group
-          // a tile range outside the stream region means a corrupt work list: flag it, load no weights
-          const bool tiles_ok = tk >= 0 && (int64_t)tk + __popc(mm) <= P.stream_tiles;
-          if (!tiles_ok) mm = 0;
-          const uint32_t stk = (it + k2) % L::NS;
-          const uint32_t st_u32 = smem_base + stk * C::STAGE_BYTES;
-          if (k2 < nb && (lane & 1) == 0) {
-            if (!tiles_ok) atomicOr(&P.ctl->err, ERR_BAD_SCHED);
-            mbar_arrive_expect_tx(full_bar(stk), C::X_BYTES + __popc(mm) * C::A_BYTES);
-          }
-          __syncwarp();
-          if (k2 < nb) {
-            if ((lane & 1) == 0)
-              tma_load_2d(st_u32, &tmX, (wk & 0xffff) * BK, tt * C::TT, full_bar(stk));
-            else if (mm)
-              bulk_load(st_u32 + C::X_BYTES, P.wstream + (int64_t)tk * C::A_BYTES, __popc(mm) * C::A_BYTES,
-                        full_bar(stk));
-          }
-          __syncwarp();
-          it += nb;
-          i += nb;
+        bool wok = true;
+        if (lane < nb) {
+          const uint32_t itk = it + lane;
+          wok = mbar_wait(empty_bar(itk % NSTAGES), ((itk / NSTAGES) & 1u) ^ 1u, abort_flag, tmo);
         }
+        if (!__all_sync(0xffffffffu, wok)) {
+          ok = false;
+          if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_EMPTY);
+          break;
+        }
+        const int e = base + (lane < nb ? lane : 0);  // the batch entry of this lane's copy
+        int c = __shfl_sync(0xffffffffu, cw, (e - win) & 31);
+        int tile = e;
+        // a chunk or tile outside the work list's ranges means a corrupt list: flag it, load tile 0
+        const bool in_range = xrole ? (c >= 0 && c < kc) : ((int64_t)tile < P.stream_tiles);
+        if (!in_range) {
+          c = 0;
+          tile = 0;
+        }
+        const uint32_t stk = (it + (uint32_t)lane) % NSTAGES;
+        const uint32_t st = smem_base + stk * STAGE_BYTES;
+        const uint32_t fb = mapa_rank(full_bar(stk), 0);
+        if (lane < nb) {
+          if (!in_range) atomicOr(&P.ctl->err, ERR_BAD_SCHED);
+          if (leader && xrole) mbar_arrive_expect_tx(full_bar(stk), 2 * STAGE_BYTES);
+          if (xrole) tma_load_2d_pair(st, &tmX, c * CHUNK_COLS, ytok, fb);
+          else tma_load_2d_pair(st + X_BYTES, &tmW, 0, tile * GROUP_FEATURES + (int)rank * HALF_FEATURES, fb);
+        }
+        __syncwarp();
+        it += nb;
       }
       if (!ok) break;
       ++ui;
-      u_cur = u_nx;
-      cur = nxt;
-      w0c = w0x;
-      toffc = toffx;
     }
     if (!ok && lane == 0) *abort_flag = 1;
-    // queue bookkeeping: the last CTA to leave resets the counters for the next launch
-    if (lane == 0) {
-      __threadfence();
-      if (atomicAdd(&P.ctl->done_ctas, 1u) == gridDim.x - 1) {
-        P.ctl->next_unit = 0;
-        P.ctl->done_ctas = 0;
+    // no copy of either CTA may still be in flight: they all complete on the leader's full barriers
+    if (leader && xrole) {
+      const uint32_t first = it > (uint32_t)NSTAGES ? it - NSTAGES : 0u;
+      for (uint32_t i = first; i < it; ++i)
+        if (!mbar_wait(full_bar(i % NSTAGES), (i / NSTAGES) & 1u, never_flag, tmo)) {
+          if (lane == 0) atomicOr(&P.ctl->err, ERR_DRAIN);
+          break;
+        }
+    }
+  } else if (warp == SCHED_WARP) {
+    // ============================================================== scheduler (leader only)
+    // Publishes each unit (or the end record) once its ring slot is free in both CTAs: the record
+    // and the unit's first 32 chunk indices, written locally and into the peer, then both CTAs'
+    // unit-full barriers. Runs up to UR units ahead of the producers.
+    if (leader) {
+      bool ok = true;
+      uint32_t fetched = 0;
+      if (lane == 0) fetched = atomicAdd(&P.ctl->next_unit, 1u);
+      for (uint32_t pub = 0;; ++pub) {
+        const uint32_t slot = pub % UR;
+        if (!mbar_wait_cluster(unite_bar(slot), ((pub / UR) & 1u) ^ 1u, abort_flag, tmo)) {
+          ok = false;
+          if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_UNIT);
+          break;
+        }
+        const uint32_t u = __shfl_sync(0xffffffffu, fetched, 0);
+        UnitInfo d;
+        if (u < total_units) {
+          d.tt = (int)(u / (uint32_t)total_slices);
+          const int rr = (int)(u % (uint32_t)total_slices);
+          int lo = 0, hi = P.n_groups - 1;  // group g with slice_ptr[g] <= rr < slice_ptr[g+1]
+          while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (slice_ptr[mid] <= rr) lo = mid;
+            else hi = mid - 1;
+          }
+          d.g = lo;
+          d.s = rr - slice_ptr[lo];
+          d.nsl = slice_ptr[lo + 1] - slice_ptr[lo];
+          const int ge0 = gent_s[lo], ge1 = gent_s[lo + 1];
+          d.e0 = min(ge0 + d.s * P.S, ge1);
+          d.e1 = min(d.e0 + P.S, ge1);
+        } else {
+          d.tt = -1; d.g = d.s = d.nsl = d.e0 = d.e1 = 0;
+        }
+        d.pad0 = d.pad1 = 0;
+        if (lane == 0 && u < total_units) fetched = atomicAdd(&P.ctl->next_unit, 1u);
+        const int wv = d.e0 + lane < d.e1 ? __ldg(entries + d.e0 + lane) : 0;
+        UnitSlot &rs = ring[slot];
+        const uint32_t remote = mapa_rank(smem_u32(&rs), 1);
+        rs.win[lane] = wv;
+        asm volatile("st.shared::cluster.b32 [%0], %1;"
+                     :: "r"(remote + (uint32_t)offsetof(UnitSlot, win) + 4u * lane), "r"(wv) : "memory");
+        if (lane == 0) {
+          rs.inf = d;
+          const int4 *v = reinterpret_cast<const int4 *>(&d);
+          st_cluster_v4(remote, v[0]);
+          st_cluster_v4(remote + 16, v[1]);
+        }
+        asm volatile("fence.acq_rel.cluster;" ::: "memory");  // every lane's writes before the signal
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(unitf_bar(slot));
+          mbar_arrive_cluster(mapa_rank(unitf_bar(slot), 1));
+        }
+        __syncwarp();
+        if (u >= total_units) break;
+      }
+      if (!ok && lane == 0) *abort_flag = 1;
+      // queue bookkeeping: the last scheduler to leave resets the counters for the next launch
+      if (lane == 0) {
         __threadfence();
+        if (atomicAdd(&P.ctl->done_ctas, 1u) == gridDim.x / 2 - 1) {
+          P.ctl->next_unit = 0;
+          P.ctl->done_ctas = 0;
+          __threadfence();
+        }
       }
     }
-    // make sure no TMA write into this CTA's smem is still in flight
-    const uint32_t first = it > (uint32_t)L::NS ? it - L::NS : 0u;
-    for (uint32_t i = first; i < it; ++i)
-      if (!mbar_wait(full_bar(i % L::NS), (i / L::NS) & 1u, never_flag, tmo)) break;
   } else if (warp < FIRST_EPI) {
-    // ============================================================== MMA issuer
-    // Arrives on a stage's empty barrier once per entry: a commit when it issued MMAs there.
-    uint32_t it = 0, ui = 0;
-    bool ok = true;
-    while (ok) {
-      const uint32_t slot = ui % L::UR, uph = (ui / L::UR) & 1u;
-      if (!mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)) {
-        ok = false;
-        if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_UNIT);
-        break;
-      }
-      const UnitInfo inf = ring[slot];
-      if (inf.tt < 0) break;
-      const uint32_t buf = ui & 1u, aph = (ui >> 1) & 1u;
-      if (!mbar_wait(acce_bar(buf), aph ^ 1u, abort_flag, tmo)) {
-        ok = false;
-        if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_ACC);
-        break;
-      }
-      tc_fence_after();
-      const uint32_t dbase = tmem_base + buf * C::BUF_COLS;
-      uint32_t touched = 0;
-      for (int e = inf.e0; e < inf.e1; ++e) {
-        const uint32_t stage = it % L::NS, ph = (it / L::NS) & 1u;
-        if (!mbar_wait(full_bar(stage), ph, abort_flag, tmo)) {
+    // ============================================================== MMA issuer (leader only)
+    if (leader) {
+      uint32_t it = 0, ui = 0;
+      bool ok = true;
+      while (ok) {
+        const uint32_t slot = ui % UR, uph = (ui / UR) & 1u;
+        if (!mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)) {
           ok = false;
-          if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_FULL);
+          if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_UNIT);
+          break;
+        }
+        const UnitInfo inf = ring[slot].inf;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(unite_bar(slot));
+        if (inf.tt < 0) break;
+        const uint32_t buf = ui & 1u, aph = (ui >> 1) & 1u;
+        // both CTAs' epilogues have read this accumulator buffer
+        if (!mbar_wait_cluster(acce_bar(buf), aph ^ 1u, abort_flag, tmo)) {
+          ok = false;
+          if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_ACC);
           break;
         }
         tc_fence_after();
-        // every entry keeps a block of its group, so every stage holds a W tile (a work list whose
-        // tile range is corrupt has its error bit set and its stage's weights left stale)
-        const uint32_t st_u32 = smem_base + stage * C::STAGE_BYTES;
+        const uint32_t dbase = tmem_base + buf * BUF_COLS;
+        for (int e = inf.e0; e < inf.e1; ++e) {
+          const uint32_t stage = it % NSTAGES, ph = (it / NSTAGES) & 1u;
+          if (!mbar_wait(full_bar(stage), ph, abort_flag, tmo)) {
+            ok = false;
+            if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_FULL);
+            break;
+          }
+          tc_fence_after();
+          const uint32_t st = smem_base + stage * STAGE_BYTES;
+          if (elect_one()) {
+#pragma unroll
+            for (int kk = 0; kk < KSTEPS; ++kk) {
+              const uint64_t adesc = smem_desc<128>(st + kk * 32);
+              const uint64_t bdesc = smem_desc<128>(st + X_BYTES + kk * 32);
+              umma_f16_pair(dbase, adesc, bdesc, IDESC, (e > inf.e0 || kk > 0) ? 1u : 0u);
+            }
+            tc_commit_pair(empty_bar(stage), 3);
+          }
+          __syncwarp();
+          ++it;
+        }
+        if (!ok) break;
         if (elect_one()) {
-          issue_entry<BK>(st_u32, dbase, touched);
-          tc_commit(empty_bar(stage));
+          if (inf.e1 > inf.e0) {
+            tc_commit_pair(accf_bar(buf), 3);
+          } else {  // nothing accumulated: the epilogue treats the sums as zero
+            mbar_arrive(accf_bar(buf));
+            mbar_arrive_cluster(mapa_rank(accf_bar(buf), 1));
+          }
         }
         __syncwarp();
-        touched = 1;
-        ++it;
+        ++ui;
       }
-      if (!ok) break;
-      if (elect_one()) {
-        if (touched) tc_commit(accf_bar(buf));
-        else mbar_arrive(accf_bar(buf));
-      }
+      if (!ok && lane == 0) *abort_flag = 1;
+      // every MMA this thread issued completes before TMEM can be freed
+      if (elect_one()) tc_commit_pair(drain_bar, 1);
       __syncwarp();
-      ++ui;
+      if (!mbar_wait(drain_bar, 0, never_flag, tmo) && lane == 0) atomicOr(&P.ctl->err, ERR_DRAIN);
     }
-    if (!ok && lane == 0) *abort_flag = 1;
-    // wait for every MMA this thread issued before TMEM can be freed
-    if (elect_one()) tc_commit(drain_bar);
-    __syncwarp();
-    if (!mbar_wait(drain_bar, 0, never_flag, tmo) && lane == 0) atomicOr(&P.ctl->err, ERR_DRAIN);
   } else {
     // ============================================================== epilogue
-    // A unit's accumulator is 128 features (TMEM lanes) x 256 tokens (columns). Per TMEM lane
-    // quarter (32 features) it forms 8 blocks of 32 tokens; the quarter's EPI_WARPS / 4 warps take
-    // them in turn.
-    const int ew = warp - FIRST_EPI;             // 0 .. EPI_WARPS - 1
-    const int q = warp & 3;                      // TMEM lane quarter this warp may access
-    const int wq = ew >> 2;                      // this warp's turn within its quarter
-    constexpr int QBLK = C::TT / 32;             // blocks per lane quarter
-    uint32_t ui = 0, sync_phase = 0;
-    uint8_t *epi_tile = smem + L::EPI_OFF + ew * L::EPI_TILE;
+    // The accumulator is 128 tokens (TMEM lanes) x 256 group rows (columns). Warp w reads lane
+    // quarter q = w % 4 (tokens 32 q .. 32 q + 31) and the 64 columns of part (w - 2) / 4.
+    const int q = warp & 3;
+    const int part = (warp - FIRST_EPI) >> 2;
+    float *bias_s = reinterpret_cast<float *>(smem + L::BIAS_OFF) + (warp - FIRST_EPI) * 64;
+    uint32_t ui = 0;
     while (true) {
-      const uint32_t slot = ui % L::UR, uph = (ui / L::UR) & 1u;
-      if (!mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)) {
+      const uint32_t slot = ui % UR, uph = (ui / UR) & 1u;
+      if (!(leader ? mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)
+                   : mbar_wait_cluster(unitf_bar(slot), uph, abort_flag, tmo))) {
         if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_UNIT); *abort_flag = 1; }
         break;
       }
-      const UnitInfo inf = ring[slot];
+      const UnitInfo inf = ring[slot].inf;
+      __syncwarp();
+      if (lane == 0) {
+        if (leader) mbar_arrive(unite_bar(slot));
+        else mbar_arrive_cluster(mapa_rank(unite_bar(slot), 0));
+      }
       if (inf.tt < 0) break;
-      // this lane's group row 32 q + lane is row (32 q + lane) % bn of the panel in slot (32 q + lane) / bn;
-      // its feature and bias are loaded while the accumulator is still being computed
-      const int grow = 32 * q + lane;
-      const int panel = __ldg(gpan + (int64_t)inf.g * MAX_GROUP_PANELS + grow / P.bn);
-      const int fl = panel >= 0 ? panel * P.bn + grow % P.bn : -1;
-      const float bb = (P.bias != nullptr && fl >= 0) ? __ldg(P.bias + fl) : 0.f;
+      // the features of this warp's 64 columns (first feature of each 16-column quarter, or -1)
+      // and their bias, staged while the accumulator is still being computed
+      int fcol[4];
+#pragma unroll
+      for (int r4 = 0; r4 < 4; ++r4) {
+        const int c = 64 * part + 16 * r4;
+        const int panel = __ldg(gpan + (int64_t)inf.g * MAX_GROUP_PANELS + c / P.bn);
+        fcol[r4] = panel >= 0 ? panel * P.bn + c % P.bn : -1;
+      }
+      if (lane < 16) {
+        const int qq = lane >> 2;  // the lane's quarter, selected without indexing the array
+        const int fq = qq == 0 ? fcol[0] : (qq == 1 ? fcol[1] : (qq == 2 ? fcol[2] : fcol[3]));
+        const int f = fq < 0 ? -1 : fq + 4 * (lane & 3);
+        float4 b4 = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (f >= 0 && P.bias != nullptr) {
+          if (P.bias_vec16) {
+            b4 = __ldg(reinterpret_cast<const float4 *>(P.bias + f));
+          } else {
+            b4 = make_float4(__ldg(P.bias + f), __ldg(P.bias + f + 1), __ldg(P.bias + f + 2), __ldg(P.bias + f + 3));
+          }
+        }
+        *reinterpret_cast<float4 *>(bias_s + 4 * lane) = b4;
+      }
+      __syncwarp();
       const uint32_t buf = ui & 1u, aph = (ui >> 1) & 1u;
       if (!mbar_wait(accf_bar(buf), aph, abort_flag, tmo)) {
         if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_ACC); *abort_flag = 1; }
         break;
       }
       tc_fence_after();
+      const int t_tile = (int)rank * CTA_TOKENS + 32 * q + lane;   // token within the unit's tile
+      const int64_t tok0 = (int64_t)inf.tt * TOKENS_PER_TILE + (int)rank * CTA_TOKENS + 32 * q;
+      const int64_t t = tok0 + lane;
+      const bool tvalid = t < P.m;
       const bool split = inf.nsl > 1;
-      float *part = nullptr;
+      float *part_row = nullptr;
       if (split)
-        part = P.partials + ((int64_t)inf.tt * total_slices + slice_ptr[inf.g] + inf.s) * (int64_t)(C::TT * 128);
+        part_row = P.partials +
+                   (((int64_t)inf.tt * total_slices + slice_ptr[inf.g] + inf.s) * P.part_rows + t_tile) * GROUP_FEATURES;
+      const bool touched = inf.e1 > inf.e0;
 #pragma unroll 1
-      for (int j = wq; j < QBLK; j += EPI_WARPS / 4) {
-        const int tok0 = 32 * j;  // first token of the block (its accumulator column)
-        const uint32_t taddr = tmem_base + ((uint32_t)(32 * q) << 16) + buf * C::BUF_COLS + tok0;
+      for (int h = 0; h < 2; ++h) {
+        const int c0 = 64 * part + 32 * h;  // first group row (accumulator column) of these 32
         float v[32];
-        if (inf.touched) {
-          tmem_ld32(taddr, v);
+        if (touched) {  // warp-uniform: the TMEM load is a warp-collective instruction
+          tmem_ld32(tmem_base + ((uint32_t)(32 * q) << 16) + buf * BUF_COLS + c0, v);
         } else {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = 0.f;
         }
         if (split) {
-          float4 *dst = reinterpret_cast<float4 *>(part + (int64_t)(32 * q + lane) * C::TT + tok0);
+          if (tvalid) {
+            float4 *dst = reinterpret_cast<float4 *>(part_row + c0);
 #pragma unroll
-          for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+            for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+          }
         } else {
-          emit32(v, bb, fl, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
+          const int fa = h == 0 ? fcol[0] : fcol[2], fb2 = h == 0 ? fcol[1] : fcol[3];
+          const uint32_t bs = smem_u32(bias_s + 32 * h);
+          float ya[16], yb[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            ya[i] = v[i];
+            yb[i] = v[16 + i];
+          }
+          if (fa >= 0) emit_run16<GELU, F32>(ya, bs, fa, tok0, P);
+          if (fb2 >= 0) emit_run16<GELU, F32>(yb, bs + 64, fb2, tok0, P);
         }
+        __syncwarp();
       }
-      // accumulator buffer and unit slot are free again
+      // the accumulator buffer is free again (the leader's MMAs wait for both CTAs' warps)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
-        mbar_arrive(acce_bar(buf));
-        mbar_arrive(unite_bar(slot));
-      }
-      if (split) {
-        // make the partial visible, take a ticket; the last slice sums all partials in order
-        __threadfence();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(episync_bar);
-        if (!mbar_wait(episync_bar, sync_phase, abort_flag, tmo)) {
-          if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_UNIT); *abort_flag = 1; }
-          break;
-        }
-        sync_phase ^= 1u;
-        if (ew == 0 && lane == 0) {
-          int32_t *tk = P.tickets + (int64_t)inf.tt * P.n_groups + inf.g;
-          const int old = atomicAdd(tk, 1);
-          const int last = old == inf.nsl - 1;
-          if (last) atomicExch(tk, 0);
-          *last_flag = last;
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(episync_bar);
-        if (!mbar_wait(episync_bar, sync_phase, abort_flag, tmo)) {
-          if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_UNIT); *abort_flag = 1; }
-          break;
-        }
-        sync_phase ^= 1u;
-        const int last = *last_flag;
-        if (last) {
-          __threadfence();
-          const float *base0 =
-              P.partials + ((int64_t)inf.tt * total_slices + slice_ptr[inf.g]) * (int64_t)(C::TT * 128);
-#pragma unroll 1
-          for (int j = wq; j < QBLK; j += EPI_WARPS / 4) {
-            const int tok0 = 32 * j;
-            float v[32];
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0.f;
-            for (int s2 = 0; s2 < inf.nsl; ++s2) {
-              const float4 *src = reinterpret_cast<const float4 *>(
-                  base0 + (int64_t)s2 * (C::TT * 128) + (int64_t)(32 * q + lane) * C::TT + tok0);
-#pragma unroll
-              for (int i = 0; i < 8; ++i) {
-                const float4 t = __ldcg(src + i);
-                v[4 * i] += t.x; v[4 * i + 1] += t.y; v[4 * i + 2] += t.z; v[4 * i + 3] += t.w;
-              }
-            }
-            emit32(v, bb, fl, (int64_t)inf.tt * C::TT + tok0, P, epi_tile);
-          }
-        }
+        if (leader) mbar_arrive(acce_bar(buf));
+        else mbar_arrive_cluster(mapa_rank(acce_bar(buf), 0));
       }
       ++ui;
     }
@@ -589,37 +643,140 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const LinearParams P)
   // ---------------------------------------------------------------- teardown
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // no signal, copy or MMA of the pair is still aimed at either CTA
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem_base, 512);
+  if (warp == 1) tmem_dealloc_pair(tmem_base, 512);
 }
+
+// Split units: Y = act(sum over the slices, in slice order, of the partial sums + bias). One thread
+// per 8 consecutive group rows of one token of one (token tile, group) with more than one slice.
+__global__ void __launch_bounds__(256) split_reduce_kernel(const ReduceParams R) {
+  __shared__ int sp[MAX_GROUPS + 1];
+  __shared__ int nslice[MAX_GROUPS];
+  const int32_t *gent = R.sched + SCHED_HDR_INTS;
+  const int32_t *gpan = R.sched + sched_gpan_offset_ints(R.n_groups);
+  if (threadIdx.x < 32) {
+    int run = 0;
+    const int lane = threadIdx.x;
+    for (int base = 0; base < R.n_groups; base += 32) {
+      const int g = base + lane;
+      int c = 0;
+      if (g < R.n_groups) {
+        const int cnt = gent[g + 1] - gent[g];
+        c = cnt <= 0 ? 1 : (cnt + R.S - 1) / R.S;
+        nslice[g] = c;
+      }
+      int incl = c;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int tv = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += tv;
+      }
+      if (g < R.n_groups) sp[g] = run + incl - c;
+      run += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) sp[R.n_groups] = run;
+  }
+  __syncthreads();
+  const int total_slices = sp[R.n_groups];
+  constexpr int VPR = GROUP_FEATURES / 8;  // 8-row pieces per token
+  const int64_t items = (int64_t)R.n_tt * R.n_groups * R.part_rows * VPR;
+  for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < items; idx += (int64_t)gridDim.x * blockDim.x) {
+    const int v = (int)(idx % VPR);
+    int64_t rest = idx / VPR;
+    const int row = (int)(rest % R.part_rows);
+    rest /= R.part_rows;
+    const int g = (int)(rest % R.n_groups);
+    const int tt = (int)(rest / R.n_groups);
+    const int nsl = nslice[g];
+    if (nsl <= 1) continue;
+    const int64_t t = (int64_t)tt * TOKENS_PER_TILE + row;
+    if (t >= R.m) continue;
+    const int c0 = 8 * v;
+    const int panel = gpan[(int64_t)g * MAX_GROUP_PANELS + c0 / R.bn];
+    if (panel < 0) continue;
+    float acc[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+    const float *p0 = R.partials + (((int64_t)tt * total_slices + sp[g]) * R.part_rows + row) * GROUP_FEATURES + c0;
+    for (int s = 0; s < nsl; ++s) {
+      const float4 *p = reinterpret_cast<const float4 *>(p0 + (int64_t)s * R.part_rows * GROUP_FEATURES);
+      const float4 a = __ldcg(p), b = __ldcg(p + 1);
+      acc[0] += a.x; acc[1] += a.y; acc[2] += a.z; acc[3] += a.w;
+      acc[4] += b.x; acc[5] += b.y; acc[6] += b.z; acc[7] += b.w;
+    }
+    {
+      const int f0 = panel * R.bn + c0 % R.bn;
+      float b8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) b8[i] = R.bias != nullptr ? R.bias[f0 + i] : 0.f;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] = R.gelu ? gelu_erf(acc[i] + b8[i]) : acc[i] + b8[i];
+      if (R.y_f32) {
+        float *dst = static_cast<float *>(R.Y) + t * R.ldy + f0;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) dst[i] = acc[i];
+      } else {
+        uint16_t *dst = static_cast<uint16_t *>(R.Y) + t * R.ldy + f0;
+#pragma unroll
+        for (int i = 0; i < 8; i += 2) {
+          uint32_t w = pack_bf16x2(acc[i], acc[i + 1]);
+          if (R.R != nullptr) {
+            const uint16_t *rp = R.R + t * R.ldr + f0;
+            const float lo = __uint_as_float(w << 16) + __uint_as_float((uint32_t)rp[i] << 16);
+            const float hi = __uint_as_float(w & 0xffff0000u) + __uint_as_float((uint32_t)rp[i + 1] << 16);
+            w = pack_bf16x2(lo, hi);
+          }
+          dst[i] = (uint16_t)(w & 0xffffu);
+          dst[i + 1] = (uint16_t)(w >> 16);
+        }
+      }
+    }
+  }
+}
+
+}  // namespace
 
 // ------------------------------------------------------------------------------------ host side
 
-template <int BK>
-int smem_bytes() { return Smem<BK>::BYTES; }
-
-template <int BK>
-cudaError_t launch_linear_t(const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s) {
+cudaError_t launch_linear(const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
+                          cudaStream_t s) {
   static bool attr_done[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(bsr_linear_kernel<BK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         Smem<BK>::BYTES);
-    if (e != cudaSuccess) return e;
+    for (auto k : {bsr_linear_kernel<false, false>, bsr_linear_kernel<true, false>, bsr_linear_kernel<false, true>,
+                   bsr_linear_kernel<true, true>}) {
+      cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem::BYTES);
+      if (e != cudaSuccess) return e;
+    }
     attr_done[dev] = true;
   }
-  bsr_linear_kernel<BK><<<grid, NUM_THREADS, Smem<BK>::BYTES, s>>>(tmX, P);
+  auto kern = P.gelu ? (P.y_f32 ? bsr_linear_kernel<true, true> : bsr_linear_kernel<true, false>)
+                     : (P.y_f32 ? bsr_linear_kernel<false, true> : bsr_linear_kernel<false, false>);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = Smem::BYTES;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kern, tmX, tmW, P);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
-cudaError_t launch_linear(int bk, const CUtensorMap &tmX, const LinearParams &P, int grid, cudaStream_t s) {
-  switch (bk) {
-    case 16: return launch_linear_t<16>(tmX, P, grid, s);
-    case 32: return launch_linear_t<32>(tmX, P, grid, s);
-    case 64: return launch_linear_t<64>(tmX, P, grid, s);
-    default: return cudaErrorInvalidValue;
-  }
+cudaError_t launch_split_reduce(const ReduceParams &R, int64_t threads, cudaStream_t s) {
+  int64_t blocks = (threads + 255) / 256;
+  if (blocks < 1) blocks = 1;
+  if (blocks > 4096) blocks = 4096;
+  split_reduce_kernel<<<(unsigned)blocks, 256, 0, s>>>(R);
+  return cudaGetLastError();
 }
 
 }  // namespace lpvit

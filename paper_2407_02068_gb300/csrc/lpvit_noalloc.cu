@@ -51,12 +51,10 @@ extern "C" lpvit_status lpvit_bsr_linear_noalloc(const lpvit_bsr *bsr, const voi
   void *ws = nullptr;
   const lpvit_status st = noalloc_scratch(&ws);
   if (st != LPVIT_OK) return st;
-  // The array keeps whatever the previous call left; the counters, error word and arrival
-  // tickets at its start must begin at zero (partial sums are always written before they are
-  // read), so clear them on the caller's stream.
-  const int64_t n_tt = (m + lpvit::TOKENS_PER_TILE - 1) / lpvit::TOKENS_PER_TILE;
-  const int64_t ng = (bsr->n + lpvit::GROUP_FEATURES - 1) / lpvit::GROUP_FEATURES;
-  size_t clear = sizeof(lpvit::Control) + (size_t)((n_tt * ng * 4 + 255) / 256 * 256);
+  // The array keeps whatever the previous call left; the work-queue counters and the error word
+  // at its start must begin at zero (partial sums are always written before they are read), so
+  // clear them on the caller's stream.
+  size_t clear = sizeof(lpvit::Control);
   if (clear > need) clear = need;
   if (cudaMemsetAsync(ws, 0, clear, static_cast<cudaStream_t>(stream)) != cudaSuccess) return LPVIT_ERR_CUDA;
   return gelu ? lpvit_bsr_linear_gelu(bsr, X, m, ldx, bias, Y, ldy, y_dtype, ws, LPVIT_NOALLOC_SCRATCH_BYTES, stream)

@@ -6,13 +6,13 @@
 // plan kernel (one CTA): per row panel r (bn rows), cnt[r] = number of kept blocks (warp
 //   reductions); row_ptr = exclusive prefix sum of cnt (warp-shuffle scan + a scan of warp
 //   totals); col_idx = kept block columns of each panel in ascending order (ballot compaction);
-//   work list: panels are grouped 128 output features (128 / bn panels) at a time, greedily by
-//   overlap of their kept block columns (one warp; consecutive panels when that is not better);
-//   for every group, one entry per block column where any panel of the group keeps a block, with
-//   that column's block index in each panel (or -1). The GEMM walks these entries.
+//   work list: the GEMM covers the weight in tiles of 256 output features by 64 input columns (a
+//   "chunk"); panels are grouped 256 features (256 / bn panels) at a time, greedily by overlap of
+//   the chunks in which they keep blocks (one warp; consecutive panels when that is not better);
+//   for every group, one entry per chunk where any panel of the group keeps a block.
 // copy kernel (grid-stride): blocks[t] = W[r*bn:(r+1)*bn, j*bk:(j+1)*bk], 16-byte vector copies,
-//   bits unchanged; then the weight stream, the same bits once more, entry by entry as the 128-row
-//   group tiles the GEMM's MMAs read (rows of removed row panels zero, 16-byte chunks swizzled).
+//   bits unchanged; then the weight stream, entry by entry: the group's 256 rows over the chunk's
+//   64 columns, row-major, removed blocks and empty slots zero.
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -66,8 +66,8 @@ __device__ int block_exclusive_scan(int *v, int count, int *warp_tot) {
 // row panels and GROUPING_MAX_WORDS words of per-panel column bitmaps.
 constexpr int GROUPING_MAX_PANELS = 1024;
 constexpr int GROUPING_MAX_WORDS = 8192;
-__host__ __device__ inline bool grouping_on(int np, int kb, int gb) {
-  const int W = (kb + 31) / 32;
+__host__ __device__ inline bool grouping_on(int np, int kc, int gb) {
+  const int W = (kc + 31) / 32;
   return gb >= 2 && np <= GROUPING_MAX_PANELS && (int64_t)np * W <= GROUPING_MAX_WORDS;
 }
 
@@ -78,9 +78,9 @@ __device__ __forceinline__ int warp_sum(int v) {
 }
 
 // Group the row panels, one warp. A group starts with the unassigned panel keeping the most blocks
-// and then takes, gb - 1 times, the unassigned panel that adds the fewest block columns to the
-// group's union (ties to the lower panel index). The work list has one entry per block column of
-// the union, so overlapping panels make fewer entries. The grouping is kept only if it gives fewer
+// and then takes, gb - 1 times, the unassigned panel that adds the fewest chunks to the group's
+// union (ties to the lower panel index). The work list has one entry per chunk of the union, so
+// overlapping panels make fewer entries. The grouping is kept only if it gives fewer
 // entries than consecutive panels; gpan is written either way.
 __device__ void group_panels(const unsigned *__restrict__ bits, int W, const int *__restrict__ kcnt, int np,
                              int gb, int ng, unsigned *U, int *asg, int32_t *__restrict__ gpan) {
@@ -232,27 +232,39 @@ __device__ void group_panels_fast(const unsigned *__restrict__ bits, int W, cons
   }
 }
 
+// Does panel r keep a block in chunk c (input columns [64 c, 64 c + 64))?
+__device__ __forceinline__ bool chunk_kept(const uint8_t *__restrict__ mask, int r, int c, int kb, int bpc) {
+  bool any = false;
+  for (int q = 0; q < bpc; ++q) {
+    const int j = c * bpc + q;
+    any |= j < kb && mask[(int64_t)r * kb + j] != 0;
+  }
+  return any;
+}
+
 // The plan of one weight, computed by one CTA of PLAN_THREADS threads (plan_smem: plan_smem_bytes).
 __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int n, int k, int bn, int bk,
                                           int32_t *__restrict__ row_ptr, int32_t *__restrict__ col_idx, int cap,
                                           int32_t *__restrict__ sched, int *plan_smem) {
   const int np = n / bn, kb = k / bk;
-  const int gb = GROUP_FEATURES / bn;  // row panels per group
+  const int kc = sched_chunks(k);          // chunks of CHUNK_COLS input columns
+  const int bpc = CHUNK_COLS / bk;         // blocks per chunk (bk divides CHUNK_COLS)
+  const int gb = GROUP_FEATURES / bn;      // row panels per group
   const int ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
-  const int W = (kb + 31) / 32;    // words of a panel's column bitmap
-  const bool grouping = grouping_on(np, kb, gb);
+  const int W = (kc + 31) / 32;            // words of a panel's chunk bitmap
+  const bool grouping = grouping_on(np, kc, gb);
   int *cnt = plan_smem;            // [np + 1]
   int *gcnt = cnt + np + 1;        // [ng + 1]
   int *warp_tot = gcnt + ng + 1;   // [33]
   int *kcnt = warp_tot + 33;       // [np] kept blocks per panel
-  unsigned *bits = reinterpret_cast<unsigned *>(kcnt + np);  // grouping: [np][W] column bitmaps
+  unsigned *bits = reinterpret_cast<unsigned *>(kcnt + np);  // grouping: [np][W] chunk bitmaps
   unsigned *U = bits + (grouping ? np * W : 0);              // grouping: [W] union of a group
   int *asg = reinterpret_cast<int *>(U + (grouping ? W : 0));  // grouping: [np] assigned flags
   int32_t *gpan = sched + sched_gpan_offset_ints(ng);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const unsigned lt = (1u << lane) - 1u;
 
-  // 1. kept blocks per panel
+  // 1. kept blocks per panel; chunk bitmaps for the grouping
   for (int r = warp; r < np; r += PLAN_WARPS) {
     int c = 0;
     for (int j = lane; j < kb; j += 32) c += mask[(int64_t)r * kb + j] != 0;
@@ -263,9 +275,9 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
       kcnt[r] = c;
     }
     if (grouping)
-      for (int base = 0; base < kb; base += 32) {
-        const int j = base + lane;
-        const unsigned bal = __ballot_sync(0xffffffffu, j < kb && mask[(int64_t)r * kb + j] != 0);
+      for (int base = 0; base < kc; base += 32) {
+        const int ch = base + lane;
+        const unsigned bal = __ballot_sync(0xffffffffu, ch < kc && chunk_kept(mask, r, ch, kb, bpc));
         if (lane == 0) bits[r * W + base / 32] = bal;
       }
   }
@@ -305,18 +317,17 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
     }
   }
   __syncthreads();
-  // 4a. entries per group: block columns where any panel of the group keeps a block
+  // 4a. entries per group: chunks where any panel of the group keeps a block
   for (int g = warp; g < ng; g += PLAN_WARPS) {
     int c = 0;
-    for (int base = 0; base < kb; base += 32) {
-      const int j = base + lane;
-      unsigned any = 0;
-      for (int p = 0; p < gb; ++p) {
+    for (int base = 0; base < kc; base += 32) {
+      const int ch = base + lane;
+      bool any = false;
+      for (int p = 0; p < gb && ch < kc; ++p) {
         const int r = gpan[g * MAX_GROUP_PANELS + p];
-        const bool keep = r >= 0 && j < kb && mask[(int64_t)r * kb + j] != 0;
-        any |= __ballot_sync(0xffffffffu, keep);
+        if (r >= 0) any |= chunk_kept(mask, r, ch, kb, bpc);
       }
-      c += __popc(any);
+      c += __popc(__ballot_sync(0xffffffffu, any));
     }
     if (lane == 0) gcnt[g] = c;
   }
@@ -335,49 +346,22 @@ __device__ __forceinline__ void plan_body(const uint8_t *__restrict__ mask, int 
     sched[5] = k;
     sched[6] = bn;
     sched[7] = bk;
-    for (int i = 8; i < SCHED_HDR_INTS; ++i) sched[i] = 0;
+    sched[8] = SCHED_VERSION;
+    for (int i = 9; i < SCHED_HDR_INTS; ++i) sched[i] = 0;
   }
-  // 4b. entries: j | (panel mask << 16), then the block index of each panel of the group (or -1),
-  //     then the entry's stream tile (its own index)
+  // 4b. entries: the chunk index, in ascending order within each group
   for (int g = warp; g < ng; g += PLAN_WARPS) {
     int e_run = gcnt[g];
-    int p_run[MAX_GROUP_PANELS];
-    int rr[MAX_GROUP_PANELS];  // the panel of each slot, or -1
-#pragma unroll
-    for (int p = 0; p < MAX_GROUP_PANELS; ++p) {
-      rr[p] = p < gb ? gpan[g * MAX_GROUP_PANELS + p] : -1;
-      p_run[p] = rr[p] >= 0 ? cnt[rr[p]] : 0;
-    }
-    for (int base = 0; base < kb; base += 32) {
-      const int j = base + lane;
-      unsigned bal[MAX_GROUP_PANELS];
-      unsigned any = 0;
-#pragma unroll
-      for (int p = 0; p < MAX_GROUP_PANELS; ++p) {
-        const int r = rr[p];
-        const bool keep = r >= 0 && j < kb && mask[(int64_t)r * kb + j] != 0;
-        bal[p] = __ballot_sync(0xffffffffu, keep);
-        any |= bal[p];
+    for (int base = 0; base < kc; base += 32) {
+      const int ch = base + lane;
+      bool any = false;
+      for (int p = 0; p < gb && ch < kc; ++p) {
+        const int r = gpan[g * MAX_GROUP_PANELS + p];
+        if (r >= 0) any |= chunk_kept(mask, r, ch, kb, bpc);
       }
-      unsigned pm = 0;
-#pragma unroll
-      for (int p = 0; p < MAX_GROUP_PANELS; ++p) pm |= ((bal[p] >> lane) & 1u) << p;
-      if ((any >> lane) & 1u) {
-        const int ei = e_run + __popc(any & lt);
-        int32_t *e = entries + (int64_t)ei * ENTRY_INTS;
-#pragma unroll
-        for (int p = 0; p < MAX_GROUP_PANELS; ++p) {
-          const bool keep = (bal[p] >> lane) & 1u;
-          e[1 + p] = keep ? p_run[p] + __popc(bal[p] & lt) : -1;
-        }
-        e[0] = (int32_t)((unsigned)j | (pm << 16));
-#pragma unroll
-        for (int q = 1 + MAX_GROUP_PANELS; q < ENTRY_INTS; ++q) e[q] = 0;
-        e[ENTRY_TILE_WORD] = ei;
-      }
-      e_run += __popc(any);
-#pragma unroll
-      for (int p = 0; p < MAX_GROUP_PANELS; ++p) p_run[p] += __popc(bal[p]);
+      const unsigned bal = __ballot_sync(0xffffffffu, any);
+      if (any) entries[e_run + __popc(bal & lt)] = ch;
+      e_run += __popc(bal);
     }
   }
 }
@@ -421,20 +405,23 @@ __device__ __forceinline__ void copy_body(const uint16_t *__restrict__ W, int n,
   }
 }
 
-// Weight-stream tiles of entries e = cta, cta + ncta, ... of one weight (after its plan).
-__device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int n, int k, int bn, int bk,
-                                            const int32_t *__restrict__ sched, int cta, int ncta) {
-  const int kb = k / bk, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
+// Weight-stream tiles of entries e = cta, cta + ncta, ... of one weight (after its plan): the
+// group's 256 rows over the entry's 64 columns, row-major, 16-byte vectors; zero where the block
+// is removed, where the slot has no panel and beyond column k.
+__device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, const uint8_t *__restrict__ mask, int n,
+                                            int k, int bn, int bk, const int32_t *__restrict__ sched, int cta,
+                                            int ncta) {
+  const int kb = k / bk, kc = sched_chunks(k), ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
   if (sched[1] != ng || sched[3] != 0) return;  // not this shape's plan, or blocks overflowed
   const int total = sched[2];
-  const int row_bytes = 2 * bk, cpr = row_bytes / 16, chunks = GROUP_FEATURES * cpr;
-  const int lcpr = __ffs(cpr) - 1, lbn = __ffs(bn) - 1;  // bk and bn are powers of 2
-  const int tile_bytes = stream_tile_bytes(bk);
-  const int64_t max_tiles = sched_stream_tiles(ng, kb);
+  constexpr int VPR = CHUNK_COLS / 8;             // 16-byte vectors per tile row
+  constexpr int VECS = GROUP_FEATURES * VPR;
+  const int lbn = __ffs(bn) - 1, lbk = __ffs(bk) - 1;  // bn and bk are powers of 2
+  const int64_t max_tiles = sched_stream_tiles(ng, kc);
   const int32_t *gent = sched + SCHED_HDR_INTS;
   const int32_t *gpan = sched + sched_gpan_offset_ints(ng);
   const int32_t *ent = sched + sched_entries_offset_ints(ng);
-  uint8_t *stream = reinterpret_cast<uint8_t *>(const_cast<int32_t *>(sched)) + sched_stream_offset_bytes(ng, kb);
+  uint8_t *stream = reinterpret_cast<uint8_t *>(const_cast<int32_t *>(sched)) + sched_stream_offset_bytes(ng, kc);
   for (int e = cta; e < total; e += ncta) {
     int lo = 0, hi = ng - 1;  // largest g with gent[g] <= e (the group holding entry e)
     while (lo < hi) {
@@ -442,32 +429,29 @@ __device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, int 
       if (gent[mid] <= e) lo = mid;
       else hi = mid - 1;
     }
-    const int g = lo;
-    const int32_t *ep = ent + (int64_t)e * ENTRY_INTS;
-    const int j = ep[0] & 0xffff;
-    const uint32_t pm = (uint32_t)ep[0] >> 16;
-    const int t = ep[ENTRY_TILE_WORD];
-    if (j >= kb || t < 0 || (int64_t)t >= max_tiles) continue;
-    uint8_t *tile = stream + (int64_t)t * tile_bytes;
-    for (int v = threadIdx.x; v < chunks; v += blockDim.x) {
-      const int r = v >> lcpr, c = v & (cpr - 1), slot = r >> lbn;
+    const int g = lo, ch = ent[e];
+    if (ch < 0 || ch >= kc || (int64_t)e >= max_tiles) continue;
+    int4 *tile = reinterpret_cast<int4 *>(stream + (int64_t)e * stream_tile_bytes());
+    for (int v = threadIdx.x; v < VECS; v += blockDim.x) {
+      const int r = v / VPR, cv = v % VPR, slot = r >> lbn;
       const int panel = gpan[g * MAX_GROUP_PANELS + slot];
+      const int col = ch * CHUNK_COLS + cv * 8;
       // the output feature of group row r (none for an empty slot)
       const int row = panel >= 0 ? (panel << lbn) + (r & (bn - 1)) : -1;
       int4 val = make_int4(0, 0, 0, 0);
-      if (((pm >> slot) & 1u) && row >= 0 && row < n)
-        val = __ldg(reinterpret_cast<const int4 *>(W + (int64_t)row * k + (int64_t)j * bk + c * 8));
-      reinterpret_cast<int4 *>(tile + r * row_bytes)[c ^ stream_chunk_swizzle(r, row_bytes)] = val;
+      if (row >= 0 && row < n && col < k && mask[(int64_t)panel * kb + (col >> lbk)] != 0)
+        val = __ldg(reinterpret_cast<const int4 *>(W + (int64_t)row * k + col));
+      tile[v] = val;
     }
   }
 }
 
 __global__ void __launch_bounds__(128)
-copy_blocks_kernel(const uint16_t *__restrict__ W, int n, int k, int bn, int bk,
+copy_blocks_kernel(const uint16_t *__restrict__ W, const uint8_t *__restrict__ mask, int n, int k, int bn, int bk,
                    const int32_t *__restrict__ row_ptr, const int32_t *__restrict__ col_idx, int cap,
                    uint16_t *__restrict__ blocks, const int32_t *__restrict__ sched) {
   copy_body(W, n, k, bn, bk, row_ptr, col_idx, cap, blocks, blockIdx.x, gridDim.x);
-  stream_body(W, n, k, bn, bk, sched, blockIdx.x, gridDim.x);
+  stream_body(W, mask, n, k, bn, bk, sched, blockIdx.x, gridDim.x);
 }
 
 // Several weights at once: every CTA takes its share of every job's kept blocks and stream tiles.
@@ -476,15 +460,16 @@ __global__ void __launch_bounds__(128) copy_many_kernel(const __grid_constant__ 
     const PackJob &w = J.job[j];
     if (w.cap > 0)
       copy_body(w.W, w.n, w.k, w.bn, w.bk, w.row_ptr, w.col_idx, w.cap, w.blocks, blockIdx.x, gridDim.x);
-    stream_body(w.W, w.n, w.k, w.bn, w.bk, w.sched, blockIdx.x, gridDim.x);
+    stream_body(w.W, w.mask, w.n, w.k, w.bn, w.bk, w.sched, blockIdx.x, gridDim.x);
   }
 }
 
 size_t plan_smem_bytes(int n, int k, int bn, int bk) {
-  const int np = n / bn, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES, kb = k / bk;
-  const int W = (kb + 31) / 32;
+  (void)bk;
+  const int np = n / bn, ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES, kc = sched_chunks(k);
+  const int W = (kc + 31) / 32;
   size_t words = (size_t)np + 1 + ng + 1 + 33 + np;
-  if (grouping_on(np, kb, GROUP_FEATURES / bn)) words += (size_t)np * W + W + np;
+  if (grouping_on(np, kc, GROUP_FEATURES / bn)) words += (size_t)np * W + W + np;
   return sizeof(int) * words;
 }
 
@@ -497,7 +482,7 @@ cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int bn
   const int max_blocks = (n / bn) * (k / bk);
   int grid = max_blocks < num_sms * 16 ? max_blocks : num_sms * 16;
   if (grid < 1) grid = 1;
-  copy_blocks_kernel<<<grid, 128, 0, s>>>(static_cast<const uint16_t *>(W), n, k, bn, bk, row_ptr, col_idx, cap,
+  copy_blocks_kernel<<<grid, 128, 0, s>>>(static_cast<const uint16_t *>(W), mask, n, k, bn, bk, row_ptr, col_idx, cap,
                                          static_cast<uint16_t *>(blocks), sched);
   return cudaGetLastError();
 }

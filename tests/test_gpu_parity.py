@@ -112,33 +112,53 @@ def test_pack_bit_exact(lp, n, k, b, sp):
     assert np.array_equal(got, bl)
 
 
+GROUP = 256    # output features of a work unit
+CHUNK = 64     # input columns of a work-list entry
+SLOTS = 16     # group table width
+
+
 def _decode_sched(w):
-    """Header, group entry pointers, entries and the group table (row panel of every slot, or -1)."""
+    """Header, group entry pointers, entries (chunk index each) and the group table (row panel of
+    every slot, or -1)."""
     raw = w.sched.cpu().numpy().view(np.int32)
     ng = int(raw[1])
     gent = raw[16:16 + ng + 1]
-    gpan = raw[16 + ng + 1:16 + ng + 1 + 8 * ng].reshape(ng, 8)
+    gpan = raw[16 + ng + 1:16 + ng + 1 + SLOTS * ng].reshape(ng, SLOTS)
     off = _entries_offset(ng)
-    ent = raw[off:off + int(gent[-1]) * 12].reshape(-1, 12)
+    ent = raw[off:off + int(gent[-1])]
     return raw[:16], gent, ent, gpan
 
 
 def _entries_offset(ng):
-    return (16 + ng + 1 + 8 * ng + 3) // 4 * 4
+    return (16 + ng + 1 + SLOTS * ng + 3) // 4 * 4
 
 
-def _grouping(M, bn):
-    """The plan's grouping rule restated: a group starts with the unassigned panel keeping the most
-    blocks, then takes the unassigned panel adding the fewest block columns to the group's union
-    (ties to the lower index); kept only if it has fewer entries than consecutive panels, and only
-    for up to 1024 panels and 8192 bitmap words."""
+def _chunk_bits(M, bk):
+    """[panels, chunks]: does the panel keep a block in each 64-column chunk?"""
     npan, kb = M.shape
-    gb = 128 // bn
+    bpc = CHUNK // bk
+    kc = -(-kb * bk // CHUNK)
+    C = np.zeros((npan, kc), dtype=bool)
+    for c in range(kc):
+        C[:, c] = M[:, c * bpc:(c + 1) * bpc].any(axis=1)
+    return C
+
+
+def _grouping(M, bn, bk):
+    """The plan's grouping rule restated: a group starts with the unassigned panel keeping the most
+    blocks, then takes the unassigned panel adding the fewest chunks to the group's union (ties to
+    the lower index); kept only if it has fewer entries than consecutive panels, and only for up to
+    1024 panels and 8192 bitmap words."""
+    npan, kb = M.shape
+    C = _chunk_bits(M, bk)
+    kc = C.shape[1]
+    gb = GROUP // bn
     ng = -(-npan // gb)
-    ident = [[g * gb + p if p < gb and g * gb + p < npan else -1 for p in range(8)] for g in range(ng)]
-    if not (gb >= 2 and npan <= 1024 and npan * ((kb + 31) // 32) <= 8192):
+    ident = [[g * gb + p if p < gb and g * gb + p < npan else -1 for p in range(SLOTS)] for g in range(ng)]
+    if not (gb >= 2 and npan <= 1024 and npan * ((kc + 31) // 32) <= 8192):
         return ident
-    rows = [set(np.nonzero(M[r])[0].tolist()) for r in range(npan)]
+    rows = [set(np.nonzero(C[r])[0].tolist()) for r in range(npan)]
+    kept = [int(M[r].sum()) for r in range(npan)]
     asg, table = [False] * npan, []
     for g in range(ng):
         t, U = [], set()
@@ -147,11 +167,11 @@ def _grouping(M, bn):
             if not cand:
                 t.append(-1)
                 continue
-            pick = min(cand, key=(lambda p: (-len(rows[p]), p)) if sl == 0 else (lambda p: (len(rows[p] - U), p)))
+            pick = min(cand, key=(lambda p: (-kept[p], p)) if sl == 0 else (lambda p: (len(rows[p] - U), p)))
             asg[pick] = True
             t.append(pick)
             U |= rows[pick]
-        table.append(t + [-1] * (8 - gb))
+        table.append(t + [-1] * (SLOTS - gb))
 
     def entries(tab):
         return sum(len(set().union(*[rows[r] for r in t if r >= 0])) for t in tab)
@@ -172,47 +192,44 @@ def test_work_list_covers_every_kept_block_once(lp, n, k, b):
     w = lp.pack_bsr(W, mask, b, count=True)
     hdr, gent, ent, gpan = _decode_sched(w)
     bn, bk = _sides(b)
-    assert (int(hdr[4]), int(hdr[5]), int(hdr[6]), int(hdr[7])) == (n, k, bn, bk)
-    gb = 128 // bn
+    assert (int(hdr[4]), int(hdr[5]), int(hdr[6]), int(hdr[7]), int(hdr[8])) == (n, k, bn, bk, 2)
+    gb = GROUP // bn
     M = mask.cpu().numpy()
+    C = _chunk_bits(M, bk)
     # the group table: every row panel in exactly one slot, as the grouping rule picks them
     used = sorted(int(r) for r in gpan.ravel() if r >= 0)
     assert used == list(range(n // bn)) and np.all(gpan[:, gb:] == -1)
-    assert gpan.tolist() == _grouping(M, bn)
-    rp, ci, _ = oracle.pack(_bits(W), M, b)
-    seen = set()
+    assert gpan.tolist() == _grouping(M, bn, bk)
+    # entries: per group the chunks where one of its panels keeps a block, ascending; so every
+    # kept block lies in exactly one entry (its panel's group, its column's chunk)
+    covered = np.zeros_like(M, dtype=np.int32)
     for g in range(int(hdr[1])):
-        js = []
-        for e in ent[gent[g]:gent[g + 1]]:
-            j, pm = int(e[0]) & 0xFFFF, (int(e[0]) >> 16) & 0xFFFF
-            js.append(j)
-            for p in range(gb):
-                r = int(gpan[g, p])
-                if (pm >> p) & 1:
-                    t = int(e[1 + p])
-                    assert r >= 0 and M[r, j] and ci[t] == j and rp[r] <= t < rp[r + 1]
-                    seen.add(t)
-                else:
-                    assert e[1 + p] == -1 and (r < 0 or not M[r, j])
-        assert js == sorted(set(js))
+        cs = [int(c) for c in ent[gent[g]:gent[g + 1]]]
         panels = [int(r) for r in gpan[g, :gb] if r >= 0]
-        want = sorted(set(np.nonzero(M[panels].any(axis=0))[0].tolist())) if panels else []
-        assert js == want
-    assert seen == set(range(len(ci)))
+        want = sorted(np.nonzero(C[panels].any(axis=0))[0].tolist()) if panels else []
+        assert cs == want
+        for c in cs:
+            for r in panels:
+                j0 = c * CHUNK // bk
+                covered[r, j0:j0 + CHUNK // bk] += 1
+    assert np.all(covered[M != 0] == 1)
 
 
 @pytest.mark.parametrize("b", [32, 16, (64, 32)])
 def test_grouping_pairs_panels_with_the_same_columns(lp, b):
-    """Row panels of two kinds keep blocks in two disjoint sets of block columns (even panels in
-    A, odd panels in B). Consecutive groups would mix the kinds and need |A u B| entries each; the
-    plan's grouping puts panels of one kind together, so each group needs |A| or |B| entries. The
-    linear on that work list still matches the oracle."""
+    """Row panels of two kinds keep blocks in two disjoint sets of chunks (even panels in A, odd
+    panels in B). Consecutive groups would mix the kinds and need |A u B| entries each; the plan's
+    grouping puts panels of one kind together, so each group needs |A| or |B| entries. The linear on
+    that work list still matches the oracle."""
     bn, bk = _sides(b)
     n, k = 1024, 512
-    npan, kb = n // bn, k // bk
+    npan, kb, kc = n // bn, k // bk, k // CHUNK
     rng = np.random.default_rng(77)
-    cols = rng.permutation(kb)
-    A, B = np.sort(cols[:kb // 3]), np.sort(cols[kb // 3:kb // 3 + kb // 4])
+    chunks = rng.permutation(kc)
+    CA, CB = np.sort(chunks[:kc // 3]), np.sort(chunks[kc // 3:kc // 3 + kc // 4])
+    bpc = CHUNK // bk
+    A = np.concatenate([np.arange(c * bpc, (c + 1) * bpc) for c in CA])
+    B = np.concatenate([np.arange(c * bpc, (c + 1) * bpc) for c in CB])
     M = np.zeros((npan, kb), np.uint8)
     M[0::2, A] = 1
     M[1::2, B] = 1
@@ -220,51 +237,46 @@ def test_grouping_pairs_panels_with_the_same_columns(lp, b):
     mask = torch.from_numpy(M).cuda()
     w = lp.pack_bsr(W, mask, b, count=True)
     hdr, gent, ent, gpan = _decode_sched(w)
-    gb = 128 // bn
-    assert gpan.tolist() == _grouping(M, bn)
+    gb = GROUP // bn
+    assert gpan.tolist() == _grouping(M, bn, bk)
     for g in range(int(hdr[1])):
         kinds = {int(r) % 2 for r in gpan[g, :gb] if r >= 0}
         assert len(kinds) == 1                       # one kind of panel per group
     ng = npan // gb
-    assert int(gent[-1]) == (ng // 2) * (len(A) + len(B))
+    assert int(gent[-1]) == (ng // 2) * (len(CA) + len(CB))
     Y = lp.bsr_linear(w, X, bias, out_dtype=torch.float32)
     ref = _oracle(X, W, mask, b, bias)
     assert _norm_err(Y.cpu().double().numpy(), ref) <= TIGHT_TOL
 
 
 def _check_weight_stream(w, W, mask):
-    """The work list's weight stream: entry by entry, the 128-row tile of the entry's group at its
-    block column (W's rows there, removed row panels zero), tiles contiguous in entry order,
-    16-byte chunk c of tile row r stored at chunk c ^ ((r * rowbytes >> 7) & (rowbytes / 16 - 1))."""
+    """The work list's weight stream: entry by entry, the 256-row tile of the entry's group over its
+    64-column chunk, row-major: row r holds W[feature of group row r] over the chunk where that
+    block is kept, zero where it is removed, where the slot has no panel and beyond column k."""
     n, k, bn, bk = w.n, w.k, w.bn, w.bk
     hdr, gent, ent, gpan = _decode_sched(w)
-    ng, kb = int(hdr[1]), k // bk
-    mp = 128
-    rb, cpr = 2 * bk, 2 * bk // 16
+    ng, kc = int(hdr[1]), -(-k // CHUNK)
     raw = w.sched.cpu().numpy().view(np.uint8)
-    ent_end = 4 * (_entries_offset(ng) + ng * kb * 12)
+    ent_end = 4 * (_entries_offset(ng) + ng * kc)
     stream = raw[(ent_end + 1023) // 1024 * 1024:]
     Wb = _bits(W).reshape(n, k)
     M = mask.cpu().numpy()
-    t_next = 0
+    # the expected tile of group g at chunk c, built from the definition
+    feat = np.full(GROUP, -1)
     for g in range(ng):
-        for e in ent[gent[g]:gent[g + 1]]:
-            j, pm = int(e[0]) & 0xFFFF, (int(e[0]) >> 16) & 0xFFFF
-            assert int(e[9]) == t_next
-            panels = [q for q in range(128 // mp) if any((pm >> ((q * mp + r) // bn)) & 1 for r in range(0, mp, bn))]
-            for i, q in enumerate(panels):
-                tile = stream[(t_next + i) * mp * rb:(t_next + i + 1) * mp * rb].reshape(mp, cpr, 16)
-                for r in range(mp):
-                    panel = int(gpan[g, (q * mp + r) // bn])
-                    row = panel * bn + (q * mp + r) % bn   # the output feature of group row r
-                    kept = (pm >> ((q * mp + r) // bn)) & 1
-                    want = Wb[row, j * bk:(j + 1) * bk] if kept else np.zeros(bk, np.uint16)
-                    if kept:
-                        assert M[row // bn, j]
-                    sw = ((r * rb) >> 7) & (cpr - 1)
-                    got = np.concatenate([tile[r, c ^ sw] for c in range(cpr)]).view(np.uint16)
-                    assert np.array_equal(got, want), (g, j, q, r)
-            t_next += len(panels)
+        for r in range(GROUP):
+            panel = int(gpan[g, r // bn])
+            feat[r] = panel * bn + r % bn if panel >= 0 else -1
+        ri = np.nonzero(feat >= 0)[0]
+        fr = feat[ri]
+        for e in range(int(gent[g]), int(gent[g + 1])):
+            c = int(ent[e])
+            want = np.zeros((GROUP, CHUNK), np.uint16)
+            cols = np.arange(c * CHUNK, min(k, (c + 1) * CHUNK))
+            keep = M[fr // bn][:, cols // bk] != 0
+            want[np.ix_(ri, cols - c * CHUNK)] = np.where(keep, Wb[fr][:, cols], 0)
+            tile = stream[e * GROUP * CHUNK * 2:(e + 1) * GROUP * CHUNK * 2].view(np.uint16).reshape(GROUP, CHUNK)
+            assert np.array_equal(tile, want), (g, c)
 
 
 @pytest.mark.parametrize("n,k,b", [(384, 256, 32), (208, 128, 16), (384, 192, 64), (96, 64, 32), (384, 128, (64, 32)),
