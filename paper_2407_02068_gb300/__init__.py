@@ -58,7 +58,7 @@ class BsrWeight:
     capacity: int
     row_ptr: torch.Tensor   # int32 [n/bn + 1]
     col_idx: torch.Tensor   # int32 [capacity]
-    blocks: torch.Tensor    # bf16 [capacity, bn, bk]
+    blocks: torch.Tensor | None  # bf16 [capacity, bn, bk]; None: index and work list only
     sched: torch.Tensor     # uint8 [sched_bytes]
     nnzb: int | None = None
 
@@ -69,13 +69,16 @@ class BsrWeight:
 
     def struct(self) -> _lib.lpvit_bsr:
         return _lib.lpvit_bsr(self.n, self.k, self.bn, self.bk, self.capacity, self.row_ptr.data_ptr(),
-                              self.col_idx.data_ptr(), self.blocks.data_ptr(), self.sched.data_ptr(),
+                              self.col_idx.data_ptr(), 0 if self.blocks is None else self.blocks.data_ptr(),
+                              self.sched.data_ptr(),
                               self.sched.numel())
 
 
-def alloc_bsr(n: int, k: int, b, capacity: int | None = None, device="cuda") -> BsrWeight:
+def alloc_bsr(n: int, k: int, b, capacity: int | None = None, device="cuda", blocks: bool = True) -> BsrWeight:
     """Device buffers for a packed n x k weight with blocks b (int or (bn, bk)); the capacity
-    defaults to every block."""
+    defaults to every block. ``blocks=False`` leaves out the BSR copy of the kept tiles: the
+    linear reads only the work list's weight stream, so packing then writes the block index and
+    the work list alone."""
     bn, bk = block_sides(b)
     if capacity is None:
         capacity = (n // bn) * (k // bk) if bn > 0 and bk > 0 and n % bn == 0 and k % bk == 0 else 0
@@ -83,7 +86,8 @@ def alloc_bsr(n: int, k: int, b, capacity: int | None = None, device="cuda") -> 
     return BsrWeight(n, k, bn, bk, capacity,
                      torch.empty(max(n // max(bn, 1), 0) + 1, dtype=torch.int32, device=device),
                      torch.empty(max(capacity, 1), dtype=torch.int32, device=device),
-                     torch.empty((max(capacity, 1), max(bn, 1), max(bk, 1)), dtype=torch.bfloat16, device=device),
+                     torch.empty((max(capacity, 1), max(bn, 1), max(bk, 1)), dtype=torch.bfloat16, device=device)
+                     if blocks else None,
                      torch.empty(max(sb, 16), dtype=torch.uint8, device=device))
 
 
@@ -244,7 +248,7 @@ def pack_bsr(W: torch.Tensor, mask: torch.Tensor, b, capacity: int | None = None
 def workspace_for(w: BsrWeight, m: int, device=None) -> torch.Tensor:
     """A zero-filled workspace of lpvit_workspace_bytes(w, m) bytes (256-byte aligned)."""
     nbytes = _lib.lpvit_workspace_bytes(w.struct(), m)
-    return torch.zeros(max(nbytes, 256), dtype=torch.uint8, device=device or w.blocks.device)
+    return torch.zeros(max(nbytes, 256), dtype=torch.uint8, device=device or w.sched.device)
 
 
 def bsr_linear(w: BsrWeight, X: torch.Tensor, bias: torch.Tensor | None = None, gelu: bool = False,

@@ -244,7 +244,7 @@ lpvit_status check_pack_args(const void *W, const uint8_t *mask, const lpvit_bsr
   if (!valid_side(bn) || !valid_side(bk)) return LPVIT_ERR_UNSUPPORTED;
   if (!shape_ok(n, k, bn, bk)) return LPVIT_ERR_INVALID_ARG;
   if (!W || !mask || !bsr->row_ptr || !bsr->sched || bsr->nnzb_capacity < 0) return LPVIT_ERR_INVALID_ARG;
-  if (bsr->nnzb_capacity > 0 && (!bsr->col_idx || !bsr->blocks)) return LPVIT_ERR_INVALID_ARG;
+  if (bsr->nnzb_capacity > 0 && !bsr->col_idx) return LPVIT_ERR_INVALID_ARG;  // blocks may be NULL
   if (!aligned(W, 16) || (bsr->blocks && !aligned(bsr->blocks, 16)) || !aligned(bsr->sched, 16) ||
       !aligned(bsr->row_ptr, 4) || (bsr->col_idx && !aligned(bsr->col_idx, 4)))
     return LPVIT_ERR_INVALID_ARG;

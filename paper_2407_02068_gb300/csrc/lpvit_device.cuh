@@ -125,6 +125,7 @@ struct PackJob {
   uint16_t *blocks;
   int32_t *sched;
   int n, k, bn, bk, cap;
+  int rot_b, rot_t;  // set by launch_pack_many: where the job's block and tile units start
 };
 constexpr int PACK_MAX_JOBS = 96;  // jobs per launch (6 KB of parameters)
 struct PackJobs {

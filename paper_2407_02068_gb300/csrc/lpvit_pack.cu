@@ -380,87 +380,125 @@ __global__ void __launch_bounds__(PLAN_THREADS, 1) plan_many_kernel(const __grid
   plan_body(w.mask, w.n, w.k, w.bn, w.bk, w.row_ptr, w.col_idx, w.cap, w.sched, plan_smem);
 }
 
-// Kept blocks t = cta, cta + ncta, ... of one weight.
+// Largest i in [0, len) with a[i] <= t, for a[] ascending and a[0] <= t; every lane of the warp
+// calls it and gets the answer. Each round splits the range into 32 parts, one load per lane.
+__device__ __forceinline__ int warp_last_le(const int32_t *__restrict__ a, int len, int t) {
+  const int lane = threadIdx.x & 31;
+  int lo = 0, hi = len;  // the answer lies in [lo, hi)
+  while (hi - lo > 1) {
+    const int step = (hi - lo + 31) >> 5;
+    const int i = lo + lane * step;
+    const unsigned le = __ballot_sync(0xffffffffu, i < hi && __ldg(a + i) <= t);
+    lo += (31 - __clz(le)) * step;  // lane 0 (i = lo) always qualifies
+    hi = min(hi, lo + step);
+  }
+  return lo;
+}
+
+constexpr int COPY_THREADS = 128;
+constexpr int COPY_WARPS = COPY_THREADS / 32;
+constexpr int COPY_CTAS_PER_SM = 6;  // resident at 80 registers a thread: the grid is one wave
+
+// Kept blocks of one weight, one warp per block: blocks t = wi, wi + nw, ... (wi the warp's index
+// among nw warps).
 __device__ __forceinline__ void copy_body(const uint16_t *__restrict__ W, int n, int k, int bn, int bk,
                                           const int32_t *__restrict__ row_ptr, const int32_t *__restrict__ col_idx,
-                                          int cap, uint16_t *__restrict__ blocks, int cta, int ncta) {
-  const int np = n / bn;
-  const int nnzb = min(row_ptr[np], cap);
+                                          int cap, uint16_t *__restrict__ blocks, int wi, int nw) {
+  const int np = n / bn, lane = threadIdx.x & 31;
+  const int nnzb = min(__ldg(row_ptr + np), cap);
   const int lvpr = __ffs(bk / 8) - 1;  // log2 of the 16-byte vectors per block row (bk is a power of 2)
-  const int vecs = bn << lvpr;
-  for (int t = cta; t < nnzb; t += ncta) {
-    int lo = 0, hi = np - 1;  // largest r with row_ptr[r] <= t (that panel holds block t)
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (row_ptr[mid] <= t) lo = mid;
-      else hi = mid - 1;
-    }
-    const int r = lo, j = col_idx[t];
-    for (int v = threadIdx.x; v < vecs; v += blockDim.x) {
-      const int c = v >> lvpr, cv = v & ((1 << lvpr) - 1);
-      const int4 *src = reinterpret_cast<const int4 *>(W + ((int64_t)r * bn + c) * k + (int64_t)j * bk + cv * 8);
-      int4 *dst = reinterpret_cast<int4 *>(blocks + ((int64_t)t * bn + c) * bk + cv * 8);
-      *dst = __ldg(src);
+  const int vecs = bn << lvpr;         // 32 .. 512, a multiple of 32
+  for (int t = wi; t < nnzb; t += nw) {
+    const int r = warp_last_le(row_ptr, np, t), j = __ldg(col_idx + t);
+    const uint16_t *src = W + (int64_t)r * bn * k + (int64_t)j * bk;
+    int4 *dst = reinterpret_cast<int4 *>(blocks + (int64_t)t * bn * bk);
+    for (int v0 = 0; v0 < vecs; v0 += 128) {  // up to four vectors per lane in flight
+      int4 val[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int v = v0 + lane + 32 * q;
+        if (v < vecs)
+          val[q] = __ldg(reinterpret_cast<const int4 *>(src + (int64_t)(v >> lvpr) * k + (v & ((1 << lvpr) - 1)) * 8));
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int v = v0 + lane + 32 * q;
+        if (v < vecs) dst[v] = val[q];
+      }
     }
   }
 }
 
 // Weight-stream tiles of entries e = cta, cta + ncta, ... of one weight (after its plan): the
 // group's 256 rows over the entry's 64 columns, row-major, 16-byte vectors; zero where the block
-// is removed, where the slot has no panel and beyond column k.
+// is removed, where the slot has no panel and beyond column k. Thread i writes vectors
+// i + COPY_THREADS * q of the tile: column vector i % 8 of rows i / 8 + 16 q.
 __device__ __forceinline__ void stream_body(const uint16_t *__restrict__ W, const uint8_t *__restrict__ mask, int n,
                                             int k, int bn, int bk, const int32_t *__restrict__ sched, int cta,
                                             int ncta) {
   const int kb = k / bk, kc = sched_chunks(k), ng = (n + GROUP_FEATURES - 1) / GROUP_FEATURES;
-  if (sched[1] != ng || sched[3] != 0) return;  // not this shape's plan, or blocks overflowed
-  const int total = sched[2];
-  constexpr int VPR = CHUNK_COLS / 8;             // 16-byte vectors per tile row
-  constexpr int VECS = GROUP_FEATURES * VPR;
+  if (__ldg(sched + 1) != ng || __ldg(sched + 3) != 0) return;  // not this shape's plan, or blocks overflowed
+  const int total = __ldg(sched + 2);
+  constexpr int VPR = CHUNK_COLS / 8;                    // 16-byte vectors per tile row
+  constexpr int RSTEP = COPY_THREADS / VPR;              // rows between a thread's vectors
+  constexpr int PER = GROUP_FEATURES / RSTEP;            // vectors per thread and tile
+  static_assert(PER % 8 == 0, "tile rows");
   const int lbn = __ffs(bn) - 1, lbk = __ffs(bk) - 1;  // bn and bk are powers of 2
   const int64_t max_tiles = sched_stream_tiles(ng, kc);
   const int32_t *gent = sched + SCHED_HDR_INTS;
   const int32_t *gpan = sched + sched_gpan_offset_ints(ng);
   const int32_t *ent = sched + sched_entries_offset_ints(ng);
   uint8_t *stream = reinterpret_cast<uint8_t *>(const_cast<int32_t *>(sched)) + sched_stream_offset_bytes(ng, kc);
+  const int cv = threadIdx.x % VPR, r0 = threadIdx.x / VPR;
   for (int e = cta; e < total; e += ncta) {
-    int lo = 0, hi = ng - 1;  // largest g with gent[g] <= e (the group holding entry e)
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (gent[mid] <= e) lo = mid;
-      else hi = mid - 1;
-    }
-    const int g = lo, ch = ent[e];
+    const int g = warp_last_le(gent, ng, e), ch = __ldg(ent + e);
     if (ch < 0 || ch >= kc || (int64_t)e >= max_tiles) continue;
     int4 *tile = reinterpret_cast<int4 *>(stream + (int64_t)e * stream_tile_bytes());
-    for (int v = threadIdx.x; v < VECS; v += blockDim.x) {
-      const int r = v / VPR, cv = v % VPR, slot = r >> lbn;
-      const int panel = gpan[g * MAX_GROUP_PANELS + slot];
-      const int col = ch * CHUNK_COLS + cv * 8;
-      // the output feature of group row r (none for an empty slot)
-      const int row = panel >= 0 ? (panel << lbn) + (r & (bn - 1)) : -1;
-      int4 val = make_int4(0, 0, 0, 0);
-      if (row >= 0 && row < n && col < k && mask[(int64_t)panel * kb + (col >> lbk)] != 0)
-        val = __ldg(reinterpret_cast<const int4 *>(W + (int64_t)row * k + col));
-      tile[v] = val;
+    const int col = ch * CHUNK_COLS + cv * 8;
+    const bool col_ok = col < k;
+    const int bc = col >> lbk;
+#pragma unroll 1
+    for (int h = 0; h < PER; h += 8) {  // eight vectors per thread in flight
+      int4 val[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int r = r0 + RSTEP * (h + q);
+        const int panel = __ldg(gpan + g * MAX_GROUP_PANELS + (r >> lbn));
+        // the output feature of group row r (none for an empty slot)
+        const int row = panel >= 0 ? (panel << lbn) + (r & (bn - 1)) : -1;
+        val[q] = make_int4(0, 0, 0, 0);
+        if (row >= 0 && row < n && col_ok && __ldg(mask + (int64_t)panel * kb + bc) != 0)
+          val[q] = __ldg(reinterpret_cast<const int4 *>(W + (int64_t)row * k + col));
+      }
+#pragma unroll
+      for (int q = 0; q < 8; ++q) tile[threadIdx.x + COPY_THREADS * (h + q)] = val[q];
     }
   }
 }
 
-__global__ void __launch_bounds__(128)
+__global__ void __launch_bounds__(COPY_THREADS, COPY_CTAS_PER_SM)
 copy_blocks_kernel(const uint16_t *__restrict__ W, const uint8_t *__restrict__ mask, int n, int k, int bn, int bk,
                    const int32_t *__restrict__ row_ptr, const int32_t *__restrict__ col_idx, int cap,
                    uint16_t *__restrict__ blocks, const int32_t *__restrict__ sched) {
-  copy_body(W, n, k, bn, bk, row_ptr, col_idx, cap, blocks, blockIdx.x, gridDim.x);
+  const int warp = threadIdx.x >> 5;
+  if (blocks != nullptr)
+    copy_body(W, n, k, bn, bk, row_ptr, col_idx, cap, blocks, blockIdx.x * COPY_WARPS + warp, gridDim.x * COPY_WARPS);
   stream_body(W, mask, n, k, bn, bk, sched, blockIdx.x, gridDim.x);
 }
 
-// Several weights at once: every CTA takes its share of every job's kept blocks and stream tiles.
-__global__ void __launch_bounds__(128) copy_many_kernel(const __grid_constant__ PackJobs J) {
+// Several weights at once. The units of job j (kept blocks, one per warp, and stream tiles, one
+// per CTA) start where the previous jobs' largest possible counts end (rot_b, rot_t), so that
+// the work of all jobs spreads over the whole grid.
+__global__ void __launch_bounds__(COPY_THREADS, COPY_CTAS_PER_SM) copy_many_kernel(const __grid_constant__ PackJobs J) {
+  const int warp = threadIdx.x >> 5;
+  const unsigned ncta = gridDim.x, nw = ncta * COPY_WARPS;
   for (int j = 0; j < J.count; ++j) {
     const PackJob &w = J.job[j];
-    if (w.cap > 0)
-      copy_body(w.W, w.n, w.k, w.bn, w.bk, w.row_ptr, w.col_idx, w.cap, w.blocks, blockIdx.x, gridDim.x);
-    stream_body(w.W, w.mask, w.n, w.k, w.bn, w.bk, w.sched, blockIdx.x, gridDim.x);
+    if (w.cap > 0 && w.blocks != nullptr) {
+      const int wi = (int)((blockIdx.x * COPY_WARPS + warp + (unsigned)w.rot_b) % nw);
+      copy_body(w.W, w.n, w.k, w.bn, w.bk, w.row_ptr, w.col_idx, w.cap, w.blocks, wi, (int)nw);
+    }
+    stream_body(w.W, w.mask, w.n, w.k, w.bn, w.bk, w.sched, (int)((blockIdx.x + (unsigned)w.rot_t) % ncta), (int)ncta);
   }
 }
 
@@ -480,9 +518,10 @@ cudaError_t launch_pack(const void *W, const uint8_t *mask, int n, int k, int bn
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const int max_blocks = (n / bn) * (k / bk);
-  int grid = max_blocks < num_sms * 16 ? max_blocks : num_sms * 16;
+  int grid = (max_blocks + COPY_WARPS - 1) / COPY_WARPS;
+  if (grid > num_sms * COPY_CTAS_PER_SM) grid = num_sms * COPY_CTAS_PER_SM;
   if (grid < 1) grid = 1;
-  copy_blocks_kernel<<<grid, 128, 0, s>>>(static_cast<const uint16_t *>(W), mask, n, k, bn, bk, row_ptr, col_idx, cap,
+  copy_blocks_kernel<<<grid, COPY_THREADS, 0, s>>>(static_cast<const uint16_t *>(W), mask, n, k, bn, bk, row_ptr, col_idx, cap,
                                          static_cast<uint16_t *>(blocks), sched);
   return cudaGetLastError();
 }
@@ -513,9 +552,20 @@ cudaError_t launch_pack_many(const PackJob *jobs, int count, int num_sms, cudaSt
     plan_many_kernel<<<J.count, PLAN_THREADS, smem, s>>>(J);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    int64_t grid = blocks_max < (int64_t)num_sms * 16 ? blocks_max : (int64_t)num_sms * 16;
+    int64_t grid = (blocks_max + COPY_WARPS - 1) / COPY_WARPS;
+    if (grid > (int64_t)num_sms * COPY_CTAS_PER_SM) grid = (int64_t)num_sms * COPY_CTAS_PER_SM;
     if (grid < 1) grid = 1;
-    copy_many_kernel<<<(int)grid, 128, 0, s>>>(J);
+    // each job's units start after the previous jobs' largest possible counts (mod the grid)
+    const int64_t nw = grid * COPY_WARPS;
+    int64_t pb = 0, pt = grid / 2;
+    for (int j = 0; j < J.count; ++j) {
+      const PackJob &w = J.job[j];
+      J.job[j].rot_b = (int)((nw - pb % nw) % nw);
+      J.job[j].rot_t = (int)((grid - pt % grid) % grid);
+      pb += (int64_t)(w.n / w.bn) * (w.k / w.bk);
+      pt += (int64_t)((w.n + GROUP_FEATURES - 1) / GROUP_FEATURES) * sched_chunks(w.k);
+    }
+    copy_many_kernel<<<(int)grid, COPY_THREADS, 0, s>>>(J);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }

@@ -313,10 +313,45 @@ def test_pack_many_matches_single_packs(lp, count):
         ha, hs, ea, es = _decode_sched(a)[0], _decode_sched(s1)[0], _decode_sched(a), _decode_sched(s1)
         assert np.array_equal(ha, hs) and np.array_equal(ea[1], es[1]) and np.array_equal(ea[2], es[2])
         assert np.array_equal(ea[3], es[3])
+        assert np.array_equal(_stream_bytes(a), _stream_bytes(s1))
         if i < 5:
             _check_weight_stream(a, Ws[i], masks[i])
         rp, ci, bl = oracle.pack(_bits(Ws[i]), masks[i].cpu().numpy(), b)
         assert np.array_equal(a.row_ptr.cpu().numpy(), rp) and np.array_equal(a.col_idx[:nnzb].cpu().numpy(), ci)
+
+
+def _stream_bytes(w):
+    """The weight-stream tiles of w's work list (entries x 256 x 64 bf16) as raw bytes."""
+    hdr, gent, ent, gpan = _decode_sched(w)
+    ng, kc = int(hdr[1]), -(-w.k // CHUNK)
+    raw = w.sched.cpu().numpy().view(np.uint8)
+    start = (4 * (_entries_offset(ng) + ng * kc) + 1023) // 1024 * 1024
+    return raw[start:start + int(hdr[2]) * GROUP * CHUNK * 2]
+
+
+@pytest.mark.parametrize("many", [False, True])
+def test_pack_without_blocks(lp, many):
+    """A weight allocated without the BSR block copy packs to the same index, work list and weight
+    stream, and its linear gives the same bits."""
+    shapes = [(1152, 384, 32, 0.5), (384, 1536, 16, 0.4), (768, 3072, (64, 32), 0.6)]
+    for i, (n, k, b, sp) in enumerate(shapes):
+        X, W, bias, mask = _case(197, n, k, b, sp, 4100 + i)
+        full = lp.pack_bsr(W, mask, b, count=True)
+        bare = lp.alloc_bsr(n, k, b, blocks=False)
+        assert bare.blocks is None
+        if many:
+            lp.pack_bsr_many_into([bare], [W.contiguous()], [mask.contiguous()])
+        else:
+            lp.pack_bsr_into(bare, W.contiguous(), mask.contiguous())
+        torch.cuda.synchronize()
+        nnzb = full.nnzb
+        assert torch.equal(bare.row_ptr, full.row_ptr) and torch.equal(bare.col_idx[:nnzb], full.col_idx[:nnzb])
+        hb, hf = _decode_sched(bare), _decode_sched(full)
+        assert all(np.array_equal(u, v) for u, v in zip(hb, hf))
+        assert np.array_equal(_stream_bytes(bare), _stream_bytes(full))
+        yb = lp.bsr_linear(bare, X, bias)
+        yf = lp.bsr_linear(full, X, bias)
+        assert torch.equal(yb.view(torch.int16), yf.view(torch.int16))
 
 
 # ------------------------------------------------------------------------------------- GEMM
