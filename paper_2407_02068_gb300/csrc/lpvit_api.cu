@@ -203,9 +203,11 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.y_f32 = y_dtype == LPVIT_F32;
   P.gelu = gelu;
   P.y_vec16 = (aligned(Y, 16) && ((size_t)ldy * ysz) % 16 == 0) ? 1 : 0;
+  P.y_vec32 = (aligned(Y, 32) && ((size_t)ldy * ysz) % 32 == 0) ? 1 : 0;
   P.bias_vec16 = (bias && aligned(bias, 16)) ? 1 : 0;
   P.R = static_cast<const uint16_t *>(R);
   P.ldr = R ? ldr : 0;
+  P.r_vec32 = (R && aligned(R, 32) && ((size_t)ldr * 2) % 32 == 0) ? 1 : 0;
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   P.ctl = reinterpret_cast<Control *>(ws);
   P.partials = reinterpret_cast<float *>(ws + W.partials_off);

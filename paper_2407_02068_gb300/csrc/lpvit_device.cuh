@@ -74,9 +74,11 @@ struct LinearParams {
   int n_tt, n_groups, S;   // token tiles, groups, max entries per slice
   int y_f32, gelu;
   int y_vec16;             // output rows may take 16-byte stores (Y 16-byte aligned, ldy * size % 16 == 0)
+  int y_vec32;             // ... and 32-byte stores (Y 32-byte aligned, ldy * size % 32 == 0)
   int bias_vec16;          // bias is 16-byte aligned
   const uint16_t *R;       // bf16 residual [m][ldr] added after rounding (bf16 output only), or nullptr
   int64_t ldr;
+  int r_vec32;             // residual rows may take 32-byte loads (else 16-byte ones)
   Control *ctl;
   float *partials;         // split units: [slice][part_rows][GROUP_FEATURES] fp32 partial sums
   int part_rows;           // token rows of one partial tile: min(m, TOKENS_PER_TILE)

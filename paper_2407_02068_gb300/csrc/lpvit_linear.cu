@@ -61,7 +61,9 @@ static_assert(CHUNK_COLS * 2 == 128, "stage rows are 128 bytes (the 128-byte swi
 static_assert(EPI_WARPS == 16 && GROUP_FEATURES == 4 * 64, "each epilogue warp takes 64 feature columns");
 
 struct UnitInfo {
-  int tt, g, s, nsl, e0, e1, pad0, pad1;
+  int tt, g, s, nsl, e0, e1;
+  int ptile;  // split units: the partial tile (token tile, group slice) the slice writes
+  int pad;
 };
 static_assert(sizeof(UnitInfo) == 32, "unit record is two 16-byte vectors");
 // A unit-ring slot: the unit and the chunk indices of its first 32 entries (0 past its end).
@@ -75,10 +77,8 @@ struct Smem {
   // barriers: full[NS], empty[NS], accf[2], acce[2], unitf[UR], unite[UR], drain
   static constexpr int NBARS = 2 * NSTAGES + 4 + 2 * UR + 1;
   static constexpr int RING_OFF = (BAR_OFF + 8 * NBARS + 31) / 32 * 32;
-  static constexpr int SLICE_OFF = RING_OFF + (int)sizeof(UnitSlot) * UR;
-  static constexpr int GENT_OFF = SLICE_OFF + 4 * (MAX_GROUPS + 1);
-  static constexpr int MISC_OFF = GENT_OFF + 4 * (MAX_GROUPS + 1);
-  static constexpr int BIAS_OFF = (MISC_OFF + 64 + 15) / 16 * 16;  // per epilogue warp: its 64 features' bias
+  static constexpr int MISC_OFF = RING_OFF + (int)sizeof(UnitSlot) * UR;
+  static constexpr int BIAS_OFF = MISC_OFF + 64;  // per epilogue warp: its 64 features' bias
   static constexpr int END = BIAS_OFF + EPI_WARPS * 64 * 4;
   static constexpr int BYTES = END + 1024;  // + alignment slack for the dynamic smem base
   static_assert(BYTES <= 227 * 1024, "shared memory per CTA");
@@ -138,39 +138,36 @@ __device__ __forceinline__ float gelu_erf(float t) {
   return t * (t >= 0.f ? 1.f - half_erfc : half_erfc);
 }
 
-// Transpose 16-byte chunks within groups of CPR lanes: lane i of a group holds chunks
-// w[4 j .. 4 j + 3] (j < CPR) of its own row; afterwards it holds chunk i of row j of the group in
-// w[4 j .. 4 j + 3] (butterfly exchange over lane bits 1, 2, 4, ...).
-template <int CPR>
-__device__ __forceinline__ void transpose_chunks(uint32_t (&w)[4 * CPR], int lane) {
-  const int i = lane & (CPR - 1);
-#pragma unroll
-  for (int sft = 1; sft < CPR; sft <<= 1) {
-    const bool hi = (i & sft) != 0;
-#pragma unroll
-    for (int j = 0; j < CPR; ++j) {
-      if (j & sft) continue;
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const uint32_t send = hi ? w[4 * j + q] : w[4 * (j ^ sft) + q];
-        const uint32_t recv = __shfl_xor_sync(0xffffffffu, send, sft);
-        if (hi) w[4 * j + q] = recv;
-        else w[4 * (j ^ sft) + q] = recv;
-      }
-    }
-  }
+__device__ __forceinline__ void st_global_32B(void *p, const uint32_t (&w)[8]) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]),
+               "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+               : "memory");
+}
+__device__ __forceinline__ void ld_global_32B(const void *p, uint32_t (&w)[8]) {
+  asm volatile("ld.global.v8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+               : "=r"(w[0]), "=r"(w[1]), "=r"(w[2]), "=r"(w[3]), "=r"(w[4]), "=r"(w[5]), "=r"(w[6]), "=r"(w[7])
+               : "l"(p));
 }
 
-// The outputs of one run of 16 consecutive group rows (features f0 .. f0 + 15) for the warp's 32
-// tokens (a lane per token, tokens tok0 .. tok0 + 31): y[0..16) are the lane's accumulated sums (or
-// zero), bs the run's bias in shared memory (the same for every lane). Adds the bias, applies GELU,
-// rounds, then exchanges 16-byte chunks between lanes so that each store instruction writes whole
-// 16-feature row segments (32 bytes bf16, 64 bytes fp32) of 32 / CPR tokens; bf16 output may add
-// the residual (each sum rounded, as a separate bf16 addition would). Warp-uniform: every lane
-// calls it.
+// Entry g of a table spread over the warp (lane l holds entries l + 32 j in t[j]); g warp-uniform.
+template <int N>
+__device__ __forceinline__ int table_at(const int (&t)[N], int g) {
+  int v = 0;
+#pragma unroll
+  for (int j = 0; j < N; ++j) {
+    const int x = __shfl_sync(0xffffffffu, t[j], g & 31);
+    v = (g >> 5) == j ? x : v;
+  }
+  return v;
+}
+
+// The outputs of one run of 16 consecutive group rows (features f0 .. f0 + 15) for the lane's token
+// t: y[0..16) are its accumulated sums (or zero), bs the run's bias in shared memory (the same for
+// every lane). Adds the bias, applies GELU, rounds and stores the lane's 32-byte (bf16) or 64-byte
+// (fp32) row segment with 32-byte stores, so that each store instruction writes whole sectors;
+// bf16 output may add the residual (each sum rounded, as a separate bf16 addition would).
 template <bool GELU, bool F32>
-__device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, int64_t tok0, const LinearParams &P) {
-  const int lane = threadIdx.x & 31;
+__device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, int64_t t, const LinearParams &P) {
 #pragma unroll
   for (int i = 0; i < 16; i += 4) {
     float4 b;
@@ -181,51 +178,57 @@ __device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, 
 #pragma unroll
     for (int i = 0; i < 16; ++i) y[i] = gelu_erf(y[i]);
   }
-  constexpr int CPR = F32 ? 4 : 2;  // 16-byte chunks per row segment
-  uint32_t w[4 * CPR];
+  if (t >= P.m) return;
   if (F32) {
+    float *dst = static_cast<float *>(P.Y) + t * P.ldy + f0;
+    if (P.y_vec32) {
 #pragma unroll
-    for (int i = 0; i < 16; ++i) w[i] = __float_as_uint(y[i]);
+      for (int h = 0; h < 2; ++h) {
+        uint32_t w[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) w[q] = __float_as_uint(y[8 * h + q]);
+        st_global_32B(dst + 8 * h, w);
+      }
+    } else if (P.y_vec16) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) reinterpret_cast<float4 *>(dst)[q] = make_float4(y[4 * q], y[4 * q + 1], y[4 * q + 2], y[4 * q + 3]);
+    } else {  // row not 16-byte aligned: element by element
+#pragma unroll
+      for (int q = 0; q < 16; ++q) dst[q] = y[q];
+    }
   } else {
+    uint32_t o[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) w[i] = pack_bf16x2(y[2 * i], y[2 * i + 1]);
-  }
-  transpose_chunks<CPR>(w, lane);
-  const int ci = lane & (CPR - 1), grp = lane / CPR;
-#pragma unroll
-  for (int j = 0; j < CPR; ++j) {
-    const int64_t t = tok0 + grp * CPR + j;
-    if (t >= P.m) continue;
-    uint32_t o[4] = {w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]};
-    if (F32) {
-      float *dst = static_cast<float *>(P.Y) + t * P.ldy + f0 + 4 * ci;
-      if (P.y_vec16) {
-        *reinterpret_cast<int4 *>(dst) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
-      } else {  // row not 16-byte aligned: element by element
-#pragma unroll
-        for (int q = 0; q < 4; ++q) dst[q] = __uint_as_float(o[q]);
+    for (int i = 0; i < 8; ++i) o[i] = pack_bf16x2(y[2 * i], y[2 * i + 1]);
+    if (P.R != nullptr) {
+      // a plain load: R may be Y itself, read and then written by this lane only
+      const uint16_t *src = P.R + t * P.ldr + f0;
+      uint32_t rw[8];
+      if (P.r_vec32) {
+        ld_global_32B(src, rw);
+      } else {
+        const int4 r0 = reinterpret_cast<const int4 *>(src)[0], r1 = reinterpret_cast<const int4 *>(src)[1];
+        rw[0] = (uint32_t)r0.x; rw[1] = (uint32_t)r0.y; rw[2] = (uint32_t)r0.z; rw[3] = (uint32_t)r0.w;
+        rw[4] = (uint32_t)r1.x; rw[5] = (uint32_t)r1.y; rw[6] = (uint32_t)r1.z; rw[7] = (uint32_t)r1.w;
       }
-    } else {
-      if (P.R != nullptr) {
-        // a plain load: R may be Y itself, read and then written by this lane only
-        const int4 rv = *reinterpret_cast<const int4 *>(P.R + t * P.ldr + f0 + 8 * ci);
-        const uint32_t rw[4] = {(uint32_t)rv.x, (uint32_t)rv.y, (uint32_t)rv.z, (uint32_t)rv.w};
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const float lo = __uint_as_float(o[q] << 16) + __uint_as_float(rw[q] << 16);
-          const float hi = __uint_as_float(o[q] & 0xffff0000u) + __uint_as_float(rw[q] & 0xffff0000u);
-          o[q] = pack_bf16x2(lo, hi);
-        }
+      for (int q = 0; q < 8; ++q) {
+        const float lo = __uint_as_float(o[q] << 16) + __uint_as_float(rw[q] << 16);
+        const float hi = __uint_as_float(o[q] & 0xffff0000u) + __uint_as_float(rw[q] & 0xffff0000u);
+        o[q] = pack_bf16x2(lo, hi);
       }
-      uint16_t *dst = static_cast<uint16_t *>(P.Y) + t * P.ldy + f0 + 8 * ci;
-      if (P.y_vec16) {
-        *reinterpret_cast<int4 *>(dst) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
-      } else {  // row not 16-byte aligned: element by element
+    }
+    uint16_t *dst = static_cast<uint16_t *>(P.Y) + t * P.ldy + f0;
+    if (P.y_vec32) {
+      st_global_32B(dst, o);
+    } else if (P.y_vec16) {
+      reinterpret_cast<int4 *>(dst)[0] = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
+      reinterpret_cast<int4 *>(dst)[1] = make_int4((int)o[4], (int)o[5], (int)o[6], (int)o[7]);
+    } else {  // row not 16-byte aligned: element by element
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          dst[2 * q] = (uint16_t)(o[q] & 0xffffu);
-          dst[2 * q + 1] = (uint16_t)(o[q] >> 16);
-        }
+      for (int q = 0; q < 8; ++q) {
+        dst[2 * q] = (uint16_t)(o[q] & 0xffffu);
+        dst[2 * q + 1] = (uint16_t)(o[q] >> 16);
       }
     }
   }
@@ -253,8 +256,6 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
   auto unite_bar = [&](int u) { return bar0 + 8u * (RB + 4 + UR + u); };
   const uint32_t drain_bar = bar0 + 8u * (RB + 4 + 2 * UR);
   UnitSlot *ring = reinterpret_cast<UnitSlot *>(smem + L::RING_OFF);
-  int *slice_ptr = reinterpret_cast<int *>(smem + L::SLICE_OFF);
-  int *gent_s = reinterpret_cast<int *>(smem + L::GENT_OFF);
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + L::MISC_OFF);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 4);
   volatile int *never_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 8);  // stays 0
@@ -295,35 +296,11 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
   // the work list must be this weight's plan: layout, group count, shape
   const bool sched_ok = P.sched[3] == 0 && P.sched[1] == P.n_groups && P.sched[4] == P.n && P.sched[5] == P.k &&
                         P.sched[6] == P.bn && P.sched[8] == SCHED_VERSION && P.n_groups <= MAX_GROUPS;
-  if (warp == 2 && sched_ok) {
-    // slices per group = max(1, ceil(entries / S)); exclusive prefix into slice_ptr
-    int run = 0;
-    for (int base = 0; base < P.n_groups; base += 32) {
-      const int g = base + lane;
-      int c = 0;
-      if (g < P.n_groups) {
-        const int cnt = gent[g + 1] - gent[g];
-        c = cnt <= 0 ? 1 : (cnt + P.S - 1) / P.S;
-      }
-      int incl = c;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int t = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += t;
-      }
-      if (g < P.n_groups) slice_ptr[g] = run + incl - c;
-      run += __shfl_sync(0xffffffffu, incl, 31);
-    }
-    if (lane == 0) slice_ptr[P.n_groups] = run;
-    for (int g = lane; g <= P.n_groups; g += 32) gent_s[g] = gent[g];
-  }
   tc_fence_before();
   __syncthreads();
   cluster_sync();  // both CTAs' barriers are initialised before any signal crosses the pair
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int total_slices = sched_ok ? slice_ptr[P.n_groups] : 0;
-  const uint32_t total_units = sched_ok ? (uint32_t)P.n_tt * (uint32_t)total_slices : 0u;
   if (!sched_ok && tid == 0 && leader) atomicOr(&P.ctl->err, P.sched[3] ? ERR_SCHED_OVERFLOW : ERR_BAD_SCHED);
 
   if (warp == 0 || warp == W_WARP) {
@@ -359,16 +336,6 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
           cw = cw_next;
           cw_next = xrole && win + 32 + lane < inf.e1 ? __ldg(entries + win + 32 + lane) : 0;
         }
-        bool wok = true;
-        if (lane < nb) {
-          const uint32_t itk = it + lane;
-          wok = mbar_wait(empty_bar(itk % NSTAGES), ((itk / NSTAGES) & 1u) ^ 1u, abort_flag, tmo);
-        }
-        if (!__all_sync(0xffffffffu, wok)) {
-          ok = false;
-          if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_EMPTY);
-          break;
-        }
         const int e = base + (lane < nb ? lane : 0);  // the batch entry of this lane's copy
         int c = __shfl_sync(0xffffffffu, cw, (e - win) & 31);
         int tile = e;
@@ -378,10 +345,18 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
           c = 0;
           tile = 0;
         }
-        const uint32_t stk = (it + (uint32_t)lane) % NSTAGES;
+        const uint32_t itk = it + (uint32_t)lane;
+        const uint32_t stk = itk % NSTAGES;
         const uint32_t st = smem_base + stk * STAGE_BYTES;
         const uint32_t fb = mapa_rank(full_bar(stk), 0);
-        if (lane < nb) {
+        bool wok = true;
+        if (lane < nb) wok = mbar_wait(empty_bar(stk), ((itk / NSTAGES) & 1u) ^ 1u, abort_flag, tmo);
+        if (!__all_sync(0xffffffffu, wok)) {
+          ok = false;
+          if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_EMPTY);
+          break;
+        }
+        if (lane < nb) {  // the batch's stages are all free: one issue step for all of them
           if (!in_range) atomicOr(&P.ctl->err, ERR_BAD_SCHED);
           if (leader && xrole) mbar_arrive_expect_tx(full_bar(stk), 2 * STAGE_BYTES);
           if (xrole) tma_load_2d_pair(st, &tmX, c * CHUNK_COLS, ytok, fb);
@@ -409,6 +384,33 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     // and the unit's first 32 chunk indices, written locally and into the peer, then both CTAs'
     // unit-full barriers. Runs up to UR units ahead of the producers.
     if (leader) {
+      // slices per group = max(1, ceil(entries / S)) and their exclusive prefix, kept in registers:
+      // lane l holds group l + 32 j in sp[j] (first slice) and ge[j] (first entry)
+      constexpr int GPL = MAX_GROUPS / 32;
+      int sp[GPL], ge[GPL];
+      int run = 0;
+#pragma unroll
+      for (int j = 0; j < GPL; ++j) {
+        const int g = 32 * j + lane;
+        int c = 0, g0 = 0;
+        if (sched_ok && g < P.n_groups) {
+          g0 = gent[g];
+          const int cnt = gent[g + 1] - g0;
+          c = cnt <= 0 ? 1 : (cnt + P.S - 1) / P.S;
+        }
+        int incl = c;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int t = __shfl_up_sync(0xffffffffu, incl, o);
+          if (lane >= o) incl += t;
+        }
+        sp[j] = run + incl - c;
+        ge[j] = g0;
+        run += __shfl_sync(0xffffffffu, incl, 31);
+      }
+      const int total_slices = run;
+      const int ge_end = sched_ok ? gent[P.n_groups] : 0;
+      const uint32_t total_units = sched_ok ? (uint32_t)P.n_tt * (uint32_t)total_slices : 0u;
       bool ok = true;
       uint32_t fetched = 0;
       if (lane == 0) fetched = atomicAdd(&P.ctl->next_unit, 1u);
@@ -424,22 +426,24 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
         if (u < total_units) {
           d.tt = (int)(u / (uint32_t)total_slices);
           const int rr = (int)(u % (uint32_t)total_slices);
-          int lo = 0, hi = P.n_groups - 1;  // group g with slice_ptr[g] <= rr < slice_ptr[g+1]
-          while (lo < hi) {
-            const int mid = (lo + hi + 1) >> 1;
-            if (slice_ptr[mid] <= rr) lo = mid;
-            else hi = mid - 1;
-          }
-          d.g = lo;
-          d.s = rr - slice_ptr[lo];
-          d.nsl = slice_ptr[lo + 1] - slice_ptr[lo];
-          const int ge0 = gent_s[lo], ge1 = gent_s[lo + 1];
+          // group g with sp[g] <= rr < sp[g + 1]: every group has a slice, so g + 1 = #{g : sp[g] <= rr}
+          int cnt = 0;
+#pragma unroll
+          for (int j = 0; j < GPL; ++j)
+            cnt += __popc(__ballot_sync(0xffffffffu, 32 * j + lane < P.n_groups && sp[j] <= rr));
+          const int g = cnt - 1;
+          const int s0 = table_at(sp, g), s1 = g + 1 < P.n_groups ? table_at(sp, g + 1) : total_slices;
+          const int ge0 = table_at(ge, g), ge1 = g + 1 < P.n_groups ? table_at(ge, g + 1) : ge_end;
+          d.g = g;
+          d.s = rr - s0;
+          d.nsl = s1 - s0;
           d.e0 = min(ge0 + d.s * P.S, ge1);
           d.e1 = min(d.e0 + P.S, ge1);
+          d.ptile = d.tt * total_slices + rr;
         } else {
-          d.tt = -1; d.g = d.s = d.nsl = d.e0 = d.e1 = 0;
+          d.tt = -1; d.g = d.s = d.nsl = d.e0 = d.e1 = d.ptile = 0;
         }
-        d.pad0 = d.pad1 = 0;
+        d.pad = 0;
         if (lane == 0 && u < total_units) fetched = atomicAdd(&P.ctl->next_unit, 1u);
         const int wv = d.e0 + lane < d.e1 ? __ldg(entries + d.e0 + lane) : 0;
         UnitSlot &rs = ring[slot];
@@ -560,7 +564,6 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       }
       if (inf.tt < 0) break;
       // the features of this warp's 64 columns (first feature of each 16-column quarter, or -1)
-      // and their bias, staged while the accumulator is still being computed
       int fcol[4];
 #pragma unroll
       for (int r4 = 0; r4 < 4; ++r4) {
@@ -568,6 +571,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
         const int panel = __ldg(gpan + (int64_t)inf.g * MAX_GROUP_PANELS + c / P.bn);
         fcol[r4] = panel >= 0 ? panel * P.bn + c % P.bn : -1;
       }
+      // and their bias, staged while the accumulator is still being computed
       if (lane < 16) {
         const int qq = lane >> 2;  // the lane's quarter, selected without indexing the array
         const int fq = qq == 0 ? fcol[0] : (qq == 1 ? fcol[1] : (qq == 2 ? fcol[2] : fcol[3]));
@@ -596,8 +600,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       const bool split = inf.nsl > 1;
       float *part_row = nullptr;
       if (split)
-        part_row = P.partials +
-                   (((int64_t)inf.tt * total_slices + slice_ptr[inf.g] + inf.s) * P.part_rows + t_tile) * GROUP_FEATURES;
+        part_row = P.partials + ((int64_t)inf.ptile * P.part_rows + t_tile) * GROUP_FEATURES;
       const bool touched = inf.e1 > inf.e0;
 #pragma unroll 1
       for (int h = 0; h < 2; ++h) {
@@ -617,15 +620,15 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
           }
         } else {
           const int fa = h == 0 ? fcol[0] : fcol[2], fb2 = h == 0 ? fcol[1] : fcol[3];
-          const uint32_t bs = smem_u32(bias_s + 32 * h);
           float ya[16], yb[16];
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
             ya[i] = v[i];
             yb[i] = v[16 + i];
           }
-          if (fa >= 0) emit_run16<GELU, F32>(ya, bs, fa, tok0, P);
-          if (fb2 >= 0) emit_run16<GELU, F32>(yb, bs + 64, fb2, tok0, P);
+          const uint32_t bs = smem_u32(bias_s + 32 * h);
+          if (fa >= 0) emit_run16<GELU, F32>(ya, bs, fa, t, P);
+          if (fb2 >= 0) emit_run16<GELU, F32>(yb, bs + 64, fb2, t, P);
         }
         __syncwarp();
       }
