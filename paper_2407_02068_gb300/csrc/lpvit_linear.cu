@@ -122,24 +122,25 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return r;
 }
 
-// GELU(t) = t * Phi(t), Phi(t) = erfc(-t / sqrt 2) / 2, with erfc(x) for x >= 0 by Abramowitz &
-// Stegun 7.1.26 (Hastings): erfc(x) = (a1 s + a2 s^2 + a3 s^3 + a4 s^4 + a5 s^5) exp(-x^2),
-// s = 1 / (1 + p x), absolute error below 1.5e-7; for t < 0 the same expression is Phi's tail
-// itself (no 1 - erf cancellation), for t >= 0 Phi = 1 - erfc(x) / 2. Branch-free, two MUFU ops.
+// GELU(t) = t * Phi(t), Phi the standard normal CDF. With h = Phi(-|t|) = erfc(|t| / sqrt 2) / 2 from
+// Abramowitz & Stegun 7.1.26 (Hastings): erfc(x) = (a1 s + a2 s^2 + a3 s^3 + a4 s^4 + a5 s^5) exp(-x^2),
+// s = 1 / (1 + p x), absolute error below 1.5e-7 (the halving folded into a1 .. a5, the 1 / sqrt 2
+// into p and into the exponent), GELU(t) = max(t, 0) - |t| h for either sign of t: t (1 - h) for
+// t >= 0, t h for t < 0, with no 1 - erf cancellation. Branch-free, two MUFU ops.
 __device__ __forceinline__ float gelu_erf(float t) {
-  const float x = fabsf(t) * 0.70710678118654752440f;
-  const float s = rcp_approx(fmaf(0.3275911f, x, 1.f));
-  float p = 1.061405429f;
-  p = fmaf(p, s, -1.453152027f);
-  p = fmaf(p, s, 1.421413741f);
-  p = fmaf(p, s, -0.284496736f);
-  p = fmaf(p, s, 0.254829592f);
-  const float half_erfc = 0.5f * p * s * ex2_approx(-1.44269504088896340736f * x * x);
-  return t * (t >= 0.f ? 1.f - half_erfc : half_erfc);
+  const float s = rcp_approx(fmaf(0.3275911f * 0.70710678118654752440f, fabsf(t), 1.f));
+  float q = 0.5f * 1.061405429f;
+  q = fmaf(q, s, 0.5f * -1.453152027f);
+  q = fmaf(q, s, 0.5f * 1.421413741f);
+  q = fmaf(q, s, 0.5f * -0.284496736f);
+  q = fmaf(q, s, 0.5f * 0.254829592f);
+  const float e = ex2_approx((t * -0.72134752044448170368f) * t);  // exp(-t^2 / 2)
+  const float h = (q * s) * e;
+  return fmaf(-fabsf(t), h, fmaxf(t, 0.f));
 }
 
 __device__ __forceinline__ void st_global_32B(void *p, const uint32_t (&w)[8]) {
-  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]),
+  asm volatile("st.global.L1::no_allocate.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]),
                "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
                : "memory");
 }
