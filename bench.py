@@ -448,7 +448,7 @@ def run_gpu(args, world, rank, local):
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "peak_source": f"{peak_src} bf16_tflops (burst, the dense bf16 cuBLAS rate)",
-                     "kernel": "lpvit::bsr_linear_kernel<32>", "launches_timed": linear_launches,
+                     "kernel": "lpvit::bsr_linear_kernel<gelu, f32_out>", "launches_timed": linear_launches,
                      "frac_of_sustained_peak": achieved / peak_sustained},
         "linear_ms_per_step": lin_ms / args.steps,
         "pack_and_gaps_ms_per_step": (elapsed_ms - lin_ms) / args.steps,

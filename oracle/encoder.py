@@ -53,6 +53,28 @@ def _bits_to_f64(bits):
     return bf16_to_f64(np.asarray(bits, dtype=np.uint16))
 
 
+def layer_forward(x_bits: np.ndarray, L, tokens: int, heads: int, eps: float = 1e-6,
+                  nthreads: int | None = None) -> np.ndarray:
+    """One encoder layer on the bf16 residual stream x_bits [images * tokens, D] (uint16 bits):
+    x + Attn(LN1(x)), then that + MLP(LN2(.)), every hand-off rounded to bf16; returns the new
+    stream as bf16 bits. ``L`` as for ``encoder_forward``."""
+    x = np.asarray(x_bits, dtype=np.uint16)
+    head_dim = x.shape[1] // heads
+    h = round_bf16(layernorm(_bits_to_f64(x), *L["ln1"], eps))
+    W, M, bias, b = L["qkv"]
+    qkv = round_bf16(linear(h, W, M, b, bias, False, nthreads))
+    a = round_bf16(attention(_bits_to_f64(qkv), tokens, heads, head_dim))
+    W, M, bias, b = L["proj"]
+    p = round_bf16(linear(a, W, M, b, bias, False, nthreads))
+    x = round_bf16(_bits_to_f64(x) + _bits_to_f64(p))
+    h = round_bf16(layernorm(_bits_to_f64(x), *L["ln2"], eps))
+    W, M, bias, b = L["fc1"]
+    f = round_bf16(linear(h, W, M, b, bias, True, nthreads))
+    W, M, bias, b = L["fc2"]
+    o = round_bf16(linear(f, W, M, b, bias, False, nthreads))
+    return round_bf16(_bits_to_f64(x) + _bits_to_f64(o))
+
+
 def encoder_forward(x_bits: np.ndarray, layers, final, tokens: int, heads: int, eps: float = 1e-6,
                     nthreads: int | None = None) -> np.ndarray:
     """The encoder on bf16 token activations x_bits [images * tokens, D] (uint16 bits); returns the
@@ -61,20 +83,6 @@ def encoder_forward(x_bits: np.ndarray, layers, final, tokens: int, heads: int, 
     ``layers``: per layer a dict with ln1 / ln2 = (gamma, beta) float32 arrays and qkv / proj / fc1 /
     fc2 = (W_bits, mask, bias, b) as for ``oracle.linear``; ``final`` = (gamma, beta)."""
     x = np.asarray(x_bits, dtype=np.uint16)
-    D = x.shape[1]
-    head_dim = D // heads
     for L in layers:
-        h = round_bf16(layernorm(_bits_to_f64(x), *L["ln1"], eps))
-        W, M, bias, b = L["qkv"]
-        qkv = round_bf16(linear(h, W, M, b, bias, False, nthreads))
-        a = round_bf16(attention(_bits_to_f64(qkv), tokens, heads, head_dim))
-        W, M, bias, b = L["proj"]
-        p = round_bf16(linear(a, W, M, b, bias, False, nthreads))
-        x = round_bf16(_bits_to_f64(x) + _bits_to_f64(p))
-        h = round_bf16(layernorm(_bits_to_f64(x), *L["ln2"], eps))
-        W, M, bias, b = L["fc1"]
-        f = round_bf16(linear(h, W, M, b, bias, True, nthreads))
-        W, M, bias, b = L["fc2"]
-        o = round_bf16(linear(f, W, M, b, bias, False, nthreads))
-        x = round_bf16(_bits_to_f64(x) + _bits_to_f64(o))
+        x = layer_forward(x, L, tokens, heads, eps, nthreads)
     return round_bf16(layernorm(_bits_to_f64(x), *final, eps))

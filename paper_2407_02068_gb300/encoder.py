@@ -59,9 +59,10 @@ class SparseEncoder:
                                  out=e(D), ws=ws)
         return self._bufs[M]
 
-    def forward(self, x: torch.Tensor) -> torch.Tensor:
+    def forward(self, x: torch.Tensor, streams: list | None = None) -> torch.Tensor:
         """x: bf16 [images * tokens, D] contiguous CUDA token activations. Returns bf16 [images * tokens, D]
-        (a buffer reused by the next call with the same shape)."""
+        (a buffer reused by the next call with the same shape). ``streams``: optional list that
+        receives a copy of the residual stream after each layer."""
         M = x.shape[0]
         B = self._buffers(M, x.device)
         # the residual stream ping-pongs between s0 and s1 (x itself is never written); proj and fc2
@@ -77,6 +78,8 @@ class SparseEncoder:
             bsr_linear(W["fc1"], B["h"], L["fc1"][2], gelu=True, out=B["f"], workspace=B["ws"]["fc1"])
             bsr_linear(W["fc2"], B["f"], L["fc2"][2], out=s_next, workspace=B["ws"]["fc2"], residual=s_cur)
             s_cur, s_next = s_next, (B["s1"] if s_next is B["s0"] else B["s0"])
+            if streams is not None:
+                streams.append(s_cur.clone())
         add_layernorm(s_cur, None, *self.final, eps=self.eps, norm_out=B["out"])
         return B["out"]
 

@@ -138,24 +138,39 @@ def test_deit_b_encoder_at_the_timed_configuration(lp):
     """The configuration `bench.py --encoder deit_b` times: DeiT-B, 12 layers, 256 images of 197
     tokens (M = 50432: its token tiles, slicing and attention grid), 32x32 blocks at the stack's
     per-GEMM sparsities. Images are independent, so the oracle runs each sampled image alone: the
-    first, the last and four seeded others, under the same gate as the DeiT-S test."""
+    first, the last and four seeded others. Layer by layer, the oracle layer applied to the GPU's
+    input stream of that layer must give the GPU's output stream under the DeiT-S gate; the final
+    LayerNorm likewise. Over all 12 layers the hand-off roundings compound (a value within the
+    accumulation error of a bf16 boundary rounds differently on the two sides, and later layers
+    carry that ulp), so end to end only the mean error is gated."""
     from paper_2407_02068_gb300.encoder import SparseEncoder
     model, b, config, images, T = inputs.DEIT_B, 32, 9, 256, 197
     D, heads = model["dim"], model["dim"] // 64
     layers, final = inputs.deit_encoder_params(model, b, config, 12, "cuda")
     enc = SparseEncoder(layers, final, heads, T, b)
     x = inputs.activations(images * T, D, inputs.seed(config, 0, "X"), "cuda")
-    y = enc.forward(x)
+    streams = []
+    y = enc.forward(x, streams)
     torch.cuda.synchronize()
+    assert len(streams) == 12
     ol, of = _oracle_layers(layers, final, b)
     rng = np.random.default_rng(20240702)
     sample = sorted({0, images - 1, *rng.choice(np.arange(1, images - 1), size=4, replace=False).tolist()})
-    xb, yb = _b(x), _b(y)
-    for img in sample:
-        rows = slice(img * T, (img + 1) * T)
-        ref = oracle.bf16_to_f64(oenc.encoder_forward(xb[rows], ol, of, T, heads))
-        got = oracle.bf16_to_f64(yb[rows])
+    sb = [_b(x)] + [_b(st) for st in streams]
+    yb = _b(y)
+
+    def gate(got_bits, ref_bits, what):
+        ref, got = oracle.bf16_to_f64(ref_bits), oracle.bf16_to_f64(got_bits)
         rms = np.sqrt(np.mean(ref ** 2))
         err = np.abs(got - ref)
-        assert np.all(err <= 2 * _ulp(ref) + 2.0 ** -7 * rms), (img, float(np.max(err / (_ulp(ref) + 1e-30))))
-        assert err.mean() <= 0.01 * rms, (img, err.mean() / rms)
+        assert np.all(err <= 2 * _ulp(ref) + 2.0 ** -7 * rms), (what, float(np.max(err / (_ulp(ref) + 1e-30))))
+        assert err.mean() <= 0.01 * rms, (what, err.mean() / rms)
+
+    for img in sample:
+        rows = slice(img * T, (img + 1) * T)
+        for li in range(12):
+            gate(sb[li + 1][rows], oenc.layer_forward(sb[li][rows], ol[li], T, heads), (img, li))
+        gate(yb[rows], oenc.encoder_forward(sb[12][rows], [], of, T, heads), (img, "final LayerNorm"))
+        ref = oracle.bf16_to_f64(oenc.encoder_forward(sb[0][rows], ol, of, T, heads))
+        got = oracle.bf16_to_f64(yb[rows])
+        assert np.abs(got - ref).mean() <= 0.01 * np.sqrt(np.mean(ref ** 2)), img
