@@ -111,32 +111,44 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
-__device__ __forceinline__ float rcp_approx(float x) {
-  float r;
-  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
-  return r;
-}
 __device__ __forceinline__ float ex2_approx(float x) {
   float r;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
   return r;
 }
 
-// GELU(t) = t * Phi(t), Phi the standard normal CDF. With h = Phi(-|t|) = erfc(|t| / sqrt 2) / 2 from
-// Abramowitz & Stegun 7.1.26 (Hastings): erfc(x) = (a1 s + a2 s^2 + a3 s^3 + a4 s^4 + a5 s^5) exp(-x^2),
-// s = 1 / (1 + p x), absolute error below 1.5e-7 (the halving folded into a1 .. a5, the 1 / sqrt 2
-// into p and into the exponent), GELU(t) = max(t, 0) - |t| h for either sign of t: t (1 - h) for
-// t >= 0, t h for t < 0, with no 1 - erf cancellation. Branch-free, two MUFU ops.
+// GELU(t) = t * Phi(t), Phi the standard normal CDF, as max(t, 0) - |t| h with h = Phi(-|t|) (t (1 - h)
+// for t >= 0, t h for t < 0, no 1 - erf cancellation). h = 2^P(x), x = min(|t|, 6), P the degree-10
+// polynomial fitted to log2 Phi(-x) on [0, 6] (least squares on Chebyshev nodes, reweighted towards
+// equal ripple): GELU within 4e-7 relative for |t| <= 0.1 and 2.5e-6 (float32 rounding included)
+// elsewhere; at x = 6 the tail is below 1e-9, so clamping there costs less than 1e-9 |t|.
+// Branch-free, one MUFU op (the erfc form with a reciprocal needs two, and MUFU throughput bounds
+// the GELU epilogue).
 __device__ __forceinline__ float gelu_erf(float t) {
-  const float s = rcp_approx(fmaf(0.3275911f * 0.70710678118654752440f, fabsf(t), 1.f));
-  float q = 0.5f * 1.061405429f;
-  q = fmaf(q, s, 0.5f * -1.453152027f);
-  q = fmaf(q, s, 0.5f * 1.421413741f);
-  q = fmaf(q, s, 0.5f * -0.284496736f);
-  q = fmaf(q, s, 0.5f * 0.254829592f);
-  const float e = ex2_approx((t * -0.72134752044448170368f) * t);  // exp(-t^2 / 2)
-  const float h = (q * s) * e;
+  const float x = fminf(fabsf(t), 6.f);
+  float p = -1.231680357705045e-08f;
+  p = fmaf(p, x, 4.146599508203508e-07f);
+  p = fmaf(p, x, -5.938332378718769e-06f);
+  p = fmaf(p, x, 4.5272547140484676e-05f);
+  p = fmaf(p, x, -0.0001642438000999391f);
+  p = fmaf(p, x, -0.00026072203763760626f);
+  p = fmaf(p, x, 0.007299995981156826f);
+  p = fmaf(p, x, -0.05271168798208237f);
+  p = fmaf(p, x, -0.45911723375320435f);
+  p = fmaf(p, x, -1.151119351387024f);
+  p = fmaf(p, x, -0.9999996423721313f);
+  const float h = ex2_approx(p);
   return fmaf(-fabsf(t), h, fmaxf(t, 0.f));
+}
+
+// mbarrier arrival without release semantics: for signals that hand over no memory written by this
+// thread (a TMEM buffer whose loads have completed, see tcgen05.wait::ld), so that the arrival does
+// not wait for this thread's outstanding global stores.
+__device__ __forceinline__ void mbar_arrive_relaxed(uint32_t bar) {
+  asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];" :: "r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_relaxed_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" :: "r"(cluster_addr) : "memory");
 }
 
 __device__ __forceinline__ void st_global_32B(void *p, const uint32_t (&w)[8]) {
@@ -549,21 +561,27 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     const int q = warp & 3;
     const int part = (warp - FIRST_EPI) >> 2;
     float *bias_s = reinterpret_cast<float *>(smem + L::BIAS_OFF) + (warp - FIRST_EPI) * 64;
-    uint32_t ui = 0;
-    while (true) {
-      const uint32_t slot = ui % UR, uph = (ui / UR) & 1u;
+    // The unit record of unit ui + 1 is taken (and its ring slot handed back) before unit ui's
+    // outputs are stored, so that this release-ordered arrival never waits for fresh stores.
+    auto take_unit = [&](uint32_t u, UnitInfo &out) -> bool {
+      const uint32_t slot = u % UR, uph = (u / UR) & 1u;
       if (!(leader ? mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)
                    : mbar_wait_cluster(unitf_bar(slot), uph, abort_flag, tmo))) {
         if (lane == 0) { atomicOr(&P.ctl->err, ERR_EPI_UNIT); *abort_flag = 1; }
-        break;
+        return false;
       }
-      const UnitInfo inf = ring[slot].inf;
+      out = ring[slot].inf;
       __syncwarp();
       if (lane == 0) {
         if (leader) mbar_arrive(unite_bar(slot));
         else mbar_arrive_cluster(mapa_rank(unite_bar(slot), 0));
       }
-      if (inf.tt < 0) break;
+      return true;
+    };
+    UnitInfo inf;
+    bool have = take_unit(0, inf);
+    uint32_t ui = 0;
+    while (have && inf.tt >= 0) {
       // the features of this warp's 64 columns (first feature of each 16-column quarter, or -1)
       int fcol[4];
 #pragma unroll
@@ -599,10 +617,13 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       const int64_t t = tok0 + lane;
       const bool tvalid = t < P.m;
       const bool split = inf.nsl > 1;
+      const bool touched = inf.e1 > inf.e0;
       float *part_row = nullptr;
       if (split)
         part_row = P.partials + ((int64_t)inf.ptile * P.part_rows + t_tile) * GROUP_FEATURES;
-      const bool touched = inf.e1 > inf.e0;
+      // the next unit's record, before this unit's stores
+      UnitInfo nxt;
+      have = take_unit(ui + 1, nxt);
 #pragma unroll 1
       for (int h = 0; h < 2; ++h) {
         const int c0 = 64 * part + 32 * h;  // first group row (accumulator column) of these 32
@@ -633,13 +654,15 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
         }
         __syncwarp();
       }
-      // the accumulator buffer is free again (the leader's MMAs wait for both CTAs' warps)
+      // the accumulator buffer is free again (the leader's MMAs wait for both CTAs' warps); its
+      // loads have completed and no memory written here is handed over, so no release ordering
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
-        if (leader) mbar_arrive(acce_bar(buf));
-        else mbar_arrive_cluster(mapa_rank(acce_bar(buf), 0));
+        if (leader) mbar_arrive_relaxed(acce_bar(buf));
+        else mbar_arrive_relaxed_cluster(mapa_rank(acce_bar(buf), 0));
       }
+      inf = nxt;
       ++ui;
     }
   }
