@@ -74,12 +74,14 @@ typedef struct {
 } lpvit_bsr;
 
 /* Bytes of the `sched` buffer needed for an n x k weight with bn x bk blocks (0 if the shape is
- * invalid). The work list groups the row panels into 128-feature groups (128 / bn panels each,
- * chosen so that the panels of a group keep blocks in overlapping columns, or consecutive panels
- * when that gives no fewer columns) and lists, per group, the block columns where any panel of the
- * group keeps a block (Sec. 3.3: one block matmul per kept block and token tile). It also holds a second copy of the kept weights, arranged entry
- * by entry as the GEMM's tensor-core tiles, so that the GEMM reads `sched` and never `blocks`;
- * that copy is sized for a dense weight: about 2*k*ceil(n/128)*128 bytes plus the list. */
+ * invalid). The work list groups the row panels into 256-feature groups (256 / bn panels each,
+ * chosen so that the panels of a group keep blocks in overlapping 64-column chunks, or
+ * consecutive panels when that gives no fewer chunks) and lists, per group, the chunks where any
+ * panel of the group keeps a block (Sec. 3.3: one block matmul per kept block and token tile; a
+ * chunk whose blocks are all removed is neither loaded nor multiplied). It also holds a second
+ * copy of the kept weights, arranged entry by entry as the GEMM's tensor-core tiles (256 rows x
+ * 64 columns, removed blocks as zeros), so that the GEMM reads `sched` and never `blocks`; that
+ * copy is sized for a dense weight: 2*64*256 bytes per (group, chunk) plus the list. */
 size_t lpvit_sched_bytes(int32_t n, int32_t k, int32_t bn, int32_t bk);
 
 /* Pack W (bf16 [n][k], row-major, 16-byte aligned) under the block mask (uint8 [n/bn][k/bk],

@@ -141,6 +141,49 @@ __device__ __forceinline__ float gelu_erf(float t) {
   return fmaf(-fabsf(t), h, fmaxf(t, 0.f));
 }
 
+// Two float32 lanes in one 64-bit register: fma / add of pairs (sm_100+ packed fp32 arithmetic,
+// each lane the IEEE float32 operation, so results equal the scalar ones).
+__device__ __forceinline__ uint64_t pk2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void unpk2(uint64_t v, float &lo, float &hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__host__ __device__ constexpr uint64_t splat2(uint32_t bits) { return ((uint64_t)bits << 32) | bits; }
+
+// gelu_erf of two values at once: the polynomial in packed pairs (half the FMA instructions).
+__device__ __forceinline__ void gelu_erf2(float &a, float &b) {
+  const uint64_t x = pk2(fminf(fabsf(a), 6.f), fminf(fabsf(b), 6.f));
+  uint64_t p = splat2(__float_as_uint(-1.231680357705045e-08f));
+  p = fma2(p, x, splat2(__float_as_uint(4.146599508203508e-07f)));
+  p = fma2(p, x, splat2(__float_as_uint(-5.938332378718769e-06f)));
+  p = fma2(p, x, splat2(__float_as_uint(4.5272547140484676e-05f)));
+  p = fma2(p, x, splat2(__float_as_uint(-0.0001642438000999391f)));
+  p = fma2(p, x, splat2(__float_as_uint(-0.00026072203763760626f)));
+  p = fma2(p, x, splat2(__float_as_uint(0.007299995981156826f)));
+  p = fma2(p, x, splat2(__float_as_uint(-0.05271168798208237f)));
+  p = fma2(p, x, splat2(__float_as_uint(-0.45911723375320435f)));
+  p = fma2(p, x, splat2(__float_as_uint(-1.151119351387024f)));
+  p = fma2(p, x, splat2(__float_as_uint(-0.9999996423721313f)));
+  float pa, pb;
+  unpk2(p, pa, pb);
+  const uint64_t h = pk2(ex2_approx(pa), ex2_approx(pb));
+  const uint64_t r = fma2(pk2(-fabsf(a), -fabsf(b)), h, pk2(fmaxf(a, 0.f), fmaxf(b, 0.f)));
+  unpk2(r, a, b);
+}
+
 // mbarrier arrival without release semantics: for signals that hand over no memory written by this
 // thread (a TMEM buffer whose loads have completed, see tcgen05.wait::ld), so that the arrival does
 // not wait for this thread's outstanding global stores.
@@ -183,13 +226,14 @@ template <bool GELU, bool F32>
 __device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, int64_t t, const LinearParams &P) {
 #pragma unroll
   for (int i = 0; i < 16; i += 4) {
-    float4 b;
-    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(b.x), "=f"(b.y), "=f"(b.z), "=f"(b.w) : "r"(bs + 4 * i));
-    y[i] += b.x; y[i + 1] += b.y; y[i + 2] += b.z; y[i + 3] += b.w;
+    uint64_t b01, b23;
+    asm volatile("ld.shared.v2.b64 {%0, %1}, [%2];" : "=l"(b01), "=l"(b23) : "r"(bs + 4 * i));
+    unpk2(add2(pk2(y[i], y[i + 1]), b01), y[i], y[i + 1]);
+    unpk2(add2(pk2(y[i + 2], y[i + 3]), b23), y[i + 2], y[i + 3]);
   }
   if (GELU) {
 #pragma unroll
-    for (int i = 0; i < 16; ++i) y[i] = gelu_erf(y[i]);
+    for (int i = 0; i < 16; i += 2) gelu_erf2(y[i], y[i + 1]);
   }
   if (t >= P.m) return;
   if (F32) {
