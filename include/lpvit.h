@@ -128,6 +128,16 @@ lpvit_status lpvit_pack_bsr_many(int32_t count, const void *const *W, const uint
 lpvit_status lpvit_taylor_block_mask(const void *W, const float *G, int32_t n, int32_t k, int32_t bn, int32_t bk,
                                      double prune_ratio, double *scores, uint8_t *mask, void *stream);
 
+/* Sec. 3.1 end to end in one call: the Taylor block mask of (W, G) at `prune_ratio` (exactly as
+ * lpvit_taylor_block_mask: scores into `scores`, the mask into `mask`) followed by the pack of W
+ * under that mask into `bsr` (exactly as lpvit_pack_bsr), all launched on `stream` with no host step
+ * between them: the mask passes from the ranking kernel to the pack through `mask` (n/bn x k/bk
+ * bytes, which the caller also gets), never through the host. Arguments as for the two calls;
+ * nnzb_host as for lpvit_pack_bsr (synchronises `stream` when not NULL).
+ * Errors: those of lpvit_taylor_block_mask and lpvit_pack_bsr. */
+lpvit_status lpvit_taylor_pack_bsr(const void *W, const float *G, double prune_ratio, double *scores, uint8_t *mask,
+                                   lpvit_bsr *bsr, int32_t *nnzb_host, void *stream);
+
 /* The first-order gradient of Sec. 3.1 / 3.5 as the mean of N per-sample gradients:
  * g[e] = (sum_i G[i][e]) / N in float32, the sum in sample order (IEEE float32 additions and
  * division: the precision of the gradients themselves).

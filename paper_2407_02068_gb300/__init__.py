@@ -8,6 +8,7 @@ or 64 (Table 2 uses 32x32, 64x32, 16x32 and 16x16). This package wraps the C lib
 
 * ``taylor_block_mask(W, G, b, alpha)`` -- the block mask from first-order Taylor scores (Sec. 3.1)
 * ``pack_bsr(W, mask, b)``  -- mask -> BSR pack + work list, on the GPU
+* ``taylor_pack_bsr(W, G, b, alpha)`` -- the Taylor mask and the pack in one call (no host step)
 * ``pack_bsr_many_into(ws, Ws, masks)`` -- the same for a list of weights in two launches
 * ``bsr_linear(w, X, bias, gelu=..., residual=...)`` -- Y = act(X (W (.) M)^T + bias), optionally
   plus a bf16 residual in the same pass (the x + sublayer(x) of a pre-norm block)
@@ -27,6 +28,7 @@ import torch
 from . import _lib
 
 __all__ = ["BsrWeight", "alloc_bsr", "pack_bsr", "pack_bsr_into", "pack_bsr_many_into", "taylor_block_mask",
+           "taylor_pack_bsr",
            "workspace_for", "bsr_linear", "check", "LpvitError", "delta_curve", "lambda_search", "mean_gradient",
            "add_layernorm", "attention"]
 
@@ -125,6 +127,30 @@ def taylor_block_mask(W: torch.Tensor, G: torch.Tensor, b, prune_ratio: float, s
     if st != _lib.LPVIT_OK:
         raise LpvitError(st, "lpvit_taylor_block_mask")
     return mask, scores
+
+
+def taylor_pack_bsr(W: torch.Tensor, G: torch.Tensor, b, prune_ratio: float, capacity: int | None = None,
+                    count: bool = False, stream=None):
+    """Sec. 3.1 end to end: the block mask from first-order Taylor scores at ``prune_ratio`` and the
+    pack of W under it, in one library call (lpvit_taylor_pack_bsr). W bf16 [n, k], G float32 [n, k],
+    both contiguous CUDA. Returns (BsrWeight, mask uint8 [n/bn, k/bk], scores float64 [n/bn, k/bk])."""
+    if W.dtype != torch.bfloat16 or not W.is_cuda or W.dim() != 2 or not W.is_contiguous():
+        raise ValueError("W must be a contiguous 2-D bf16 CUDA tensor")
+    if G.dtype != torch.float32 or G.shape != W.shape or not G.is_contiguous() or G.device != W.device:
+        raise ValueError("G must be a contiguous float32 tensor shaped like W on W's device")
+    n, k = W.shape
+    bn, bk = block_sides(b)
+    if bn <= 0 or bk <= 0 or n % bn or k % bk:
+        raise ValueError("n and k must be multiples of the block sides")
+    w = alloc_bsr(n, k, b, capacity, W.device)
+    scores = torch.empty((n // bn, k // bk), dtype=torch.float64, device=W.device)
+    mask = torch.empty((n // bn, k // bk), dtype=torch.uint8, device=W.device)
+    st, nnzb = _lib.lpvit_taylor_pack_bsr(W.data_ptr(), G.data_ptr(), prune_ratio, scores.data_ptr(),
+                                          mask.data_ptr(), w.struct(), count, _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_taylor_pack_bsr")
+    w.nnzb = nnzb
+    return w, mask, scores
 
 
 def delta_curve(W: torch.Tensor, G: torch.Tensor, b, steps: int, kappa: float, workspace: torch.Tensor | None = None,

@@ -21,7 +21,7 @@ LPVIT_ERR_WORKSPACE = 5
 LPVIT_BF16 = 0
 LPVIT_F32 = 1
 
-EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_workspace_bytes", "lpvit_bsr_linear",
+EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_taylor_pack_bsr", "lpvit_workspace_bytes", "lpvit_bsr_linear",
            "lpvit_bsr_linear_gelu", "lpvit_bsr_linear_noalloc", "lpvit_check", "lpvit_status_string",
            "lpvit_selftest_wait", "lpvit_pack_bsr_many", "lpvit_taylor_block_mask",
            "lpvit_delta_curve_workspace_bytes", "lpvit_delta_curve", "lpvit_lambda_search", "lpvit_mean_gradient",
@@ -65,6 +65,8 @@ def load(path: str | None = None):
         lib.lpvit_sched_bytes.argtypes = [I32, I32, I32, I32]
         lib.lpvit_pack_bsr.restype = ctypes.c_int
         lib.lpvit_pack_bsr.argtypes = [V, V, BP, ctypes.POINTER(I32), V]
+        lib.lpvit_taylor_pack_bsr.restype = ctypes.c_int
+        lib.lpvit_taylor_pack_bsr.argtypes = [V, V, ctypes.c_double, V, V, BP, ctypes.POINTER(I32), V]
         lib.lpvit_taylor_block_mask.restype = ctypes.c_int
         lib.lpvit_taylor_block_mask.argtypes = [V, V, I32, I32, I32, I32, ctypes.c_double, V, V, V]
         lib.lpvit_delta_curve_workspace_bytes.restype = SZ
@@ -114,6 +116,15 @@ def lpvit_pack_bsr(W_ptr: int, mask_ptr: int, bsr: lpvit_bsr, want_count: bool, 
     cnt = ctypes.c_int32(0)
     st = load().lpvit_pack_bsr(W_ptr, mask_ptr, ctypes.byref(bsr), ctypes.byref(cnt) if want_count else None,
                                stream)
+    return st, (cnt.value if want_count else None)
+
+
+def lpvit_taylor_pack_bsr(W_ptr: int, G_ptr: int, prune_ratio: float, scores_ptr: int, mask_ptr: int,
+                          bsr: lpvit_bsr, want_count: bool, stream: int):
+    """Returns (status, nnzb or None)."""
+    cnt = ctypes.c_int32(0)
+    st = load().lpvit_taylor_pack_bsr(W_ptr, G_ptr, prune_ratio, scores_ptr, mask_ptr, ctypes.byref(bsr),
+                                      ctypes.byref(cnt) if want_count else None, stream)
     return st, (cnt.value if want_count else None)
 
 

@@ -1,5 +1,6 @@
 // C ABI of liblpvit.so (declared in include/lpvit.h): argument checks, TMA tensor-map encoding,
 // work sizing, and launches on the caller's stream. No allocation happens here.
+#include <cmath>
 #include <cstdint>
 #include <cstring>
 #include <mutex>
@@ -9,6 +10,7 @@
 
 #include "lpvit.h"
 #include "lpvit_device.cuh"
+#include "lpvit_taylor.h"
 
 namespace lpvit {
 
@@ -81,12 +83,19 @@ bool shape_ok(int n, int k, int bn, int bk) {
 int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
 // Entries per slice. With at least half as many (token tile, group) units as CTA pairs, a unit
-// covers the whole group; otherwise the group's chunks are cut into slices so that about one unit
-// per pair exists, and the reduction kernel adds the slices' partial sums.
+// covers the whole group. Otherwise a group's chunks are cut into slices, whose fp32 partial sums a
+// second kernel adds, to bring the unit count towards one per pair, but only while every slice
+// keeps at least MIN_SLICE_CHUNKS chunks: below that the partial sums and the reduction launch cost
+// more than the extra pairs gain (DeiT batch 1, M = 197: K = 384 and 768 run 1.4-1.8x faster
+// unsplit, K = 3072 fastest in four slices).
+constexpr int MIN_SLICE_CHUNKS = 12;
 int choose_slice(int64_t n_tt, int n_groups, int kc, int pairs) {
   const int64_t units = n_tt * n_groups;
   if (2 * units >= pairs) return kc;
-  const int64_t nsl = ceil_div(pairs, units);
+  int64_t nsl = ceil_div(pairs, units);
+  const int64_t most = kc / MIN_SLICE_CHUNKS;
+  if (nsl > most) nsl = most;
+  if (nsl < 1) nsl = 1;
   const int64_t s = ceil_div(kc, nsl);
   return (int)(s < 1 ? 1 : (s > kc ? kc : s));
 }
@@ -277,6 +286,38 @@ lpvit_status lpvit_pack_bsr(const void *W, const uint8_t *mask, lpvit_bsr *bsr, 
   lpvit_status st = LPVIT_OK;
   if (!device_info(&sms, &st)) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = launch_pack(W, mask, n, k, bn, bk, bsr->row_ptr, bsr->col_idx, bsr->nnzb_capacity, bsr->blocks,
+                              static_cast<int32_t *>(bsr->sched), sms, s);
+  if (e != cudaSuccess) return LPVIT_ERR_CUDA;
+  if (nnzb_host) {
+    int32_t v = 0;
+    e = cudaMemcpyAsync(&v, bsr->row_ptr + n / bn, sizeof(v), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return LPVIT_ERR_CUDA;
+    *nnzb_host = v;
+    if (v > bsr->nnzb_capacity) return LPVIT_ERR_WORKSPACE;
+  }
+  return LPVIT_OK;
+}
+
+lpvit_status lpvit_taylor_pack_bsr(const void *W, const float *G, double prune_ratio, double *scores, uint8_t *mask,
+                                   lpvit_bsr *bsr, int32_t *nnzb_host, void *stream) {
+  const lpvit_status chk = check_pack_args(W, mask, bsr);
+  if (chk != LPVIT_OK) return chk;
+  const int n = bsr->n, k = bsr->k, bn = bsr->bn, bk = bsr->bk;
+  if (!(prune_ratio >= 0.0 && prune_ratio <= 1.0)) return LPVIT_ERR_INVALID_ARG;  // also rejects NaN
+  if (!G || !scores || !aligned(G, 16) || !aligned(scores, 8)) return LPVIT_ERR_INVALID_ARG;
+  const int64_t total = (int64_t)(n / bn) * (k / bk);
+  if (total > (int64_t)1 << 20) return LPVIT_ERR_UNSUPPORTED;
+  int sms = 0;
+  lpvit_status st = LPVIT_OK;
+  if (!device_info(&sms, &st)) return st;
+  // eliminated = round(alpha * blocks), half away from zero (as lpvit_taylor_block_mask)
+  const int64_t keep = total - (int64_t)floor(prune_ratio * (double)total + 0.5);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (launch_block_scores(static_cast<const uint16_t *>(W), G, n, k, bn, bk, scores, s) != cudaSuccess ||
+      launch_block_rank(scores, total, keep, mask, nullptr, s) != cudaSuccess)
+    return LPVIT_ERR_CUDA;
   cudaError_t e = launch_pack(W, mask, n, k, bn, bk, bsr->row_ptr, bsr->col_idx, bsr->nnzb_capacity, bsr->blocks,
                               static_cast<int32_t *>(bsr->sched), sms, s);
   if (e != cudaSuccess) return LPVIT_ERR_CUDA;

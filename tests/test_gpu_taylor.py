@@ -99,3 +99,45 @@ def test_mask_drives_pack_and_linear(lp):
     ref = oracle.linear(inputs.bf16_bits(X), inputs.bf16_bits(W), got_m, b, bias.cpu().numpy(), False)
     err = np.max(np.abs(Y.cpu().double().numpy() - ref)) / np.sqrt(np.mean(ref ** 2))
     assert err <= 1e-4 and w.nnzb == int(got_m.sum())
+
+
+@pytest.mark.parametrize("n,k,b,alpha", [(384, 256, 32, 0.5), (768, 3072, 32, 0.3), (1152, 384, 16, 0.6),
+                                         (768, 3072, (64, 32), 0.615), (384, 1536, (16, 32), 0.287),
+                                         (256, 512, 64, 1.0), (256, 512, 32, 0.0)])
+def test_fused_taylor_pack_matches_mask_then_pack(lp, n, k, b, alpha):
+    """lpvit_taylor_pack_bsr (mask and pack in one call, no host step) gives bit for bit the scores,
+    mask, BSR arrays and work list of lpvit_taylor_block_mask followed by lpvit_pack_bsr; its mask
+    agrees with the oracle's away from the cut-off and its pack with the oracle's pack of that mask;
+    a linear on it matches the oracle."""
+    bn, bk = inputs.block_sides(b)
+    W, G = _wg(n, k, 6100 + n + k + (bn if bn == bk else 100 * bn + bk))
+    wf, mf, sf = lp.taylor_pack_bsr(W, G, b, alpha, count=True)
+    ms, ss = lp.taylor_block_mask(W, G, b, alpha)
+    ws = lp.pack_bsr(W, ms, b, count=True)
+    torch.cuda.synchronize()
+    assert torch.equal(sf.view(torch.int64), ss.view(torch.int64)) and torch.equal(mf, ms)
+    assert wf.nnzb == ws.nnzb and torch.equal(wf.row_ptr, ws.row_ptr)
+    assert torch.equal(wf.col_idx[:wf.nnzb], ws.col_idx[:ws.nnzb])
+    assert torch.equal(wf.blocks[:wf.nnzb].view(torch.int16), ws.blocks[:ws.nnzb].view(torch.int16))
+    hdr = wf.sched[:64].view(torch.int32).cpu().numpy()
+    ng, kc = int(hdr[1]), -(-k // 64)
+    table_end = 4 * (16 + ng + 1 + 16 * ng)              # header, group pointers, group table
+    ent0 = 4 * ((16 + ng + 1 + 16 * ng + 3) // 4 * 4)   # entries (after padding to 16 bytes)
+    ent_end = ent0 + 4 * int(hdr[2])
+    stream = (4 * ((16 + ng + 1 + 16 * ng + 3) // 4 * 4 + ng * kc) + 1023) // 1024 * 1024
+    used = stream + int(hdr[2]) * 256 * 64 * 2
+    assert torch.equal(wf.sched[:table_end], ws.sched[:table_end])
+    assert torch.equal(wf.sched[ent0:ent_end], ws.sched[ent0:ent_end])
+    assert torch.equal(wf.sched[stream:used], ws.sched[stream:used])
+    exact = oracle.block_scores(inputs.bf16_bits(W), G.cpu().numpy(), b)
+    got_m = mf.cpu().numpy()
+    assert_mask_matches_away_from_cutoff(got_m, exact, alpha, bn, bk)
+    rp, ci, bl = oracle.pack(inputs.bf16_bits(W), got_m, b)
+    assert np.array_equal(wf.row_ptr.cpu().numpy(), rp) and np.array_equal(wf.col_idx[:wf.nnzb].cpu().numpy(), ci)
+    assert np.array_equal(wf.blocks[:wf.nnzb].contiguous().view(torch.int16).cpu().numpy().view(np.uint16), bl)
+    X = inputs.activations(197, k, 6200 + n, "cuda")
+    bias = inputs.bias(n, 6300 + n, "cuda")
+    Y = lp.bsr_linear(wf, X, bias, out_dtype=torch.float32)
+    ref = oracle.linear(inputs.bf16_bits(X), inputs.bf16_bits(W), got_m, b, bias.cpu().numpy())
+    err = np.max(np.abs(Y.cpu().double().numpy() - ref)) / max(np.sqrt(np.mean(ref ** 2)), 1e-30)
+    assert err <= 1e-4

@@ -48,7 +48,8 @@ def _err(y, ref):
 
 
 @pytest.mark.parametrize("m,n,k,b,gelu", [(20000, 512, 384, 32, False),   # one slice per group
-                                          (197, 384, 256, 32, True),       # split slices + fix-up
+                                          (197, 768, 3072, 32, True),      # split slices + fix-up
+                                          (197, 384, 256, 32, True),       # short: one slice per group
                                           (300, 256, 128, 16, False),
                                           (600, 256, 512, 64, True)])
 def test_noalloc_matches_existing_entry_point_twice(lp, m, n, k, b, gelu):
@@ -68,7 +69,7 @@ def test_noalloc_matches_existing_entry_point_twice(lp, m, n, k, b, gelu):
 
 def test_noalloc_rejects_work_beyond_its_array(lp):
     from paper_2407_02068_gb300 import _lib
-    m, n, k, b = 197, 3072, 768, 32   # small m, many groups: the split partial sums need > 8 MiB
+    m, n, k, b = 197, 3072, 3072, 32   # small m, long k, many groups: the split partial sums need > 8 MiB
     X, W, bias, mask = _case(m, n, k, b, 77)
     w = lp.pack_bsr(W, mask, b)
     assert _lib.lpvit_workspace_bytes(w.struct(), m) > _lib.LPVIT_NOALLOC_SCRATCH_BYTES
