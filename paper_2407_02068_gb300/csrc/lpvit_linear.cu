@@ -13,7 +13,8 @@
 //               every copy completing on the leader's full barrier.
 //   warp 18     weight producer: the same walk, loading the weight tiles (a second issuing warp:
 //               a tensor copy keeps its issuing thread for a few hundred cycles).
-//   warp 19     scheduler (leader only): takes units from a global atomic queue and publishes each,
+//   warp 19     scheduler (leader only): takes units (pair p's first unit is unit p, the rest come
+//               from a global atomic queue) and publishes each,
 //               with the chunk indices of its first 32 entries, to both CTAs' unit rings, up to
 //               UR units ahead of the producers.
 //   warp 1      MMA issuer (leader only): per stage four MMAs, the commit multicast to both CTAs'
@@ -328,22 +329,24 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     tmem_alloc_pair(smem_u32(tmem_slot), 512);  // one warp of each CTA, together
     tmem_relinquish_pair();
   }
-  if (tid == 0) {
-    for (int i = 0; i < NSTAGES; ++i) {
-      mbar_init(full_bar(i), 1);
-      mbar_init(empty_bar(i), 1);
+  if (warp == 0) {  // the barriers initialised by the lanes of one warp, one or two each
+    if (lane < NSTAGES) {
+      mbar_init(full_bar(lane), 1);
+      mbar_init(empty_bar(lane), 1);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(accf_bar(b), 1);
-      mbar_init(acce_bar(b), 2 * EPI_WARPS);
+    if (lane < 2) {
+      mbar_init(accf_bar(lane), 1);
+      mbar_init(acce_bar(lane), 2 * EPI_WARPS);
     }
-    for (int u = 0; u < UR; ++u) {
-      mbar_init(unitf_bar(u), 1);
-      mbar_init(unite_bar(u), UNIT_CONSUMERS);
+    if (lane < UR) {
+      mbar_init(unitf_bar(lane), 1);
+      mbar_init(unite_bar(lane), UNIT_CONSUMERS);
     }
-    mbar_init(drain_bar, 1);
-    *abort_flag = 0;
-    *never_flag = 0;
+    if (lane == 0) {
+      mbar_init(drain_bar, 1);
+      *abort_flag = 0;
+      *never_flag = 0;
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0 && lane == 0) {
@@ -469,8 +472,10 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       const int ge_end = sched_ok ? gent[P.n_groups] : 0;
       const uint32_t total_units = sched_ok ? (uint32_t)P.n_tt * (uint32_t)total_slices : 0u;
       bool ok = true;
-      uint32_t fetched = 0;
-      if (lane == 0) fetched = atomicAdd(&P.ctl->next_unit, 1u);
+      // the first unit of pair p is unit p (no queue round trip before the first copies); the queue
+      // hands out the units after the first gridDim.x / 2
+      const uint32_t npairs = gridDim.x / 2;
+      uint32_t fetched = blockIdx.x / 2;
       for (uint32_t pub = 0;; ++pub) {
         const uint32_t slot = pub % UR;
         if (!mbar_wait_cluster(unite_bar(slot), ((pub / UR) & 1u) ^ 1u, abort_flag, tmo)) {
@@ -501,7 +506,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
           d.tt = -1; d.g = d.s = d.nsl = d.e0 = d.e1 = d.ptile = 0;
         }
         d.pad = 0;
-        if (lane == 0 && u < total_units) fetched = atomicAdd(&P.ctl->next_unit, 1u);
+        if (lane == 0 && u < total_units) fetched = npairs + atomicAdd(&P.ctl->next_unit, 1u);
         const int wv = d.e0 + lane < d.e1 ? __ldg(entries + d.e0 + lane) : 0;
         UnitSlot &rs = ring[slot];
         const uint32_t remote = mapa_rank(smem_u32(&rs), 1);
