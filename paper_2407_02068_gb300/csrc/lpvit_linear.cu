@@ -44,7 +44,8 @@ constexpr int W_BYTES = HALF_FEATURES * CHUNK_COLS * 2;   // 16 KB: this CTA's w
 constexpr int STAGE_BYTES = X_BYTES + W_BYTES;
 constexpr int KSTEPS = CHUNK_COLS / 16;
 constexpr int BUF_COLS = GROUP_FEATURES;                  // TMEM columns of one accumulator
-constexpr int UR = 8;                                     // unit ring depth
+constexpr int UR = 3;                                     // unit ring depth: units are handed out at most
+                                                          // three ahead, so the queue's last units stay balanced
 constexpr int BATCH = 2;                                  // stages per producer batch
 static_assert(32 % BATCH == 0, "producer batches tile the 32-entry windows");
 constexpr int FIRST_EPI = 2;
