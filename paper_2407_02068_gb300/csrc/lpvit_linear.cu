@@ -38,12 +38,17 @@ namespace lpvit {
 
 namespace {
 
-constexpr int NSTAGES = 6;
+// Stages of the copy pipeline: six when the epilogue stages its bias in shared memory, seven when it
+// reads the bias from the L1-cached global copy instead (the fourth kilobyte of that staging is what
+// a seventh stage needs). Long-K launches (many entries per unit) are bound by the copy feed and take
+// the deeper ring; short-K launches are bound by their epilogue and keep the staged bias.
+template <bool DEEP> struct Depth { static constexpr int NSTAGES = DEEP ? 7 : 6; };
 constexpr int X_BYTES = CTA_TOKENS * CHUNK_COLS * 2;      // 16 KB: this CTA's tokens x 64 columns
 constexpr int W_BYTES = HALF_FEATURES * CHUNK_COLS * 2;   // 16 KB: this CTA's weight rows x 64 columns
 constexpr int STAGE_BYTES = X_BYTES + W_BYTES;
 constexpr int KSTEPS = CHUNK_COLS / 16;
 constexpr int BUF_COLS = GROUP_FEATURES;                  // TMEM columns of one accumulator
+constexpr int DEEP_MIN_CHUNKS = 24;                       // units of >= 24 entries take seven stages
 constexpr int UR = 3;                                     // unit ring depth: units are handed out at most
                                                           // three ahead, so the queue's last units stay balanced
 constexpr int BATCH = 2;                                  // stages per producer batch
@@ -74,14 +79,16 @@ struct UnitSlot {
   int win[32];
 };
 
+template <bool DEEP>
 struct Smem {
+  static constexpr int NSTAGES = Depth<DEEP>::NSTAGES;
   static constexpr int BAR_OFF = NSTAGES * STAGE_BYTES;
   // barriers: full[NS], empty[NS], accf[2], acce[2], unitf[UR], unite[UR], drain
   static constexpr int NBARS = 2 * NSTAGES + 4 + 2 * UR + 1;
   static constexpr int RING_OFF = (BAR_OFF + 8 * NBARS + 31) / 32 * 32;
   static constexpr int MISC_OFF = RING_OFF + (int)sizeof(UnitSlot) * UR;
   static constexpr int BIAS_OFF = MISC_OFF + 64;  // per epilogue warp: its 64 features' bias
-  static constexpr int END = BIAS_OFF + EPI_WARPS * 64 * 4;
+  static constexpr int END = BIAS_OFF + (DEEP ? 0 : EPI_WARPS * 64 * 4);
   static constexpr int BYTES = END + 1024;  // + alignment slack for the dynamic smem base
   static_assert(BYTES <= 227 * 1024, "shared memory per CTA");
 };
@@ -224,12 +231,24 @@ __device__ __forceinline__ int table_at(const int (&t)[N], int g) {
 // every lane). Adds the bias, applies GELU, rounds and stores the lane's 32-byte (bf16) or 64-byte
 // (fp32) row segment with 32-byte stores, so that each store instruction writes whole sectors;
 // bf16 output may add the residual (each sum rounded, as a separate bf16 addition would).
-template <bool GELU, bool F32>
+template <bool GELU, bool F32, bool BIASG>
 __device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, int64_t t, const LinearParams &P) {
 #pragma unroll
   for (int i = 0; i < 16; i += 4) {
-    uint64_t b01, b23;
-    asm volatile("ld.shared.v2.b64 {%0, %1}, [%2];" : "=l"(b01), "=l"(b23) : "r"(bs + 4 * i));
+    uint64_t b01 = 0, b23 = 0;
+    if (!BIASG) {
+      asm volatile("ld.shared.v2.b64 {%0, %1}, [%2];" : "=l"(b01), "=l"(b23) : "r"(bs + 4 * i));
+    } else if (P.bias != nullptr) {  // the same 16 features for every lane: a broadcast load from L1
+      float4 bb;
+      if (P.bias_vec16) {
+        bb = __ldg(reinterpret_cast<const float4 *>(P.bias + f0 + i));
+      } else {
+        bb = make_float4(__ldg(P.bias + f0 + i), __ldg(P.bias + f0 + i + 1), __ldg(P.bias + f0 + i + 2),
+                         __ldg(P.bias + f0 + i + 3));
+      }
+      b01 = pk2(bb.x, bb.y);
+      b23 = pk2(bb.z, bb.w);
+    }
     unpk2(add2(pk2(y[i], y[i + 1]), b01), y[i], y[i + 1]);
     unpk2(add2(pk2(y[i + 2], y[i + 3]), b23), y[i + 2], y[i + 3]);
   }
@@ -293,11 +312,12 @@ __device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, 
   }
 }
 
-template <bool GELU, bool F32>
+template <bool GELU, bool F32, bool DEEP>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
 bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
                   const LinearParams P) {
-  using L = Smem;
+  using L = Smem<DEEP>;
+  constexpr int NSTAGES = L::NSTAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t smem_base = smem_u32(smem);
@@ -610,7 +630,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     // quarter q = w % 4 (tokens 32 q .. 32 q + 31) and the 64 columns of part (w - 2) / 4.
     const int q = warp & 3;
     const int part = (warp - FIRST_EPI) >> 2;
-    float *bias_s = reinterpret_cast<float *>(smem + L::BIAS_OFF) + (warp - FIRST_EPI) * 64;
+    float *bias_s = reinterpret_cast<float *>(smem + L::BIAS_OFF) + (warp - FIRST_EPI) * 64;  // (not DEEP)
     // The unit record of unit ui + 1 is taken (and its ring slot handed back) before unit ui's
     // outputs are stored, so that this release-ordered arrival never waits for fresh stores.
     auto take_unit = [&](uint32_t u, UnitInfo &out) -> bool {
@@ -641,7 +661,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
         fcol[r4] = panel >= 0 ? panel * P.bn + c % P.bn : -1;
       }
       // and their bias, staged while the accumulator is still being computed
-      if (lane < 16) {
+      if (!DEEP && lane < 16) {
         const int qq = lane >> 2;  // the lane's quarter, selected without indexing the array
         const int fq = qq == 0 ? fcol[0] : (qq == 1 ? fcol[1] : (qq == 2 ? fcol[2] : fcol[3]));
         const int f = fq < 0 ? -1 : fq + 4 * (lane & 3);
@@ -699,8 +719,8 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
             yb[i] = v[16 + i];
           }
           const uint32_t bs = smem_u32(bias_s + 32 * h);
-          if (fa >= 0) emit_run16<GELU, F32>(ya, bs, fa, t, P);
-          if (fb2 >= 0) emit_run16<GELU, F32>(yb, bs + 64, fb2, t, P);
+          if (fa >= 0) emit_run16<GELU, F32, DEEP>(ya, bs, fa, t, P);
+          if (fb2 >= 0) emit_run16<GELU, F32, DEEP>(yb, bs + 64, fb2, t, P);
         }
         __syncwarp();
       }
@@ -822,19 +842,28 @@ cudaError_t launch_linear(const CUtensorMap &tmX, const CUtensorMap &tmW, const 
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    for (auto k : {bsr_linear_kernel<false, false>, bsr_linear_kernel<true, false>, bsr_linear_kernel<false, true>,
-                   bsr_linear_kernel<true, true>}) {
-      cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem::BYTES);
+    for (auto k : {bsr_linear_kernel<false, false, false>, bsr_linear_kernel<true, false, false>,
+                   bsr_linear_kernel<false, true, false>, bsr_linear_kernel<true, true, false>}) {
+      cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<false>::BYTES);
+      if (e != cudaSuccess) return e;
+    }
+    for (auto k : {bsr_linear_kernel<false, false, true>, bsr_linear_kernel<true, false, true>,
+                   bsr_linear_kernel<false, true, true>, bsr_linear_kernel<true, true, true>}) {
+      cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, Smem<true>::BYTES);
       if (e != cudaSuccess) return e;
     }
     attr_done[dev] = true;
   }
-  auto kern = P.gelu ? (P.y_f32 ? bsr_linear_kernel<true, true> : bsr_linear_kernel<true, false>)
-                     : (P.y_f32 ? bsr_linear_kernel<false, true> : bsr_linear_kernel<false, false>);
+  // long K (at least DEEP_MIN_CHUNKS entries per unit): the seven-stage variant
+  const bool deep = sched_chunks(P.k) >= DEEP_MIN_CHUNKS && P.S >= DEEP_MIN_CHUNKS;
+  auto kern = deep ? (P.gelu ? (P.y_f32 ? bsr_linear_kernel<true, true, true> : bsr_linear_kernel<true, false, true>)
+                             : (P.y_f32 ? bsr_linear_kernel<false, true, true> : bsr_linear_kernel<false, false, true>))
+                   : (P.gelu ? (P.y_f32 ? bsr_linear_kernel<true, true, false> : bsr_linear_kernel<true, false, false>)
+                             : (P.y_f32 ? bsr_linear_kernel<false, true, false> : bsr_linear_kernel<false, false, false>));
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3(NUM_THREADS);
-  cfg.dynamicSmemBytes = Smem::BYTES;
+  cfg.dynamicSmemBytes = deep ? Smem<true>::BYTES : Smem<false>::BYTES;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
