@@ -494,8 +494,10 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       const uint32_t total_units = sched_ok ? (uint32_t)P.n_tt * (uint32_t)total_slices : 0u;
       bool ok = true;
       // the first unit of pair p is unit p (no queue round trip before the first copies); the queue
-      // hands out the units after the first gridDim.x / 2
+      // hands out the units after the first gridDim.x / 2. When every unit is such a first unit
+      // (small token counts), no pair touches the queue or its counters.
       const uint32_t npairs = gridDim.x / 2;
+      const bool queued = total_units > npairs;  // the same in every pair
       uint32_t fetched = blockIdx.x / 2;
       for (uint32_t pub = 0;; ++pub) {
         const uint32_t slot = pub % UR;
@@ -527,7 +529,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
           d.tt = -1; d.g = d.s = d.nsl = d.e0 = d.e1 = d.ptile = 0;
         }
         d.pad = 0;
-        if (lane == 0 && u < total_units) fetched = npairs + atomicAdd(&P.ctl->next_unit, 1u);
+        if (lane == 0 && u < total_units) fetched = queued ? npairs + atomicAdd(&P.ctl->next_unit, 1u) : total_units;
         const int wv = d.e0 + lane < d.e1 ? __ldg(entries + d.e0 + lane) : 0;
         UnitSlot &rs = ring[slot];
         const uint32_t remote = mapa_rank(smem_u32(&rs), 1);
@@ -551,7 +553,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       }
       if (!ok && lane == 0) *abort_flag = 1;
       // queue bookkeeping: the last scheduler to leave resets the counters for the next launch
-      if (lane == 0) {
+      if (lane == 0 && queued) {
         __threadfence();
         if (atomicAdd(&P.ctl->done_ctas, 1u) == gridDim.x / 2 - 1) {
           P.ctl->next_unit = 0;
