@@ -14,9 +14,9 @@
  * square 16x16, 32x32, 64x64 and the paper's 64x32 and 16x32 of Table 2 are all covered),
  * act = identity (lpvit_bsr_linear) or the exact GELU
  * 0.5*y*(1+erf(y/sqrt 2)) (lpvit_bsr_linear_gelu, the DeiT fc1 activation). Only the kept
- * blocks are stored, and removed blocks are never read. The GEMM multiplies, per 128-output group,
- * only the block columns where the group keeps a block (rows of removed blocks there enter as
- * zeros), so its work follows those group columns rather than exactly the kept blocks that the
+ * blocks are stored, and removed blocks are never read. The GEMM multiplies, per 256-output group,
+ * only the 64-column chunks where the group keeps a block (rows of removed blocks there enter as
+ * zeros), so its work follows those group chunks rather than exactly the kept blocks that the
  * power model of Sec. 3.3 (Eq. for P) counts.
  *
  * Conventions for every call:
@@ -209,10 +209,11 @@ lpvit_status lpvit_attention(const void *qkv, int64_t images, int32_t tokens, in
                              void *out, void *stream);
 
 /* Bytes of device workspace lpvit_bsr_linear[_gelu] needs for m tokens. The workspace holds
- * scheduler counters, the device error word and, for small m, fp32 partial sums of split
- * work units. It must be zero-filled once before its first use (cudaMemset); every call
- * leaves its counters at zero again. Calls that may run concurrently must not share a
- * workspace. */
+ * scheduler counters, the device error word and, where few token tiles cannot fill the GPU, room
+ * for fp32 partial sums of split work units (token counts up to 256 run a single-launch kernel
+ * that needs only the counters and the error word; the size asked for does not depend on that).
+ * It must be zero-filled once before its first use (cudaMemset); every call leaves its counters
+ * at zero again. Calls that may run concurrently must not share a workspace. */
 size_t lpvit_workspace_bytes(const lpvit_bsr *bsr, int64_t m);
 
 /* Y = X W~^T + bias for m tokens.
@@ -222,6 +223,10 @@ size_t lpvit_workspace_bytes(const lpvit_bsr *bsr, int64_t m);
  *         only columns [0, n) of rows [0, m) are written. X and Y must not overlap.
  *   workspace / ws_bytes: see lpvit_workspace_bytes.
  * Output columns of a panel with no kept block equal bias (or GELU(bias)).
+ * m <= 256 (a ViT at batch 1: 197 tokens) runs one launch of plain CTAs, each 128 tokens x 32
+ * features of one group over a share of its chunks, a long K cut over the CTAs of a cluster and
+ * added in a fixed order; larger m runs the persistent CTA-pair kernel. Both are deterministic:
+ * repeated calls give the same bits.
  * Errors: LPVIT_ERR_INVALID_ARG, LPVIT_ERR_UNSUPPORTED, LPVIT_ERR_WORKSPACE, LPVIT_ERR_CUDA. */
 lpvit_status lpvit_bsr_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias,
                               void *Y, int64_t ldy, lpvit_dtype y_dtype, void *workspace, size_t ws_bytes,

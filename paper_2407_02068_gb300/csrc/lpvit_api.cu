@@ -166,36 +166,9 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   if (!device_info(&sms, &st)) return st;
   const WsLayout W = ws_layout(m, n, k, sms);
   if (ws_bytes < W.total) return LPVIT_ERR_WORKSPACE;
-  EncodeTiledFn enc = encode_fn();
-  if (!enc) return LPVIT_ERR_CUDA;
-
   const int ng = (int)ceil_div(n, GROUP_FEATURES);
   const int kc = sched_chunks(k);
   const int64_t stream_tiles = sched_stream_tiles(ng, kc);
-  cuuint32_t es[2] = {1, 1};
-  // X: [m rows][k columns], boxes of 64 columns x 128 tokens (one CTA's half of a token tile);
-  // rows beyond m and columns beyond k read as zero
-  CUtensorMap tmX, tmW;
-  {
-    cuuint64_t dims[2] = {(cuuint64_t)k, (cuuint64_t)m};
-    cuuint64_t strides[1] = {(cuuint64_t)ldx * 2};
-    cuuint32_t box[2] = {(cuuint32_t)CHUNK_COLS, (cuuint32_t)CTA_TOKENS};
-    if (enc(&tmX, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(X), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return LPVIT_ERR_INVALID_ARG;
-  }
-  // the weight stream: tiles of 256 rows x 64 columns, boxes of 128 rows (one CTA's half)
-  {
-    void *wstream = static_cast<uint8_t *>(bsr->sched) + sched_stream_offset_bytes(ng, kc);
-    cuuint64_t dims[2] = {(cuuint64_t)CHUNK_COLS, (cuuint64_t)(stream_tiles * GROUP_FEATURES)};
-    cuuint64_t strides[1] = {(cuuint64_t)CHUNK_COLS * 2};
-    cuuint32_t box[2] = {(cuuint32_t)CHUNK_COLS, (cuuint32_t)HALF_FEATURES};
-    if (enc(&tmW, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, wstream, dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return LPVIT_ERR_INVALID_ARG;
-  }
   LinearParams P;
   P.sched = static_cast<const int32_t *>(bsr->sched);
   P.stream_tiles = stream_tiles;
@@ -222,10 +195,43 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.partials = reinterpret_cast<float *>(ws + W.partials_off);
   P.part_rows = W.part_rows;
   P.timeout_ns = TIMEOUT_NS;
+  P.X = static_cast<const uint16_t *>(X);
+  P.ldx = ldx;
+  P.wstream = reinterpret_cast<const uint16_t *>(static_cast<const uint8_t *>(bsr->sched) +
+                                                 sched_stream_offset_bytes(ng, kc));
+  P.kp = 1;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (m <= SMALL_M_MAX) return cuda_status(launch_linear_small(P, sms, s));
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return LPVIT_ERR_CUDA;
+
+  cuuint32_t es[2] = {1, 1};
+  // X: [m rows][k columns], boxes of 64 columns x 128 tokens (one CTA's half of a token tile);
+  // rows beyond m and columns beyond k read as zero
+  CUtensorMap tmX, tmW;
+  {
+    cuuint64_t dims[2] = {(cuuint64_t)k, (cuuint64_t)m};
+    cuuint64_t strides[1] = {(cuuint64_t)ldx * 2};
+    cuuint32_t box[2] = {(cuuint32_t)CHUNK_COLS, (cuuint32_t)CTA_TOKENS};
+    if (enc(&tmX, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(X), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return LPVIT_ERR_INVALID_ARG;
+  }
+  // the weight stream: tiles of 256 rows x 64 columns, boxes of 128 rows (one CTA's half)
+  {
+    void *wstream = static_cast<uint8_t *>(bsr->sched) + sched_stream_offset_bytes(ng, kc);
+    cuuint64_t dims[2] = {(cuuint64_t)CHUNK_COLS, (cuuint64_t)(stream_tiles * GROUP_FEATURES)};
+    cuuint64_t strides[1] = {(cuuint64_t)CHUNK_COLS * 2};
+    cuuint32_t box[2] = {(cuuint32_t)CHUNK_COLS, (cuuint32_t)HALF_FEATURES};
+    if (enc(&tmW, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, wstream, dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return LPVIT_ERR_INVALID_ARG;
+  }
   const int pairs = sms / 2;
   const int64_t units_max = (int64_t)P.n_tt * P.n_groups * ceil_div(kc, P.S);
   const int grid = 2 * (int)(units_max < pairs ? units_max : pairs);
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
   cudaError_t e = launch_linear(tmX, tmW, P, grid, s);
   if (e != cudaSuccess || !W.split) return cuda_status(e);
   ReduceParams RP;

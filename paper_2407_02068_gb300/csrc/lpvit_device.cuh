@@ -83,6 +83,11 @@ struct LinearParams {
   float *partials;         // split units: [slice][part_rows][GROUP_FEATURES] fp32 partial sums
   int part_rows;           // token rows of one partial tile: min(m, TOKENS_PER_TILE)
   uint64_t timeout_ns;     // limit of every device-side wait
+  // read by the small-m kernel only (the pair kernel reaches X and the stream through tensor maps)
+  const uint16_t *X;       // bf16 [m][ldx]
+  int64_t ldx;
+  const uint16_t *wstream; // the work list's weight stream
+  int kp;                  // K parts per (group, row slice, token tile): the CTAs of one cluster
 };
 
 // Parameter block of the split-slice reduction (after the linear kernel, same stream).
@@ -139,6 +144,10 @@ cudaError_t launch_pack_many(const PackJob *jobs, int count, int num_sms, cudaSt
 cudaError_t launch_linear(const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
                           cudaStream_t s);
 cudaError_t launch_split_reduce(const ReduceParams &R, int64_t threads, cudaStream_t s);
+// Token counts up to SMALL_M_MAX take the small-m kernel (one launch, no workspace beyond the
+// control block); it sets P.kp itself.
+constexpr int SMALL_M_MAX = 256;
+cudaError_t launch_linear_small(LinearParams P, int num_sms, cudaStream_t s);
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 

@@ -834,6 +834,295 @@ __global__ void __launch_bounds__(256) split_reduce_kernel(const ReduceParams R)
   }
 }
 
+// ------------------------------------------------------------------------------------ small m
+// Token counts up to SMALL_M_MAX (batch 1 of a ViT is 197 tokens): the pair kernel's fixed cost --
+// cluster launch, TMEM allocation for 512 columns, the scheduler's dependent loads, a second launch
+// for split slices -- is most of such a call. Here plain CTAs of four warps each compute 128 tokens x
+// 32 group rows of one group over a share of the group's entries, from the same work list and
+// weight stream. All 128 threads copy each entry's X and weight rows with 16-byte cp.async into a
+// five-stage ring (two CTAs per SM), in the 128-byte-swizzled K-major layout the tensor core reads (piece j of row r
+// at j ^ (r mod 8) inside 1024-byte atoms); one thread issues the entry's four tcgen05 MMAs
+// (M = 128 tokens, N = 32 rows, K = 16) into 32 TMEM columns and commits them to the stage's
+// mbarrier, which frees the stage for its next copy. A long K is cut into kp parts run by the kp
+// CTAs of one cluster; their partial sums meet in distributed shared memory and are added in rank
+// order (deterministic), each CTA finishing 128 / kp of the tokens.
+constexpr int SM_TOK = 128;                           // tokens per CTA: the MMA's M (a lane each)
+constexpr int SM_ROWS = 32;                           // group rows per CTA: the MMA's N
+constexpr int SM_SLICES = GROUP_FEATURES / SM_ROWS;   // row slices per group
+constexpr int SM_THREADS = 128;
+constexpr int SM_STAGES = 5;
+constexpr int SM_XB = SM_TOK * CHUNK_COLS * 2;        // 16 KB of X per stage
+constexpr int SM_WB = SM_ROWS * CHUNK_COLS * 2;       // 4 KB of the weight stream per stage
+constexpr int SM_STAGE = SM_XB + SM_WB;
+constexpr int SM_PSTRIDE = SM_ROWS + 4;               // floats per token row of the partial tile
+constexpr int SM_CHUNK_OFF = SM_STAGES * SM_STAGE;    // then the CTA's chunk indices (kc ints)
+constexpr uint32_t SM_IDESC = idesc_bf16(SM_TOK, SM_ROWS);
+static_assert(SM_STAGE % 1024 == 0 && SM_XB % 1024 == 0, "stages and their weight rows start on swizzle atoms");
+static_assert(SM_TOK * SM_PSTRIDE * 4 <= SM_STAGES * SM_STAGE, "the partial tile reuses the ring");
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" :: "r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" :: "n"(N) : "memory"); }
+// Byte offset of 16-byte piece j of row r in a tile of 128-byte rows (the 128-byte swizzle).
+__device__ __forceinline__ uint32_t sw_off(int r, int j) { return (uint32_t)(r * 128 + ((j ^ (r & 7)) << 4)); }
+__device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+  return v;
+}
+
+// Bias, GELU, rounding, residual and store of 8 consecutive features f0 .. f0 + 7 of token t (the
+// same operations, in the same order, as the pair kernel's epilogue).
+template <bool GELU, bool F32>
+__device__ __forceinline__ void finish8(float *v, const float *b8, int f0, int64_t t, const LinearParams &P) {
+  if (P.bias != nullptr) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] += b8[i];
+  }
+  if (GELU) {
+#pragma unroll
+    for (int i = 0; i < 8; i += 2) gelu_erf2(v[i], v[i + 1]);
+  }
+  if (F32) {
+    float *dst = static_cast<float *>(P.Y) + t * P.ldy + f0;
+    if (P.y_vec16) {
+      reinterpret_cast<float4 *>(dst)[0] = make_float4(v[0], v[1], v[2], v[3]);
+      reinterpret_cast<float4 *>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) dst[i] = v[i];
+    }
+  } else {
+    uint32_t o[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) o[i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
+    if (P.R != nullptr) {  // 16-byte rows (checked on the host); R may be Y itself, read before written
+      const int4 r4 = *reinterpret_cast<const int4 *>(P.R + t * P.ldr + f0);
+      const uint32_t rw[4] = {(uint32_t)r4.x, (uint32_t)r4.y, (uint32_t)r4.z, (uint32_t)r4.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float lo = __uint_as_float(o[q] << 16) + __uint_as_float(rw[q] << 16);
+        const float hi = __uint_as_float(o[q] & 0xffff0000u) + __uint_as_float(rw[q] & 0xffff0000u);
+        o[q] = pack_bf16x2(lo, hi);
+      }
+    }
+    uint16_t *dst = static_cast<uint16_t *>(P.Y) + t * P.ldy + f0;
+    if (P.y_vec16) {
+      *reinterpret_cast<int4 *>(dst) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
+    } else {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        dst[2 * q] = (uint16_t)(o[q] & 0xffffu);
+        dst[2 * q + 1] = (uint16_t)(o[q] >> 16);
+      }
+    }
+  }
+}
+
+// Grid: kp x SM_SLICES x n_groups x ceil(m / SM_TOK) CTAs, clusters of kp along x.
+template <bool GELU, bool F32>
+__global__ void __launch_bounds__(SM_THREADS) bsr_linear_small_kernel(const LinearParams P) {
+  extern __shared__ uint8_t sm_raw[];
+  uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(sm_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ __align__(8) uint64_t mma_bar[SM_STAGES];
+  __shared__ __align__(16) float bias_s[SM_ROWS];  // the slice's bias (0 where the row has no panel)
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_flag;  // stays 0: the waits end only by completion or their time limit
+  const uint32_t ring = smem_u32(sm);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int kp = P.kp;
+  const int part = (int)(blockIdx.x % (unsigned)kp);  // the cluster rank (clusters of kp along x)
+  int idx = (int)(blockIdx.x / (unsigned)kp);
+  const int rs = idx % SM_SLICES;
+  idx /= SM_SLICES;
+  const int g = idx % P.n_groups;
+  const int tt = idx / P.n_groups;
+  const int kc = sched_chunks(P.k);
+  // one wave of independent loads: the header words, the group's entry range, this slice's panels
+  // (one or two slots); every early return below depends only on data shared by the whole cluster
+  const int32_t *gpan = P.sched + sched_gpan_offset_ints(P.n_groups) + (int64_t)g * MAX_GROUP_PANELS;
+  const int32_t *gent = P.sched + SCHED_HDR_INTS;
+  const int slot0 = rs * SM_ROWS / P.bn, slot1 = (rs * SM_ROWS + SM_ROWS - 1) / P.bn;
+  const int h1 = __ldg(P.sched + 1), h3 = __ldg(P.sched + 3), h4 = __ldg(P.sched + 4), h5 = __ldg(P.sched + 5);
+  const int h6 = __ldg(P.sched + 6), h8 = __ldg(P.sched + 8);
+  const int ga = __ldg(gent + g), gb = __ldg(gent + g + 1);
+  const int p0 = __ldg(gpan + slot0), p1 = __ldg(gpan + slot1);
+  const bool sched_ok = h3 == 0 && h1 == P.n_groups && h4 == P.n && h5 == P.k && h6 == P.bn && h8 == SCHED_VERSION;
+  if (!sched_ok) {
+    if (blockIdx.x == 0 && tid == 0) atomicOr(&P.ctl->err, h3 ? ERR_SCHED_OVERFLOW : ERR_BAD_SCHED);
+    return;
+  }
+  if (p0 < 0 && p1 < 0) return;  // a row slice with no panel (the last group of an n that is not a multiple of 256)
+  if (ga < 0 || gb < ga || gb - ga > kc || (int64_t)gb > P.stream_tiles) {
+    if (part == 0 && rs == 0 && tt == 0 && tid == 0) atomicOr(&P.ctl->err, ERR_BAD_SCHED);
+    return;
+  }
+  const int cnt = gb - ga;
+  const int e0 = ga + cnt * part / kp, e1 = ga + cnt * (part + 1) / kp;
+  const int ne = e1 - e0;
+
+  if (warp == 0) {
+    tmem_alloc(smem_u32(&tmem_slot), SM_ROWS);
+    tmem_relinquish();
+  }
+  if (tid == 0) {
+    for (int i = 0; i < SM_STAGES; ++i) mbar_init(smem_u32(&mma_bar[i]), 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (tid < SM_ROWS) {
+    const int gr = rs * SM_ROWS + tid;
+    const int panel = gr / P.bn == slot0 ? p0 : p1;
+    bias_s[tid] = P.bias != nullptr && panel >= 0 ? __ldg(P.bias + panel * P.bn + gr % P.bn) : 0.f;
+  }
+  int *chunk = reinterpret_cast<int *>(sm + SM_CHUNK_OFF);
+  const int32_t *entries = P.sched + sched_entries_offset_ints(P.n_groups);
+  for (int i = tid; i < ne; i += SM_THREADS) {
+    int c = __ldg(entries + e0 + i);
+    if (c < 0 || c >= kc) {  // a corrupt list: flag it, read chunk 0
+      atomicOr(&P.ctl->err, ERR_BAD_SCHED);
+      c = 0;
+    }
+    chunk[i] = c;
+  }
+
+  // stage s <- entry i: this slice's 32 stream rows (they need only the entry's index), X rows
+  // tt*128 .. +128 of the entry's chunk (zero beyond m and k)
+  auto load_w = [&](int i, int s) {
+    const uint32_t wsm = ring + s * SM_STAGE + SM_XB;
+    const uint16_t *tile = P.wstream + ((int64_t)(e0 + i) * GROUP_FEATURES + rs * SM_ROWS) * CHUNK_COLS;
+#pragma unroll
+    for (int q = 0; q < SM_WB / 16 / SM_THREADS; ++q) {
+      const int pc = tid + q * SM_THREADS, r = pc >> 3, j = pc & 7;
+      cp_async16(wsm + sw_off(r, j), tile + r * CHUNK_COLS + j * 8, 16u);
+    }
+  };
+  auto load_x = [&](int i, int s) {
+    const int c = chunk[i];
+    const uint32_t xs = ring + s * SM_STAGE;
+#pragma unroll
+    for (int q = 0; q < SM_XB / 16 / SM_THREADS; ++q) {
+      const int pc = tid + q * SM_THREADS, r = pc >> 3, j = pc & 7;
+      const int64_t t = (int64_t)tt * SM_TOK + r;
+      const int col = c * CHUNK_COLS + j * 8;  // k is a multiple of 16: a piece is all in or all out
+      const bool in = t < P.m && col < P.k;
+      cp_async16(xs + sw_off(r, j), in ? P.X + t * P.ldx + col : P.X, in ? 16u : 0u);
+    }
+  };
+  // the first stages' weight rows go out before the chunk indices are shared (they join the first
+  // commit group, which only makes them complete no later than their stage needs them)
+#pragma unroll
+  for (int s = 0; s < SM_STAGES - 1; ++s)
+    if (s < ne) load_w(s, s);
+  tc_fence_before();
+  __syncthreads();  // chunk indices, barriers and the TMEM address visible
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+#pragma unroll
+  for (int s = 0; s < SM_STAGES - 1; ++s) {
+    if (s < ne) load_x(s, s);
+    cp_async_commit();
+  }
+
+  bool ok = true;
+  for (int i = 0; i < ne; ++i) {
+    cp_async_wait<SM_STAGES - 2>();
+    fence_proxy_async_smem();  // this thread's copies of entry i, visible to the tensor core
+    __syncthreads();
+    const int s = i % SM_STAGES;
+    if (tid == 0) {
+      tc_fence_after();
+      const uint32_t xs = ring + s * SM_STAGE;
+#pragma unroll
+      for (int kk = 0; kk < CHUNK_COLS / 16; ++kk)
+        umma_f16(tmem, smem_desc<128>(xs + kk * 32), smem_desc<128>(xs + SM_XB + kk * 32), SM_IDESC,
+                 (i > 0 || kk > 0) ? 1u : 0u);
+      tc_commit(smem_u32(&mma_bar[s]));
+    }
+    // refill the stage entry i - 1 used once its MMAs have read it
+    const int nx = i + SM_STAGES - 1;
+    if (nx < ne) {
+      if (i >= 1 && !mbar_wait(smem_u32(&mma_bar[(i - 1) % SM_STAGES]), ((i - 1) / SM_STAGES) & 1u, &abort_flag,
+                               P.timeout_ns))
+        ok = false;
+      load_w(nx, nx % SM_STAGES);
+      load_x(nx, nx % SM_STAGES);
+    }
+    cp_async_commit();
+  }
+  cp_async_wait<0>();
+  // every MMA done (they complete in order: the last commit covers them all)
+  if (ne > 0 && !mbar_wait(smem_u32(&mma_bar[(ne - 1) % SM_STAGES]), ((ne - 1) / SM_STAGES) & 1u, &abort_flag,
+                           P.timeout_ns))
+    ok = false;
+  if (!ok) atomicOr(&P.ctl->err, ERR_MMA_ACC);
+  tc_fence_after();
+
+  // warp w holds tokens 32 w .. 32 w + 31 (TMEM lanes), the slice's 32 group rows (columns)
+  float v[SM_ROWS];
+  if (ne > 0) {
+    tmem_ld32(tmem + ((uint32_t)(32 * warp) << 16), v);
+  } else {
+#pragma unroll
+    for (int c = 0; c < SM_ROWS; ++c) v[c] = 0.f;
+  }
+  const int r_own = 32 * warp + lane;
+  if (kp == 1) {
+    const int64_t t = (int64_t)tt * SM_TOK + r_own;
+    if (t < P.m) {
+#pragma unroll
+      for (int run = 0; run < SM_ROWS / 8; ++run) {
+        const int gr = rs * SM_ROWS + run * 8;  // the run's first group row; a run stays inside one panel
+        const int panel = gr / P.bn == slot0 ? p0 : p1;
+        if (panel >= 0) finish8<GELU, F32>(v + run * 8, bias_s + run * 8, panel * P.bn + gr % P.bn, t, P);
+      }
+    }
+  } else {
+    __syncthreads();  // every thread is past its last copy: the ring takes the partial tile
+    float *pt = reinterpret_cast<float *>(sm);
+#pragma unroll
+    for (int c = 0; c < SM_ROWS; c += 4)
+      *reinterpret_cast<float4 *>(pt + r_own * SM_PSTRIDE + c) = make_float4(v[c], v[c + 1], v[c + 2], v[c + 3]);
+    cluster_sync();
+    // rows part * 128 / kp ..: the kp partial tiles added in rank order, then the epilogue
+    const int rows = SM_TOK / kp, r0 = part * rows;
+    for (int it = tid; it < rows * (SM_ROWS / 8); it += SM_THREADS) {
+      const int r = r0 + it / (SM_ROWS / 8), run = it % (SM_ROWS / 8);
+      const int64_t t = (int64_t)tt * SM_TOK + r;
+      const int gr = rs * SM_ROWS + run * 8;
+      const int panel = gr / P.bn == slot0 ? p0 : p1;
+      if (t >= P.m || panel < 0) continue;
+      const uint32_t off = smem_u32(pt + r * SM_PSTRIDE + run * 8);
+      // every part's values requested first (one remote latency), then added in rank order
+      float4 lo[8], hi[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (q < kp) {
+          const uint32_t rem = mapa_rank(off, (uint32_t)q);
+          lo[q] = ld_cluster_f4(rem);
+          hi[q] = ld_cluster_f4(rem + 16);
+        }
+      }
+      float y[8] = {lo[0].x, lo[0].y, lo[0].z, lo[0].w, hi[0].x, hi[0].y, hi[0].z, hi[0].w};
+#pragma unroll
+      for (int q = 1; q < 8; ++q) {
+        if (q < kp) {
+          y[0] += lo[q].x; y[1] += lo[q].y; y[2] += lo[q].z; y[3] += lo[q].w;
+          y[4] += hi[q].x; y[5] += hi[q].y; y[6] += hi[q].z; y[7] += hi[q].w;
+        }
+      }
+      finish8<GELU, F32>(y, bias_s + run * 8, panel * P.bn + gr % P.bn, t, P);
+    }
+    cluster_sync();  // no CTA leaves while another still reads its partial tile
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, SM_ROWS);
+}
+
 }  // namespace
 
 // ------------------------------------------------------------------------------------ host side
@@ -875,6 +1164,48 @@ cudaError_t launch_linear(const CUtensorMap &tmX, const CUtensorMap &tmW, const 
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, tmX, tmW, P);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+cudaError_t launch_linear_small(LinearParams P, int num_sms, cudaStream_t s) {
+  static bool attr_done[64] = {false};
+  const int kc = sched_chunks(P.k);
+  const size_t smem = (size_t)SM_CHUNK_OFF + (size_t)kc * sizeof(int) + 1024;  // + alignment slack
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+    // the largest request: kc <= 1024 chunk indices
+    const int most = SM_CHUNK_OFF + 1024 * (int)sizeof(int) + 1024;
+    for (auto k : {bsr_linear_small_kernel<false, false>, bsr_linear_small_kernel<true, false>,
+                   bsr_linear_small_kernel<false, true>, bsr_linear_small_kernel<true, true>}) {
+      cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+      if (e != cudaSuccess) return e;
+    }
+    attr_done[dev] = true;
+  }
+  const int64_t ctas = ((P.m + SM_TOK - 1) / SM_TOK) * (int64_t)P.n_groups * SM_SLICES;
+  // K parts: double while the grid stays resident at two CTAs per SM (the ring's shared memory)
+  // and each part keeps at least 8 chunks. An entry costs a CTA ~0.45 us at batch 1 and the
+  // cluster's reduction (two cluster barriers, remote reads) ~2.7 us, so shorter parts lose.
+  int kp = 1;
+  while (kp < 8 && ctas * kp * 2 <= 2 * (int64_t)num_sms && kc / (2 * kp) >= 8) kp *= 2;
+  P.kp = kp;
+  auto kern = P.gelu ? (P.y_f32 ? bsr_linear_small_kernel<true, true> : bsr_linear_small_kernel<true, false>)
+                     : (P.y_f32 ? bsr_linear_small_kernel<false, true> : bsr_linear_small_kernel<false, false>);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(ctas * kp));
+  cfg.blockDim = dim3(SM_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)kp;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = kp > 1 ? 1 : 0;  // no cluster when K is not cut
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kern, P);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

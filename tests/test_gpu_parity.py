@@ -371,9 +371,10 @@ def test_linear_fp32_out(lp, b, m):
     assert err <= TIGHT_TOL
 
 
+@pytest.mark.parametrize("m", [520, 200])   # the pair kernel; the small-m kernel
 @pytest.mark.parametrize("b", BLOCKS)
-def test_linear_integer_inputs_bit_exact(lp, b):
-    m, n, k = 520, 256, 512
+def test_linear_integer_inputs_bit_exact(lp, b, m):
+    n, k = 256, 512
     X, W, bias, mask = _case(m, n, k, b, 0.5, 200 + _sid(b), int_valued=True)
     w = lp.pack_bsr(W, mask, b)
     Y = lp.bsr_linear(w, X, bias, out_dtype=torch.float32)
@@ -448,9 +449,10 @@ def test_all_zero_mask_is_bias(lp, b):
     assert torch.count_nonzero(Yn) == 0
 
 
+@pytest.mark.parametrize("m", [300, 120])
 @pytest.mark.parametrize("b", BLOCKS)
-def test_pruned_blocks_never_read(lp, b):
-    m, n, k = 300, 256, 256
+def test_pruned_blocks_never_read(lp, b, m):
+    n, k = 256, 256
     X, W, bias, mask = _case(m, n, k, b, 0.5, 600 + _sid(b))
     bn, bk = _sides(b)
     keep = mask.repeat_interleave(bn, 0).repeat_interleave(bk, 1).bool()
@@ -463,8 +465,9 @@ def test_pruned_blocks_never_read(lp, b):
     assert torch.equal(Yp, Yz) and torch.isfinite(Yp).all()
 
 
-def test_single_block_closed_form(lp):
-    m, n, k, b = 290, 256, 256, 32
+@pytest.mark.parametrize("m", [290, 100])
+def test_single_block_closed_form(lp, m):
+    n, k, b = 256, 256, 32
     X, W, bias, _ = _case(m, n, k, b, 0.5, 700, int_valued=True)
     mask = torch.zeros(n // b, k // b, dtype=torch.uint8, device="cuda")
     mask[3, 5] = 1
@@ -475,8 +478,9 @@ def test_single_block_closed_form(lp):
     assert torch.equal(Y.double().cpu(), expect)
 
 
-def test_strided_input_output_and_guard_band(lp):
-    m, n, k, b = 400, 256, 128, 32
+@pytest.mark.parametrize("m", [400, 150])
+def test_strided_input_output_and_guard_band(lp, m):
+    n, k, b = 256, 128, 32
     X, W, bias, mask = _case(m, n, k, b, 0.5, 800)
     Xw = torch.zeros(m, k + 64, dtype=torch.bfloat16, device="cuda")
     Xw[:, 64:] = X
@@ -489,12 +493,13 @@ def test_strided_input_output_and_guard_band(lp):
     assert torch.all(Yw[m:] == canary) and torch.all(Yw[:, :16] == canary) and torch.all(Yw[:, 16 + n:] == canary)
 
 
+@pytest.mark.parametrize("m", [301, 101])
 @pytest.mark.parametrize("col0,extra", [(1, 33), (2, 34)])
-def test_bf16_output_offsets_and_row_strides(lp, col0, extra):
+def test_bf16_output_offsets_and_row_strides(lp, col0, extra, m):
     """bf16 output inside a larger buffer, with bases and row strides that rule out 16-byte stores
     (element stores instead); the canary around the output region survives and the values are
     those of a contiguous output."""
-    m, n, k, b = 301, 256, 128, 32
+    n, k, b = 256, 128, 32
     X, W, bias, mask = _case(m, n, k, b, 0.5, 850 + col0)
     canary = torch.tensor(-777.0, dtype=torch.bfloat16)
     Yw = torch.full((m + 3, n + extra), canary.item(), dtype=torch.bfloat16, device="cuda")
@@ -510,11 +515,12 @@ def test_bf16_output_offsets_and_row_strides(lp, col0, extra):
 
 
 @pytest.mark.parametrize("b,m,n,k,gelu", [(32, 333, 256, 256, False), (16, 197, 768, 3072, False),
-                                          ((64, 32), 300, 384, 512, True)])
+                                          ((64, 32), 300, 384, 512, True), (16, 300, 768, 3072, False)])
 def test_residual_linear_is_the_bf16_sum(lp, b, m, n, k, gelu):
     """lpvit_bsr_linear_residual: Y equals, bit for bit, the plain linear's bf16 output plus R
     rounded to bf16 (the sum formed in float32), into a new tensor and in place (R = Y); the
-    197-row case splits its units (the fix-up path)."""
+    197-row case runs the small-m kernel with K cut over a cluster, the 300-row K = 3072 case the
+    pair kernel's split units (the fix-up path)."""
     X, W, bias, mask = _case(m, n, k, b, 0.5, 1300 + _sid(b))
     w = lp.pack_bsr(W, mask, b)
     R = torch.randn(m, n, generator=torch.Generator().manual_seed(9)).to(torch.bfloat16).cuda()
@@ -527,9 +533,10 @@ def test_residual_linear_is_the_bf16_sum(lp, b, m, n, k, gelu):
     assert torch.equal(Z, want)
 
 
+@pytest.mark.parametrize("m", [197, 300])   # small-m kernel (K over a cluster); pair kernel split units
 @pytest.mark.parametrize("b", [32, (64, 32), (16, 32)])
-def test_deterministic_repeats(lp, b):
-    m, n, k = 197, 768, 3072   # small m: split slices + fix-up path
+def test_deterministic_repeats(lp, b, m):
+    n, k = 768, 3072
     X, W, bias, mask = _case(m, n, k, b, 0.5, 900 + (0 if b == 32 else _sid(b)))
     w = lp.pack_bsr(W, mask, b)
     ws = lp.workspace_for(w, m)
@@ -539,6 +546,50 @@ def test_deterministic_repeats(lp, b):
     assert torch.equal(Y1, Y2)
     ref = _oracle(X, W, mask, b, bias)
     assert _norm_err(Y1.cpu().double().numpy(), ref) <= TIGHT_TOL
+
+
+# ------------------------------------------------------------------------------ small m
+
+# (m, n, k, b, gelu, f32): one token, a 256-feature weight and K = 3072 (eight K parts in one
+# cluster); 17 tokens (eight parts); k = 400, not a multiple of the 64-column chunk (the last
+# chunk reads zeros past k); n = 1152, 4.5 groups (row slices with no panel); 197 tokens over
+# 64 x 32 blocks with GELU; m = 256, the largest the small-m kernel takes (four parts).
+SMALL_M_CASES = [(1, 256, 3072, 32, False, True), (17, 768, 3072, 16, True, True),
+                 (64, 384, 400, 16, False, True), (65, 1152, 384, 32, True, False),
+                 (197, 3072, 768, (64, 32), True, False), (256, 512, 1536, (16, 32), False, True)]
+
+
+@pytest.mark.parametrize("m,n,k,b,gelu,f32", SMALL_M_CASES)
+def test_small_m_kernel_against_oracle(lp, m, n, k, b, gelu, f32):
+    """Token counts up to 256 run the small-m kernel: fp32 output within the tight gate of the
+    oracle, bf16 output within one bf16 ulp plus the fp32 accumulation bound, and the workspace
+    error word clear."""
+    X, W, bias, mask = _case(m, n, k, b, 0.5, 1500 + m + _sid(b))
+    w = lp.pack_bsr(W, mask, b)
+    ws = lp.workspace_for(w, m)
+    Y = lp.bsr_linear(w, X, bias, gelu=gelu, out_dtype=torch.float32 if f32 else torch.bfloat16, workspace=ws)
+    lp.check(ws)
+    ref = _oracle(X, W, mask, b, bias, gelu=gelu)
+    y = Y.float().cpu().double().numpy()
+    if f32:
+        assert _norm_err(y, ref) <= TIGHT_TOL
+    else:
+        assert np.all(np.abs(y - ref) <= _bf16_tol(ref, X, W, mask, b, bias, gelu=gelu))
+
+
+def test_small_and_pair_kernels_agree_at_the_boundary(lp):
+    """m = 256 (small-m kernel) and m = 257 (pair kernel) on the same weight: the first 256 rows
+    agree within the fp32 accumulation bound of two summation orders, and both meet the oracle."""
+    n, k, b = 768, 1536, 32
+    X, W, bias, mask = _case(257, n, k, b, 0.5, 1600)
+    w = lp.pack_bsr(W, mask, b)
+    Ys = lp.bsr_linear(w, X[:256], bias, out_dtype=torch.float32)
+    Yp = lp.bsr_linear(w, X, bias, out_dtype=torch.float32)
+    bound = 2 * _acc_bound(X[:256], W, mask, b, bias)
+    assert np.all(np.abs(Ys.cpu().double().numpy() - Yp[:256].cpu().double().numpy()) <= bound)
+    ref = _oracle(X, W, mask, b, bias)
+    assert _norm_err(Yp.cpu().double().numpy(), ref) <= TIGHT_TOL
+    assert _norm_err(Ys.cpu().double().numpy(), ref[:256]) <= TIGHT_TOL
 
 
 @pytest.mark.parametrize("b", [16, 64, (16, 32)])
