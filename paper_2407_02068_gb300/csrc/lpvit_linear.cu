@@ -633,8 +633,10 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     const int q = warp & 3;
     const int part = (warp - FIRST_EPI) >> 2;
     float *bias_s = reinterpret_cast<float *>(smem + L::BIAS_OFF) + (warp - FIRST_EPI) * 64;  // (not DEEP)
-    // The unit record of unit ui + 1 is taken (and its ring slot handed back) before unit ui's
-    // outputs are stored, so that this release-ordered arrival never waits for fresh stores.
+    // Takes the record of unit u and hands its ring slot back. The hand-back orders nothing but
+    // this warp's reads of the slot, so it is a relaxed arrival made data-dependent on them: a vote
+    // over every lane's loaded record (pad is always 0) completes only once all the reads have
+    // returned. A release arrival would also wait for the previous unit's output stores.
     auto take_unit = [&](uint32_t u, UnitInfo &out) -> bool {
       const uint32_t slot = u % UR, uph = (u / UR) & 1u;
       if (!(leader ? mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)
@@ -643,10 +645,11 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
         return false;
       }
       out = ring[slot].inf;
-      __syncwarp();
-      if (lane == 0) {
-        if (leader) mbar_arrive(unite_bar(slot));
-        else mbar_arrive_cluster(mapa_rank(unite_bar(slot), 0));
+      const uint32_t read = __ballot_sync(0xffffffffu, (out.tt ^ out.g ^ out.s ^ out.nsl ^ out.e0 ^ out.e1 ^ out.ptile) !=
+                                                           0x7fffffff || out.pad == 0);
+      if (lane == 0 && read != 0u) {
+        if (leader) mbar_arrive_relaxed(unite_bar(slot));
+        else mbar_arrive_relaxed_cluster(mapa_rank(unite_bar(slot), 0));
       }
       return true;
     };
