@@ -6,23 +6,24 @@
 //   is null), then y = (s - mean) / sqrt(var + eps) * gamma + beta over the row in float32 (biased
 //   variance, two passes over the row held in registers), stored as bf16; s is stored too when r
 //   is given (the new residual stream).
-// attention_kernel (one CTA of ATT_WARPS = 7 warps per image and head; head_dim 64, at most 208
-//   tokens): Q, K and V of the head are staged in shared memory by asynchronous 16-byte copies (rows
-//   padded to 144 bytes: ldmatrix rows fall in distinct banks); each warp takes 16-query tiles in
-//   turn (13 tiles for 197 tokens, two rounds). Per tile the keys stream in chunks of 64 with an
-//   online softmax: S = Q K^T for the chunk with bf16 tensor-core MMAs (mma.sync m16n8k16, fp32
-//   accumulation), scaled by 1/sqrt(64) (folded into base-2 exponentials), padded keys masked,
-//   the running row max and sum updated over the four lanes sharing a row and the partial output
-//   rescaled when the max grows; P = exp(S - max) rounded to bf16 is the A operand of O += P V (V
-//   fragments by ldmatrix.trans); O / sum is stored as bf16. Attention is about 8% of the FLOPs of a
-//   DeiT-B layer at 50% block density (30.5 GFLOP per layer at batch 256); these warp-level MMAs
-//   are the legacy tensor path, kept because the kernel is latency-bound at 197 tokens per head.
+// attention_kernel (tcgen05; one CTA of four warps per image, head and 128-query tile; head_dim 64,
+//   at most 208 tokens): the tile's Q rows and the head's K rows are copied by 16-byte cp.async into
+//   K-major tiles of 128-byte rows in the 128-byte swizzle, V's rows as they are; while the first
+//   MMAs run, the threads transpose V in shared memory into K-major tiles (the 64 dims as rows, keys
+//   along K, two keys per 32-bit store). S = Q K^T is four tcgen05 MMAs (M = 128
+//   queries, N = the keys rounded up to 16, K = 16) into TMEM; each thread then takes one query row
+//   of S from TMEM: the row max over the valid keys, p = 2^((s - max) log2(e) / sqrt(64)) for them
+//   (ex2.approx.ftz; 0 for padding keys), their float32 sum, and p rounded to bf16 into the K-major P tiles (written
+//   over Q, K and V's rows, no longer read). O = P V is one MMA per 16 keys (N = 64)
+//   into the first TMEM columns, where S was; O / sum is rounded to bf16 and stored. Attention is
+//   about 8% of the FLOPs of a DeiT-B layer at 50% block density (30.5 GFLOP per layer at batch 256).
 #include <cmath>
 #include <cstdint>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include "lpvit.h"
+#include "lpvit_device.cuh"
 
 namespace lpvit {
 
@@ -32,12 +33,20 @@ constexpr int LN_THREADS = 256;
 constexpr int LN_MAX_D = 1024;
 constexpr int LN_VPL = LN_MAX_D / 8 / 32;  // 16-byte vectors per lane at most
 
-constexpr int ATT_WARPS = 7;             // 13 query tiles of 16 in two rounds
-constexpr int KCHUNK = 8;                // key tiles of 8 per online-softmax chunk (64 keys)
-constexpr int HD = 64;                   // head dimension
-constexpr int MAX_TOKENS = 208;          // 13 tiles of 16
-constexpr int ROW = HD + 8;              // shared-memory row in bf16 (144 bytes)
-constexpr int ATT_SMEM = 3 * MAX_TOKENS * ROW * 2;
+constexpr int HD = 64;                      // head dimension
+constexpr int MAX_TOKENS = 208;             // 13 key tiles of 16
+constexpr int AT_Q = 128;                   // queries per CTA: the MMA's M, one TMEM lane each
+constexpr int AT_THREADS = 128;
+constexpr int AT_K_OFF = AT_Q * 128;        // K's rows after the 128 Q rows
+constexpr int AT_V_OFF = AT_K_OFF + MAX_TOKENS * 128;  // V's rows as they are (128-byte rows)
+constexpr int AT_P_CHUNK = AT_Q * 128;      // P: four 64-key chunks of [128 rows x 128 bytes], from 0
+constexpr int AT_VT_OFF = 68 * 1024;        // V^T: four 64-key chunks of [64 dims x 128 bytes]
+constexpr int AT_VT_CHUNK = HD * 128;
+constexpr int AT_TMEM_COLS = 256;           // S (up to 208 columns); O reuses the first 64
+constexpr int AT_SMEM = AT_VT_OFF + 4 * AT_VT_CHUNK + 1024;  // + alignment slack (101 KB: two CTAs per SM)
+constexpr float AT_SCALE_LOG2 = 0.125f * 1.4426950408889634f;  // 1/sqrt(64) * log2(e)
+constexpr uint64_t AT_WAIT_NS = 2000000000ull;
+static_assert(AT_V_OFF + MAX_TOKENS * 128 <= AT_VT_OFF && 4 * AT_P_CHUNK <= AT_VT_OFF, "Q, K, V and P before V^T");
 
 __device__ __forceinline__ float warp_sum_f(float v) {
 #pragma unroll
@@ -113,157 +122,171 @@ add_layernorm_kernel(const __nv_bfloat16 *__restrict__ x, const __nv_bfloat16 *_
   }
 }
 
-__device__ __forceinline__ uint32_t smem_addr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &a0, uint32_t &a1, uint32_t &a2, uint32_t &a3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(a0), "=r"(a1), "=r"(a2), "=r"(a3) : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t &b0, uint32_t &b1) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];" : "=r"(b0), "=r"(b1) : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x2_trans(uint32_t addr, uint32_t &b0, uint32_t &b1) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0,%1}, [%2];" : "=r"(b0), "=r"(b1) : "r"(addr));
-}
-// D (16x8 fp32) += A (16x16 bf16, row) * B (16x8 bf16, col)
-__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
-                                         uint32_t b0, uint32_t b1) {
-  asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-               "{%0,%1,%2,%3};"
-               : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-               : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-  __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t *>(&p);
+// V's staged rows: piece j of key row r at j ^ ((r / 2) mod 8), so that the transpose's reads of one
+// piece of 32 consecutive even (or odd) keys fall in distinct bank groups.
+__device__ __forceinline__ uint32_t v_off(int r, int j) { return (uint32_t)(r * 128 + ((j ^ ((r >> 1) & 7)) << 4)); }
+__device__ __forceinline__ float ex2_ftz(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
-// One CTA per (image, head): Q, K, V of the head staged in shared memory by asynchronous copies;
-// each warp takes 16-query tiles and streams the keys in chunks of 64 with an online softmax
-// (running row max and sum, rescaling the partial output when the max grows), so a chunk's scores
-// stay in 32 registers per thread. Scores and exponentials in float32 (base 2, the 1/sqrt(64) scale
-// folded into log2 e), P rounded to bf16 for the P V products, fp32 accumulation.
-__global__ void __launch_bounds__(32 * ATT_WARPS, 2)
+// Grid: images x heads x ceil(tokens / 128) CTAs; qkv [images * tokens][3 D] (q | k | v, head h at
+// columns h * 64 of each), out [images * tokens][D], D = heads * 64.
+__global__ void __launch_bounds__(AT_THREADS)
 attention_kernel(const __nv_bfloat16 *__restrict__ qkv, int tokens, int heads, __nv_bfloat16 *__restrict__ out) {
-  extern __shared__ __align__(16) __nv_bfloat16 att_smem[];
-  __nv_bfloat16 *Qs = att_smem, *Ks = Qs + MAX_TOKENS * ROW, *Vs = Ks + MAX_TOKENS * ROW;
-  const int img = blockIdx.x / heads, h = blockIdx.x - img * heads;
+  extern __shared__ uint8_t at_raw[];
+  uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(at_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ __align__(8) uint64_t bars[2];
+  __shared__ uint32_t tmem_slot;
+  __shared__ int abort_flag;  // stays 0: the waits end by completion or their time limit
+  const uint32_t base = smem_u32(sm);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nqt = (tokens + AT_Q - 1) / AT_Q;
+  const int qt = (int)(blockIdx.x % (unsigned)nqt);
+  const int bh = (int)(blockIdx.x / (unsigned)nqt);
+  const int img = bh / heads, h = bh - img * heads;
   const int D = heads * HD;
-  const int tp = (tokens + 15) / 16 * 16;  // padded token count
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // stage Q, K, V of this head (8 vectors of 16 bytes per row each) with asynchronous copies, all
-  // in flight together; padded rows are zero
-  for (int idx = threadIdx.x; idx < tp * 8 * 3; idx += blockDim.x) {
-    const int m = idx / (tp * 8), rem = idx - m * tp * 8, row = rem >> 3, c = rem & 7;
-    uint4 *dst = reinterpret_cast<uint4 *>(att_smem + (m * MAX_TOKENS + row) * ROW) + c;
-    if (row < tokens) {
-      const uint4 *src =
-          reinterpret_cast<const uint4 *>(qkv + ((int64_t)img * tokens + row) * 3 * D + m * D + h * HD) + c;
-      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" :: "r"(smem_addr(dst)), "l"(src) : "memory");
-    } else {
-      *dst = make_uint4(0, 0, 0, 0);
-    }
+  const int64_t row0 = (int64_t)img * tokens;  // the image's first token row
+  const int64_t ld = 3 * (int64_t)D;           // elements per qkv row
+  const int nkeys = (tokens + 15) & ~15;       // S's N
+  const uint32_t bar_s = smem_u32(&bars[0]), bar_o = smem_u32(&bars[1]);
+
+  if (warp == 0) {
+    tmem_alloc(smem_u32(&tmem_slot), AT_TMEM_COLS);
+    tmem_relinquish();
   }
-  asm volatile("cp.async.wait_all;" ::: "memory");
+  if (tid == 0) {
+    mbar_init(bar_s, 1);
+    mbar_init(bar_o, 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  // the tile's Q rows and the head's K rows (zero past the tokens)
+  for (int pc = tid; pc < AT_Q * 8; pc += AT_THREADS) {
+    const int r = pc >> 3, j = pc & 7, t = qt * AT_Q + r;
+    const bool in = t < tokens;
+    cp_async16(base + sw_off(r, j), qkv + (in ? (row0 + t) * ld + h * HD + j * 8 : 0), in ? 16u : 0u);
+  }
+  for (int pc = tid; pc < nkeys * 8; pc += AT_THREADS) {
+    const int r = pc >> 3, j = pc & 7;
+    const bool in = r < tokens;
+    cp_async16(base + AT_K_OFF + sw_off(r, j), qkv + (in ? (row0 + r) * ld + D + h * HD + j * 8 : 0), in ? 16u : 0u);
+  }
+  for (int pc = tid; pc < nkeys * 8; pc += AT_THREADS) {
+    const int r = pc >> 3, j = pc & 7;
+    const bool in = r < tokens;
+    cp_async16(base + AT_V_OFF + v_off(r, j), qkv + (in ? (row0 + r) * ld + 2 * D + h * HD + j * 8 : 0),
+               in ? 16u : 0u);
+  }
+  cp_async_commit();
+  cp_async_wait<0>();
+  fence_proxy_async_smem();  // this thread's copies, visible to the tensor core
+  tc_fence_before();
   __syncthreads();
-  constexpr float kScaleLog2 = 0.125f * 1.4426950408889634f;  // 1/sqrt(64) * log2(e)
-  const int ntiles = tp / 8, kq = lane & 3, rq = lane >> 2;
-  for (int mt = warp; mt < tp / 16; mt += ATT_WARPS) {
-    uint32_t qa[HD / 16][4];
+  tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+  if (tid == 0) {
 #pragma unroll
-    for (int ks = 0; ks < HD / 16; ++ks)
-      ldsm_x4(smem_addr(Qs + (16 * mt + (lane & 15)) * ROW + 16 * ks + (lane >> 4) * 8), qa[ks][0], qa[ks][1],
-              qa[ks][2], qa[ks][3]);
-    float o[HD / 8][4];
+    for (int kk = 0; kk < HD / 16; ++kk)
+      umma_f16(tmem, smem_desc<128>(base + kk * 32), smem_desc<128>(base + AT_K_OFF + kk * 32),
+               idesc_bf16(AT_Q, nkeys), kk > 0 ? 1u : 0u);
+    tc_commit(bar_s);
+  }
+  // V^T while S is computed: dims 8 dp .. 8 dp + 7 of keys r, r + 1 become columns r, r + 1 of rows
+  // 8 dp .. 8 dp + 7 of key chunk r / 64 (consecutive threads take consecutive key pairs)
+  for (int it = tid; it < 4 * nkeys; it += AT_THREADS) {
+    const int dp = it / (nkeys / 2), r = 2 * (it - dp * (nkeys / 2));
+    uint4 a, b;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w)
+                 : "r"(base + AT_V_OFF + v_off(r, dp)));
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(b.x), "=r"(b.y), "=r"(b.z), "=r"(b.w)
+                 : "r"(base + AT_V_OFF + v_off(r + 1, dp)));
+    const uint32_t wa[4] = {a.x, a.y, a.z, a.w}, wb[4] = {b.x, b.y, b.z, b.w};
+    const uint32_t col = base + AT_VT_OFF + (r >> 6) * AT_VT_CHUNK + 2 * (r & 7);
 #pragma unroll
-    for (int nd = 0; nd < HD / 8; ++nd) o[nd][0] = o[nd][1] = o[nd][2] = o[nd][3] = 0.f;
-    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;  // rows rq and rq + 8 of the tile
-    for (int kc = 0; kc < ntiles; kc += KCHUNK) {
-      // S = Q K^T for keys 8 kc .. 8 (kc + KCHUNK)
-      float s[KCHUNK][4];
-#pragma unroll
-      for (int nt = 0; nt < KCHUNK; ++nt) {
-        s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-        if (kc + nt < ntiles) {
-#pragma unroll
-          for (int ks = 0; ks < HD / 16; ++ks) {
-            uint32_t b0, b1;
-            ldsm_x2(smem_addr(Ks + (8 * (kc + nt) + (lane & 7)) * ROW + 16 * ks + ((lane >> 3) & 1) * 8), b0, b1);
-            mma_bf16(s[nt], qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], b0, b1);
-          }
-        }
-      }
-      float cm0 = -INFINITY, cm1 = -INFINITY;
-#pragma unroll
-      for (int nt = 0; nt < KCHUNK; ++nt) {
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int col = 8 * (kc + nt) + 2 * kq + (e & 1);
-          s[nt][e] = col < tokens ? s[nt][e] * kScaleLog2 : -INFINITY;
-        }
-        cm0 = fmaxf(cm0, fmaxf(s[nt][0], s[nt][1]));
-        cm1 = fmaxf(cm1, fmaxf(s[nt][2], s[nt][3]));
-      }
-      cm0 = fmaxf(cm0, __shfl_xor_sync(0xffffffffu, cm0, 1));
-      cm0 = fmaxf(cm0, __shfl_xor_sync(0xffffffffu, cm0, 2));
-      cm1 = fmaxf(cm1, __shfl_xor_sync(0xffffffffu, cm1, 1));
-      cm1 = fmaxf(cm1, __shfl_xor_sync(0xffffffffu, cm1, 2));
-      // the first chunk always holds key 0, so the running max is finite from here on
-      const float n0 = fmaxf(m0, cm0), n1 = fmaxf(m1, cm1);
-      const float a0 = exp2f(m0 - n0), a1 = exp2f(m1 - n1);  // 0 on the first chunk
-      m0 = n0;
-      m1 = n1;
-      l0 *= a0;
-      l1 *= a1;
-#pragma unroll
-      for (int nd = 0; nd < HD / 8; ++nd) {
-        o[nd][0] *= a0;
-        o[nd][1] *= a0;
-        o[nd][2] *= a1;
-        o[nd][3] *= a1;
-      }
-#pragma unroll
-      for (int nt = 0; nt < KCHUNK; ++nt) {
-        s[nt][0] = exp2f(s[nt][0] - n0);
-        s[nt][1] = exp2f(s[nt][1] - n0);
-        s[nt][2] = exp2f(s[nt][2] - n1);
-        s[nt][3] = exp2f(s[nt][3] - n1);
-        l0 += s[nt][0] + s[nt][1];
-        l1 += s[nt][2] + s[nt][3];
-      }
-      // O += P V over the chunk's keys, 16 at a time (ntiles is even)
-#pragma unroll
-      for (int kt = 0; kt < KCHUNK / 2; ++kt) {
-        if (kc + 2 * kt < ntiles) {
-          const uint32_t p0 = pack_bf16(s[2 * kt][0], s[2 * kt][1]), p1 = pack_bf16(s[2 * kt][2], s[2 * kt][3]);
-          const uint32_t p2 = pack_bf16(s[2 * kt + 1][0], s[2 * kt + 1][1]);
-          const uint32_t p3 = pack_bf16(s[2 * kt + 1][2], s[2 * kt + 1][3]);
-#pragma unroll
-          for (int nd = 0; nd < HD / 8; ++nd) {
-            uint32_t b0, b1;
-            ldsm_x2_trans(smem_addr(Vs + (8 * kc + 16 * kt + (lane & 15)) * ROW + 8 * nd), b0, b1);
-            mma_bf16(o[nd], p0, p1, p2, p3, b0, b1);
-          }
-        }
-      }
-    }
-    l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-    l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-    l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-    const float inv0 = 1.f / l0, inv1 = 1.f / l1;
-    const int r0 = 16 * mt + rq, r1 = r0 + 8;
-#pragma unroll
-    for (int nd = 0; nd < HD / 8; ++nd) {
-      const int col = h * HD + 8 * nd + 2 * kq;
-      if (r0 < tokens)
-        *reinterpret_cast<uint32_t *>(out + ((int64_t)img * tokens + r0) * D + col) =
-            pack_bf16(o[nd][0] * inv0, o[nd][1] * inv0);
-      if (r1 < tokens)
-        *reinterpret_cast<uint32_t *>(out + ((int64_t)img * tokens + r1) * D + col) =
-            pack_bf16(o[nd][2] * inv1, o[nd][3] * inv1);
+    for (int e = 0; e < 8; ++e) {
+      const uint32_t lo = (e & 1) ? (wa[e >> 1] >> 16) : (wa[e >> 1] & 0xffffu);
+      const uint32_t hi = (e & 1) ? (wb[e >> 1] >> 16) : (wb[e >> 1] & 0xffffu);
+      asm volatile("st.shared.b32 [%0], %1;" :: "r"(col + sw_off(dp * 8 + e, (r & 63) >> 3)), "r"(lo | (hi << 16))
+                   : "memory");
     }
   }
+  __syncthreads();  // V's rows are read: P may be written over them
+  bool ok = mbar_wait(bar_s, 0, &abort_flag, AT_WAIT_NS);
+  tc_fence_after();
+
+  // softmax of this thread's query row (TMEM lane r), in chunks of 32 keys
+  const int r = 32 * warp + lane;
+  const uint32_t trow = tmem + ((uint32_t)(32 * warp) << 16);
+  const int nch = (nkeys + 31) / 32;
+  float m = -INFINITY;
+  for (int c = 0; c < nch; ++c) {
+    float v[32];
+    tmem_ld32(trow + 32 * c, v);
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      m = 32 * c + i < tokens ? fmaxf(m, v[i]) : m;
+  }
+  const float mb = m * AT_SCALE_LOG2;
+  float sum = 0.f;
+  for (int c = 0; c < nch; ++c) {
+    float v[32];
+    tmem_ld32(trow + 32 * c, v);
+    uint32_t pk[16];
+    const bool full = 32 * c + 32 <= tokens;  // warp-uniform: only the last chunk holds padding keys
+#pragma unroll
+    for (int i = 0; i < 32; i += 2) {
+      float p0 = ex2_ftz(fmaf(v[i], AT_SCALE_LOG2, -mb)), p1 = ex2_ftz(fmaf(v[i + 1], AT_SCALE_LOG2, -mb));
+      if (!full) {
+        p0 = 32 * c + i < tokens ? p0 : 0.f;
+        p1 = 32 * c + i + 1 < tokens ? p1 : 0.f;
+      }
+      sum += p0 + p1;
+      asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(pk[i / 2]) : "f"(p1), "f"(p0));
+    }
+    // keys 32 c .. 32 c + 31: chunk c / 2, 16-byte pieces 4 (c % 2) .. 4 (c % 2) + 3 of row r
+    const uint32_t prow = base + (c >> 1) * AT_P_CHUNK;
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(prow + sw_off(r, (c & 1) * 4 + q)),
+                   "r"(pk[4 * q]), "r"(pk[4 * q + 1]), "r"(pk[4 * q + 2]), "r"(pk[4 * q + 3]) : "memory");
+  }
+  fence_proxy_async_smem();
+  tc_fence_before();  // every thread's S loads are complete: O may overwrite those columns
+  __syncthreads();
+  tc_fence_after();
+  if (tid == 0) {
+    for (int st = 0; st < nkeys / 16; ++st) {
+      const int c = st >> 2, kk = st & 3;
+      umma_f16(tmem, smem_desc<128>(base + c * AT_P_CHUNK + kk * 32),
+               smem_desc<128>(base + AT_VT_OFF + c * AT_VT_CHUNK + kk * 32), idesc_bf16(AT_Q, HD),
+               st > 0 ? 1u : 0u);
+    }
+    tc_commit(bar_o);
+  }
+  ok = mbar_wait(bar_o, 0, &abort_flag, AT_WAIT_NS) && ok;
+  tc_fence_after();
+
+  const int t = qt * AT_Q + r;
+  const float inv = 1.f / sum;
+#pragma unroll
+  for (int half = 0; half < 2; ++half) {
+    float o[32];
+    tmem_ld32(trow + 32 * half, o);
+    if (ok && t < tokens) {
+      uint32_t w[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(w[i]) : "f"(o[2 * i + 1] * inv), "f"(o[2 * i] * inv));
+      uint4 *dst = reinterpret_cast<uint4 *>(out + (row0 + t) * D + h * HD + half * 32);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) dst[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, AT_TMEM_COLS);
 }
 
 bool aligned_to(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -296,17 +319,18 @@ lpvit_status lpvit_attention(const void *qkv, int64_t images, int32_t tokens, in
   if (head_dim != HD || tokens < 1 || tokens > MAX_TOKENS) return LPVIT_ERR_UNSUPPORTED;
   if (images < 0 || heads < 1 || heads > 64) return LPVIT_ERR_INVALID_ARG;
   if (images == 0) return LPVIT_OK;
-  if (images * heads > 0x7fffffffLL) return LPVIT_ERR_INVALID_ARG;
+  const int64_t ctas = images * heads * ((tokens + AT_Q - 1) / AT_Q);
+  if (ctas > 0x7fffffffLL) return LPVIT_ERR_INVALID_ARG;
   if (!qkv || !out || !aligned_to(qkv, 16) || !aligned_to(out, 16)) return LPVIT_ERR_INVALID_ARG;
   static bool attr_done[64] = {false};
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 0 && dev < 64 && !attr_done[dev]) {
-    if (cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, ATT_SMEM) != cudaSuccess)
+    if (cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, AT_SMEM) != cudaSuccess)
       return LPVIT_ERR_CUDA;
     attr_done[dev] = true;
   }
-  attention_kernel<<<(int)(images * heads), 32 * ATT_WARPS, ATT_SMEM, static_cast<cudaStream_t>(stream)>>>(
+  attention_kernel<<<(int)ctas, AT_THREADS, AT_SMEM, static_cast<cudaStream_t>(stream)>>>(
       static_cast<const __nv_bfloat16 *>(qkv), tokens, heads, static_cast<__nv_bfloat16 *>(out));
   return cudaGetLastError() == cudaSuccess ? LPVIT_OK : LPVIT_ERR_CUDA;
 }

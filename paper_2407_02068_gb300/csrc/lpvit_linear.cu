@@ -863,14 +863,6 @@ constexpr uint32_t SM_IDESC = idesc_bf16(SM_TOK, SM_ROWS);
 static_assert(SM_STAGE % 1024 == 0 && SM_XB % 1024 == 0, "stages and their weight rows start on swizzle atoms");
 static_assert(SM_TOK * SM_PSTRIDE * 4 <= SM_STAGES * SM_STAGE, "the partial tile reuses the ring");
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" :: "r"(dst), "l"(src), "r"(src_bytes) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" :: "n"(N) : "memory"); }
-// Byte offset of 16-byte piece j of row r in a tile of 128-byte rows (the 128-byte swizzle).
-__device__ __forceinline__ uint32_t sw_off(int r, int j) { return (uint32_t)(r * 128 + ((j ^ (r & 7)) << 4)); }
 __device__ __forceinline__ float4 ld_cluster_f4(uint32_t addr) {
   float4 v;
   asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
