@@ -59,7 +59,7 @@ def test_add_layernorm(lp, D, rows, with_r):
 
 
 @pytest.mark.parametrize("tokens,heads,images", [(197, 6, 3), (197, 12, 1), (49, 3, 5), (1, 2, 2), (208, 1, 2),
-                                                 (16, 4, 1), (33, 2, 2)])
+                                                 (16, 4, 1), (33, 2, 2), (128, 3, 2), (129, 2, 3), (177, 1, 2)])
 def test_attention(lp, tokens, heads, images):
     g = torch.Generator(device="cuda").manual_seed(tokens * 100 + heads)
     qkv = (torch.randn(images * tokens, 3 * heads * 64, generator=g, device="cuda")).to(torch.bfloat16)
