@@ -35,6 +35,10 @@ BLOCK = 32
 CONFIG_ID = 4             # seeds of the 12-layer stack workload
 WORKLOAD = "deit_b_12layer_linear_stack_batch256"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# GB300 datasheet figures, reported beside the measured denominators: dense bf16 tensor throughput
+# (without 2:4 sparsity) and HBM3e bandwidth
+NOMINAL_BF16_TFLOPS = 2250.0
+NOMINAL_HBM_GBS = 8000.0
 PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "bsr_linear_deit_b_stack_traffic.txt")
 # single GEMMs of the stack's shapes (profiling cases): (k, n, b, sparsity, gelu, m)
 CASES = {
@@ -484,7 +488,9 @@ def run_gpu(args, world, rank, local):
                      "peak_source": f"{peak_src} bf16_tflops (burst, the dense bf16 cuBLAS rate)",
                      "kernel": "lpvit::bsr_linear_kernel<gelu, f32_out>", "launches_timed": linear_launches,
                      "launch_timing": "an event pair around every linear, in K steps run after the timed ones",
-                     "frac_of_sustained_peak": achieved / peak_sustained},
+                     "frac_of_sustained_peak": achieved / peak_sustained,
+                     "frac_of_nominal_peak": achieved / NOMINAL_BF16_TFLOPS,
+                     "nominal_peak": "GB300 dense bf16 2250 TFLOP/s (datasheet, without 2:4 sparsity)"},
         "linear_ms_per_step": lin_ms / args.steps,
         "pack_and_gaps_ms_per_step": (elapsed_ms - lin_ms) / args.steps,
         "hbm_gbs_linears": stack.algorithmic_bytes() * args.steps / (lin_ms / 1e3) / 1e9,
@@ -660,7 +666,9 @@ def run_config(args, local):
                 "roofline": {"bound": bound, "achieved": achieved, "peak": BW if bound == "hbm" else P,
                              "unit": "GB/s" if bound == "hbm" else "TFLOP/s", "frac": achieved / (BW if bound == "hbm" else P),
                              "frac_of_roofline_time": t_roof / t, "peak_source": src,
-                             "frac_tensor_burst": F / (t / 1e3) / 1e12 / P, "frac_hbm": B / (t / 1e3) / 1e9 / BW},
+                             "frac_tensor_burst": F / (t / 1e3) / 1e12 / P, "frac_hbm": B / (t / 1e3) / 1e9 / BW,
+                             "frac_tensor_nominal": F / (t / 1e3) / 1e12 / NOMINAL_BF16_TFLOPS,
+                             "frac_hbm_nominal": B / (t / 1e3) / 1e9 / NOMINAL_HBM_GBS},
                 "algorithmic_bytes": B, "effective_flops": F,
                 "graph": graph, "pack_ms_median": statistics.median(pack),
                 "dense_torch_ms_median": statistics.median(dense),
