@@ -377,6 +377,33 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
   // the work list must be this weight's plan: layout, group count, shape
   const bool sched_ok = P.sched[3] == 0 && P.sched[1] == P.n_groups && P.sched[4] == P.n && P.sched[5] == P.k &&
                         P.sched[6] == P.bn && P.sched[8] == SCHED_VERSION && P.n_groups <= MAX_GROUPS;
+  // When no group is cut into slices (S >= the chunk count), pair p's first unit is unit p: token
+  // tile p / n_groups, group p % n_groups, all of that group's entries. The producers and the MMA
+  // issuer take it from the work list themselves rather than wait for the scheduler's record (which
+  // is the same); the group's entry range is requested here, so the load overlaps the prologue.
+  const uint32_t u0 = blockIdx.x / 2;
+  const uint32_t unsplit_units = (uint32_t)P.n_tt * (uint32_t)P.n_groups;
+  const bool first_local = sched_ok && P.S >= kc && (warp == 0 || warp == 1 || warp == W_WARP);
+  int f_ga = 0, f_gb = 0;
+  if (first_local && u0 < unsplit_units) {
+    const int g = (int)(u0 % (uint32_t)P.n_groups);
+    f_ga = __ldg(gent + g);
+    f_gb = __ldg(gent + g + 1);
+  }
+  auto first_unit = [&](UnitInfo &d) {
+    if (u0 < unsplit_units) {
+      d.tt = (int)(u0 / (uint32_t)P.n_groups);
+      d.g = (int)(u0 % (uint32_t)P.n_groups);
+      d.s = 0;
+      d.nsl = 1;
+      d.e0 = f_ga;
+      d.e1 = f_gb;
+      d.ptile = (int)u0;
+    } else {
+      d.tt = -1; d.g = d.s = d.nsl = d.e0 = d.e1 = d.ptile = 0;
+    }
+    d.pad = 0;
+  };
   tc_fence_before();
   __syncthreads();
   cluster_sync();  // both CTAs' barriers are initialised before any signal crosses the pair
@@ -391,13 +418,20 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     bool ok = true;
     while (ok) {
       const uint32_t slot = ui % UR, uph = (ui / UR) & 1u;
-      if (!mbar_wait_cluster(unitf_bar(slot), uph, abort_flag, tmo)) {
-        ok = false;
-        if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_UNIT);
-        break;
+      UnitInfo inf;
+      int cw;  // chunk indices of entries win .. win + 31, one per lane
+      if (ui == 0 && first_local) {
+        first_unit(inf);
+        cw = inf.e0 + lane < inf.e1 ? __ldg(entries + inf.e0 + lane) : 0;
+      } else {
+        if (!mbar_wait_cluster(unitf_bar(slot), uph, abort_flag, tmo)) {
+          ok = false;
+          if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_UNIT);
+          break;
+        }
+        inf = ring[slot].inf;
+        cw = ring[slot].win[lane];
       }
-      const UnitInfo inf = ring[slot].inf;
-      int cw = ring[slot].win[lane];  // chunk indices of entries win .. win + 31, one per lane
       __syncwarp();
       if (lane == 0) {
         if (leader) mbar_arrive(unite_bar(slot));
@@ -569,12 +603,17 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       bool ok = true;
       while (ok) {
         const uint32_t slot = ui % UR, uph = (ui / UR) & 1u;
-        if (!mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)) {
-          ok = false;
-          if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_UNIT);
-          break;
+        UnitInfo inf;
+        if (ui == 0 && first_local) {
+          first_unit(inf);
+        } else {
+          if (!mbar_wait(unitf_bar(slot), uph, abort_flag, tmo)) {
+            ok = false;
+            if (lane == 0) atomicOr(&P.ctl->err, ERR_MMA_UNIT);
+            break;
+          }
+          inf = ring[slot].inf;
         }
-        const UnitInfo inf = ring[slot].inf;
         __syncwarp();
         if (lane == 0) mbar_arrive(unite_bar(slot));
         if (inf.tt < 0) break;
