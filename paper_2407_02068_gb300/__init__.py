@@ -283,7 +283,8 @@ def bsr_linear(w: BsrWeight, X: torch.Tensor, bias: torch.Tensor | None = None, 
     """Y = act(X W~^T + bias). X: bf16 [m, k] CUDA (a row-strided view with unit column stride is
     fine); bias: fp32 [n] or None. Returns Y [m, n] (or writes ``out``). With ``residual`` (bf16
     [m, n], 16-byte rows; may be ``out`` itself) Y = round(round(act(...)) + residual), bf16
-    (lpvit_bsr_linear_residual)."""
+    (lpvit_bsr_linear_residual). The library picks the kernel: m <= 256 runs one launch of the
+    small-m kernel, larger m the persistent CTA-pair kernel."""
     if X.dtype != torch.bfloat16 or X.dim() != 2 or X.stride(1) != 1:
         raise ValueError("X must be a 2-D bf16 tensor with unit column stride")
     m = X.shape[0]
