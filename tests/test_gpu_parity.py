@@ -408,8 +408,8 @@ def test_linear_gelu(lp, b):
 def test_gelu_epilogue_over_the_float32_range(lp):
     """All-zero mask: the output is GELU(bias). Biases sweep [-14, 14], tiny, huge and signed-zero
     values, against the oracle's exact GELU: float32 output within 5e-4 relative plus 2^-21 |t|
-    (single-precision MUFU approximations of the reciprocal and the exponential), relative alone
-    where t > -3; bf16 output within one bf16 ulp plus that."""
+    (the epilogue's GELU: a polynomial for log2 of the normal tail and one single-precision MUFU
+    exponential), relative alone where t > -3; bf16 output within one bf16 ulp plus that."""
     f32 = np.float32
     special = [0.0, -0.0, 1e-30, -1e-30, 1e-6, -1e-6, 20.0, -20.0, 1e4, -1e4, 3.0, -3.0]
     sweep = np.linspace(-14.0, 14.0, 4096 - len(special))
