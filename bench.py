@@ -99,6 +99,9 @@ def parse_args():
     p.add_argument("--cpu-budget-s", type=float, default=15.0, help="CPU seconds for the oracle baseline sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-dense", action="store_true")
+    p.add_argument("--launch", choices=["chain", "per-linear"], default="chain",
+                   help="the stack's 48 linears as one lpvit_bsr_linear_chain call (one persistent launch), "
+                        "or one lpvit_bsr_linear[_gelu] call each")
     p.add_argument("--case", default="stack", choices=["stack"] + sorted(CASES),
                    help="stack (the benchmarked workload) or one GEMM of it, for profiling")
     p.add_argument("--calibrate", action="store_true",
@@ -138,9 +141,9 @@ def kernel_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic():
-    """DRAM bytes per launch of the linear kernel from the committed ncu summary, if it was
-    taken on the current kernel source (else None)."""
+def profiled_traffic(key: str = "dram_bytes_per_stack_linear_launch"):
+    """DRAM bytes per launch of the linear kernel (per chain launch: key dram_bytes_per_chain_launch)
+    from the committed ncu summary, if it was taken on the current kernel source (else None)."""
     try:
         kv = {}
         with open(PROFILE_TRAFFIC) as f:
@@ -150,7 +153,7 @@ def profiled_traffic():
                     kv[k.strip()] = v.strip()
         if kv.get("kernel_source_sha") != kernel_source_hash():
             return None
-        return float(kv["dram_bytes_per_stack_linear_launch"])
+        return float(kv[key])
     except (OSError, KeyError, ValueError):
         return None
 
@@ -346,9 +349,11 @@ def run_gpu(args, world, rank, local):
     stack.h_in.copy_(h0)
     s = torch.cuda.current_stream()
     ngemm = len(stack.gemms)
+    chain = args.launch == "chain"
+    nev = 1 if chain else ngemm  # event pairs per step: one per library call
 
     for _ in range(max(args.warmup, 3)):
-        stack.step()
+        stack.step(chain=chain)
     stack.check()
     torch.cuda.synchronize()
 
@@ -361,21 +366,30 @@ def run_gpu(args, world, rank, local):
     time.sleep(0.3)
     start.record(s)
     for k in range(args.steps):
-        stack.step()
+        stack.step(chain=chain)
     end.record(s)
     torch.cuda.synchronize()
     # ---------------- the linear kernel's launch durations (roofline): K more steps with an event
-    # pair around every linear (the records cost the stream time, so they stay out of the step time)
-    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(ngemm)]
+    # pair around every library call, i.e. every linear or the chain call (the records cost the
+    # stream time, so they stay out of the step time)
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(nev)]
           for _ in range(args.steps)]
+    ev_step = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
     for k in range(args.steps):
-        stack.step(events=ev[k])
+        ev_step[k][0].record(s)
+        stack.step(events=ev[k], chain=chain)
+        ev_step[k][1].record(s)
     torch.cuda.synchronize()
     barrier(world)
     clk = clocks.stop()
     stack.check()
     elapsed_ms = start.elapsed_time(end)
     lin_ms = sum(a.elapsed_time(b) for row in ev for (a, b) in row)
+    # the same pass split three ways: pack (step start to the first linear), the linears, and the
+    # gaps between consecutive linears (the rest of that pass's step)
+    pack_ms = sum(a.elapsed_time(row[0][0]) for (a, _), row in zip(ev_step, ev))
+    evpass_ms = sum(a.elapsed_time(b) for (a, b) in ev_step)
     elapsed_max = max_over_ranks(elapsed_ms, world, dev)
     flops_step = stack.effective_flops()
     value = weak_scaling_value(flops_step, args.steps, world, elapsed_max)
@@ -384,8 +398,8 @@ def run_gpu(args, world, rank, local):
     peaks, peak_src = load_peaks()
     peak = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
     peak_sustained = float(peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
-    traffic = profiled_traffic()
-    linear_launches = ngemm * args.steps
+    traffic = profiled_traffic("dram_bytes_per_chain_launch" if chain else "dram_bytes_per_stack_linear_launch")
+    linear_launches = ((ngemm + 47) // 48 if chain else ngemm) * args.steps
 
     # ---------------- e2e through the public API: pinned host in, pinned host out, every step
     # Each step copies its input from pinned host memory and its result back to pinned host memory,
@@ -398,7 +412,7 @@ def run_gpu(args, world, rank, local):
     out_host = torch.empty_like(h0_host).pin_memory()
     stage = torch.empty_like(stack.out)
     cs = torch.cuda.Stream(device=dev)
-    lin_ev = [(torch.cuda.Event(), torch.cuda.Event()) for _ in range(ngemm)]
+    lin_ev = [(torch.cuda.Event(), torch.cuda.Event()) for _ in range(nev)]
     in_ready, out_ready, out_done = torch.cuda.Event(), torch.cuda.Event(), torch.cuda.Event()
 
     def e2e_run(nsteps):
@@ -411,7 +425,7 @@ def run_gpu(args, world, rank, local):
             out_done.record(cs)
         for k in range(nsteps):
             s.wait_event(in_ready)
-            out = stack.step(events=lin_ev)
+            out = stack.step(events=lin_ev, chain=chain)
             if k + 1 < nsteps:
                 cs.wait_event(lin_ev[0][1])
                 with torch.cuda.stream(cs):
@@ -481,22 +495,28 @@ def run_gpu(args, world, rank, local):
         "config": {"workload": WORKLOAD, "M": M_TOKENS, "block": BLOCK, "gemms": ngemm,
                    "sparsity": "per-GEMM U[0.30,0.70], antithetic layer pairs, mean 0.50",
                    "step": "pack all 48 weights + 48 chained block-sparse linears (fc1 with GELU)",
+                   "launch": "one lpvit_bsr_linear_chain call (one launch)" if chain else "one call per linear",
                    "l2": "no flush: each step streams ~15 GB (> 129 MB L2)",
                    "parallelism": f"replicas x{world} (token batches per rank, no collective)"},
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "traffic": traffic,
                      "peak_source": f"{peak_src} bf16_tflops (burst, the dense bf16 cuBLAS rate)",
-                     "kernel": "lpvit::bsr_linear_kernel<gelu, f32_out>", "launches_timed": linear_launches,
-                     "launch_timing": "an event pair around every linear, in K steps run after the timed ones",
+                     "kernel": ("lpvit::bsr_linear_chain_kernel" if chain
+                                else "lpvit::bsr_linear_kernel<gelu, f32_out, deep>"),
+                     "launches_timed": linear_launches,
+                     "launch_timing": ("an event pair around every chain call" if chain else
+                                       "an event pair around every linear") + ", in K steps run after the timed ones",
                      "frac_of_sustained_peak": achieved / peak_sustained,
                      "frac_of_nominal_peak": achieved / NOMINAL_BF16_TFLOPS,
                      "nominal_peak": "GB300 dense bf16 2250 TFLOP/s (datasheet, without 2:4 sparsity)"},
         "linear_ms_per_step": lin_ms / args.steps,
-        "pack_and_gaps_ms_per_step": (elapsed_ms - lin_ms) / args.steps,
+        "pack_ms_per_step": pack_ms / args.steps,
+        "gaps_ms_per_step": (evpass_ms - pack_ms - lin_ms) / args.steps,
+        "events_pass_ms_per_step": evpass_ms / args.steps,
         "hbm_gbs_linears": stack.algorithmic_bytes() * args.steps / (lin_ms / 1e3) / 1e9,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": io_bytes, "d2h_bytes_per_step": io_bytes,
                 "steps": e2e_steps},
-        "gpu_launches": args.steps * stack.launches_per_step(),
+        "gpu_launches": args.steps * stack.launches_per_step(chain),
         "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"],
                    "power_w_median": clk.get("power_w_median"), "samples": clk["samples"]},
         "cpu_baseline": cpu,

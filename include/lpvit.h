@@ -58,7 +58,10 @@ typedef enum { LPVIT_BF16 = 0, LPVIT_F32 = 1 } lpvit_dtype;
  *   [j*bk, (j+1)*bk);  k/bk block columns.
  *   row_ptr [n/bn + 1]         int32   exclusive prefix sum of kept blocks per panel
  *   col_idx [nnzb_capacity]    int32   kept block columns of each panel, ascending
- *   blocks  [nnzb_capacity][bn][bk] bf16 kept tiles of W, row-major inside the tile, bits unchanged
+ *   blocks  [nnzb_capacity][bn][bk] bf16 kept tiles of W, row-major inside the tile, bits unchanged;
+ *                                      may be NULL: the linear reads only `sched`, so the pack then
+ *                                      writes row_ptr, col_idx and the work list alone, and the
+ *                                      packed weight holds one copy of its kept tiles
  *   sched   [sched_bytes]      bytes   work list for lpvit_bsr_linear (layout private to the
  *                                      library; see lpvit_sched_bytes)
  * nnzb_capacity must be >= the number of kept blocks; (n/bn)*(k/bk) always suffices. */
@@ -250,6 +253,45 @@ lpvit_status lpvit_bsr_linear_gelu(const lpvit_bsr *bsr, const void *X, int64_t 
 lpvit_status lpvit_bsr_linear_residual(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx,
                                        const float *bias, int32_t gelu, const void *R, int64_t ldr, void *Y,
                                        int64_t ldy, void *workspace, size_t ws_bytes, void *stream);
+
+/* One linear of a chain: Y = act(X W~^T + bias) with bf16 output, act = GELU when gelu == 1.
+ * bsr, X / ldx, bias, Y / ldy and gelu mean what they mean for lpvit_bsr_linear[_gelu]. */
+typedef struct {
+  const lpvit_bsr *bsr;
+  const void *X;
+  int64_t ldx;
+  const float *bias;
+  void *Y;
+  int64_t ldy;
+  int32_t gelu;
+} lpvit_chain_link;
+
+/* Bytes of device workspace lpvit_bsr_linear_chain needs for these links at m tokens (0 for a
+ * null or empty list, or a link whose weight shape is invalid). Zero-filled once before its first
+ * use; every call leaves it ready for the next (as lpvit_workspace_bytes). */
+size_t lpvit_chain_workspace_bytes(const lpvit_chain_link *links, int32_t count, int64_t m);
+
+/* The linears links[0], links[1], ... links[count-1] over the same m tokens, in that order, as if
+ * each were a separate lpvit_bsr_linear (gelu 0) / lpvit_bsr_linear_gelu (gelu 1) call with bf16
+ * output on `stream`; the results are bit-identical to those calls. A link may read what earlier
+ * links wrote (the layer chain of Sec. 3.3's block matmuls, one after another, e.g. fc1 -> fc2).
+ * Consecutive links run in one persistent launch (up to 48 links per launch): the units of a
+ * link follow those of the link before it, and a unit of 256 tokens starts its copies once the
+ * previous link has stored every output of those 256 tokens, so one link's last units overlap the
+ * next link's first and the launch start and end are paid once per launch, not per link.
+ * Rules: row r of every X and Y holds token r. Where a link's X or Y overlaps an earlier link's X
+ * or Y, the two must have the same leading dimension and overlap only row for row (a column range
+ * of the same rows, e.g. X = the last third of an earlier Y's columns); a link that breaks this,
+ * one whose work would be cut into slices (few token tiles: m <= 256, or too few units to fill the
+ * GPU), and m <= 256 generally, start a new launch or run on their own. No Y may overlap a weight,
+ * work list or bias of the chain.
+ *   workspace / ws_bytes: >= lpvit_chain_workspace_bytes(links, count, m), 256-byte aligned.
+ * Every link is checked before anything is launched; nothing runs if one fails.
+ * Errors: LPVIT_ERR_INVALID_ARG (count < 0, null links or workspace, gelu not 0 or 1, and the
+ * checks of lpvit_bsr_linear for each link), LPVIT_ERR_UNSUPPORTED, LPVIT_ERR_WORKSPACE,
+ * LPVIT_ERR_CUDA. count == 0 or m == 0 does nothing and returns LPVIT_OK. */
+lpvit_status lpvit_bsr_linear_chain(const lpvit_chain_link *links, int32_t count, int64_t m, void *workspace,
+                                    size_t ws_bytes, void *stream);
 
 /* Size of the library-held scratch array used by lpvit_bsr_linear_noalloc (8 MiB). */
 #define LPVIT_NOALLOC_SCRATCH_BYTES (8 * 1024 * 1024)

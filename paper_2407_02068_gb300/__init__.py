@@ -29,7 +29,7 @@ from . import _lib
 
 __all__ = ["BsrWeight", "alloc_bsr", "pack_bsr", "pack_bsr_into", "pack_bsr_many_into", "taylor_block_mask",
            "taylor_pack_bsr",
-           "workspace_for", "bsr_linear", "check", "LpvitError", "delta_curve", "lambda_search", "mean_gradient",
+           "workspace_for", "bsr_linear", "bsr_linear_chain", "check", "LpvitError", "delta_curve", "lambda_search", "mean_gradient",
            "add_layernorm", "attention"]
 
 LpvitError = _lib.LpvitError
@@ -315,6 +315,35 @@ def bsr_linear(w: BsrWeight, X: torch.Tensor, bias: torch.Tensor | None = None, 
     if st != _lib.LPVIT_OK:
         raise LpvitError(st, "lpvit_bsr_linear_gelu" if gelu else "lpvit_bsr_linear")
     return out
+
+
+def bsr_linear_chain(steps, workspace: torch.Tensor | None = None, stream=None) -> None:
+    """Consecutive linears over the same m tokens in one library call (lpvit_bsr_linear_chain).
+    ``steps``: a sequence of (w, X, bias, out, gelu): X and out bf16 [m, k] / [m, n] CUDA tensors with
+    unit column stride (row-strided views are fine; a later X may be an earlier out, or a column range
+    of it), bias fp32 [n] or None. Each out = act(X W~^T + bias), in order, bit-identical to separate
+    bsr_linear calls. The workspace defaults to a zero-filled one of lpvit_chain_workspace_bytes."""
+    steps = list(steps)
+    if not steps:
+        return
+    m = steps[0][1].shape[0]
+    rows = []
+    for w, X, bias, out, gelu in steps:
+        for t in (X, out):
+            if t.dtype != torch.bfloat16 or t.dim() != 2 or t.stride(1) != 1 or t.shape[0] != m:
+                raise ValueError("X and out must be 2-D bf16 tensors of m rows with unit column stride")
+        if bias is not None and (bias.dtype != torch.float32 or not bias.is_contiguous()):
+            raise ValueError("bias must be a contiguous fp32 tensor")
+        rows.append((w.struct(), X.data_ptr(), X.stride(0), bias.data_ptr() if bias is not None else None,
+                     out.data_ptr(), out.stride(0), 1 if gelu else 0))
+    links = _lib.chain_links(rows)
+    if workspace is None:
+        nbytes = _lib.lpvit_chain_workspace_bytes(links, len(rows), m)
+        workspace = torch.zeros(max(nbytes, 256), dtype=torch.uint8, device=steps[0][1].device)
+    st = _lib.lpvit_bsr_linear_chain(links, len(rows), m, workspace.data_ptr(), workspace.numel(),
+                                     _stream_handle(stream))
+    if st != _lib.LPVIT_OK:
+        raise LpvitError(st, "lpvit_bsr_linear_chain")
 
 
 def check(workspace: torch.Tensor, stream=None) -> None:

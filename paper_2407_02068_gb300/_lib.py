@@ -25,7 +25,8 @@ EXPORTS = ("lpvit_sched_bytes", "lpvit_pack_bsr", "lpvit_taylor_pack_bsr", "lpvi
            "lpvit_bsr_linear_gelu", "lpvit_bsr_linear_noalloc", "lpvit_check", "lpvit_status_string",
            "lpvit_selftest_wait", "lpvit_pack_bsr_many", "lpvit_taylor_block_mask",
            "lpvit_delta_curve_workspace_bytes", "lpvit_delta_curve", "lpvit_lambda_search", "lpvit_mean_gradient",
-           "lpvit_add_layernorm", "lpvit_attention", "lpvit_bsr_linear_residual")
+           "lpvit_add_layernorm", "lpvit_attention", "lpvit_bsr_linear_residual", "lpvit_chain_workspace_bytes",
+           "lpvit_bsr_linear_chain")
 LPVIT_NOALLOC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 
@@ -35,6 +36,13 @@ class lpvit_bsr(ctypes.Structure):
         ("nnzb_capacity", ctypes.c_int32),
         ("row_ptr", ctypes.c_void_p), ("col_idx", ctypes.c_void_p), ("blocks", ctypes.c_void_p),
         ("sched", ctypes.c_void_p), ("sched_bytes", ctypes.c_size_t),
+    ]
+
+
+class lpvit_chain_link(ctypes.Structure):
+    _fields_ = [
+        ("bsr", ctypes.POINTER(lpvit_bsr)), ("X", ctypes.c_void_p), ("ldx", ctypes.c_int64),
+        ("bias", ctypes.c_void_p), ("Y", ctypes.c_void_p), ("ldy", ctypes.c_int64), ("gelu", ctypes.c_int32),
     ]
 
 
@@ -91,6 +99,11 @@ def load(path: str | None = None):
             f.argtypes = [BP, V, I64, I64, V, V, I64, ctypes.c_int, V, SZ, V]
         lib.lpvit_bsr_linear_residual.restype = ctypes.c_int
         lib.lpvit_bsr_linear_residual.argtypes = [BP, V, I64, I64, V, ctypes.c_int32, V, I64, V, I64, V, SZ, V]
+        CL = ctypes.POINTER(lpvit_chain_link)
+        lib.lpvit_chain_workspace_bytes.restype = SZ
+        lib.lpvit_chain_workspace_bytes.argtypes = [CL, I32, I64]
+        lib.lpvit_bsr_linear_chain.restype = ctypes.c_int
+        lib.lpvit_bsr_linear_chain.argtypes = [CL, I32, I64, V, SZ, V]
         lib.lpvit_bsr_linear_noalloc.restype = ctypes.c_int
         lib.lpvit_bsr_linear_noalloc.argtypes = [BP, V, I64, I64, V, V, I64, ctypes.c_int, ctypes.c_int, V]
         lib.lpvit_check.restype = ctypes.c_int
@@ -200,6 +213,24 @@ def lpvit_bsr_linear_residual(bsr, X_ptr, m, ldx, bias_ptr, gelu, R_ptr, ldr, Y_
                               stream) -> int:
     return load().lpvit_bsr_linear_residual(ctypes.byref(bsr), X_ptr, m, ldx, bias_ptr, int(gelu), R_ptr,
                                             ldr, Y_ptr, ldy, ws_ptr, ws_bytes, stream)
+
+
+def chain_links(rows) -> ctypes.Array:
+    """A ctypes array of lpvit_chain_link from (bsr, X_ptr, ldx, bias_ptr, Y_ptr, ldy, gelu) tuples; the
+    lpvit_bsr structs must outlive the array."""
+    arr = (lpvit_chain_link * len(rows))()
+    for i, (bsr, X_ptr, ldx, bias_ptr, Y_ptr, ldy, gelu) in enumerate(rows):
+        arr[i] = lpvit_chain_link(ctypes.pointer(bsr) if bsr is not None else None, X_ptr, ldx, bias_ptr, Y_ptr,
+                                  ldy, int(gelu))
+    return arr
+
+
+def lpvit_chain_workspace_bytes(links, count: int, m: int) -> int:
+    return int(load().lpvit_chain_workspace_bytes(links, count, m))
+
+
+def lpvit_bsr_linear_chain(links, count: int, m: int, ws_ptr, ws_bytes, stream) -> int:
+    return load().lpvit_bsr_linear_chain(links, count, m, ws_ptr, ws_bytes, stream)
 
 
 def lpvit_bsr_linear_noalloc(bsr, X_ptr, m, ldx, bias_ptr, Y_ptr, ldy, y_dtype, gelu, stream) -> int:

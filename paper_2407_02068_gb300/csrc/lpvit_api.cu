@@ -3,6 +3,7 @@
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#include <memory>
 #include <mutex>
 #include <vector>
 #include <cuda.h>
@@ -128,16 +129,30 @@ lpvit_status cuda_status(cudaError_t e) { return e == cudaSuccess ? LPVIT_OK : L
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias, void *Y,
-                        int64_t ldy, lpvit_dtype y_dtype, void *workspace, size_t ws_bytes, void *stream, int gelu,
-                        const void *R = nullptr, int64_t ldr = 0) {
+// One linear call, checked and parameterised, ready to launch.
+struct Prepared {
+  LinearParams P;
+  CUtensorMap tmX, tmW;  // the pair kernel's tensor maps (large m)
+  WsLayout W;
+  int sms = 0;
+  bool empty = false;    // m == 0: nothing to do
+  bool small = false;    // m <= SMALL_M_MAX: the small-m kernel
+};
+
+// The argument checks of a linear call, then its parameter block and tensor maps. Launches nothing.
+lpvit_status prepare_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias, void *Y,
+                            int64_t ldy, lpvit_dtype y_dtype, void *workspace, size_t ws_bytes, int gelu,
+                            const void *R, int64_t ldr, Prepared &pr) {
   if (!bsr) return LPVIT_ERR_INVALID_ARG;
   const int n = bsr->n, k = bsr->k, bn = bsr->bn, bk = bsr->bk;
   if (!valid_side(bn) || !valid_side(bk)) return LPVIT_ERR_UNSUPPORTED;
   if (!shape_ok(n, k, bn, bk)) return LPVIT_ERR_INVALID_ARG;
   if (m < 0) return LPVIT_ERR_INVALID_ARG;
   if (y_dtype != LPVIT_BF16 && y_dtype != LPVIT_F32) return LPVIT_ERR_INVALID_ARG;
-  if (m == 0) return LPVIT_OK;
+  if (m == 0) {
+    pr.empty = true;
+    return LPVIT_OK;
+  }
   if (!X || !Y || !bsr->sched || !workspace) return LPVIT_ERR_INVALID_ARG;
   if (bsr->nnzb_capacity < 0) return LPVIT_ERR_INVALID_ARG;
   if (ldx < k || ldx % 8 != 0 || !aligned(X, 16)) return LPVIT_ERR_INVALID_ARG;
@@ -161,15 +176,14 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
     if (!in_place && r0 < y1 && y0 < r1) return LPVIT_ERR_INVALID_ARG;
   }
   if (bsr->sched_bytes < lpvit_sched_bytes(n, k, bn, bk)) return LPVIT_ERR_WORKSPACE;
-  int sms = 0;
   lpvit_status st = LPVIT_OK;
-  if (!device_info(&sms, &st)) return st;
-  const WsLayout W = ws_layout(m, n, k, sms);
-  if (ws_bytes < W.total) return LPVIT_ERR_WORKSPACE;
+  if (!device_info(&pr.sms, &st)) return st;
+  pr.W = ws_layout(m, n, k, pr.sms);
+  if (ws_bytes < pr.W.total) return LPVIT_ERR_WORKSPACE;
   const int ng = (int)ceil_div(n, GROUP_FEATURES);
   const int kc = sched_chunks(k);
   const int64_t stream_tiles = sched_stream_tiles(ng, kc);
-  LinearParams P;
+  LinearParams &P = pr.P;
   P.sched = static_cast<const int32_t *>(bsr->sched);
   P.stream_tiles = stream_tiles;
   P.bias = bias;
@@ -181,7 +195,7 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.bn = bn;
   P.n_tt = (int)ceil_div(m, TOKENS_PER_TILE);
   P.n_groups = ng;
-  P.S = W.S;
+  P.S = pr.W.S;
   P.y_f32 = y_dtype == LPVIT_F32;
   P.gelu = gelu;
   P.y_vec16 = (aligned(Y, 16) && ((size_t)ldy * ysz) % 16 == 0) ? 1 : 0;
@@ -192,28 +206,29 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
   P.r_vec32 = (R && aligned(R, 32) && ((size_t)ldr * 2) % 32 == 0) ? 1 : 0;
   uint8_t *ws = static_cast<uint8_t *>(workspace);
   P.ctl = reinterpret_cast<Control *>(ws);
-  P.partials = reinterpret_cast<float *>(ws + W.partials_off);
-  P.part_rows = W.part_rows;
+  P.partials = reinterpret_cast<float *>(ws + pr.W.partials_off);
+  P.part_rows = pr.W.part_rows;
   P.timeout_ns = TIMEOUT_NS;
   P.X = static_cast<const uint16_t *>(X);
   P.ldx = ldx;
   P.wstream = reinterpret_cast<const uint16_t *>(static_cast<const uint8_t *>(bsr->sched) +
                                                  sched_stream_offset_bytes(ng, kc));
   P.kp = 1;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (m <= SMALL_M_MAX) return cuda_status(launch_linear_small(P, sms, s));
+  if (m <= SMALL_M_MAX) {
+    pr.small = true;
+    return LPVIT_OK;
+  }
   EncodeTiledFn enc = encode_fn();
   if (!enc) return LPVIT_ERR_CUDA;
 
   cuuint32_t es[2] = {1, 1};
   // X: [m rows][k columns], boxes of 64 columns x 128 tokens (one CTA's half of a token tile);
   // rows beyond m and columns beyond k read as zero
-  CUtensorMap tmX, tmW;
   {
     cuuint64_t dims[2] = {(cuuint64_t)k, (cuuint64_t)m};
     cuuint64_t strides[1] = {(cuuint64_t)ldx * 2};
     cuuint32_t box[2] = {(cuuint32_t)CHUNK_COLS, (cuuint32_t)CTA_TOKENS};
-    if (enc(&tmX, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(X), dims, strides, box, es,
+    if (enc(&pr.tmX, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(X), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return LPVIT_ERR_INVALID_ARG;
@@ -224,34 +239,102 @@ lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t 
     cuuint64_t dims[2] = {(cuuint64_t)CHUNK_COLS, (cuuint64_t)(stream_tiles * GROUP_FEATURES)};
     cuuint64_t strides[1] = {(cuuint64_t)CHUNK_COLS * 2};
     cuuint32_t box[2] = {(cuuint32_t)CHUNK_COLS, (cuuint32_t)HALF_FEATURES};
-    if (enc(&tmW, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, wstream, dims, strides, box, es,
+    if (enc(&pr.tmW, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, wstream, dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return LPVIT_ERR_INVALID_ARG;
   }
-  const int pairs = sms / 2;
+  return LPVIT_OK;
+}
+
+// Launches a prepared call: the small-m kernel, or the pair kernel (+ the slice reduction).
+lpvit_status launch_prepared(const Prepared &pr, cudaStream_t s) {
+  if (pr.empty) return LPVIT_OK;
+  const LinearParams &P = pr.P;
+  if (pr.small) return cuda_status(launch_linear_small(P, pr.sms, s));
+  const int pairs = pr.sms / 2;
+  const int kc = sched_chunks(P.k);
   const int64_t units_max = (int64_t)P.n_tt * P.n_groups * ceil_div(kc, P.S);
   const int grid = 2 * (int)(units_max < pairs ? units_max : pairs);
-  cudaError_t e = launch_linear(tmX, tmW, P, grid, s);
-  if (e != cudaSuccess || !W.split) return cuda_status(e);
+  cudaError_t e = launch_linear(pr.tmX, pr.tmW, P, grid, s);
+  if (e != cudaSuccess || !pr.W.split) return cuda_status(e);
   ReduceParams RP;
   RP.sched = P.sched;
   RP.partials = P.partials;
-  RP.bias = bias;
-  RP.Y = Y;
-  RP.ldy = ldy;
-  RP.m = m;
-  RP.n = n;
-  RP.bn = bn;
+  RP.bias = P.bias;
+  RP.Y = P.Y;
+  RP.ldy = P.ldy;
+  RP.m = P.m;
+  RP.n = P.n;
+  RP.bn = P.bn;
   RP.n_tt = P.n_tt;
-  RP.n_groups = ng;
+  RP.n_groups = P.n_groups;
   RP.S = P.S;
   RP.part_rows = P.part_rows;
   RP.y_f32 = P.y_f32;
-  RP.gelu = gelu;
+  RP.gelu = P.gelu;
   RP.R = P.R;
   RP.ldr = P.ldr;
-  return cuda_status(launch_split_reduce(RP, (int64_t)P.n_tt * ng * P.part_rows * (GROUP_FEATURES / 8), s));
+  return cuda_status(launch_split_reduce(RP, (int64_t)P.n_tt * P.n_groups * P.part_rows * (GROUP_FEATURES / 8), s));
+}
+
+lpvit_status run_linear(const lpvit_bsr *bsr, const void *X, int64_t m, int64_t ldx, const float *bias, void *Y,
+                        int64_t ldy, lpvit_dtype y_dtype, void *workspace, size_t ws_bytes, void *stream, int gelu,
+                        const void *R = nullptr, int64_t ldr = 0) {
+  Prepared pr;
+  const lpvit_status st = prepare_linear(bsr, X, m, ldx, bias, Y, ldy, y_dtype, workspace, ws_bytes, gelu, R, ldr, pr);
+  if (st != LPVIT_OK) return st;
+  return launch_prepared(pr, static_cast<cudaStream_t>(stream));
+}
+
+// ---------------------------------------------------------------- chains
+// A chain's workspace: the control block and room for the split-unit partial sums of the largest
+// of its linears (those run on their own), then the per-(linear, token tile) counters of a launch.
+struct ChainWs {
+  size_t counters_off, total;
+};
+size_t align256(size_t x) { return (x + 255) / 256 * 256; }
+ChainWs chain_ws_layout(const lpvit_chain_link *links, int32_t count, int64_t m, int sms) {
+  size_t most = sizeof(Control);
+  for (int32_t i = 0; i < count; ++i) {
+    const size_t t = ws_layout(m, links[i].bsr->n, links[i].bsr->k, sms).total;
+    if (t > most) most = t;
+  }
+  ChainWs L;
+  L.counters_off = align256(most);
+  const int jobs = count < CHAIN_MAX_JOBS ? count : CHAIN_MAX_JOBS;
+  L.total = L.counters_off + align256((size_t)jobs * (size_t)ceil_div(m, TOKENS_PER_TILE) * sizeof(uint32_t));
+  return L;
+}
+
+// A linear joins a chain launch when it runs on the pair kernel without slices.
+bool chainable(const Prepared &pr) { return !pr.empty && !pr.small && !pr.W.split && !pr.P.R && !pr.P.y_f32; }
+
+// Row r of two bf16 buffers (base a, row width wa, stride la; base b, wb, lb; in elements) may
+// overlap only within token row r: then each linear of a chain touches, in any buffer, only the rows
+// of the token tiles it computes, and the tile counters order every access.
+bool rows_disjoint_or_aligned(const void *a, int64_t wa, int64_t la, const void *b, int64_t wb, int64_t lb,
+                              int64_t m) {
+  const intptr_t a0 = reinterpret_cast<intptr_t>(a), b0 = reinterpret_cast<intptr_t>(b);
+  const intptr_t a1 = a0 + (intptr_t)((m - 1) * la + wa) * 2, b1 = b0 + (intptr_t)((m - 1) * lb + wb) * 2;
+  if (a1 <= b0 || b1 <= a0) return true;
+  if (la != lb) return false;
+  const intptr_t d = a0 - b0, row = (intptr_t)la * 2;
+  return d >= 2 * (intptr_t)wb - row && d + 2 * (intptr_t)wa <= row;
+}
+
+// Link j may join a launch that holds links [i, j): every buffer it writes or reads overlaps the
+// others' only row for row.
+bool joins(const lpvit_chain_link *L, int32_t i, int32_t j, int64_t m) {
+  const lpvit_chain_link &c = L[j];
+  for (int32_t q = i; q < j; ++q) {
+    const lpvit_chain_link &e = L[q];
+    if (!rows_disjoint_or_aligned(c.Y, c.bsr->n, c.ldy, e.X, e.bsr->k, e.ldx, m) ||
+        !rows_disjoint_or_aligned(c.Y, c.bsr->n, c.ldy, e.Y, e.bsr->n, e.ldy, m) ||
+        !rows_disjoint_or_aligned(c.X, c.bsr->k, c.ldx, e.Y, e.bsr->n, e.ldy, m))
+      return false;
+  }
+  return true;
 }
 
 // The checks lpvit_pack_bsr applies to one weight.
@@ -393,6 +476,76 @@ lpvit_status lpvit_bsr_linear_residual(const lpvit_bsr *bsr, const void *X, int6
                                        int64_t ldy, void *workspace, size_t ws_bytes, void *stream) {
   if (!R || (gelu != 0 && gelu != 1)) return LPVIT_ERR_INVALID_ARG;
   return run_linear(bsr, X, m, ldx, bias, Y, ldy, LPVIT_BF16, workspace, ws_bytes, stream, gelu, R, ldr);
+}
+
+size_t lpvit_chain_workspace_bytes(const lpvit_chain_link *links, int32_t count, int64_t m) {
+  if (!links || count <= 0 || m < 0) return 0;
+  for (int32_t i = 0; i < count; ++i)
+    if (!links[i].bsr || !shape_ok(links[i].bsr->n, links[i].bsr->k, links[i].bsr->bn, links[i].bsr->bk)) return 0;
+  int sms = 0;
+  lpvit_status st = LPVIT_OK;
+  if (!device_info(&sms, &st)) sms = 152;  // sizing only; the call itself reports the device error
+  return chain_ws_layout(links, count, m > 0 ? m : 1, sms).total;
+}
+
+lpvit_status lpvit_bsr_linear_chain(const lpvit_chain_link *links, int32_t count, int64_t m, void *workspace,
+                                    size_t ws_bytes, void *stream) {
+  if (count < 0 || m < 0) return LPVIT_ERR_INVALID_ARG;
+  if (count == 0 || m == 0) return LPVIT_OK;
+  if (!links || !workspace || !aligned(workspace, 256)) return LPVIT_ERR_INVALID_ARG;
+  // every link is checked before anything is launched
+  for (int32_t i = 0; i < count; ++i)
+    if (!links[i].bsr || (links[i].gelu != 0 && links[i].gelu != 1)) return LPVIT_ERR_INVALID_ARG;
+  std::vector<Prepared> pr((size_t)count);
+  for (int32_t i = 0; i < count; ++i) {
+    const lpvit_chain_link &c = links[i];
+    const lpvit_status st = prepare_linear(c.bsr, c.X, m, c.ldx, c.bias, c.Y, c.ldy, LPVIT_BF16, workspace, ws_bytes,
+                                           c.gelu, nullptr, 0, pr[(size_t)i]);
+    if (st != LPVIT_OK) return st;
+  }
+  const ChainWs CW = chain_ws_layout(links, count, m, pr[0].sms);
+  if (ws_bytes < CW.total) return LPVIT_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int n_tt = (int)ceil_div(m, TOKENS_PER_TILE);
+  std::unique_ptr<ChainParams> C(new ChainParams());
+  for (int32_t i = 0; i < count;) {
+    // the longest run from link i that one launch takes
+    int32_t j = i + 1;
+    uint64_t units = chainable(pr[(size_t)i]) ? (uint64_t)n_tt * pr[(size_t)i].P.n_groups : 0;
+    if (chainable(pr[(size_t)i]))
+      while (j < count && j - i < CHAIN_MAX_JOBS && chainable(pr[(size_t)j]) && joins(links, i, j, m) &&
+             units + (uint64_t)n_tt * pr[(size_t)j].P.n_groups <= 0x7fffffffull) {
+        units += (uint64_t)n_tt * pr[(size_t)j].P.n_groups;
+        ++j;
+      }
+    if (j - i == 1) {  // a run of one: the linear's own launch
+      const lpvit_status st = launch_prepared(pr[(size_t)i], s);
+      if (st != LPVIT_OK) return st;
+      i = j;
+      continue;
+    }
+    uint32_t u0 = 0;
+    for (int32_t q = i; q < j; ++q) {
+      ChainJob &J = C->job[q - i];
+      const Prepared &p = pr[(size_t)q];
+      J.tmX = p.tmX;
+      J.tmW = p.tmW;
+      J.P = p.P;
+      J.unit0 = u0;
+      J.units = (uint32_t)n_tt * (uint32_t)p.P.n_groups;
+      u0 += J.units;
+    }
+    C->tile_done = reinterpret_cast<uint32_t *>(static_cast<uint8_t *>(workspace) + CW.counters_off);
+    C->total_units = u0;
+    C->njobs = j - i;
+    C->n_tt = n_tt;
+    const int pairs = pr[0].sms / 2;
+    const int grid = 2 * (int)((int64_t)u0 < pairs ? (int64_t)u0 : pairs);
+    const cudaError_t e = launch_linear_chain(*C, grid, s);
+    if (e != cudaSuccess) return LPVIT_ERR_CUDA;
+    i = j;
+  }
+  return LPVIT_OK;
 }
 
 lpvit_status lpvit_check(void *workspace, void *stream) {

@@ -57,7 +57,8 @@ struct Control {
   unsigned int done_ctas;   // CTAs that found the queue empty; the last one resets both
   unsigned int err;         // device error word (bit set per failing wait site), read by lpvit_check
   unsigned int err_detail;
-  unsigned int pad[60];
+  unsigned int chain_ctas;  // chain launches: CTAs that have finished; the last one resets the tile counters
+  unsigned int pad[59];
 };
 static_assert(sizeof(Control) == 256, "control block is 256 bytes");
 
@@ -117,6 +118,7 @@ enum ErrBits : unsigned int {
   ERR_DRAIN = 1u << 7,
   ERR_SCHED_OVERFLOW = 1u << 8,
   ERR_BAD_SCHED = 1u << 9,
+  ERR_CHAIN_WAIT = 1u << 10,
 };
 
 // Launchers (host side, defined next to their kernels).
@@ -144,6 +146,27 @@ cudaError_t launch_pack_many(const PackJob *jobs, int count, int num_sms, cudaSt
 cudaError_t launch_linear(const CUtensorMap &tmX, const CUtensorMap &tmW, const LinearParams &P, int grid,
                           cudaStream_t s);
 cudaError_t launch_split_reduce(const ReduceParams &R, int64_t threads, cudaStream_t s);
+// A chain: consecutive linears over the same m tokens in one persistent launch of the pair kernel.
+// Linear j's units follow linear j - 1's in the unit order; a unit of linear j > 0 loads its X tile
+// only once every unit of linear j - 1 for the same token tile has stored its outputs (both CTAs of
+// each of its n_groups units: 2 n_groups arrivals on tile_done[j - 1][tile]). Only linears whose
+// groups are not cut into slices, with bf16 output and no residual, are chained.
+struct ChainJob {
+  CUtensorMap tmX;   // this linear's input (any earlier linear's output, or the chain's input)
+  CUtensorMap tmW;   // its weight stream
+  LinearParams P;
+  uint32_t unit0;    // index of its first unit in the chain's unit order
+  uint32_t units;    // n_tt * n_groups
+};
+constexpr int CHAIN_MAX_JOBS = 48;  // linears per launch (the whole table travels in the parameters)
+struct ChainParams {
+  ChainJob job[CHAIN_MAX_JOBS];
+  uint32_t *tile_done;   // [njobs][n_tt] stored-unit arrivals per (linear, token tile); zero at entry
+  uint32_t total_units;
+  int njobs, n_tt;
+};
+static_assert(sizeof(ChainParams) <= 32764, "kernel parameter space");
+cudaError_t launch_linear_chain(const ChainParams &C, int grid, cudaStream_t s);
 // Token counts up to SMALL_M_MAX take the small-m kernel (one launch, no workspace beyond the
 // control block); it sets P.kp itself.
 constexpr int SMALL_M_MAX = 256;

@@ -26,6 +26,11 @@
 // Accumulators are double-buffered in TMEM (2 x 256 columns), so one unit's epilogue overlaps the
 // next unit's MMAs. Every wait is bounded: on timeout the CTA records an error bit, drains its own
 // copies and MMAs, frees TMEM and returns.
+// A chain launch runs several linears over the same tokens in one launch (units of linear j after
+// those of linear j - 1): each CTA counts a unit's stores on a per-(linear, token tile) counter with
+// a gpu-scope release, and the X producer of a unit of linear j waits (acquire, then a proxy fence)
+// for linear j - 1's count on its token tile before its tensor copies. No launch boundary separates
+// the linears: one linear's last units overlap the next one's first.
 #include <cstddef>
 #include <cstdint>
 #include <cuda.h>
@@ -83,8 +88,8 @@ template <bool DEEP>
 struct Smem {
   static constexpr int NSTAGES = Depth<DEEP>::NSTAGES;
   static constexpr int BAR_OFF = NSTAGES * STAGE_BYTES;
-  // barriers: full[NS], empty[NS], accf[2], acce[2], unitf[UR], unite[UR], drain
-  static constexpr int NBARS = 2 * NSTAGES + 4 + 2 * UR + 1;
+  // barriers: full[NS], empty[NS], accf[2], acce[2], unitf[UR], unite[UR], drain, stored[2] (chain)
+  static constexpr int NBARS = 2 * NSTAGES + 4 + 2 * UR + 3;
   static constexpr int RING_OFF = (BAR_OFF + 8 * NBARS + 31) / 32 * 32;
   static constexpr int MISC_OFF = RING_OFF + (int)sizeof(UnitSlot) * UR;
   static constexpr int BIAS_OFF = MISC_OFF + 64;  // per epilogue warp: its 64 features' bias
@@ -203,6 +208,30 @@ __device__ __forceinline__ void mbar_arrive_relaxed_cluster(uint32_t cluster_add
   asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" :: "r"(cluster_addr) : "memory");
 }
 
+// Chain counters: a gpu-scope release increment (cumulative: it publishes the stores that this thread
+// has acquired, i.e. those of every epilogue warp of the CTA) and its acquiring, bounded wait.
+__device__ __forceinline__ void red_release_gpu_add(uint32_t *p, uint32_t v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+// Warp-collective: true once every lane has read a count >= need (each lane's own acquire); false
+// after limit_ns or once the CTA's abort flag is up.
+__device__ __forceinline__ bool wait_count(const uint32_t *p, uint32_t need, const volatile int *abort_flag,
+                                           uint64_t limit_ns) {
+  if (__all_sync(0xffffffffu, ld_acquire_gpu(p) >= need)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (;;) {
+    __nanosleep(128);
+    if (__all_sync(0xffffffffu, ld_acquire_gpu(p) >= need)) return true;
+    if (__any_sync(0xffffffffu, *abort_flag != 0)) return false;
+    if (__any_sync(0xffffffffu, globaltimer_ns() - t0 > limit_ns)) return false;
+  }
+}
+
 __device__ __forceinline__ void st_global_32B(void *p, const uint32_t (&w)[8]) {
   asm volatile("st.global.L1::no_allocate.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]), "r"(w[1]), "r"(w[2]),
                "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
@@ -230,9 +259,11 @@ __device__ __forceinline__ int table_at(const int (&t)[N], int g) {
 // t: y[0..16) are its accumulated sums (or zero), bs the run's bias in shared memory (the same for
 // every lane). Adds the bias, applies GELU, rounds and stores the lane's 32-byte (bf16) or 64-byte
 // (fp32) row segment with 32-byte stores, so that each store instruction writes whole sectors;
-// bf16 output may add the residual (each sum rounded, as a separate bf16 addition would).
+// bf16 output may add the residual (each sum rounded, as a separate bf16 addition would). GELU
+// compiles the activation in; do_gelu applies it (a chain decides per linear).
 template <bool GELU, bool F32, bool BIASG>
-__device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, int64_t t, const LinearParams &P) {
+__device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, int64_t t, const LinearParams &P,
+                                           bool do_gelu) {
 #pragma unroll
   for (int i = 0; i < 16; i += 4) {
     uint64_t b01 = 0, b23 = 0;
@@ -252,7 +283,7 @@ __device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, 
     unpk2(add2(pk2(y[i], y[i + 1]), b01), y[i], y[i + 1]);
     unpk2(add2(pk2(y[i + 2], y[i + 3]), b23), y[i + 2], y[i + 3]);
   }
-  if (GELU) {
+  if (GELU && do_gelu) {
 #pragma unroll
     for (int i = 0; i < 16; i += 2) gelu_erf2(y[i], y[i + 1]);
   }
@@ -312,10 +343,12 @@ __device__ __forceinline__ void emit_run16(float (&y)[16], uint32_t bs, int f0, 
   }
 }
 
-template <bool GELU, bool F32, bool DEEP>
-__global__ void __launch_bounds__(NUM_THREADS, 1)
-bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
-                  const LinearParams P) {
+// The pair kernel. One linear: tensor maps tmX0 / tmW0 and parameters P, C unused. A chain (CHAIN):
+// C the launch's table, P its first linear's parameters (workspace, token count, timeout), GELU
+// compiled in and applied to the linears that ask for it.
+template <bool GELU, bool F32, bool DEEP, bool CHAIN>
+__device__ __forceinline__ void pair_body(const CUtensorMap *tmX0, const CUtensorMap *tmW0, const LinearParams &P,
+                                          const ChainParams *C) {
   using L = Smem<DEEP>;
   constexpr int NSTAGES = L::NSTAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -334,10 +367,18 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
   auto unitf_bar = [&](int u) { return bar0 + 8u * (RB + 4 + u); };
   auto unite_bar = [&](int u) { return bar0 + 8u * (RB + 4 + UR + u); };
   const uint32_t drain_bar = bar0 + 8u * (RB + 4 + 2 * UR);
+  auto stored_bar = [&](int b) { return bar0 + 8u * (RB + 5 + 2 * UR + b); };  // chain: a unit's stores
   UnitSlot *ring = reinterpret_cast<UnitSlot *>(smem + L::RING_OFF);
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + L::MISC_OFF);
   volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 4);
   volatile int *never_flag = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 8);  // stays 0
+  volatile int *chain_ok_s = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 12);  // chain: plans checked
+  volatile int *last_cta_s = reinterpret_cast<volatile int *>(smem + L::MISC_OFF + 16);  // chain: last CTA out
+  // the parameters of the unit's linear (a chain's record names it; one linear: P)
+  auto jobp = [&](int j) -> const LinearParams & {
+    if constexpr (CHAIN) return C->job[j].P;
+    else return P;
+  };
 
   const int32_t *gent = P.sched + SCHED_HDR_INTS;
   const int32_t *gpan = P.sched + sched_gpan_offset_ints(P.n_groups);
@@ -358,6 +399,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     if (lane < 2) {
       mbar_init(accf_bar(lane), 1);
       mbar_init(acce_bar(lane), 2 * EPI_WARPS);
+      if (CHAIN) mbar_init(stored_bar(lane), EPI_WARPS);
     }
     if (lane < UR) {
       mbar_init(unitf_bar(lane), 1);
@@ -370,20 +412,41 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 0 && lane == 0) {
-    prefetch_tensormap(&tmX);
-    prefetch_tensormap(&tmW);
+  if constexpr (CHAIN) {
+    if (warp == 0)
+      for (int j = lane; j < C->njobs; j += 32) {
+        prefetch_tensormap(&C->job[j].tmX);
+        prefetch_tensormap(&C->job[j].tmW);
+      }
+  } else if (warp == 0 && lane == 0) {
+    prefetch_tensormap(tmX0);
+    prefetch_tensormap(tmW0);
   }
   // the work list must be this weight's plan: layout, group count, shape
-  const bool sched_ok = P.sched[3] == 0 && P.sched[1] == P.n_groups && P.sched[4] == P.n && P.sched[5] == P.k &&
-                        P.sched[6] == P.bn && P.sched[8] == SCHED_VERSION && P.n_groups <= MAX_GROUPS;
+  auto plan_ok = [](const LinearParams &Q) {
+    return Q.sched[3] == 0 && Q.sched[1] == Q.n_groups && Q.sched[4] == Q.n && Q.sched[5] == Q.k &&
+           Q.sched[6] == Q.bn && Q.sched[8] == SCHED_VERSION && Q.n_groups <= MAX_GROUPS;
+  };
+  bool sched_ok = !CHAIN && plan_ok(P);
+  if constexpr (CHAIN) {
+    if (warp == SCHED_WARP) {  // every linear's plan, a lane per linear (1 ok, 2 overflowed, 0 bad)
+      bool ok = true, ovf = false;
+      for (int j = lane; j < C->njobs; j += 32) {
+        ok = ok && plan_ok(C->job[j].P);
+        ovf = ovf || C->job[j].P.sched[3] != 0;
+      }
+      ok = __all_sync(0xffffffffu, ok);
+      ovf = __any_sync(0xffffffffu, ovf);
+      if (lane == 0) *chain_ok_s = ok ? 1 : (ovf ? 2 : 0);
+    }
+  }
   // When no group is cut into slices (S >= the chunk count), pair p's first unit is unit p: token
   // tile p / n_groups, group p % n_groups, all of that group's entries. The producers and the MMA
   // issuer take it from the work list themselves rather than wait for the scheduler's record (which
   // is the same); the group's entry range is requested here, so the load overlaps the prologue.
   const uint32_t u0 = blockIdx.x / 2;
   const uint32_t unsplit_units = (uint32_t)P.n_tt * (uint32_t)P.n_groups;
-  const bool first_local = sched_ok && P.S >= kc && (warp == 0 || warp == 1 || warp == W_WARP);
+  const bool first_local = !CHAIN && sched_ok && P.S >= kc && (warp == 0 || warp == 1 || warp == W_WARP);
   int f_ga = 0, f_gb = 0;
   if (first_local && u0 < unsplit_units) {
     const int g = (int)(u0 % (uint32_t)P.n_groups);
@@ -409,7 +472,11 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
   cluster_sync();  // both CTAs' barriers are initialised before any signal crosses the pair
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  if (!sched_ok && tid == 0 && leader) atomicOr(&P.ctl->err, P.sched[3] ? ERR_SCHED_OVERFLOW : ERR_BAD_SCHED);
+  if constexpr (CHAIN) sched_ok = *chain_ok_s == 1;
+  if (!sched_ok && tid == 0 && leader) {
+    const bool ovf = CHAIN ? *chain_ok_s == 2 : P.sched[3] != 0;
+    atomicOr(&P.ctl->err, ovf ? ERR_SCHED_OVERFLOW : ERR_BAD_SCHED);
+  }
 
   if (warp == 0 || warp == W_WARP) {
     // ============================================================== producers
@@ -438,24 +505,44 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
         else mbar_arrive_cluster(mapa_rank(unite_bar(slot), 0));
       }
       if (inf.tt < 0) break;
+      const LinearParams &Q = jobp(inf.pad);
+      const CUtensorMap *mX = tmX0, *mW = tmW0;
+      const int32_t *ents = entries;
+      int kcq = kc;
+      if constexpr (CHAIN) {
+        mX = &C->job[inf.pad].tmX;
+        mW = &C->job[inf.pad].tmW;
+        ents = Q.sched + sched_entries_offset_ints(Q.n_groups);
+        kcq = sched_chunks(Q.k);
+        if (xrole && inf.pad > 0 && inf.e1 > inf.e0) {
+          // the previous linear's outputs of this token tile, all of them stored, before the copies
+          const uint32_t need = 2u * (uint32_t)C->job[inf.pad - 1].P.n_groups;
+          if (!wait_count(C->tile_done + (size_t)(inf.pad - 1) * C->n_tt + inf.tt, need, abort_flag, tmo)) {
+            ok = false;
+            if (lane == 0) atomicOr(&P.ctl->err, ERR_CHAIN_WAIT);
+            break;
+          }
+          asm volatile("fence.proxy.async.global;" ::: "memory");  // order the tensor copies after the acquire
+        }
+      }
       // Stages: a batch of up to BATCH consecutive entries; lane i < nb waits for stage i's empty
       // barrier, then issues its stage's copy (this warp's kind), completing on the leader's full
       // barrier; the leader's X producer posts the stage's expected bytes (both kinds, both CTAs).
       const int ytok = inf.tt * TOKENS_PER_TILE + (int)rank * CTA_TOKENS;
       int win = inf.e0;
-      int cw_next = xrole && win + 32 + lane < inf.e1 ? __ldg(entries + win + 32 + lane) : 0;
+      int cw_next = xrole && win + 32 + lane < inf.e1 ? __ldg(ents + win + 32 + lane) : 0;
       for (int base = inf.e0; base < inf.e1 && ok; base += BATCH) {
         const int nb = min(BATCH, inf.e1 - base);
         if (base >= win + 32) {  // BATCH divides 32: a batch never straddles two windows
           win += 32;
           cw = cw_next;
-          cw_next = xrole && win + 32 + lane < inf.e1 ? __ldg(entries + win + 32 + lane) : 0;
+          cw_next = xrole && win + 32 + lane < inf.e1 ? __ldg(ents + win + 32 + lane) : 0;
         }
         const int e = base + (lane < nb ? lane : 0);  // the batch entry of this lane's copy
         int c = __shfl_sync(0xffffffffu, cw, (e - win) & 31);
         int tile = e;
         // a chunk or tile outside the work list's ranges means a corrupt list: flag it, load tile 0
-        const bool in_range = xrole ? (c >= 0 && c < kc) : ((int64_t)tile < P.stream_tiles);
+        const bool in_range = xrole ? (c >= 0 && c < kcq) : ((int64_t)tile < Q.stream_tiles);
         if (!in_range) {
           c = 0;
           tile = 0;
@@ -474,8 +561,8 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
         if (lane < nb) {  // the batch's stages are all free: one issue step for all of them
           if (!in_range) atomicOr(&P.ctl->err, ERR_BAD_SCHED);
           if (leader && xrole) mbar_arrive_expect_tx(full_bar(stk), 2 * STAGE_BYTES);
-          if (xrole) tma_load_2d_pair(st, &tmX, c * CHUNK_COLS, ytok, fb);
-          else tma_load_2d_pair(st + X_BYTES, &tmW, 0, tile * GROUP_FEATURES + (int)rank * HALF_FEATURES, fb);
+          if (xrole) tma_load_2d_pair(st, mX, c * CHUNK_COLS, ytok, fb);
+          else tma_load_2d_pair(st + X_BYTES, mW, 0, tile * GROUP_FEATURES + (int)rank * HALF_FEATURES, fb);
         }
         __syncwarp();
         it += nb;
@@ -499,72 +586,23 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     // and the unit's first 32 chunk indices, written locally and into the peer, then both CTAs'
     // unit-full barriers. Runs up to UR units ahead of the producers.
     if (leader) {
-      // slices per group = max(1, ceil(entries / S)) and their exclusive prefix, kept in registers:
-      // lane l holds group l + 32 j in sp[j] (first slice) and ge[j] (first entry)
-      constexpr int GPL = MAX_GROUPS / 32;
-      int sp[GPL], ge[GPL];
-      int run = 0;
-#pragma unroll
-      for (int j = 0; j < GPL; ++j) {
-        const int g = 32 * j + lane;
-        int c = 0, g0 = 0;
-        if (sched_ok && g < P.n_groups) {
-          g0 = gent[g];
-          const int cnt = gent[g + 1] - g0;
-          c = cnt <= 0 ? 1 : (cnt + P.S - 1) / P.S;
-        }
-        int incl = c;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int t = __shfl_up_sync(0xffffffffu, incl, o);
-          if (lane >= o) incl += t;
-        }
-        sp[j] = run + incl - c;
-        ge[j] = g0;
-        run += __shfl_sync(0xffffffffu, incl, 31);
-      }
-      const int total_slices = run;
-      const int ge_end = sched_ok ? gent[P.n_groups] : 0;
-      const uint32_t total_units = sched_ok ? (uint32_t)P.n_tt * (uint32_t)total_slices : 0u;
-      bool ok = true;
+      bool ok = true, queued = false;
       // the first unit of pair p is unit p (no queue round trip before the first copies); the queue
       // hands out the units after the first gridDim.x / 2. When every unit is such a first unit
       // (small token counts), no pair touches the queue or its counters.
       const uint32_t npairs = gridDim.x / 2;
-      const bool queued = total_units > npairs;  // the same in every pair
       uint32_t fetched = blockIdx.x / 2;
-      for (uint32_t pub = 0;; ++pub) {
+      // waits for ring slot `pub` to be free in both CTAs
+      auto slot_free = [&](uint32_t pub) -> bool {
+        if (mbar_wait_cluster(unite_bar(pub % UR), ((pub / UR) & 1u) ^ 1u, abort_flag, tmo)) return true;
+        ok = false;
+        if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_UNIT);
+        return false;
+      };
+      // writes record d and its first 32 chunk indices (from ents) into slot `pub` of both CTAs
+      auto publish = [&](uint32_t pub, const UnitInfo &d, const int32_t *ents) {
         const uint32_t slot = pub % UR;
-        if (!mbar_wait_cluster(unite_bar(slot), ((pub / UR) & 1u) ^ 1u, abort_flag, tmo)) {
-          ok = false;
-          if (lane == 0) atomicOr(&P.ctl->err, ERR_PRODUCER_UNIT);
-          break;
-        }
-        const uint32_t u = __shfl_sync(0xffffffffu, fetched, 0);
-        UnitInfo d;
-        if (u < total_units) {
-          d.tt = (int)(u / (uint32_t)total_slices);
-          const int rr = (int)(u % (uint32_t)total_slices);
-          // group g with sp[g] <= rr < sp[g + 1]: every group has a slice, so g + 1 = #{g : sp[g] <= rr}
-          int cnt = 0;
-#pragma unroll
-          for (int j = 0; j < GPL; ++j)
-            cnt += __popc(__ballot_sync(0xffffffffu, 32 * j + lane < P.n_groups && sp[j] <= rr));
-          const int g = cnt - 1;
-          const int s0 = table_at(sp, g), s1 = g + 1 < P.n_groups ? table_at(sp, g + 1) : total_slices;
-          const int ge0 = table_at(ge, g), ge1 = g + 1 < P.n_groups ? table_at(ge, g + 1) : ge_end;
-          d.g = g;
-          d.s = rr - s0;
-          d.nsl = s1 - s0;
-          d.e0 = min(ge0 + d.s * P.S, ge1);
-          d.e1 = min(d.e0 + P.S, ge1);
-          d.ptile = d.tt * total_slices + rr;
-        } else {
-          d.tt = -1; d.g = d.s = d.nsl = d.e0 = d.e1 = d.ptile = 0;
-        }
-        d.pad = 0;
-        if (lane == 0 && u < total_units) fetched = queued ? npairs + atomicAdd(&P.ctl->next_unit, 1u) : total_units;
-        const int wv = d.e0 + lane < d.e1 ? __ldg(entries + d.e0 + lane) : 0;
+        const int wv = d.e0 + lane < d.e1 ? __ldg(ents + d.e0 + lane) : 0;
         UnitSlot &rs = ring[slot];
         const uint32_t remote = mapa_rank(smem_u32(&rs), 1);
         rs.win[lane] = wv;
@@ -583,7 +621,95 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
           mbar_arrive_cluster(mapa_rank(unitf_bar(slot), 1));
         }
         __syncwarp();
-        if (u >= total_units) break;
+      };
+      if constexpr (CHAIN) {
+        // units in order: linear 0's (token-tile-major), then linear 1's, ...; a unit never cut
+        const uint32_t total_units = sched_ok ? C->total_units : 0u;
+        queued = total_units > npairs;
+        int jc = 0;  // the linear of the last unit taken (units come in increasing order)
+        for (uint32_t pub = 0;; ++pub) {
+          if (!slot_free(pub)) break;
+          const uint32_t u = __shfl_sync(0xffffffffu, fetched, 0);
+          UnitInfo d;
+          const int32_t *ents = nullptr;
+          if (u < total_units) {
+            while (jc + 1 < C->njobs && u >= C->job[jc].unit0 + C->job[jc].units) ++jc;
+            const LinearParams &Q = C->job[jc].P;
+            const uint32_t r = u - C->job[jc].unit0;
+            d.tt = (int)(r / (uint32_t)Q.n_groups);
+            d.g = (int)(r % (uint32_t)Q.n_groups);
+            d.s = 0;
+            d.nsl = 1;
+            d.e0 = __ldg(Q.sched + SCHED_HDR_INTS + d.g);
+            d.e1 = __ldg(Q.sched + SCHED_HDR_INTS + d.g + 1);
+            d.ptile = (int)r;
+            d.pad = jc;
+            ents = Q.sched + sched_entries_offset_ints(Q.n_groups);
+          } else {
+            d.tt = -1; d.g = d.s = d.nsl = d.e0 = d.e1 = d.ptile = d.pad = 0;
+          }
+          if (lane == 0 && u < total_units) fetched = queued ? npairs + atomicAdd(&P.ctl->next_unit, 1u) : total_units;
+          publish(pub, d, ents);
+          if (u >= total_units) break;
+        }
+      } else {
+        // slices per group = max(1, ceil(entries / S)) and their exclusive prefix, kept in registers:
+        // lane l holds group l + 32 j in sp[j] (first slice) and ge[j] (first entry)
+        constexpr int GPL = MAX_GROUPS / 32;
+        int sp[GPL], ge[GPL];
+        int run = 0;
+#pragma unroll
+        for (int j = 0; j < GPL; ++j) {
+          const int g = 32 * j + lane;
+          int c = 0, g0 = 0;
+          if (sched_ok && g < P.n_groups) {
+            g0 = gent[g];
+            const int cnt = gent[g + 1] - g0;
+            c = cnt <= 0 ? 1 : (cnt + P.S - 1) / P.S;
+          }
+          int incl = c;
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += t;
+          }
+          sp[j] = run + incl - c;
+          ge[j] = g0;
+          run += __shfl_sync(0xffffffffu, incl, 31);
+        }
+        const int total_slices = run;
+        const int ge_end = sched_ok ? gent[P.n_groups] : 0;
+        const uint32_t total_units = sched_ok ? (uint32_t)P.n_tt * (uint32_t)total_slices : 0u;
+        queued = total_units > npairs;  // the same in every pair
+        for (uint32_t pub = 0;; ++pub) {
+          if (!slot_free(pub)) break;
+          const uint32_t u = __shfl_sync(0xffffffffu, fetched, 0);
+          UnitInfo d;
+          if (u < total_units) {
+            d.tt = (int)(u / (uint32_t)total_slices);
+            const int rr = (int)(u % (uint32_t)total_slices);
+            // group g with sp[g] <= rr < sp[g + 1]: every group has a slice, so g + 1 = #{g : sp[g] <= rr}
+            int cnt = 0;
+#pragma unroll
+            for (int j = 0; j < GPL; ++j)
+              cnt += __popc(__ballot_sync(0xffffffffu, 32 * j + lane < P.n_groups && sp[j] <= rr));
+            const int g = cnt - 1;
+            const int s0 = table_at(sp, g), s1 = g + 1 < P.n_groups ? table_at(sp, g + 1) : total_slices;
+            const int ge0 = table_at(ge, g), ge1 = g + 1 < P.n_groups ? table_at(ge, g + 1) : ge_end;
+            d.g = g;
+            d.s = rr - s0;
+            d.nsl = s1 - s0;
+            d.e0 = min(ge0 + d.s * P.S, ge1);
+            d.e1 = min(d.e0 + P.S, ge1);
+            d.ptile = d.tt * total_slices + rr;
+          } else {
+            d.tt = -1; d.g = d.s = d.nsl = d.e0 = d.e1 = d.ptile = 0;
+          }
+          d.pad = 0;
+          if (lane == 0 && u < total_units) fetched = queued ? npairs + atomicAdd(&P.ctl->next_unit, 1u) : total_units;
+          publish(pub, d, entries);
+          if (u >= total_units) break;
+        }
       }
       if (!ok && lane == 0) *abort_flag = 1;
       // queue bookkeeping: the last scheduler to leave resets the counters for the next launch
@@ -685,7 +811,7 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       }
       out = ring[slot].inf;
       const uint32_t read = __ballot_sync(0xffffffffu, (out.tt ^ out.g ^ out.s ^ out.nsl ^ out.e0 ^ out.e1 ^ out.ptile) !=
-                                                           0x7fffffff || out.pad == 0);
+                                                           0x7fffffff || out.pad >= 0);
       if (lane == 0 && read != 0u) {
         if (leader) mbar_arrive_relaxed(unite_bar(slot));
         else mbar_arrive_relaxed_cluster(mapa_rank(unite_bar(slot), 0));
@@ -696,13 +822,15 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
     bool have = take_unit(0, inf);
     uint32_t ui = 0;
     while (have && inf.tt >= 0) {
+      const LinearParams &Q = jobp(inf.pad);
+      const int32_t *gp = CHAIN ? Q.sched + sched_gpan_offset_ints(Q.n_groups) : gpan;
       // the features of this warp's 64 columns (first feature of each 16-column quarter, or -1)
       int fcol[4];
 #pragma unroll
       for (int r4 = 0; r4 < 4; ++r4) {
         const int c = 64 * part + 16 * r4;
-        const int panel = __ldg(gpan + (int64_t)inf.g * MAX_GROUP_PANELS + c / P.bn);
-        fcol[r4] = panel >= 0 ? panel * P.bn + c % P.bn : -1;
+        const int panel = __ldg(gp + (int64_t)inf.g * MAX_GROUP_PANELS + c / Q.bn);
+        fcol[r4] = panel >= 0 ? panel * Q.bn + c % Q.bn : -1;
       }
       // and their bias, staged while the accumulator is still being computed
       if (!DEEP && lane < 16) {
@@ -710,11 +838,11 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
         const int fq = qq == 0 ? fcol[0] : (qq == 1 ? fcol[1] : (qq == 2 ? fcol[2] : fcol[3]));
         const int f = fq < 0 ? -1 : fq + 4 * (lane & 3);
         float4 b4 = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (f >= 0 && P.bias != nullptr) {
-          if (P.bias_vec16) {
-            b4 = __ldg(reinterpret_cast<const float4 *>(P.bias + f));
+        if (f >= 0 && Q.bias != nullptr) {
+          if (Q.bias_vec16) {
+            b4 = __ldg(reinterpret_cast<const float4 *>(Q.bias + f));
           } else {
-            b4 = make_float4(__ldg(P.bias + f), __ldg(P.bias + f + 1), __ldg(P.bias + f + 2), __ldg(P.bias + f + 3));
+            b4 = make_float4(__ldg(Q.bias + f), __ldg(Q.bias + f + 1), __ldg(Q.bias + f + 2), __ldg(Q.bias + f + 3));
           }
         }
         *reinterpret_cast<float4 *>(bias_s + 4 * lane) = b4;
@@ -732,6 +860,17 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       const bool tvalid = t < P.m;
       const bool split = inf.nsl > 1;
       const bool touched = inf.e1 > inf.e0;
+      if constexpr (CHAIN) {
+        // a unit with no entries loads nothing, so no copy waited for the previous linear: its
+        // stores wait here, so that they follow every earlier linear's use of this token tile
+        if (!touched && inf.pad > 0 &&
+            !wait_count(C->tile_done + (size_t)(inf.pad - 1) * C->n_tt + inf.tt,
+                        2u * (uint32_t)C->job[inf.pad - 1].P.n_groups, abort_flag, tmo)) {
+          if (lane == 0) { atomicOr(&P.ctl->err, ERR_CHAIN_WAIT); *abort_flag = 1; }
+          break;
+        }
+      }
+      const bool do_gelu = !CHAIN || Q.gelu != 0;
       float *part_row = nullptr;
       if (split)
         part_row = P.partials + ((int64_t)inf.ptile * P.part_rows + t_tile) * GROUP_FEATURES;
@@ -763,10 +902,17 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
             yb[i] = v[16 + i];
           }
           const uint32_t bs = smem_u32(bias_s + 32 * h);
-          if (fa >= 0) emit_run16<GELU, F32, DEEP>(ya, bs, fa, t, P);
-          if (fb2 >= 0) emit_run16<GELU, F32, DEEP>(yb, bs + 64, fb2, t, P);
+          if (fa >= 0) emit_run16<GELU, F32, DEEP>(ya, bs, fa, t, Q, do_gelu);
+          if (fb2 >= 0) emit_run16<GELU, F32, DEEP>(yb, bs + 64, fb2, t, Q, do_gelu);
         }
         __syncwarp();
+      }
+      if constexpr (CHAIN) {
+        // this warp's stores of the unit are done (a CTA-scope release); arriving before the
+        // accumulator hand-back means a stored barrier phase always completes before the MMAs of
+        // the unit two ahead, which reuses it, can start
+        __syncwarp();
+        if (lane == 0) mbar_arrive(stored_bar((int)(ui & 1u)));
       }
       // the accumulator buffer is free again (the leader's MMAs wait for both CTAs' warps); its
       // loads have completed and no memory written here is handed over, so no release ordering
@@ -775,6 +921,18 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
       if (lane == 0) {
         if (leader) mbar_arrive_relaxed(acce_bar(buf));
         else mbar_arrive_relaxed_cluster(mapa_rank(acce_bar(buf), 0));
+      }
+      if constexpr (CHAIN) {
+        // one epilogue warp per unit, in turn, publishes the CTA's stores of it to the next linear:
+        // it acquires the 16 warps' arrivals, then counts them with a gpu-scope release (which waits
+        // for the stores to complete; taking turns spreads that wait over the warps)
+        if (warp == FIRST_EPI + (int)(ui % (uint32_t)EPI_WARPS)) {
+          if (!mbar_wait(stored_bar((int)(ui & 1u)), (ui >> 1) & 1u, abort_flag, tmo)) {
+            if (lane == 0) { atomicOr(&P.ctl->err, ERR_CHAIN_WAIT); *abort_flag = 1; }
+            break;
+          }
+          if (lane == 0) red_release_gpu_add(C->tile_done + (size_t)inf.pad * C->n_tt + inf.tt, 1u);
+        }
       }
       inf = nxt;
       ++ui;
@@ -787,6 +945,35 @@ bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant
   cluster_sync();  // no signal, copy or MMA of the pair is still aimed at either CTA
   tc_fence_after();
   if (warp == 1) tmem_dealloc_pair(tmem_base, 512);
+  if constexpr (CHAIN) {
+    // the last CTA out (every other CTA has finished its waits and counts) clears the tile
+    // counters for the next chain launch on this workspace
+    if (tid == 0) {
+      __threadfence();
+      *last_cta_s = atomicAdd(&P.ctl->chain_ctas, 1u) == gridDim.x - 1 ? 1 : 0;
+    }
+    __syncthreads();
+    if (*last_cta_s) {
+      __threadfence();
+      const int count = C->njobs * C->n_tt;
+      for (int i = tid; i < count; i += NUM_THREADS) C->tile_done[i] = 0u;
+      if (tid == 0) P.ctl->chain_ctas = 0u;
+      __threadfence();
+    }
+  }
+}
+
+template <bool GELU, bool F32, bool DEEP>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+bsr_linear_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
+                  const LinearParams P) {
+  pair_body<GELU, F32, DEEP, false>(&tmX, &tmW, P, nullptr);
+}
+
+// Chains: bf16 outputs, six stages with the staged bias (the long-K linears lose their seventh
+// stage), GELU per linear.
+__global__ void __launch_bounds__(NUM_THREADS, 1) bsr_linear_chain_kernel(const __grid_constant__ ChainParams C) {
+  pair_body<true, false, false, true>(nullptr, nullptr, C.job[0].P, &C);
 }
 
 // Split units: Y = act(sum over the slices, in slice order, of the partial sums + bias). One thread
@@ -1198,6 +1385,33 @@ cudaError_t launch_linear(const CUtensorMap &tmX, const CUtensorMap &tmW, const 
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kern, tmX, tmW, P);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
+cudaError_t launch_linear_chain(const ChainParams &C, int grid, cudaStream_t s) {
+  static bool attr_done[64] = {false};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 0 && dev < 64 && !attr_done[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(bsr_linear_chain_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         Smem<false>::BYTES);
+    if (e != cudaSuccess) return e;
+    attr_done[dev] = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = Smem<false>::BYTES;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, bsr_linear_chain_kernel, C);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

@@ -13,6 +13,9 @@ layer on one stream:
 Attention, LayerNorm and residuals are not part of this path. All buffers are allocated once;
 a step allocates nothing, so it can be captured in a CUDA graph. The C entry points are called
 through pre-marshalled ctypes argument lists to keep host overhead per call at a few microseconds.
+The linears run either as one library call each or, with ``chain=True``, as one chain call
+(lpvit_bsr_linear_chain: the 48 linears in one persistent launch, each token tile of a linear
+starting once the previous linear has stored it); both give the same bits.
 """
 from __future__ import annotations
 
@@ -34,6 +37,7 @@ class DeitLinearStack:
         self._pack_fn = lib.lpvit_pack_bsr
         self._pack_many_fn = lib.lpvit_pack_bsr_many
         self._lin = {False: lib.lpvit_bsr_linear, True: lib.lpvit_bsr_linear_gelu}
+        self._chain_fn = lib.lpvit_bsr_linear_chain
         d = layers[0]["qkv"]["W"].shape[1]
         h = layers[0]["fc1"]["W"].shape[0]
         self.d, self.h = d, h
@@ -55,6 +59,8 @@ class DeitLinearStack:
                                    "gelu": bool(g["gelu"]), "w": w, "struct": w.struct(),
                                    "nnzb": int((g["mask"] != 0).sum())})
         ws_bytes = max(_lib.lpvit_workspace_bytes(G["struct"], m) for G in self.gemms)
+        sizing = _lib.chain_links([(G["struct"], 0, 0, 0, 0, 0, 0) for G in self.gemms])
+        ws_bytes = max(ws_bytes, _lib.lpvit_chain_workspace_bytes(sizing, len(self.gemms), m))
         self.ws = torch.zeros(max(ws_bytes, 256), dtype=torch.uint8, device=device)
         self._calls = None
 
@@ -72,10 +78,11 @@ class DeitLinearStack:
             tot += 2 * self.m * k + 2 * self.m * n + 2 * G["nnzb"] * bn * bk + 4 * G["nnzb"] + 4 * (n // bn + 1) + 4 * n
         return tot
 
-    def launches_per_step(self) -> int:
-        """Kernel launches of one step: one per linear, two per batched pack of up to 96 weights."""
+    def launches_per_step(self, chain: bool = False) -> int:
+        """Kernel launches of one step: one per linear (or one per 48 linears of a chain call), two per
+        batched pack of up to 96 weights."""
         n = len(self.gemms)
-        return n + 2 * ((n + 95) // 96)
+        return ((n + 47) // 48 if chain else n) + 2 * ((n + 95) // 96)
 
     # ------------------------------------------------------------------ launches
     def _build_calls(self, stream: int):
@@ -89,6 +96,7 @@ class DeitLinearStack:
         wsn = ctypes.c_size_t(self.ws.numel())
         st = V(stream)
         src = self.h_in
+        links = []
         for gi, G in enumerate(self.gemms):
             pack_args = (V(G["W"].data_ptr()), V(G["mask"].data_ptr()), ctypes.byref(G["struct"]), None, st)
             name = G["name"]
@@ -105,7 +113,10 @@ class DeitLinearStack:
                         V(G["bias"].data_ptr()), V(Y.data_ptr()), ctypes.c_int64(Y.stride(0)),
                         ctypes.c_int(_lib.LPVIT_BF16), ws, wsn, st)
             calls.append((pack_args, self._lin[G["gelu"]], lin_args))
+            links.append((G["struct"], X.data_ptr(), ldx, G["bias"].data_ptr(), Y.data_ptr(), Y.stride(0), G["gelu"]))
         self.out = src
+        arr = _lib.chain_links(links)
+        self._chain_args = (arr, ctypes.c_int32(len(links)), ctypes.c_int64(self.m), ws, wsn, st)
         return calls
 
     def _calls_for(self, stream: int):
@@ -129,11 +140,21 @@ class DeitLinearStack:
             if rc != 0:
                 raise _lib.LpvitError(rc, "lpvit_pack_bsr")
 
-    def forward(self, stream=None, events=None):
+    def forward(self, stream=None, events=None, chain: bool = False):
         """Chain the 4L linears from ``h_in``; returns the output buffer. ``events``: optional list of
-        (start, end) CUDA event pairs, one per linear, recorded around each launch."""
+        (start, end) CUDA event pairs recorded around each library call: one per linear, or one for
+        the whole chain call (``chain=True``)."""
         s = stream or torch.cuda.current_stream()
         calls = self._calls_for(int(s.cuda_stream))
+        if chain:
+            if events is not None:
+                events[0][0].record(s)
+            rc = self._chain_fn(*self._chain_args)
+            if events is not None:
+                events[0][1].record(s)
+            if rc != 0:
+                raise _lib.LpvitError(rc, "lpvit_bsr_linear_chain")
+            return self.out
         for i, (_, fn, lin_args) in enumerate(calls):
             if events is not None:
                 events[i][0].record(s)
@@ -144,10 +165,10 @@ class DeitLinearStack:
                 raise _lib.LpvitError(rc, "lpvit_bsr_linear")
         return self.out
 
-    def step(self, stream=None, events=None):
+    def step(self, stream=None, events=None, chain: bool = False):
         """One pass of the whole path: pack every weight, then run every linear."""
         self.pack_all(stream)
-        return self.forward(stream, events)
+        return self.forward(stream, events, chain)
 
     def check(self, stream=None):
         st = _lib.lpvit_check(self.ws.data_ptr(), int((stream or torch.cuda.current_stream()).cuda_stream))

@@ -175,3 +175,48 @@ def test_encoder_kernel_arguments_are_checked_without_a_gpu(lib):
     assert at(0x1000, 0, 197, 6, 64, 0x2000, None) == lib.LPVIT_OK                 # no images
     assert at(0x1008, 2, 197, 6, 64, 0x2000, None) == lib.LPVIT_ERR_INVALID_ARG
     assert at(0x1000, 2, 197, 0, 64, 0x2000, None) == lib.LPVIT_ERR_INVALID_ARG
+
+
+def test_chain_arguments_are_checked_without_a_gpu(lib):
+    """lpvit_bsr_linear_chain checks every link (as lpvit_bsr_linear would) before launching, and
+    sizes its workspace as the control block, the largest split partials and a counter per
+    (linear, token tile) of one launch."""
+    L = lib.load()
+    sched = 0x400000
+    b_qkv = lib.lpvit_bsr(2304, 768, 32, 32, 1728, None, None, None, sched, 1 << 24)
+    b_proj = lib.lpvit_bsr(768, 768, 32, 32, 576, None, None, None, sched, 1 << 24)
+    X, Y, ws = 0x1000000, 0x8000000, 0x100000
+    m = 50432
+    rows = [(b_qkv, X, 768, None, Y, 2304, 0), (b_proj, Y + 2 * 1536, 2304, None, 0x20000000, 768, 0)]
+    links = lib.chain_links(rows)
+    # a counter per (linear, 256-token tile) after the 256-byte control block (no split at this m)
+    tiles = (m + 255) // 256
+    assert lib.lpvit_chain_workspace_bytes(links, 2, m) == 256 + (2 * tiles * 4 + 255) // 256 * 256
+    assert lib.lpvit_chain_workspace_bytes(None, 2, m) == 0
+    assert lib.lpvit_chain_workspace_bytes(links, 0, m) == 0
+    bad = lib.chain_links([(lib.lpvit_bsr(2304, 770, 32, 32, 1, None, None, None, sched, 1 << 24),
+                            X, 776, None, Y, 2304, 0)])
+    assert lib.lpvit_chain_workspace_bytes(bad, 1, m) == 0
+    chain = L.lpvit_bsr_linear_chain
+    assert chain(links, 0, m, ws, 1 << 20, None) == lib.LPVIT_OK          # nothing to do
+    assert chain(links, 2, 0, ws, 1 << 20, None) == lib.LPVIT_OK          # no tokens
+    assert chain(links, -1, m, ws, 1 << 20, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert chain(None, 2, m, ws, 1 << 20, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert chain(links, 2, m, None, 1 << 20, None) == lib.LPVIT_ERR_INVALID_ARG
+    assert chain(links, 2, m, ws + 16, 1 << 20, None) == lib.LPVIT_ERR_INVALID_ARG   # workspace alignment
+    assert chain(links, 2, -5, ws, 1 << 20, None) == lib.LPVIT_ERR_INVALID_ARG
+
+    def one(**kw):
+        r = dict(bsr=b_qkv, X=X, ldx=768, bias=None, Y=Y, ldy=2304, gelu=0)
+        r.update(kw)
+        return chain(lib.chain_links([tuple(r.values())]), 1, m, ws, 1 << 20, None)
+    assert one(gelu=2) == lib.LPVIT_ERR_INVALID_ARG
+    assert one(bsr=None) == lib.LPVIT_ERR_INVALID_ARG
+    assert one(X=X + 2) == lib.LPVIT_ERR_INVALID_ARG        # X not 16-byte aligned
+    assert one(ldx=772) == lib.LPVIT_ERR_INVALID_ARG        # ldx % 8
+    assert one(ldy=2300) == lib.LPVIT_ERR_INVALID_ARG       # ldy < n
+    assert one(Y=X) == lib.LPVIT_ERR_INVALID_ARG            # Y overlaps X
+    assert one(bsr=bad[0].bsr.contents) == lib.LPVIT_ERR_INVALID_ARG   # k not a multiple of bk
+    # a bad second link stops the call before the first one runs
+    rows_bad = [rows[0], (b_proj, Y + 2 * 1536, 2304, None, 0x20000000, 768, 5)]
+    assert chain(lib.chain_links(rows_bad), 2, m, ws, 1 << 20, None) == lib.LPVIT_ERR_INVALID_ARG

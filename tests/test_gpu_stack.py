@@ -28,11 +28,16 @@ def stack_run():
     st.check()
     out2 = st.step().clone()
     st.check()
-    return layers, h0, out, out2
+    # the same step with the 48 linears as one chain call, twice on the same workspace
+    chained = []
+    for _ in range(2):
+        chained.append(st.step(chain=True).clone())
+        st.check()
+    return layers, h0, out, out2, chained
 
 
 def test_stack_sampled_rows_match_oracle(stack_run):
-    layers, h0, out, _ = stack_run
+    layers, h0, out, _, _ = stack_run
     m = out.shape[0]
     rows = np.unique(np.concatenate([np.random.default_rng(1).choice(m, 24, replace=False), [0, 1, m - 2, m - 1]]))
     olayers = [{n: (inputs.bf16_bits(L[n]["W"]), L[n]["mask"].numpy(), L[n]["bias"].cpu().numpy(), 32)
@@ -53,5 +58,12 @@ def test_stack_sampled_rows_match_oracle(stack_run):
 
 
 def test_stack_step_is_deterministic(stack_run):
-    _, _, out, out2 = stack_run
+    _, _, out, out2, _ = stack_run
     assert torch.equal(out, out2)
+
+
+def test_chained_stack_step_gives_the_same_bits(stack_run):
+    """lpvit_bsr_linear_chain over the 48 linears (one persistent launch) against the per-linear
+    launches of the same step, at the benchmarked size."""
+    _, _, out, _, chained = stack_run
+    assert torch.equal(chained[0], out) and torch.equal(chained[1], out)
