@@ -274,17 +274,18 @@ size_t lpvit_chain_workspace_bytes(const lpvit_chain_link *links, int32_t count,
 /* The linears links[0], links[1], ... links[count-1] over the same m tokens, in that order, as if
  * each were a separate lpvit_bsr_linear (gelu 0) / lpvit_bsr_linear_gelu (gelu 1) call with bf16
  * output on `stream`; the results are bit-identical to those calls. A link may read what earlier
- * links wrote (the layer chain of Sec. 3.3's block matmuls, one after another, e.g. fc1 -> fc2).
+ * links wrote (a model's pruned linears one after another, e.g. fc1 -> fc2, each the block-sparse
+ * matmul of Sec. 3.3).
  * Consecutive links run in one persistent launch (up to 48 links per launch): the units of a
  * link follow those of the link before it, and a unit of 256 tokens starts its copies once the
  * previous link has stored every output of those 256 tokens, so one link's last units overlap the
  * next link's first and the launch start and end are paid once per launch, not per link.
- * Rules: row r of every X and Y holds token r. Where a link's X or Y overlaps an earlier link's X
- * or Y, the two must have the same leading dimension and overlap only row for row (a column range
- * of the same rows, e.g. X = the last third of an earlier Y's columns); a link that breaks this,
- * one whose work would be cut into slices (few token tiles: m <= 256, or too few units to fill the
- * GPU), and m <= 256 generally, start a new launch or run on their own. No Y may overlap a weight,
- * work list or bias of the chain.
+ * Row r of every X and Y holds token r. Links share a launch only where their buffers overlap row
+ * for row (same leading dimension, a column range of the same rows, e.g. X = the last third of an
+ * earlier Y's columns); a link whose buffers overlap an earlier link's otherwise starts a new
+ * launch. A link that lpvit_bsr_linear would run on the small-m kernel (m <= 256) or cut into slices
+ * (too few 256-token tiles to fill the GPU) runs on its own, as that call would. No Y may overlap
+ * a weight, work list or bias of the chain.
  *   workspace / ws_bytes: >= lpvit_chain_workspace_bytes(links, count, m), 256-byte aligned.
  * Every link is checked before anything is launched; nothing runs if one fails.
  * Errors: LPVIT_ERR_INVALID_ARG (count < 0, null links or workspace, gelu not 0 or 1, and the
