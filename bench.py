@@ -5,10 +5,12 @@ Workload (one "step" = one pass of the whole block-sparse path over one batch): 
 DeiT-B linear stack (48 GEMMs: qkv 768->2304, proj 768->768, fc1 768->3072 + GELU,
 fc2 3072->768) at batch 256 (M = 50432 tokens), 32x32 blocks, per-GEMM block sparsity drawn
 U[30%, 70%] as antithetic layer pairs (mean exactly 50%); every weight is packed (mask -> BSR +
-work list) and every linear runs, chained layer to layer. Inputs are seeded synthetic bf16 tensors
-resident in HBM; each step streams ~15 GB, far more than the 129 MB L2, so no flush is needed.
+work list) and every linear runs, chained layer to layer: by default as one lpvit_bsr_linear_chain
+call (the 48 linears in one persistent launch), or with --launch per-linear one call per linear.
+Inputs are seeded synthetic bf16 tensors resident in HBM; each step streams ~15 GB, far more than
+the 129 MB L2, so no flush is needed.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl lpvit|reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl lpvit|reference] [--launch chain|per-linear]
 
 Prints one JSON line (rank 0). ``--impl reference`` times the CPU oracle (fp64 C loops on the
 host cores) on a bounded row sample of the same workload.
