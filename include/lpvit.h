@@ -267,8 +267,12 @@ typedef struct {
 } lpvit_chain_link;
 
 /* Bytes of device workspace lpvit_bsr_linear_chain needs for these links at m tokens (0 for a
- * null or empty list, or a link whose weight shape is invalid). Zero-filled once before its first
- * use; every call leaves it ready for the next (as lpvit_workspace_bytes). */
+ * null or empty list, or a link whose weight shape is invalid): the control block, room for the
+ * split-unit partial sums of any link that runs on its own, then the chain's tile counters.
+ * Zero-filled once before its first use; every chain call leaves it ready for the next. The same
+ * workspace may also serve lpvit_bsr_linear[_gelu] calls on these links' weights at the same m
+ * (their scratch lies below the counters); other calls can leave scratch data where the counters
+ * are, so give them a workspace of their own. */
 size_t lpvit_chain_workspace_bytes(const lpvit_chain_link *links, int32_t count, int64_t m);
 
 /* The linears links[0], links[1], ... links[count-1] over the same m tokens, in that order, as if
