@@ -17,12 +17,16 @@
  * blocks are stored, and removed blocks are never read. The GEMM multiplies, per 256-output group,
  * only the 64-column chunks where the group keeps a block (rows of removed blocks there enter as
  * zeros), so its work follows those group chunks rather than exactly the kept blocks that the
- * power model of Sec. 3.3 (Eq. for P) counts.
+ * power model of Sec. 3.3 (Eq. for P) counts. lpvit_bsr_linear_chain runs a list of such linears
+ * (a model's layers, one feeding the next) in one persistent launch.
  *
  * Conventions for every call:
- *  - All pointers except nnzb_host are DEVICE pointers owned by the caller; the library never
- *    allocates, frees or keeps them. All calls are asynchronous on `stream` (a cudaStream_t
- *    passed as void*, NULL = legacy default stream) unless stated otherwise.
+ *  - Array and matrix pointers are DEVICE pointers owned by the caller; the library never
+ *    allocates, frees or keeps them. The exceptions live in host memory: nnzb_host, the
+ *    lpvit_bsr and lpvit_chain_link structs (and the arrays of them passed to the _many and
+ *    _chain calls), which are plain host values holding device pointers, and the host arrays of
+ *    lpvit_pack_bsr_many and lpvit_lambda_search. All calls are asynchronous on `stream` (a
+ *    cudaStream_t passed as void*, NULL = legacy default stream) unless stated otherwise.
  *  - bf16 means IEEE-754 bfloat16 (raw 16-bit storage); all matrices are row-major.
  *  - A status is returned synchronously for argument errors; CUDA launch errors map to
  *    LPVIT_ERR_CUDA. Errors raised inside a running kernel (a bounded wait that ran out)
@@ -105,7 +109,7 @@ lpvit_status lpvit_pack_bsr(const void *W, const uint8_t *mask, lpvit_bsr *bsr, 
  * arrays of device pointers) are packed into bsr[i] (a host array of count descriptors, set up as
  * for lpvit_pack_bsr). Every job is checked as lpvit_pack_bsr checks its arguments before anything
  * is launched; the first failing check is returned and nothing runs. The jobs travel in the launch
- * parameters (96 per launch), so the call allocates nothing: all plans run in one launch, one CTA
+ * parameters (96 per launch), so the call allocates no device memory: all plans run in one launch, one CTA
  * per weight, then all block copies in one more. Results are bit-identical to count calls of
  * lpvit_pack_bsr. There is no kept-block count output; a capacity overflow is reported as for
  * lpvit_pack_bsr (the work list is marked invalid and lpvit_check reports it after a linear).
